@@ -1,0 +1,412 @@
+"""Pins of the CPU oracle: checks against what the paper and the mathematics fix.
+
+Each ``check_*`` raises AssertionError on failure.  ``test_oracle_pins.py`` runs
+them against the oracle as built, and against copies of the oracle source with
+a planted mistake (each mutant must fail at least one check).
+
+Sources of the expected values:
+  * Philox4x32-10 known-answer vectors (Salmon et al., SC'11 / Random123);
+  * the two worked examples of the group-size rule (Sec. 4.3);
+  * hand-worked cases of Eq. 1 / Alg. 1 l.13-15, Alg. 2 and Alg. 3
+    (``tests/golden/*.txt``, each derived in its comment header);
+  * exhaustive brute force of the +-1 dot product, N - 2 popcount(a XOR w);
+  * exact rational arithmetic for the reinforcement threshold, a binomial
+    bound on the reinforcement rate, and the closed form of Alg. 1 l.21;
+  * invariants of Alg. 3 (odd h, |h| <= h_max, one lattice unit per event,
+    reinforcement moves away from 0) and the learnability of a separable task.
+"""
+from __future__ import annotations
+
+import math
+from decimal import Decimal, getcontext
+from fractions import Fraction
+
+import numpy as np
+
+import oracle as O
+from conftest import read_golden
+
+
+# -- random stream ---------------------------------------------------------------
+
+def check_philox_kat():
+    for line in read_golden("philox4x32_10_kat.txt"):
+        v = [int(t, 16) for t in line.split()]
+        out = O.philox4x32_10(v[0:4], v[4:6])
+        assert [int(o) for o in out] == v[6:10], (line, [hex(int(o)) for o in out])
+
+
+# -- group size ----------------------------------------------------------------
+
+def check_gamma_golden():
+    for line in read_golden("gamma_rule.txt"):
+        K, g = (int(t) for t in line.split())
+        assert O.gamma_rule(K) == g, (K, O.gamma_rule(K), g)
+
+
+# -- forward ---------------------------------------------------------------------
+
+def _all_pm1(N):
+    codes = np.arange(2 ** N)
+    bits = (codes[:, None] >> np.arange(N)[None, :]) & 1
+    return codes, np.where(bits == 1, 1, -1).astype(np.int8)
+
+
+def check_dot_bruteforce(Nmax=8):
+    """z = N - 2 popcount(a XOR w) over every pair of +-1 vectors, N <= Nmax."""
+    for N in range(1, Nmax + 1):
+        codes, V = _all_pm1(N)
+        # hidden weights: odd integers whose sign is V, magnitudes 1..7
+        mag = 1 + 2 * (np.arange(V.size).reshape(V.shape) % 4)
+        H = (V.astype(np.int32) * mag).T.copy()        # N x 2^N, column w = vector w
+        z, a = O.layer_forward(V, H)
+        pc = np.array([bin(int(c)).count("1") for c in range(2 ** N)])
+        expect = N - 2 * pc[codes[:, None] ^ codes[None, :]]
+        assert np.array_equal(z, expect), N
+        assert np.array_equal(a, np.where(expect >= 0, 1, -1)), N
+
+
+def check_sign_zero():
+    """sign(0) = +1 for activations (reading O1): z = 0 gives a = +1."""
+    a_prev = np.array([[1, -1], [1, 1], [-1, -1]], np.int8)
+    H = np.array([[1], [1]], np.int32)
+    z, a = O.layer_forward(a_prev, H)
+    assert z[:, 0].tolist() == [0, 2, -2]
+    assert a[:, 0].tolist() == [1, 1, -1]
+
+
+def check_local_output_popcount(seed=0):
+    rng = np.random.default_rng(seed)
+    for (b, K, c) in [(5, 1, 2), (7, 63, 3), (9, 130, 10), (3, 257, 100)]:
+        a = np.where(rng.random((b, K)) < 0.5, 1, -1).astype(np.int8)
+        P = np.where(rng.random((K, c)) < 0.5, 1, -1).astype(np.int8)
+        yhat = O.local_output(a, P)
+        dis = (a[:, :, None] != P[None, :, :]).sum(axis=1)
+        assert np.array_equal(yhat, K - 2 * dis)
+
+
+# -- local loss and marking ------------------------------------------------------
+
+def check_local_loss_golden():
+    for line in read_golden("local_loss_cases.txt"):
+        head, yh, exp = (s.split() for s in line.split("|"))
+        K, y = int(head[0]), int(head[1])
+        yhat = np.array([[int(v) for v in yh]], np.int32)
+        pred, ell, tau, mark = O.local_loss(yhat, np.array([y]), K, 1, 4)
+        got = [int(pred[0]), int(ell[0]), int(tau[0]), int(mark[0])]
+        assert got == [int(v) for v in exp], (line, got)
+
+
+def check_local_loss_special(seed=1):
+    """r = 0 marks exactly the errors; a huge r marks every pattern."""
+    rng = np.random.default_rng(seed)
+    yhat = rng.integers(-20, 21, size=(200, 7)).astype(np.int32)
+    y = rng.integers(0, 7, size=200).astype(np.int32)
+    pred, ell, tau, mark = O.local_loss(yhat, y, 64, 0, 1)
+    assert np.array_equal(mark, ell)
+    pred, ell, tau, mark = O.local_loss(yhat, y, 64, 10 ** 6, 1)
+    assert mark.all()
+    srt = np.sort(yhat, axis=1)
+    assert np.array_equal(tau, srt[:, -1] - srt[:, -2])
+
+
+# -- selection -------------------------------------------------------------------
+
+def _parse_select():
+    z, rho, sels, marks = [], [], [], []
+    y = gamma = None
+    for line in read_golden("select_case.txt"):
+        t = line.split()
+        if t[0] == "z":
+            z.append([int(v) for v in t[1:]])
+        elif t[0] == "rho":
+            rho.append([int(v) for v in t[1:]])
+        elif t[0] == "y":
+            y = [int(v) for v in t[1:]]
+        elif t[0] == "gamma":
+            gamma = int(t[1])
+        elif t[0] == "mark":
+            marks.append([int(v) for v in t[1:]])
+            sels.append([])
+        elif t[0] == "sel":
+            sels[-1].append([int(v) for v in t[1:]])
+    return (np.array(z, np.int32), np.array(rho, np.int8), np.array(y, np.int32), gamma,
+            marks, sels)
+
+
+def check_select_golden():
+    z, rho, y, gamma, marks, sels = _parse_select()
+    for mark, sel in zip(marks, sels):
+        got = O.select(z, rho, y, np.array(mark, np.uint8), gamma)
+        assert got.tolist() == sel, (mark, got.tolist(), sel)
+
+
+def check_select_special(seed=2):
+    """gamma = 1: every neuron with negative stability is selected (Alg. 2 with
+    G = K_l); gamma = K_l: one selection per pattern, the largest negative delta."""
+    rng = np.random.default_rng(seed)
+    b, K, c = 20, 24, 5
+    z = rng.integers(-9, 10, size=(b, K)).astype(np.int32)
+    P = np.where(rng.random((K, c)) < 0.5, 1, -1).astype(np.int8)
+    y = rng.integers(0, c, size=b).astype(np.int32)
+    mark = np.ones(b, np.uint8)
+    delta = z * P[:, y].T
+    sel1 = O.select(z, P, y, mark, 1)
+    assert np.array_equal(sel1, np.where(delta < 0, np.arange(K)[None, :], -1))
+    selK = O.select(z, P, y, mark, K)
+    for mu in range(b):
+        neg = [k for k in range(K) if delta[mu, k] < 0]
+        if not neg:
+            assert selK[mu, 0] == -1
+        else:
+            best = max(delta[mu, k] for k in neg)
+            assert selK[mu, 0] == min(k for k in neg if delta[mu, k] == best)
+
+
+# -- perceptron level --------------------------------------------------------------
+
+def _parse_perceptron():
+    d = {}
+    for line in read_golden("perceptron_case.txt"):
+        t = line.split()
+        d.setdefault(t[0], []).append([int(v) for v in t[1:]])
+    return d
+
+
+def check_perceptron_golden():
+    d = _parse_perceptron()
+    H = np.array(d["H"], np.int32)
+    a = np.array(d["a"], np.int8)
+    y = np.array(d["y"][0], np.int32)
+    rho = np.array(d["rho"], np.int8)
+    sel = np.array(d["sel"], np.int32)
+    cp = O.perceptron_update(H, a, y, rho, sel, 3, 0, 7, 1, 0)
+    assert cp.tolist() == d["cp"], cp.tolist()
+    cpr = O.perceptron_update(H, a, y, rho, sel, 3, 1 << 32, 7, 1, 0)
+    assert cpr.tolist() == d["cpr"], cpr.tolist()
+
+
+def check_threshold_exact():
+    """U < T  <=>  U / 2^32 < q, checked in exact rational arithmetic, and q is
+    p_r sqrt(2 / (pi K)) to within 2 ulp (40-digit decimal evaluation)."""
+    getcontext().prec = 40
+    pi = Decimal("3.141592653589793238462643383279502884197")
+    for p_r in (0.5, 0.25, 0.1234567, 1e-3, 0.9):
+        for K in (1, 2, 10, 64, 256, 784, 1024, 4096, 8192):
+            q = O.reinforce_prob(p_r, K)
+            qd = Decimal(p_r) * (Decimal(2) / (pi * K)).sqrt()
+            assert abs(Decimal(q) - qd) <= 2 * Decimal(math.ulp(q)), (p_r, K)
+            T = O.reinforce_threshold(p_r, K)
+            if q >= 1:
+                assert T == 1 << 32
+                continue
+            qf = Fraction(q)
+            assert Fraction(T - 1, 1 << 32) < qf <= Fraction(T, 1 << 32), (p_r, K, T)
+    assert O.reinforce_threshold(0.0, 100) == 0
+
+
+def check_reinforce_rate():
+    """Reinforcement alone (no tuples): each weight moves with probability q, by
+    exactly 2 sign(h); the count obeys a binomial bound; draws repeat for the
+    same step and differ between steps."""
+    Kp, K = 512, 512
+    rng = np.random.default_rng(3)
+    H = (np.where(rng.random((Kp, K)) < 0.5, 1, -1) * (1 + 2 * rng.integers(0, 3, (Kp, K))))
+    H = H.astype(np.int32)
+    a = np.ones((1, Kp), np.int8)
+    sel = -np.ones((1, K), np.int32)
+    rho = np.ones((K, 2), np.int8)
+    y = np.zeros(1, np.int32)
+    q = 0.02
+    T = math.ceil(q * 2 ** 32)
+    H1 = O.perceptron_update(H, a, y, rho, sel, 255, T, 11, 2, 5)
+    d = H1 - H
+    moved = d != 0
+    n = moved.sum()
+    mean, sd = q * H.size, math.sqrt(q * (1 - q) * H.size)
+    assert abs(n - mean) < 5 * sd, (n, mean, sd)
+    assert np.array_equal(d[moved], 2 * np.sign(H[moved]))
+    H1b = O.perceptron_update(H, a, y, rho, sel, 255, T, 11, 2, 5)
+    assert np.array_equal(H1, H1b)
+    H2 = O.perceptron_update(H, a, y, rho, sel, 255, T, 11, 2, 6)
+    overlap = ((H2 - H) != 0) & moved
+    assert overlap.sum() < 5 * q * n + 10
+
+
+def check_uniform_bits(n=40000):
+    """The 32-bit draws are uniform: each bit is set with frequency 1/2 and the
+    top 4 bits are uniform over 16 bins (chi-square, 15 dof, p ~ 1e-6 cut)."""
+    vals = np.array([O.uniform32(5, 1, k, i, 3) for k in range(n // 200) for i in range(200)],
+                    np.uint64)
+    for bit in range(32):
+        f = ((vals >> np.uint64(bit)) & np.uint64(1)).mean()
+        assert abs(f - 0.5) < 5 * math.sqrt(0.25 / vals.size), bit
+    counts = np.bincount((vals >> np.uint64(28)).astype(np.int64), minlength=16)
+    e = vals.size / 16
+    chi2 = ((counts - e) ** 2 / e).sum()
+    assert chi2 < 50, chi2
+
+
+def check_update_invariants(seed=4):
+    """One CP tuple changes each h of its neuron by exactly one lattice unit (2)
+    unless clipped; reinforcement never flips a sign; h stays odd and bounded."""
+    rng = np.random.default_rng(seed)
+    Kp, K, c, h_max = 40, 12, 3, 5
+    H = (np.where(rng.random((Kp, K)) < 0.5, 1, -1) *
+         (1 + 2 * rng.integers(0, 3, (Kp, K)))).astype(np.int32)
+    a = np.where(rng.random((3, Kp)) < 0.5, 1, -1).astype(np.int8)
+    y = rng.integers(0, c, 3).astype(np.int32)
+    rho = np.where(rng.random((K, c)) < 0.5, 1, -1).astype(np.int8)
+    sel = -np.ones((3, 1), np.int32)
+    sel[1, 0] = 7                       # one tuple: (mu=1, k=7), gamma = K
+    H1 = O.perceptron_update(H, a, y, rho, sel, h_max, 0, 1, 1, 0)
+    d = H1 - H
+    assert np.all(d[:, [k for k in range(K) if k != 7]] == 0)
+    step = 2 * a[1] * rho[7, y[1]]
+    want = np.clip(H[:, 7] + step, -h_max, h_max)
+    assert np.array_equal(H1[:, 7], want)
+    assert np.all(np.abs(d[:, 7]) <= 2)
+    assert np.all((d[:, 7] == 0) == (np.abs(H[:, 7] + step) > h_max))
+    # reinforcement only, probability 1
+    H2 = O.perceptron_update(H, a, y, rho, -np.ones((3, 1), np.int32), h_max, 1 << 32, 1, 1, 0)
+    assert np.array_equal(np.sign(H2), np.sign(H))
+    assert np.array_equal(H2, np.clip(H + 2 * np.sign(H), -h_max, h_max))
+    for M in (H1, H2):
+        assert np.all(M % 2 != 0) and np.all(np.abs(M) <= h_max)
+
+
+# -- the whole rule ------------------------------------------------------------
+
+def _bias_data(rng, n, K, c):
+    x = np.where(rng.random((n, K)) < 0.5, 1, -1).astype(np.int8)
+    y = rng.integers(0, c, n).astype(np.int32)
+    return x, y
+
+
+def check_training_invariants(seed=5):
+    """Over whole training runs with a small h_max (lots of clipping): h odd,
+    |h| <= h_max, every h changes by at most 2 (n_k + 1) per step."""
+    rng = np.random.default_rng(seed)
+    widths, c, h_max = [50, 24, 16], 3, 7
+    m = O.OracleModel(widths, c, h_max=h_max, seed=9, bs=10, p_r0=0.9, gamma=[4, 4])
+    x, y = _bias_data(rng, 60, widths[0], c)
+    prev = [m.H(l) for l in (1, 2)]
+    for s in range(6):
+        m.train(x[10 * s:10 * s + 10], y[10 * s:10 * s + 10])
+        for l in (1, 2):
+            H = m.H(l)
+            assert np.all(H % 2 != 0) and np.all(np.abs(H) <= h_max)
+            # at most bs tuples per neuron per step, plus one reinforcement event
+            assert np.all(np.abs(H - prev[l - 1]) <= 2 * (10 + 1))
+            prev[l - 1] = H
+    assert m.step == 6
+
+
+def check_no_mark_no_update(seed=6):
+    """When no pattern of a layer is marked, the layer is not updated at all --
+    not even reinforced (reading O6).  Labels = the model's own predictions with
+    r = 0 leave M_L empty."""
+    rng = np.random.default_rng(seed)
+    m = O.OracleModel([30, 40], 2, seed=12, bs=25, r=(0, 1), p_r0=1.0)
+    x, _ = _bias_data(rng, 100, 30, 2)
+    y = m.predict(x)
+    H0 = m.H(1)
+    err = m.train(x, y)
+    assert err == 0
+    assert np.array_equal(m.H(1), H0)
+    assert m.step == 4
+
+
+def check_epoch_end_pr(seed=7):
+    """Alg. 1 l.21: p_r <- p_r sqrt(E^e), E^e the epoch's error fraction."""
+    getcontext().prec = 40
+    rng = np.random.default_rng(seed)
+    m = O.OracleModel([20, 32, 32], 4, seed=2, bs=10, p_r0=0.5)
+    x, y = _bias_data(rng, 50, 20, 4)
+    e1 = m.train(x[:30], y[:30])
+    e2 = m.train(x[30:], y[30:], epoch_end=True)
+    want = Decimal(0.5) * (Decimal(e1 + e2) / Decimal(50)).sqrt()
+    assert abs(Decimal(m.p_r) - want) <= 2 * Decimal(math.ulp(float(want))), (m.p_r, want)
+    pr1 = m.p_r
+    e3 = m.train(x, y, epoch_end=True)
+    want2 = Decimal(pr1) * (Decimal(e3) / Decimal(50)).sqrt()
+    assert abs(Decimal(m.p_r) - want2) <= 2 * Decimal(math.ulp(float(want2)) + 1e-300)
+
+
+def margin_teacher_task(seed, n, K0=64, c=4, margin=8):
+    """A linearly separable +-1 task with a margin: labels = argmax of a random
+    +-1 teacher x V, keeping only samples whose top-1 minus top-2 score >= margin."""
+    rng = np.random.default_rng(seed)
+    V = np.where(rng.random((K0, c)) < 0.5, 1, -1)
+    xs, ys, have = [], [], 0
+    while have < n:
+        x = np.where(rng.random((4096, K0)) < 0.5, 1, -1)
+        s = x @ V
+        o = np.sort(s, axis=1)
+        keep = (o[:, -1] - o[:, -2]) >= margin
+        xs.append(x[keep])
+        ys.append(np.argmax(s[keep], axis=1))
+        have += int(keep.sum())
+    x = np.concatenate(xs)[:n].astype(np.int8)
+    y = np.concatenate(ys)[:n].astype(np.int32)
+    return x, y
+
+
+LEARN_MIN_TRAIN_ACC = 0.95   # observed: 0.994 after 5 epochs (seed 3 model, seed 1 data)
+
+
+def check_learnable():
+    """The rule learns a separable teacher task: 64 -> 256 -> 4, 1000 samples,
+    bs = 100, 5 epochs; train accuracy >= 0.95."""
+    x, y = margin_teacher_task(1, 1500)
+    xtr, ytr, xte, yte = x[:1000], y[:1000], x[1000:], y[1000:]
+    m = O.OracleModel([64, 256], 4, seed=3, bs=100)
+    for _ in range(5):
+        m.train(xtr, ytr, epoch_end=True)
+    acc = (m.predict(xtr) == ytr).mean()
+    assert acc >= LEARN_MIN_TRAIN_ACC, acc
+    return acc, (m.predict(xte) == yte).mean()
+
+
+def check_resume_equivalence(seed=8):
+    """Training in one call equals training in two calls split at a batch
+    boundary, and a model rebuilt from the saved state continues identically."""
+    rng = np.random.default_rng(seed)
+    x, y = _bias_data(rng, 120, 33, 3)
+    a = O.OracleModel([33, 20, 16], 3, seed=4, bs=20, gamma=[5, 4])
+    a.train(x, y)
+    b = O.OracleModel([33, 20, 16], 3, seed=4, bs=20, gamma=[5, 4])
+    b.train(x[:60], y[:60])
+    c = O.OracleModel([33, 20, 16], 3, seed=4, bs=20, gamma=[5, 4])
+    for l in (1, 2):
+        c.set_H(l, b.H(l))
+    c.set_scalars(b.p_r, b.step)
+    b.train(x[60:], y[60:])
+    c.train(x[60:], y[60:])
+    for l in (1, 2):
+        assert np.array_equal(a.H(l), b.H(l))
+        assert np.array_equal(a.H(l), c.H(l))
+    assert a.step == b.step == c.step == 6
+
+
+ALL_CHECKS = [
+    check_philox_kat,
+    check_gamma_golden,
+    check_dot_bruteforce,
+    check_sign_zero,
+    check_local_output_popcount,
+    check_local_loss_golden,
+    check_local_loss_special,
+    check_select_golden,
+    check_select_special,
+    check_perceptron_golden,
+    check_threshold_exact,
+    check_reinforce_rate,
+    check_uniform_bits,
+    check_update_invariants,
+    check_training_invariants,
+    check_no_mark_no_update,
+    check_epoch_end_pr,
+    check_learnable,
+    check_resume_equivalence,
+]

@@ -1,0 +1,61 @@
+"""The CPU oracle against its pins (no GPU), and planted mistakes in copies of
+the oracle source, each of which some pin must catch."""
+import os
+
+import pytest
+
+import oracle_pins as P
+
+
+@pytest.mark.parametrize("check", P.ALL_CHECKS, ids=lambda f: f.__name__)
+def test_pin(oracle_mod, check):
+    check()
+
+
+def test_learnable_records_accuracy(oracle_mod):
+    acc_train, acc_test = P.check_learnable()
+    assert acc_train >= P.LEARN_MIN_TRAIN_ACC
+    assert acc_test >= 0.7, acc_test
+
+
+# Plausible mistakes: (name, exact text in bmlp_oracle.c, replacement).
+MUTANTS = [
+    ("sign_zero_negative", "static int32_t sign_of(int32_t v) { return v >= 0 ? +1 : -1; }",
+     "static int32_t sign_of(int32_t v) { return v > 0 ? +1 : -1; }"),
+    ("argmax_ties_high", "      if (v[j] > v[jmax]) jmax = j;\n    int32_t second",
+     "      if (v[j] >= v[jmax]) jmax = j;\n    int32_t second"),
+    ("tau_distinct_values", "if (j != jmax && v[j] > second)", "if (v[j] != v[jmax] && v[j] > second)"),
+    ("margin_not_strict", "(int64_t)t * r_den < (int64_t)r_num * K", "(int64_t)t * r_den <= (int64_t)r_num * K"),
+    ("select_most_negative", "delta[k] > delta[best]", "delta[k] < delta[best]"),
+    ("select_allows_zero", "if (delta[k] < 0 &&", "if (delta[k] <= 0 &&"),
+    ("cp_sign_flipped", "*h = clip(*h + 2 * a_prev[(int64_t)mu * K_prev + i] * rho, h_max);",
+     "*h = clip(*h - 2 * a_prev[(int64_t)mu * K_prev + i] * rho, h_max);"),
+    ("cp_no_clip", "*h = clip(*h + 2 * a_prev[(int64_t)mu * K_prev + i] * rho, h_max);",
+     "*h = *h + 2 * a_prev[(int64_t)mu * K_prev + i] * rho;"),
+    ("cp_descending_mu", "  for (int32_t mu = 0; mu < b; mu++)\n    for (int32_t g = 0; g < G; g++) {\n      int32_t k = sel",
+     "  for (int32_t mu = b - 1; mu >= 0; mu--)\n    for (int32_t g = 0; g < G; g++) {\n      int32_t k = sel"),
+    ("reinforce_toward_zero", "*h = clip(*h + 2 * (*h > 0 ? 1 : -1), h_max);",
+     "*h = clip(*h - 2 * (*h > 0 ? 1 : -1), h_max);"),
+    ("threshold_floor", "return (uint64_t)ceil(q * 4294967296.0);", "return (uint64_t)floor(q * 4294967296.0);"),
+    ("philox_7_rounds", "for (int round = 0; round < 10; round++)", "for (int round = 0; round < 7; round++)"),
+    ("update_without_marks", "if (!any) continue; /* O6 */", "(void)any;"),
+    ("gamma_ties_small", "(dist == best_dist && g > best)", "(dist == best_dist && g < best)"),
+    ("pr_without_sqrt", "m->p_r = m->p_r * sqrt(E);", "m->p_r = m->p_r * E;"),
+    ("forward_drops_sign", "zr[k] += ai * (hrow[k] > 0 ? 1 : -1);", "zr[k] += ai * hrow[k];"),
+]
+
+
+@pytest.mark.parametrize("name,old,new", MUTANTS, ids=[m[0] for m in MUTANTS])
+def test_planted_mistake_is_caught(oracle_mod, tmp_path, name, old, new):
+    src = oracle_mod.source()
+    assert src.count(old) == 1, "mutation anchor not found exactly once: " + name
+    path = oracle_mod.compile_variant(src.replace(old, new), os.path.join(tmp_path, name + ".so"))
+    caught = []
+    with oracle_mod.use_library(path):
+        for check in P.ALL_CHECKS:
+            try:
+                check()
+            except AssertionError:
+                caught.append(check.__name__)
+                break
+    assert caught, "no pin caught the planted mistake " + name
