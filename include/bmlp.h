@@ -1,0 +1,178 @@
+/*
+ * bmlp.h -- C-ABI of the GB300 (sm_103a) library that trains and evaluates
+ * binary multi-layer perceptrons (BMLPs) with the fully binary, gradient-free
+ * rule of "Training multi-layer binary neural networks with random local binary
+ * error signals" (arXiv 2412.00119).
+ *
+ * What the library computes (paper notation; layers l = 1..L, widths K_0..K_L,
+ * c classes):
+ *   - H_l (K_{l-1} x K_l) integer "hidden metaplastic" weights, W_l = sign(H_l)
+ *     the visible binary weights, P_l (K_l x c) a fixed random +-1 local
+ *     classifier per layer (Sec. 3.1);
+ *   - per mini-batch of bs patterns (Alg. 1): z_l = a_{l-1} W_l, a_l = sign(z_l),
+ *     yhat_l = a_l P_l, the 01-loss of Eq. 1 and the robustness margin tau of
+ *     Alg. 1 l.13-15 marking the patterns M_l to learn from;
+ *   - the layer-level selection of Alg. 2: per group of gamma neurons the
+ *     perceptron with the negative stability z_k rho_{k,y} closest to 0;
+ *   - the perceptron-level CP + R rule of Alg. 3 with hidden weights clipped to
+ *     [-h_max, h_max], W_l re-derived and re-packed in the same pass;
+ *   - the end-of-epoch rescale p_r <- p_r sqrt(E^e) (Alg. 1 l.21);
+ *   - forward-only evaluation: argmax of a_L P_L (Sec. 3.1).
+ * Conventions where the paper is silent: sign(0) = +1; argmax ties go to the
+ * lowest class; groups are contiguous (neuron k in group k / gamma); tuples are
+ * applied in ascending pattern order with clipping after each; LayerUpdate runs
+ * only when M_l is non-empty; Uniform(0,1) is a 32-bit Philox4x32-10 integer U
+ * with p = U / 2^32 and "p < q" evaluated exactly.  Every result is an integer
+ * or a bit and is reproducible bit for bit.
+ *
+ * Data formats
+ *   packed +-1 vectors: a vector of K values is ceil(K/64) little-endian uint64
+ *     words; bit j of word w is element 64 w + j; a set bit means +1; pad bits
+ *     must be 0.  A batch of n vectors is n such rows, row after row.
+ *   labels: int32 in 0..c-1.
+ *   H (state export): int16, K_l rows of K_{l-1} (neuron-major: element
+ *     [k * K_{l-1} + i] is h_{ik}), odd values in [-h_max, h_max].
+ *   W (state export): uint64, K_l rows of ceil(K_{l-1}/64) words, bit = (h > 0).
+ *   P (state export): int8, K_l rows of c values rho_{kj} in {-1, +1}.
+ *
+ * Pointers and streams
+ *   Batch inputs and outputs (x_packed, labels, labels_out) may be device or
+ *   host pointers; the library asks the CUDA runtime which.  Host buffers are
+ *   staged through library-owned device buffers with cudaMemcpyAsync on the
+ *   given stream (pinned host memory makes the copies asynchronous).  The
+ *   caller owns every buffer it passes in and must keep it alive until the
+ *   work on `cuda_stream` has completed; the library owns the model state.
+ *   `cuda_stream` is a cudaStream_t (NULL = the legacy default stream).
+ *   Calls are asynchronous on that stream, except those that return host
+ *   values (n_errors_out, BMLP_EPOCH_END, bmlp_get_state, bmlp_set_state),
+ *   which synchronise it.
+ *
+ * Errors
+ *   Every int-returning call returns BMLP_OK (0) or a negative BMLP_E* code and
+ *   never throws or aborts; bmlp_last_error() gives a one-line reason.  Labels
+ *   outside 0..c-1 in device memory are not read out of bounds: the kernels
+ *   count them, and the next call that synchronises returns BMLP_EINVAL.
+ *
+ * One handle is used by one host thread at a time.
+ */
+#ifndef BMLP_H_
+#define BMLP_H_
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define BMLP_OK 0
+#define BMLP_EINVAL (-1)   /* bad argument or bad label values */
+#define BMLP_ENOMEM (-2)   /* device or host allocation failed */
+#define BMLP_ECUDA (-3)    /* a CUDA runtime call or kernel launch failed */
+#define BMLP_ETIMEOUT (-4) /* a bounded device-side wait gave up */
+#define BMLP_ESTATE (-5)   /* state blob inconsistent with the model */
+#define BMLP_ENODEV (-6)   /* no usable sm_103 device */
+
+#define BMLP_MAX_LAYERS 16
+#define BMLP_MAX_BS 1024
+#define BMLP_MAX_CLASSES 1024
+
+/* bmlp_train flags */
+#define BMLP_EPOCH_END 1u  /* after these n patterns, close the epoch (Alg. 1 l.21) */
+
+/* forward-contraction engines (hparams.fwd_impl) */
+#define BMLP_FWD_AUTO 0     /* library's choice */
+#define BMLP_FWD_POPC 1     /* CUDA-core XOR + popcount */
+#define BMLP_FWD_TCGEN05 2  /* 5th-gen tensor cores, +-1 as e4m3, fp32 accumulate (exact) */
+
+typedef struct bmlp bmlp_t;
+
+/* Hyperparameters (Alg. 1 header).  Zero-initialise and set what you need:
+ * a zero / negative field selects the paper's setting of Sec. 4.2. */
+typedef struct bmlp_hparams {
+  int32_t bs;            /* mini-batch size, 1..BMLP_MAX_BS; 0 -> 100 */
+  int32_t r_num, r_den;  /* robustness r = r_num / r_den; r_den == 0 -> r = 1/4 */
+  double p_r0;           /* initial reinforcement probability; < 0 -> 0.5 */
+  const int32_t* gamma;  /* L group sizes, each dividing K_l; NULL -> Sec. 4.3 rule */
+  int32_t fwd_impl;      /* BMLP_FWD_*; 0 -> auto */
+} bmlp_hparams;
+
+/* Create a model and initialise H_l, P_l uniformly on {+-1} from `seed`
+ * (Alg. 1 l.2).  widths: K_0..K_L (n_widths = L + 1, 2..BMLP_MAX_LAYERS + 1,
+ * each >= 1); classes: 2..BMLP_MAX_CLASSES; h_max: odd, 1..32767 (255 = 8-bit
+ * hidden weights, Table 4); hp may be NULL (paper defaults).  Allocates the
+ * model state on the current CUDA device.  On success *out owns it. */
+int bmlp_create(const int32_t* widths, int32_t n_widths, int32_t classes, int16_t h_max,
+                uint64_t seed, const bmlp_hparams* hp, bmlp_t** out);
+
+/* Free the model (synchronises the device first).  NULL is accepted. */
+void bmlp_destroy(bmlp_t* h);
+
+/* One pass of NetworkUpdate (Alg. 1 l.4-20) over n patterns in the given
+ * order, in mini-batches of bs (a last shorter batch is processed as a batch of
+ * its own size).  x_packed: n packed rows of K_0 bits; labels: n int32.
+ * flags & BMLP_EPOCH_END: afterwards set E = (last-layer 01-loss count since the
+ * previous epoch end) / (patterns since then) and p_r <- p_r sqrt(E).
+ * n_errors_out (host, may be NULL): last-layer 01-loss count of these n
+ * patterns, measured in the training forward pass.  n == 0 is a no-op. */
+int bmlp_train(bmlp_t* h, const uint64_t* x_packed, const int32_t* labels, int64_t n,
+               uint32_t flags, void* cuda_stream, int64_t* n_errors_out);
+
+/* Forward-only evaluation (Sec. 3.1): labels_out[mu] = argmax_j (a_L P_L)_{mu j}
+ * (lowest index on ties) for n packed rows of K_0 bits.  Does not change state. */
+int bmlp_predict(bmlp_t* h, const uint64_t* x_packed, int64_t n, int32_t* labels_out,
+                 void* cuda_stream);
+
+/* Copy layer `layer` (1..L) to host buffers (each may be NULL; formats above),
+ * plus the current p_r and step counter t (mini-batches since creation). */
+int bmlp_get_state(const bmlp_t* h, int32_t layer, int16_t* H_out, uint64_t* W_out,
+                   int8_t* P_out, double* p_r_out, int64_t* step_out);
+
+/* Resume: load H of layer `layer` (host, format above; NULL keeps it) and
+ * re-derive W from it; set p_r and the step counter (step < 0 keeps both).
+ * Values must be odd and within [-h_max, h_max], else BMLP_ESTATE and nothing
+ * changes.  The epoch's error and pattern counters restart at 0. */
+int bmlp_set_state(bmlp_t* h, int32_t layer, const int16_t* H_in, double p_r, int64_t step);
+
+/* Model shape: any output may be NULL.  widths_out: L + 1 values; gamma_out: L. */
+int bmlp_get_info(const bmlp_t* h, int32_t* n_layers, int32_t* widths_out, int32_t* classes,
+                  int32_t* gamma_out, int32_t* bs, int32_t* fwd_impl);
+
+/* One-line description of the last error on this handle ("" if none).  With
+ * h == NULL: the last error of a call that had no handle (e.g. bmlp_create). */
+const char* bmlp_last_error(const bmlp_t* h);
+
+/* Group size chosen by the rule of Sec. 4.3 for a layer of K neurons: the
+ * divisor of K closest to [75, 105], the largest among equally close ones;
+ * -1 for K < 1.  Host only. */
+int32_t bmlp_gamma_rule(int32_t K);
+
+/* Reinforcement threshold of Alg. 3 l.8 for the current p_r and layer width K:
+ * q = p_r sqrt(2 / (pi K)) in IEEE double, returned as T = ceil(q 2^32)
+ * clamped to [0, 2^32], so that a 32-bit U reinforces iff U < T.  Host only. */
+uint64_t bmlp_reinforce_threshold(double p_r, int32_t K);
+
+/* Debug view of the most recent training mini-batch (synchronises): for layer
+ * `layer`, Z (bs x K_l int16 pre-activations), A (bs x ceil(K_l/64) packed
+ * activations), mark (bs uint8, 1 = pattern in M_l), sel (bs x G_l int16,
+ * selected neuron per group or -1).  Rows beyond the batch's size are stale.
+ * Any output may be NULL. */
+int bmlp_debug_last_step(const bmlp_t* h, int32_t layer, int16_t* Z, uint64_t* A,
+                         uint8_t* mark, int16_t* sel);
+
+/* Per-kernel timing.  With profiling on, train/predict launch kernels one by
+ * one with CUDA events around each (no CUDA graph) and accumulate, per kernel
+ * kind, the launch count and the summed device time.  kinds: 0 forward
+ * (train), 1 local classifier + selection, 2 update (CP + R + repack),
+ * 3 forward (predict), 4 predict output, 5 host-buffer copies.
+ * bmlp_launch_count: kernels this handle has launched since creation (graph
+ * replays count each node). */
+int bmlp_set_profiling(bmlp_t* h, int32_t on);
+int bmlp_get_profile(const bmlp_t* h, int32_t kind, int64_t* launches, double* total_ms);
+int bmlp_reset_profile(bmlp_t* h);
+int64_t bmlp_launch_count(const bmlp_t* h);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* BMLP_H_ */

@@ -367,6 +367,7 @@ int or_create(const int32_t* widths, int32_t n_widths, int32_t classes, int32_t 
       or_destroy(m);
       return OR_ENOMEM;
     }
+#pragma omp parallel for schedule(static)
     for (int32_t i = 0; i < Kp; i++)
       for (int32_t k = 0; k < K; k++) m->H[l][(int64_t)i * K + k] = or_init_h(seed, l, k, i);
     for (int32_t k = 0; k < K; k++)

@@ -1,0 +1,621 @@
+// bmlp_api.cu -- host side of the C-ABI declared in include/bmlp.h.
+//
+// One training mini-batch is L forward launches, one local-classifier +
+// selection launch and one update launch.  All of them read the batch index s
+// and the step counter t from a device-resident control block that the update
+// kernel advances, so a single captured CUDA graph replays step after step with
+// no host work between steps.  Batch pointers live in a device-resident
+// parameter block that a stream-ordered copy refreshes at the start of a call.
+#include <algorithm>
+#include <cmath>
+#include <cstddef>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include "bmlp_internal.cuh"
+
+using namespace bk;
+
+namespace {
+
+thread_local std::string g_create_error;
+
+enum ProfKind { kProfTrainFwd = 0, kProfCls = 1, kProfUpd = 2, kProfEvalFwd = 3, kProfOut = 4,
+                kProfCopy = 5, kProfKinds = 6 };
+
+}  // namespace
+
+struct bmlp {
+  int device = 0;
+  int L = 0, c = 0, h_max = 0, bs = 0, r_num = 0, r_den = 1, fwd_impl = BMLP_FWD_POPC;
+  uint64_t seed = 0;
+  std::vector<int> K, gamma;
+  double p_r = 0.5;
+  int64_t epoch_n = 0;  // patterns since the last epoch end
+  int64_t t_host = 0;   // host mirror of ctrl->t
+  StepParams hp{};      // host copy of the parameter block
+  StepParams* dP = nullptr;
+  Ctrl* dCtrl = nullptr;
+  unsigned long long* dT = nullptr;
+  std::vector<void*> allocs;
+  // evaluation scratch (grown on demand)
+  uint64_t* evA[2] = {nullptr, nullptr};
+  int64_t evCap = 0;
+  // staging for host batches
+  uint64_t* stX = nullptr;
+  int32_t* stY = nullptr;
+  int32_t* stOut = nullptr;
+  int64_t stCap = 0;
+  unsigned long long* hostPinned = nullptr;  // [4] D2H landing zone
+  // graph of one training step
+  cudaGraphExec_t stepExec = nullptr;
+  cudaStream_t capStream = nullptr;
+  int updCtas = 0;
+  size_t updSmem = 0;
+  // profiling
+  bool profiling = false;
+  std::vector<cudaEvent_t> evPool;
+  size_t evUsed = 0;
+  std::vector<std::pair<int, size_t>> evPairs;  // (kind, index of start event)
+  int64_t profN[kProfKinds] = {0};
+  double profMs[kProfKinds] = {0};
+  int64_t launches = 0;
+  std::string err;
+};
+
+namespace {
+
+int fail(bmlp_t* h, int code, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof(buf), fmt, ap);
+  va_end(ap);
+  if (h) h->err = buf; else g_create_error = buf;
+  return code;
+}
+
+int cuda_fail(bmlp_t* h, cudaError_t e, const char* what) {
+  return fail(h, e == cudaErrorMemoryAllocation ? BMLP_ENOMEM : BMLP_ECUDA, "%s: %s", what,
+              cudaGetErrorString(e));
+}
+
+#define CK(h, call)                                   \
+  do {                                                \
+    cudaError_t e_ = (call);                          \
+    if (e_ != cudaSuccess) return cuda_fail(h, e_, #call); \
+  } while (0)
+
+template <typename T>
+int dalloc(bmlp_t* h, T** p, size_t count) {
+  void* q = nullptr;
+  cudaError_t e = cudaMalloc(&q, count * sizeof(T) > 0 ? count * sizeof(T) : 16);
+  if (e != cudaSuccess) return cuda_fail(h, e, "cudaMalloc");
+  h->allocs.push_back(q);
+  *p = static_cast<T*>(q);
+  return BMLP_OK;
+}
+
+bool is_device_ptr(const void* p) {
+  cudaPointerAttributes a;
+  if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
+    (void)cudaGetLastError();
+    return false;
+  }
+  return a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged;
+}
+
+int words_of(int K) { return (K + 63) / 64; }
+
+int upload_thresholds(bmlp_t* h, cudaStream_t st) {
+  unsigned long long T[BMLP_MAX_LAYERS];
+  for (int l = 1; l <= h->L; ++l) T[l - 1] = bmlp_reinforce_threshold(h->p_r, h->K[l]);
+  CK(h, cudaMemcpyAsync(h->dT, T, sizeof(unsigned long long) * h->L, cudaMemcpyHostToDevice, st));
+  return BMLP_OK;
+}
+
+// event-bracketed launch in profiling mode
+cudaEvent_t next_event(bmlp_t* h) {
+  if (h->evUsed == h->evPool.size()) {
+    cudaEvent_t e;
+    if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+    h->evPool.push_back(e);
+  }
+  return h->evPool[h->evUsed++];
+}
+
+void prof_begin(bmlp_t* h, int kind, cudaStream_t st) {
+  if (!h->profiling) return;
+  cudaEvent_t a = next_event(h);
+  cudaEvent_t b = next_event(h);
+  if (!a || !b) return;
+  h->evPairs.push_back({kind, h->evUsed - 2});
+  cudaEventRecord(a, st);
+}
+
+void prof_end(bmlp_t* h, cudaStream_t st) {
+  if (!h->profiling || h->evPairs.empty()) return;
+  cudaEventRecord(h->evPool[h->evPairs.back().second + 1], st);
+}
+
+int prof_collect(bmlp_t* h, cudaStream_t st) {
+  if (!h->profiling || h->evPairs.empty()) return BMLP_OK;
+  CK(h, cudaStreamSynchronize(st));
+  for (auto& pr : h->evPairs) {
+    float ms = 0.f;
+    CK(h, cudaEventElapsedTime(&ms, h->evPool[pr.second], h->evPool[pr.second + 1]));
+    h->profMs[pr.first] += ms;
+    h->profN[pr.first] += 1;
+  }
+  h->evPairs.clear();
+  h->evUsed = 0;
+  return BMLP_OK;
+}
+
+// Enqueue the kernels of one training mini-batch on `st`.
+int enqueue_step(bmlp_t* h, cudaStream_t st) {
+  for (int l = 1; l <= h->L; ++l) {
+    prof_begin(h, kProfTrainFwd, st);
+    k_train_forward<<<train_forward_grid(h->bs, h->K[l]), train_forward_block(), 0, st>>>(h->dP, l);
+    prof_end(h, st);
+  }
+  prof_begin(h, kProfCls, st);
+  k_cls_select<<<dim3((unsigned)h->bs, (unsigned)h->L), kClsThreads, 0, st>>>(h->dP);
+  prof_end(h, st);
+  prof_begin(h, kProfUpd, st);
+  k_update<<<h->updCtas, kUpdThreads, h->updSmem, st>>>(h->dP);
+  prof_end(h, st);
+  CK(h, cudaGetLastError());
+  return BMLP_OK;
+}
+
+int ensure_graph(bmlp_t* h) {
+  if (h->stepExec) return BMLP_OK;
+  if (!h->capStream) CK(h, cudaStreamCreateWithFlags(&h->capStream, cudaStreamNonBlocking));
+  cudaGraph_t g = nullptr;
+  CK(h, cudaStreamBeginCapture(h->capStream, cudaStreamCaptureModeThreadLocal));
+  const bool prof = h->profiling;
+  h->profiling = false;
+  int rc = enqueue_step(h, h->capStream);
+  h->profiling = prof;
+  cudaError_t e = cudaStreamEndCapture(h->capStream, &g);
+  if (rc != BMLP_OK) {
+    if (g) cudaGraphDestroy(g);
+    return rc;
+  }
+  if (e != cudaSuccess) return cuda_fail(h, e, "cudaStreamEndCapture");
+  e = cudaGraphInstantiate(&h->stepExec, g, 0);
+  cudaGraphDestroy(g);
+  if (e != cudaSuccess) return cuda_fail(h, e, "cudaGraphInstantiate");
+  return BMLP_OK;
+}
+
+// Train on n device-resident patterns.
+int run_steps(bmlp_t* h, const uint64_t* xd, const int32_t* yd, int64_t n, cudaStream_t st) {
+  h->hp.x = xd;
+  h->hp.y = yd;
+  h->hp.n = n;
+  const size_t head = offsetof(StepParams, x);
+  CK(h, cudaMemcpyAsync(reinterpret_cast<char*>(h->dP) + head, reinterpret_cast<char*>(&h->hp) + head,
+                        sizeof(StepParams) - head, cudaMemcpyHostToDevice, st));
+  CK(h, cudaMemsetAsync(&h->dCtrl->s, 0, sizeof(uint32_t), st));
+  const int64_t steps = (n + h->bs - 1) / h->bs;
+  if (h->profiling) {
+    for (int64_t s = 0; s < steps; ++s) {
+      int rc = enqueue_step(h, st);
+      if (rc != BMLP_OK) return rc;
+    }
+  } else {
+    int rc = ensure_graph(h);
+    if (rc != BMLP_OK) return rc;
+    for (int64_t s = 0; s < steps; ++s) CK(h, cudaGraphLaunch(h->stepExec, st));
+  }
+  h->launches += steps * (h->L + 2);
+  h->t_host += steps;
+  return BMLP_OK;
+}
+
+int ensure_staging(bmlp_t* h, int64_t rows) {
+  if (rows <= h->stCap) return BMLP_OK;
+  int rc;
+  if ((rc = dalloc(h, &h->stX, (size_t)rows * h->hp.nw0)) != BMLP_OK) return rc;
+  if ((rc = dalloc(h, &h->stY, (size_t)rows)) != BMLP_OK) return rc;
+  if ((rc = dalloc(h, &h->stOut, (size_t)rows)) != BMLP_OK) return rc;
+  h->stCap = rows;
+  return BMLP_OK;
+}
+
+int ensure_eval(bmlp_t* h, int64_t rows) {
+  if (rows <= h->evCap) return BMLP_OK;
+  int nwmax = 0;
+  for (int l = 1; l <= h->L; ++l) nwmax = std::max(nwmax, words_of(h->K[l]));
+  int rc;
+  if ((rc = dalloc(h, &h->evA[0], (size_t)rows * nwmax)) != BMLP_OK) return rc;
+  if ((rc = dalloc(h, &h->evA[1], (size_t)rows * nwmax)) != BMLP_OK) return rc;
+  h->evCap = rows;
+  return BMLP_OK;
+}
+
+constexpr int64_t kEvalChunk = 65536;
+constexpr int64_t kStageRows = 65536;
+
+}  // namespace
+
+// ---------------------------------------------------------------------------
+extern "C" {
+
+int32_t bmlp_gamma_rule(int32_t K) {
+  if (K < 1) return -1;
+  int32_t best = -1, bestd = 0;
+  for (int32_t g = 1; g <= K; ++g) {
+    if (K % g) continue;
+    const int32_t d = g < 75 ? 75 - g : (g > 105 ? g - 105 : 0);
+    if (best < 0 || d < bestd || (d == bestd && g > best)) {
+      best = g;
+      bestd = d;
+    }
+  }
+  return best;
+}
+
+uint64_t bmlp_reinforce_threshold(double p_r, int32_t K) {
+  if (K < 1) return 0;
+  const double pi = 3.14159265358979323846;
+  const double q = p_r * std::sqrt(2.0 / (pi * (double)K));
+  if (!(q > 0.0)) return 0;
+  if (q >= 1.0) return 1ull << 32;
+  return (uint64_t)std::ceil(q * 4294967296.0);
+}
+
+const char* bmlp_last_error(const bmlp_t* h) {
+  return h ? h->err.c_str() : g_create_error.c_str();
+}
+
+int bmlp_create(const int32_t* widths, int32_t n_widths, int32_t classes, int16_t h_max,
+                uint64_t seed, const bmlp_hparams* hpin, bmlp_t** out) {
+  g_create_error.clear();
+  if (!out) return fail(nullptr, BMLP_EINVAL, "out is NULL");
+  *out = nullptr;
+  if (!widths) return fail(nullptr, BMLP_EINVAL, "widths is NULL");
+  if (n_widths < 2 || n_widths > BMLP_MAX_LAYERS + 1)
+    return fail(nullptr, BMLP_EINVAL, "n_widths must be in 2..%d", BMLP_MAX_LAYERS + 1);
+  for (int i = 0; i < n_widths; ++i)
+    if (widths[i] < 1 || widths[i] > (1 << 20))
+      return fail(nullptr, BMLP_EINVAL, "width %d out of range (1..2^20)", i);
+  if (classes < 2 || classes > BMLP_MAX_CLASSES)
+    return fail(nullptr, BMLP_EINVAL, "classes must be in 2..%d", BMLP_MAX_CLASSES);
+  if (h_max < 1 || (h_max % 2) == 0) return fail(nullptr, BMLP_EINVAL, "h_max must be odd and >= 1");
+  bmlp_hparams hp{};
+  if (hpin) hp = *hpin;
+  const int bs = hp.bs == 0 ? 100 : hp.bs;
+  if (bs < 1 || bs > BMLP_MAX_BS) return fail(nullptr, BMLP_EINVAL, "bs must be in 1..%d", BMLP_MAX_BS);
+  int r_num = hp.r_num, r_den = hp.r_den;
+  if (r_den == 0) { r_num = 1; r_den = 4; }
+  if (r_den < 0 || r_num < 0) return fail(nullptr, BMLP_EINVAL, "r must be non-negative");
+  const double p_r0 = hp.p_r0 < 0 ? 0.5 : hp.p_r0;
+  if (!(p_r0 >= 0.0) || !std::isfinite(p_r0)) return fail(nullptr, BMLP_EINVAL, "p_r0 invalid");
+  int fwd = hp.fwd_impl == BMLP_FWD_AUTO ? BMLP_FWD_POPC : hp.fwd_impl;
+  if (fwd != BMLP_FWD_POPC) return fail(nullptr, BMLP_EINVAL, "fwd_impl %d not available", hp.fwd_impl);
+  const int L = n_widths - 1;
+  std::vector<int> gam(L + 1, 0);
+  for (int l = 1; l <= L; ++l) {
+    const int g = hp.gamma ? hp.gamma[l - 1] : bmlp_gamma_rule(widths[l]);
+    if (g < 1 || widths[l] % g) return fail(nullptr, BMLP_EINVAL, "gamma of layer %d must divide K_l", l);
+    gam[l] = g;
+  }
+  int ndev = 0;
+  if (cudaGetDeviceCount(&ndev) != cudaSuccess || ndev == 0) {
+    (void)cudaGetLastError();
+    return fail(nullptr, BMLP_ENODEV, "no CUDA device");
+  }
+
+  bmlp_t* h = new (std::nothrow) bmlp_t();
+  if (!h) return fail(nullptr, BMLP_ENOMEM, "host allocation failed");
+  cudaGetDevice(&h->device);
+  cudaDeviceProp prop;
+  cudaFuncAttributes fa;
+  if (cudaGetDeviceProperties(&prop, h->device) != cudaSuccess || prop.major != 10 ||
+      cudaFuncGetAttributes(&fa, k_update) != cudaSuccess) {
+    (void)cudaGetLastError();
+    delete h;
+    return fail(nullptr, BMLP_ENODEV, "device has no sm_103a kernel image (needs a GB300)");
+  }
+  h->L = L; h->c = classes; h->h_max = h_max; h->bs = bs; h->r_num = r_num; h->r_den = r_den;
+  h->fwd_impl = fwd; h->seed = seed; h->p_r = p_r0;
+  h->K.assign(widths, widths + n_widths);
+  h->gamma = gam;
+
+  auto bail = [&](int rc) { std::string m = h->err; bmlp_destroy(h); g_create_error = m; return rc; };
+  int rc;
+  StepParams& P = h->hp;
+  std::memset(&P, 0, sizeof(P));
+  P.L = L; P.c = classes; P.bs = bs; P.h_max = h_max; P.r_num = r_num; P.r_den = r_den;
+  P.nw0 = words_of(widths[0]);
+  P.key0 = (uint32_t)(seed & 0xffffffffu);
+  P.key1 = (uint32_t)(seed >> 32);
+  int cta = 0;
+  for (int l = 1; l <= L; ++l) {
+    DevLayer& D = P.layer[l - 1];
+    D.Kin = h->K[l - 1]; D.Kout = h->K[l];
+    D.nw_in = words_of(D.Kin); D.nw_out = words_of(D.Kout);
+    D.ldh = 64 * D.nw_in; D.gamma = gam[l]; D.G = D.Kout / D.gamma;
+    D.upd_cta_base = cta;
+    D.upd_ctas = D.G * ((D.gamma + kUpdRowsPerCta - 1) / kUpdRowsPerCta);
+    cta += D.upd_ctas;
+    if ((rc = dalloc(h, &D.H, (size_t)D.Kout * D.ldh)) ||
+        (rc = dalloc(h, &D.W, (size_t)D.Kout * D.nw_in)) ||
+        (rc = dalloc(h, &D.PT, (size_t)classes * D.nw_out)) ||
+        (rc = dalloc(h, &D.rho, (size_t)D.Kout * classes)) ||
+        (rc = dalloc(h, &D.Z, (size_t)bs * D.Kout)) ||
+        (rc = dalloc(h, &D.A, (size_t)bs * D.nw_out)) ||
+        (rc = dalloc(h, &D.mark, (size_t)bs)) ||
+        (rc = dalloc(h, &D.sel, (size_t)bs * D.G)))
+      return bail(rc);
+  }
+  h->updCtas = cta;
+  P.upd_ctas_total = cta;
+  h->updSmem = sizeof(int32_t) * ((size_t)(bs + 1) / 2 + (size_t)(kUpdThreads / 32) * bs);
+  if ((rc = dalloc(h, &h->dP, 1)) || (rc = dalloc(h, &h->dCtrl, 1)) ||
+      (rc = dalloc(h, &h->dT, BMLP_MAX_LAYERS)))
+    return bail(rc);
+  P.ctrl = h->dCtrl;
+  P.T = h->dT;
+  if (cudaMallocHost(&h->hostPinned, 4 * sizeof(unsigned long long)) != cudaSuccess) {
+    h->hostPinned = nullptr;
+    return bail(fail(h, BMLP_ENOMEM, "cudaMallocHost failed"));
+  }
+  // initial state (Alg. 1 l.2)
+  for (int l = 1; l <= L; ++l) {
+    DevLayer& D = P.layer[l - 1];
+    const int64_t n1 = (int64_t)D.Kout * (D.ldh >> 3);
+    k_init_hw<<<(unsigned)((n1 + 255) / 256), 256>>>(D.H, D.W, D.Kin, D.Kout, D.ldh, D.nw_in, l,
+                                                       P.key0, P.key1);
+    const int64_t n2 = (int64_t)D.Kout * classes;
+    k_init_rho<<<(unsigned)((n2 + 255) / 256), 256>>>(D.rho, D.Kout, classes, l, P.key0, P.key1);
+    const int64_t n3 = (int64_t)classes * D.nw_out;
+    k_pack_pt<<<(unsigned)((n3 + 255) / 256), 256>>>(D.rho, D.PT, D.Kout, classes, D.nw_out);
+  }
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return bail(cuda_fail(h, e, "init kernels"));
+  if ((e = cudaMemset(h->dCtrl, 0, sizeof(Ctrl))) != cudaSuccess) return bail(cuda_fail(h, e, "memset"));
+  if ((e = cudaMemcpy(h->dP, &P, sizeof(P), cudaMemcpyHostToDevice)) != cudaSuccess)
+    return bail(cuda_fail(h, e, "param upload"));
+  if ((rc = upload_thresholds(h, 0)) != BMLP_OK) return bail(rc);
+  if ((e = cudaDeviceSynchronize()) != cudaSuccess) return bail(cuda_fail(h, e, "init"));
+  h->launches += 3 * L;
+  *out = h;
+  return BMLP_OK;
+}
+
+void bmlp_destroy(bmlp_t* h) {
+  if (!h) return;
+  cudaDeviceSynchronize();
+  if (h->stepExec) cudaGraphExecDestroy(h->stepExec);
+  if (h->capStream) cudaStreamDestroy(h->capStream);
+  for (auto e : h->evPool) cudaEventDestroy(e);
+  for (void* p : h->allocs) cudaFree(p);
+  if (h->hostPinned) cudaFreeHost(h->hostPinned);
+  delete h;
+}
+
+int bmlp_train(bmlp_t* h, const uint64_t* x, const int32_t* labels, int64_t n, uint32_t flags,
+               void* cuda_stream, int64_t* n_errors_out) {
+  if (!h) return BMLP_EINVAL;
+  h->err.clear();
+  if (n < 0) return fail(h, BMLP_EINVAL, "n < 0");
+  if (n > 0 && (!x || !labels)) return fail(h, BMLP_EINVAL, "x or labels is NULL");
+  if ((n + h->bs - 1) / h->bs > 0xffffffffLL) return fail(h, BMLP_EINVAL, "n too large");
+  cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
+  const bool want_count = n_errors_out != nullptr;
+  if (want_count) {
+    CK(h, cudaMemcpyAsync(&h->hostPinned[0], &h->dCtrl->err, sizeof(unsigned long long),
+                          cudaMemcpyDeviceToHost, st));
+  }
+  int rc = BMLP_OK;
+  if (n > 0) {
+    const bool xdev = is_device_ptr(x), ydev = is_device_ptr(labels);
+    if (xdev && ydev) {
+      rc = run_steps(h, x, labels, n, st);
+    } else {
+      if (!ydev)
+        for (int64_t i = 0; i < n; ++i)
+          if (labels[i] < 0 || labels[i] >= h->c) return fail(h, BMLP_EINVAL, "label %lld out of range", (long long)i);
+      const int64_t chunk = (kStageRows / h->bs) * h->bs;
+      if ((rc = ensure_staging(h, chunk)) != BMLP_OK) return rc;
+      for (int64_t s0 = 0; s0 < n && rc == BMLP_OK; s0 += chunk) {
+        const int64_t m = std::min(chunk, n - s0);
+        const uint64_t* xs = x + s0 * h->hp.nw0;
+        const int32_t* ys = labels + s0;
+        prof_begin(h, kProfCopy, st);
+        if (!xdev) CK(h, cudaMemcpyAsync(h->stX, xs, sizeof(uint64_t) * m * h->hp.nw0, cudaMemcpyHostToDevice, st));
+        if (!ydev) CK(h, cudaMemcpyAsync(h->stY, ys, sizeof(int32_t) * m, cudaMemcpyHostToDevice, st));
+        prof_end(h, st);
+        rc = run_steps(h, xdev ? xs : h->stX, ydev ? ys : h->stY, m, st);
+      }
+    }
+    if (rc != BMLP_OK) return rc;
+  }
+  h->epoch_n += n;
+  const bool epoch_end = (flags & BMLP_EPOCH_END) != 0;
+  if (want_count || epoch_end) {
+    CK(h, cudaMemcpyAsync(&h->hostPinned[1], &h->dCtrl->err, sizeof(unsigned long long),
+                          cudaMemcpyDeviceToHost, st));
+    CK(h, cudaMemcpyAsync(&h->hostPinned[2], &h->dCtrl->bad_labels, sizeof(unsigned long long),
+                          cudaMemcpyDeviceToHost, st));
+    CK(h, cudaStreamSynchronize(st));
+    if (h->hostPinned[2] != 0) {
+      CK(h, cudaMemsetAsync(&h->dCtrl->bad_labels, 0, sizeof(unsigned long long), st));
+      return fail(h, BMLP_EINVAL, "%llu labels outside 0..c-1", (unsigned long long)h->hostPinned[2]);
+    }
+    if (want_count) *n_errors_out = (int64_t)(h->hostPinned[1] - h->hostPinned[0]);
+    if (epoch_end) {
+      const double E = h->epoch_n > 0 ? (double)h->hostPinned[1] / (double)h->epoch_n : 0.0;
+      h->p_r = h->p_r * std::sqrt(E);
+      h->epoch_n = 0;
+      CK(h, cudaMemsetAsync(&h->dCtrl->err, 0, sizeof(unsigned long long), st));
+      if ((rc = upload_thresholds(h, st)) != BMLP_OK) return rc;
+    }
+  }
+  return prof_collect(h, st);
+}
+
+int bmlp_predict(bmlp_t* h, const uint64_t* x, int64_t n, int32_t* out, void* cuda_stream) {
+  if (!h) return BMLP_EINVAL;
+  h->err.clear();
+  if (n < 0) return fail(h, BMLP_EINVAL, "n < 0");
+  if (n == 0) return BMLP_OK;
+  if (!x || !out) return fail(h, BMLP_EINVAL, "x or labels_out is NULL");
+  cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
+  const bool xdev = is_device_ptr(x), odev = is_device_ptr(out);
+  int rc;
+  const int64_t chunk = std::min<int64_t>(kEvalChunk, n);
+  if ((rc = ensure_eval(h, chunk)) != BMLP_OK) return rc;
+  if ((!xdev || !odev) && (rc = ensure_staging(h, kStageRows)) != BMLP_OK) return rc;
+  const int nw0 = h->hp.nw0;
+  for (int64_t s0 = 0; s0 < n; s0 += chunk) {
+    const int64_t m = std::min(chunk, n - s0);
+    const uint64_t* in = x + s0 * nw0;
+    if (!xdev) {
+      prof_begin(h, kProfCopy, st);
+      CK(h, cudaMemcpyAsync(h->stX, in, sizeof(uint64_t) * m * nw0, cudaMemcpyHostToDevice, st));
+      prof_end(h, st);
+      in = h->stX;
+    }
+    int cur = 0;
+    for (int l = 1; l <= h->L; ++l) {
+      const DevLayer& D = h->hp.layer[l - 1];
+      prof_begin(h, kProfEvalFwd, st);
+      k_forward_eval<<<eval_forward_grid(m, D.Kout), eval_forward_block(), 0, st>>>(
+          in, m, D.nw_in, D.W, D.Kout, D.Kin, h->evA[cur], D.nw_out);
+      prof_end(h, st);
+      in = h->evA[cur];
+      cur ^= 1;
+    }
+    const DevLayer& DL = h->hp.layer[h->L - 1];
+    int32_t* o = odev ? out + s0 : h->stOut;
+    prof_begin(h, kProfOut, st);
+    k_predict_out<<<(unsigned)((m + 7) / 8), 256, 0, st>>>(in, m, DL.nw_out, DL.PT, h->c, DL.Kout, o);
+    prof_end(h, st);
+    CK(h, cudaGetLastError());
+    h->launches += h->L + 1;
+    if (!odev) {
+      prof_begin(h, kProfCopy, st);
+      CK(h, cudaMemcpyAsync(out + s0, h->stOut, sizeof(int32_t) * m, cudaMemcpyDeviceToHost, st));
+      prof_end(h, st);
+    }
+  }
+  if (!odev) CK(h, cudaStreamSynchronize(st));
+  return prof_collect(h, st);
+}
+
+int bmlp_get_state(const bmlp_t* hc, int32_t layer, int16_t* H_out, uint64_t* W_out, int8_t* P_out,
+                   double* p_r_out, int64_t* step_out) {
+  bmlp_t* h = const_cast<bmlp_t*>(hc);
+  if (!h) return BMLP_EINVAL;
+  h->err.clear();
+  if (layer < 1 || layer > h->L) return fail(h, BMLP_EINVAL, "layer must be in 1..%d", h->L);
+  CK(h, cudaDeviceSynchronize());
+  const DevLayer& D = h->hp.layer[layer - 1];
+  if (H_out)
+    CK(h, cudaMemcpy2D(H_out, sizeof(int16_t) * D.Kin, D.H, sizeof(int16_t) * D.ldh,
+                       sizeof(int16_t) * D.Kin, D.Kout, cudaMemcpyDeviceToHost));
+  if (W_out) CK(h, cudaMemcpy(W_out, D.W, sizeof(uint64_t) * D.Kout * D.nw_in, cudaMemcpyDeviceToHost));
+  if (P_out) CK(h, cudaMemcpy(P_out, D.rho, (size_t)D.Kout * h->c, cudaMemcpyDeviceToHost));
+  if (p_r_out) *p_r_out = h->p_r;
+  if (step_out) {
+    unsigned long long t = 0;
+    CK(h, cudaMemcpy(&t, &h->dCtrl->t, sizeof(t), cudaMemcpyDeviceToHost));
+    *step_out = (int64_t)t;
+  }
+  return BMLP_OK;
+}
+
+int bmlp_set_state(bmlp_t* h, int32_t layer, const int16_t* H_in, double p_r, int64_t step) {
+  if (!h) return BMLP_EINVAL;
+  h->err.clear();
+  if (layer < 1 || layer > h->L) return fail(h, BMLP_EINVAL, "layer must be in 1..%d", h->L);
+  const DevLayer& D = h->hp.layer[layer - 1];
+  if (H_in) {
+    const int64_t cnt = (int64_t)D.Kout * D.Kin;
+    for (int64_t i = 0; i < cnt; ++i) {
+      const int v = H_in[i];
+      if ((v % 2) == 0 || v > h->h_max || v < -h->h_max)
+        return fail(h, BMLP_ESTATE, "hidden weight %lld = %d is not odd within [-h_max, h_max]", (long long)i, v);
+    }
+  }
+  if (step >= 0 && (!(p_r >= 0.0) || !std::isfinite(p_r))) return fail(h, BMLP_ESTATE, "p_r invalid");
+  CK(h, cudaDeviceSynchronize());
+  if (H_in) {
+    CK(h, cudaMemcpy2D(D.H, sizeof(int16_t) * D.ldh, H_in, sizeof(int16_t) * D.Kin,
+                       sizeof(int16_t) * D.Kin, D.Kout, cudaMemcpyHostToDevice));
+    const int64_t nwt = (int64_t)D.Kout * D.nw_in;
+    k_repack_w<<<(unsigned)((nwt + 255) / 256), 256>>>(D.H, D.W, D.Kin, D.Kout, D.ldh, D.nw_in);
+    CK(h, cudaGetLastError());
+    h->launches += 1;
+  }
+  if (step >= 0) {
+    h->p_r = p_r;
+    unsigned long long t = (unsigned long long)step;
+    CK(h, cudaMemcpy(&h->dCtrl->t, &t, sizeof(t), cudaMemcpyHostToDevice));
+    h->t_host = step;
+    int rc = upload_thresholds(h, 0);
+    if (rc != BMLP_OK) return rc;
+  }
+  CK(h, cudaMemset(&h->dCtrl->err, 0, sizeof(unsigned long long)));
+  h->epoch_n = 0;
+  CK(h, cudaDeviceSynchronize());
+  return BMLP_OK;
+}
+
+int bmlp_get_info(const bmlp_t* h, int32_t* n_layers, int32_t* widths_out, int32_t* classes,
+                  int32_t* gamma_out, int32_t* bs, int32_t* fwd_impl) {
+  if (!h) return BMLP_EINVAL;
+  if (n_layers) *n_layers = h->L;
+  if (widths_out) for (int l = 0; l <= h->L; ++l) widths_out[l] = h->K[l];
+  if (classes) *classes = h->c;
+  if (gamma_out) for (int l = 1; l <= h->L; ++l) gamma_out[l - 1] = h->gamma[l];
+  if (bs) *bs = h->bs;
+  if (fwd_impl) *fwd_impl = h->fwd_impl;
+  return BMLP_OK;
+}
+
+int bmlp_debug_last_step(const bmlp_t* hc, int32_t layer, int16_t* Z, uint64_t* A, uint8_t* mark,
+                         int16_t* sel) {
+  bmlp_t* h = const_cast<bmlp_t*>(hc);
+  if (!h) return BMLP_EINVAL;
+  h->err.clear();
+  if (layer < 1 || layer > h->L) return fail(h, BMLP_EINVAL, "layer must be in 1..%d", h->L);
+  CK(h, cudaDeviceSynchronize());
+  const DevLayer& D = h->hp.layer[layer - 1];
+  if (Z) CK(h, cudaMemcpy(Z, D.Z, sizeof(int16_t) * h->bs * D.Kout, cudaMemcpyDeviceToHost));
+  if (A) CK(h, cudaMemcpy(A, D.A, sizeof(uint64_t) * h->bs * D.nw_out, cudaMemcpyDeviceToHost));
+  if (mark) CK(h, cudaMemcpy(mark, D.mark, (size_t)h->bs, cudaMemcpyDeviceToHost));
+  if (sel) CK(h, cudaMemcpy(sel, D.sel, sizeof(int16_t) * h->bs * D.G, cudaMemcpyDeviceToHost));
+  return BMLP_OK;
+}
+
+int bmlp_set_profiling(bmlp_t* h, int32_t on) {
+  if (!h) return BMLP_EINVAL;
+  h->profiling = on != 0;
+  return BMLP_OK;
+}
+
+int bmlp_get_profile(const bmlp_t* h, int32_t kind, int64_t* launches, double* total_ms) {
+  if (!h || kind < 0 || kind >= kProfKinds) return BMLP_EINVAL;
+  if (launches) *launches = h->profN[kind];
+  if (total_ms) *total_ms = h->profMs[kind];
+  return BMLP_OK;
+}
+
+int bmlp_reset_profile(bmlp_t* h) {
+  if (!h) return BMLP_EINVAL;
+  for (int i = 0; i < kProfKinds; ++i) { h->profN[i] = 0; h->profMs[i] = 0.0; }
+  return BMLP_OK;
+}
+
+int64_t bmlp_launch_count(const bmlp_t* h) { return h ? h->launches : -1; }
+
+}  // extern "C"

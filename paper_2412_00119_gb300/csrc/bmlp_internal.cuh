@@ -1,0 +1,132 @@
+// bmlp_internal.cuh -- device-side data layout and shared device helpers of the
+// BMLP library (fully binary training rule of arXiv 2412.00119, Alg. 1-3).
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "../../include/bmlp.h"
+
+namespace bk {
+
+// ---------------------------------------------------------------------------
+// HBM layout of one layer l (K_in = K_{l-1}, K_out = K_l):
+//   H    int16 [K_out][ldh]      hidden weights, neuron-major; ldh = 64*nw_in;
+//                                 entries i >= K_in are padding (never read as weights)
+//   W    uint64 [K_out][nw_in]    packed sign(H), bit (i%64) of word i/64 = (h_ik > 0)
+//   PT   uint64 [c][nw_out]       packed P_l^T, bit (k%64) of word k/64 = (rho_kj > 0)
+//   rho  int8  [K_out][c]         P_l itself, for the stability rho_{k,y}
+//   Z    int16 [bs][K_out]        pre-activations of the current mini-batch
+//   A    uint64 [bs][nw_out]      packed activations a_l of the current mini-batch
+//   mark uint8 [bs]               1 iff the pattern is in M_l
+//   sel  int16 [bs][G]            selected neuron per (pattern, group), -1 = none
+// ---------------------------------------------------------------------------
+struct DevLayer {
+  int16_t* H;
+  uint64_t* W;
+  uint64_t* PT;
+  int8_t* rho;
+  int16_t* Z;
+  uint64_t* A;
+  uint8_t* mark;
+  int16_t* sel;
+  int32_t Kin, Kout, nw_in, nw_out, ldh, gamma, G;
+  int32_t upd_cta_base;  // first CTA of this layer in the update grid
+  int32_t upd_ctas;      // CTAs of this layer in the update grid
+};
+
+// Device-resident step control.  The update kernel's last CTA advances t and s
+// and clears the per-step flags, so that one captured graph replays step after
+// step without host involvement.
+struct Ctrl {
+  unsigned long long t;         // global mini-batch counter since creation
+  unsigned long long err;       // last-layer 01-loss count since the last epoch end
+  unsigned long long bad_labels;// labels outside 0..c-1 seen by the kernels
+  uint32_t s;                   // mini-batch index within the current train call
+  uint32_t done;                // CTAs of the update kernel finished this step
+  uint32_t any_mark[BMLP_MAX_LAYERS];
+};
+
+struct StepParams {
+  DevLayer layer[BMLP_MAX_LAYERS];
+  const uint64_t* x;            // packed inputs of the current train call
+  const int32_t* y;             // labels of the current train call
+  int64_t n;                    // patterns in the current train call
+  const unsigned long long* T;  // [L] reinforcement thresholds (Alg. 3 l.8)
+  Ctrl* ctrl;
+  int32_t L, c, bs, h_max, r_num, r_den, nw0, upd_ctas_total;
+  uint32_t key0, key1;          // Philox key = (seed mod 2^32, seed div 2^32)
+};
+
+// Rows of one group handled by one update CTA.
+constexpr int kUpdRowsPerCta = 16;
+constexpr int kUpdThreads = 256;
+constexpr int kClsThreads = 256;
+
+// ---------------------------------------------------------------------------
+// Philox4x32-10 (Salmon, Moraes, Dror, Shaw, SC'11), device version.
+// Counter layout of the library's random streams (purpose tag in c2):
+//   initial h_ik of layer l : (i/4, k, 1*2^16 + l, 0)   word i%4, +1 iff bit 31
+//   rho_kj of P_l           : (j/4, k, 2*2^16 + l, 0)   word j%4, +1 iff bit 31
+//   reinforcement draw U of h_ik at step t: high 16 bits = lane i%8 of
+//     (i/8, k, 3*2^16 + l, t), low 16 bits = lane i%8 of (i/8, k, 4*2^16 + l, t);
+//     lane j of (w0..w3) is the 16-bit half j%2 (low half first) of w_{j/2}.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ uint4 philox4x32_10(uint4 ctr, uint32_t k0, uint32_t k1) {
+#pragma unroll
+  for (int r = 0; r < 10; ++r) {
+    const uint32_t lo0 = 0xD2511F53u * ctr.x;
+    const uint32_t hi0 = __umulhi(0xD2511F53u, ctr.x);
+    const uint32_t lo1 = 0xCD9E8D57u * ctr.z;
+    const uint32_t hi1 = __umulhi(0xCD9E8D57u, ctr.z);
+    ctr = make_uint4(hi1 ^ ctr.y ^ k0, lo1, hi0 ^ ctr.w ^ k1, lo0);
+    k0 += 0x9E3779B9u;
+    k1 += 0xBB67AE85u;
+  }
+  return ctr;
+}
+
+__device__ __forceinline__ uint32_t lane16(const uint4& w, int j) {
+  const uint32_t word = (j < 2) ? w.x : (j < 4) ? w.y : (j < 6) ? w.z : w.w;
+  return (j & 1) ? (word >> 16) : (word & 0xFFFFu);
+}
+
+__device__ __forceinline__ int clip_h(int h, int h_max) {
+  return h > h_max ? h_max : (h < -h_max ? -h_max : h);
+}
+
+// ---------------------------------------------------------------------------
+// Kernels
+// ---------------------------------------------------------------------------
+// Forward of layer l (1-based) for the current training mini-batch.
+__global__ void k_train_forward(const StepParams* P, int l);
+// Local classifier, 01-loss, margin, marks, and the group selection, all layers.
+__global__ void k_cls_select(const StepParams* P);
+// CP + R + repack of every layer with a non-empty M_l, then advance the step.
+__global__ void k_update(const StepParams* P);
+// Generic forward for evaluation: A (M x nw_in) against W -> Aout (M x nw_out).
+__global__ void k_forward_eval(const uint64_t* __restrict__ A, int64_t M, int nw_in,
+                               const uint64_t* __restrict__ W, int N, int Kin,
+                               uint64_t* __restrict__ Aout, int nw_out);
+// Final classifier argmax for evaluation.
+__global__ void k_predict_out(const uint64_t* __restrict__ A, int64_t M, int nw,
+                              const uint64_t* __restrict__ PT, int c, int K,
+                              int32_t* __restrict__ out);
+// Initialisation of H, W of one layer and rho, PT.
+__global__ void k_init_hw(int16_t* H, uint64_t* W, int Kin, int Kout, int ldh, int nw_in,
+                          int l, uint32_t key0, uint32_t key1);
+__global__ void k_init_rho(int8_t* rho, int Kout, int c, int l, uint32_t key0, uint32_t key1);
+__global__ void k_pack_pt(const int8_t* rho, uint64_t* PT, int Kout, int c, int nw_out);
+// Re-derive W from H for one layer (after set_state).
+__global__ void k_repack_w(const int16_t* H, uint64_t* W, int Kin, int Kout, int ldh, int nw_in);
+// Tensor-core forward (tcgen05), training layer l.
+__global__ void k_train_forward_tc(const StepParams* P, int l);
+
+// Launch helpers implemented in the kernel files (grid shapes live next to the
+// kernels they describe).
+dim3 train_forward_grid(int bs, int Kout);
+dim3 train_forward_block();
+dim3 eval_forward_grid(int64_t M, int Kout);
+dim3 eval_forward_block();
+
+}  // namespace bk

@@ -1,0 +1,76 @@
+"""The C-ABI library without a GPU: it loads, exports every entry point that
+include/bmlp.h declares, validates arguments before touching CUDA, and its
+host-side arithmetic agrees with the oracle's independent version."""
+import ctypes as C
+import os
+import re
+
+import pytest
+
+from conftest import ROOT
+
+import paper_2412_00119_gb300 as pkg
+from paper_2412_00119_gb300 import bmlp as B
+
+
+def declared_functions():
+    with open(os.path.join(ROOT, "include", "bmlp.h")) as f:
+        text = f.read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(bmlp_[a-z_0-9]+)\s*\(", text)))
+
+
+def test_library_exports_every_declared_symbol():
+    lib = pkg.lib()
+    names = declared_functions()
+    assert len(names) >= 15
+    for name in names:
+        assert hasattr(lib, name), name
+    assert sorted(n for n, _, _ in B.SIGNATURES) == names
+
+
+def test_gamma_rule_matches_oracle(oracle_mod):
+    for K in list(range(1, 400)) + [525, 784, 1024, 1035, 2025, 2048, 4096, 8192, 10000]:
+        assert B.bmlp_gamma_rule(K) == oracle_mod.gamma_rule(K), K
+    assert B.bmlp_gamma_rule(0) == -1
+
+
+def test_threshold_matches_oracle(oracle_mod):
+    for p_r in (0.0, 1e-9, 0.01, 0.1234567, 0.25, 0.5, 0.9, 1.0, 3.0):
+        for K in (1, 2, 3, 10, 64, 100, 256, 784, 1024, 4096, 8192, 65536):
+            assert B.bmlp_reinforce_threshold(p_r, K) == oracle_mod.reinforce_threshold(p_r, K), (p_r, K)
+
+
+@pytest.mark.parametrize("kw,msg", [
+    (dict(widths=[10], classes=2), "n_widths"),
+    (dict(widths=[10, 0], classes=2), "width"),
+    (dict(widths=[10, 8], classes=1), "classes"),
+    (dict(widths=[10, 8], classes=2, h_max=4), "h_max"),
+    (dict(widths=[10, 8], classes=2, bs=2000), "bs"),
+    (dict(widths=[10, 8], classes=2, gamma=[3]), "gamma"),
+    (dict(widths=[10, 8], classes=2, r=(-1, 4)), "r must"),
+    (dict(widths=[10, 8], classes=2, fwd_impl=7), "fwd_impl"),
+])
+def test_create_rejects_bad_arguments(kw, msg):
+    with pytest.raises(B.BmlpError) as ei:
+        B.bmlp_create(**kw)
+    assert ei.value.code == B.BMLP_EINVAL
+    assert msg in str(ei.value)
+
+
+def test_create_without_gpu_reports_no_device():
+    import torch
+    if torch.cuda.is_available():
+        pytest.skip("a GPU is present")
+    with pytest.raises(B.BmlpError) as ei:
+        B.bmlp_create([16, 8], 2)
+    assert ei.value.code == B.BMLP_ENODEV
+
+
+def test_null_handle_calls_fail_cleanly():
+    lib = pkg.lib()
+    assert lib.bmlp_train(None, None, None, 0, 0, None, None) == B.BMLP_EINVAL
+    assert lib.bmlp_predict(None, None, 0, None, None) == B.BMLP_EINVAL
+    assert lib.bmlp_get_state(None, 1, None, None, None, None, None) == B.BMLP_EINVAL
+    assert lib.bmlp_launch_count(None) == -1
+    lib.bmlp_destroy(None)

@@ -1,0 +1,249 @@
+"""GPU path vs the CPU oracle, bit for bit (tolerance 0: every quantity of the
+rule is an integer or a bit).
+
+Small cases span several tiles, ragged widths (not multiples of 64 or 8), tail
+batches and the rule's degenerate settings.  The five workload shapes are
+covered at full width: the 784 -> 256 -> 10 run for its whole epoch, the
+784 -> 1024 x3 -> 10 run for one full epoch, and the larger ones on a prefix of
+mini-batch steps (the oracle's cost grows with K_{l-1} K_l), plus the
+65,536-sample forward-only sweep checked on a sample of its outputs."""
+import os
+
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+import workloads as W
+from paper_2412_00119_gb300 import bmlp as B
+
+pytestmark = pytest.mark.gpu
+
+DEV = "cuda:0"
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _setup():
+    if not torch.cuda.is_available():
+        pytest.skip("needs a GPU")
+    torch.cuda.set_device(DEV)
+    O.set_threads(os.cpu_count() or 1)
+    B.lib()
+
+
+def dev_x(xp):
+    return torch.from_numpy(np.ascontiguousarray(xp).view(np.int64)).to(DEV)
+
+
+def dev_y(y):
+    return torch.from_numpy(np.ascontiguousarray(y, dtype=np.int32)).to(DEV)
+
+
+def assert_same_state(gpu, ref, where=""):
+    L = ref.L
+    for l in range(1, L + 1):
+        H, Wp, P, p_r, step = gpu.state(l)
+        Hr = ref.H(l).T
+        assert np.array_equal(H.astype(np.int32), Hr), "H differs, layer %d %s" % (l, where)
+        assert np.array_equal(Wp, W.pack(np.where(Hr > 0, 1, -1))), "W differs, layer %d %s" % (l, where)
+        assert np.array_equal(P, ref.P(l)), "P differs, layer %d" % l
+    assert p_r == ref.p_r, (p_r, ref.p_r, where)
+    assert step == ref.step, (step, ref.step, where)
+
+
+def run_pair(widths, classes, n_train, n_test=64, epochs=2, seed=5, bs=100, gamma=None, h_max=255,
+             r=(1, 4), p_r0=0.5, gen="bias", host=False, profiling=False, teacher_hidden=16,
+             data_number=99):
+    cfg = W.small_config(widths, classes, n_train, n_test, gen=gen, teacher_hidden=teacher_hidden,
+                         number=data_number)
+    tr = W.make_split(cfg, "train")
+    gpu = B.BMLP(widths, classes, h_max=h_max, seed=seed, bs=bs, r=r, p_r0=p_r0, gamma=gamma)
+    ref = O.OracleModel(list(widths), classes, h_max=h_max, seed=seed, bs=bs, r=r, p_r0=p_r0,
+                        gamma=gamma)
+    if profiling:
+        B.bmlp_set_profiling(gpu.h, True)
+    assert_same_state(gpu, ref, "after init")
+    x_t, y_t = (tr.xp, tr.y) if host else (dev_x(tr.xp), dev_y(tr.y))
+    xo = tr.pm1()
+    for e in range(epochs):
+        eg = gpu.train(x_t, y_t, epoch_end=True, count_errors=True)
+        er = ref.train(xo, tr.y, epoch_end=True)
+        assert eg == er, ("errors", e, eg, er)
+        assert_same_state(gpu, ref, "after epoch %d" % e)
+    if n_test:
+        te = W.make_split(cfg, "test")
+        if host:
+            out = np.full(n_test, -7, np.int32)
+            gpu.predict(te.xp, out)
+        else:
+            o = torch.full((n_test,), -7, dtype=torch.int32, device=DEV)
+            gpu.predict(dev_x(te.xp), o)
+            out = o.cpu().numpy()
+        assert np.array_equal(out, ref.predict(te.pm1()))
+    return gpu, ref
+
+
+CASES = {
+    "ragged_3layer": dict(widths=(200, 130, 70), classes=10, n_train=300, bs=50, gamma=[13, 7]),
+    "tail_batch": dict(widths=(64, 64), classes=4, n_train=250),
+    "single_input_bit": dict(widths=(1, 8), classes=2, n_train=30, bs=7, gamma=[2]),
+    "gamma_1_and_K": dict(widths=(65, 63, 127), classes=3, n_train=99, bs=33, gamma=[1, 127]),
+    "hundred_classes": dict(widths=(100, 96, 40), classes=100, n_train=200, teacher_hidden=64),
+    "h_max_1": dict(widths=(300, 256, 256), classes=10, n_train=200, h_max=1),
+    "h_max_3_clipping": dict(widths=(150, 192), classes=5, n_train=400, h_max=3, p_r0=1.0),
+    "always_reinforce": dict(widths=(50, 2), classes=2, n_train=60, bs=10, p_r0=2.0, gamma=[1]),
+    "never_reinforce": dict(widths=(90, 60), classes=3, n_train=120, p_r0=0.0),
+    "r_zero": dict(widths=(80, 64), classes=4, n_train=200, r=(0, 1)),
+    "r_huge": dict(widths=(80, 64), classes=4, n_train=200, r=(1000, 1)),
+    "bs_1": dict(widths=(40, 32), classes=3, n_train=20, bs=1, gamma=[8]),
+    "bs_max": dict(widths=(64, 128), classes=4, n_train=2048, bs=1024),
+    "multi_tile_k": dict(widths=(1100, 320, 200), classes=10, n_train=300, bs=100),
+    "field_inputs": dict(widths=(3072, 128), classes=10, n_train=200, gen="field", teacher_hidden=32),
+}
+
+
+@pytest.mark.parametrize("name", sorted(CASES))
+def test_small_case(name):
+    gpu, _ = run_pair(**CASES[name])
+    gpu.close()
+
+
+def test_host_buffers_match_device_buffers():
+    gpu, _ = run_pair(widths=(130, 96), classes=5, n_train=300, host=True)
+    gpu.close()
+
+
+def test_profiling_mode_matches():
+    gpu, _ = run_pair(widths=(130, 96, 64), classes=5, n_train=300, profiling=True)
+    prof = B.bmlp_get_profile(gpu.h)
+    assert prof["update"][0] == 2 * 3 and prof["train_forward"][0] == 2 * 3 * 2
+    assert prof["update"][1] > 0
+    gpu.close()
+
+
+def test_one_step_intermediates():
+    """Z, A, marks and selections of one mini-batch equal the oracle's Alg. 1
+    and Alg. 2 steps computed from the same pre-step weights."""
+    widths, c, bs = (200, 130, 70), 10, 50
+    cfg = W.small_config(widths, c, bs, 0, teacher_hidden=16)
+    tr = W.make_split(cfg, "train")
+    gamma = [13, 7]
+    gpu = B.BMLP(widths, c, seed=11, bs=bs, gamma=gamma)
+    ref = O.OracleModel(list(widths), c, seed=11, bs=bs, gamma=gamma)
+    Hs = [ref.H(l) for l in (1, 2)]
+    gpu.train(dev_x(tr.xp), dev_y(tr.y))
+    a = tr.pm1()
+    for l in (1, 2):
+        z, a_new = O.layer_forward(a, Hs[l - 1])
+        yhat = O.local_output(a_new, ref.P(l))
+        pred, ell, tau, mark = O.local_loss(yhat, tr.y, widths[l], 1, 4)
+        sel = O.select(z, ref.P(l), tr.y, mark, gamma[l - 1])
+        Zg, Ag, mg, sg = B.bmlp_debug_last_step(gpu.h, l)
+        assert np.array_equal(Zg.astype(np.int32), z)
+        assert np.array_equal(Ag, W.pack(a_new))
+        assert np.array_equal(mg, mark)
+        assert np.array_equal(sg.astype(np.int32), sel)
+        a = a_new
+    gpu.close()
+
+
+def test_resume_from_state():
+    widths, c = (150, 128, 64), 6
+    cfg = W.small_config(widths, c, 300, 0)
+    tr = W.make_split(cfg, "train")
+    x, y = dev_x(tr.xp), dev_y(tr.y)
+    a = B.BMLP(widths, c, seed=3, bs=60)
+    a.train(x, y, epoch_end=True)
+    b = B.BMLP(widths, c, seed=3, bs=60)
+    for l in (1, 2):
+        H, _, _, p_r, step = a.state(l)
+        b.set_state(l, H, p_r, step)
+    a.train(x, y, epoch_end=True)
+    b.train(x, y, epoch_end=True)
+    for l in (1, 2):
+        sa, sb = a.state(l), b.state(l)
+        for u, v in zip(sa, sb):
+            assert np.array_equal(np.asarray(u), np.asarray(v))
+    bad = a.state(1)[0].copy()
+    bad[0, 0] = 2
+    with pytest.raises(B.BmlpError) as ei:
+        a.set_state(1, bad, 0.5, 0)
+    assert ei.value.code == B.BMLP_ESTATE
+    a.close()
+    b.close()
+
+
+def test_bad_labels_are_reported():
+    gpu = B.BMLP((64, 64), 4, seed=1, bs=10)
+    xp = W.pack(np.ones((20, 64), np.int8))
+    y = np.zeros(20, np.int32)
+    y[13] = 4
+    with pytest.raises(B.BmlpError) as ei:
+        gpu.train(dev_x(xp), dev_y(y), count_errors=True)
+    assert ei.value.code == B.BMLP_EINVAL
+    y[13] = -1
+    with pytest.raises(B.BmlpError) as ei:
+        gpu.train(xp, y)              # host labels are checked before any work
+    assert ei.value.code == B.BMLP_EINVAL
+    gpu.close()
+
+
+def test_zero_patterns_is_a_noop():
+    gpu = B.BMLP((64, 64), 4, seed=1, bs=10)
+    before = gpu.state(1)
+    gpu.train(torch.empty((0, 1), dtype=torch.int64, device=DEV),
+              torch.empty(0, dtype=torch.int32, device=DEV), count_errors=True)
+    gpu.predict(torch.empty((0, 1), dtype=torch.int64, device=DEV),
+                torch.empty(0, dtype=torch.int32, device=DEV))
+    after = gpu.state(1)
+    assert np.array_equal(before[0], after[0]) and before[4] == after[4] == 0
+    gpu.close()
+
+
+# -- the workload shapes at full width ------------------------------------------
+
+def _full_width(key, steps=None, n_test=None, sweep=False):
+    cfg = W.CONFIGS[key]
+    n = cfg.n_train if steps is None else steps * 100
+    xp = W.make_inputs(cfg, "train", n)
+    teacher = W.make_teacher(cfg)
+    y = W.teacher_labels_pm1(teacher, W.unpack(xp, cfg.widths[0]))
+    gpu = B.BMLP(cfg.widths, cfg.classes, seed=cfg.model_seed, bs=100)
+    ref = O.OracleModel(list(cfg.widths), cfg.classes, seed=cfg.model_seed, bs=100)
+    eg = gpu.train(dev_x(xp), dev_y(y), epoch_end=steps is None, count_errors=True)
+    er = ref.train(W.unpack(xp, cfg.widths[0]), y, epoch_end=steps is None)
+    assert eg == er
+    assert_same_state(gpu, ref, key)
+    if n_test:
+        xt = W.make_inputs(cfg, "test", n_test)
+        o = torch.empty(n_test, dtype=torch.int32, device=DEV)
+        gpu.predict(dev_x(xt), o)
+        got = o.cpu().numpy()
+        if sweep:
+            rng = np.random.default_rng(0)
+            idx = np.concatenate([np.arange(256), rng.choice(n_test, 256, replace=False)])
+            want = ref.predict(W.unpack(xt[idx], cfg.widths[0]))
+            assert np.array_equal(got[idx], want)
+        else:
+            assert np.array_equal(got, ref.predict(W.unpack(xt, cfg.widths[0])))
+    gpu.close()
+
+
+def test_c1_784_256_full_epoch():
+    _full_width("C1", n_test=500)
+
+
+def test_c2_784_1024x3_first_epoch():
+    _full_width("C2", n_test=2000)
+
+
+def test_c3_3072_2048x3_prefix():
+    _full_width("C3", steps=12, n_test=500)
+
+
+def test_c4_3072_4096x4_100cls_prefix():
+    _full_width("C4", steps=3, n_test=200)
+
+
+def test_c5_8192x5_prefix_and_sweep():
+    _full_width("C5", steps=2, n_test=65536, sweep=True)
