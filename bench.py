@@ -1,0 +1,459 @@
+"""Throughput of the fully binary BMLP training rule (arXiv 2412.00119) on GB300.
+
+Workload (default): the 8192 -> 8192 x4 -> 10 throughput-stress network, bs 100,
+trained on a seeded 1,000,000-sample stream of i.i.d. +-1 inputs labelled by a
++-1 teacher 8192 -> 1024 -> 10.  One bench step = one bmlp_train call over
+100,000 consecutive samples (1,000 mini-batches: forward, local classifiers,
+selection, CP + R + repack of every layer); every 10th step closes the epoch
+(p_r rescale), so ten steps are one pass over the stream.  The stream (1 GB
+packed) and the model state (512 MiB of int16 hidden weights) are far larger
+than L2, so no flush is needed between steps.
+
+Printed (rank 0, one JSON line): samples/s over all ranks, XNOR-popcount
+Gbop/s, the roofline of the dominant kernel measured live with CUDA events on
+a sample of the timed mini-batches, the oracle's CPU throughput on a bounded
+sample, the end-to-end number through the C-ABI with host (pinned) buffers,
+SM clocks sampled during the timed region, and the forward-only evaluation
+sweep (65,536 samples at batch 65,536).
+
+--impl reference times the CPU oracle (plain C, all host cores) on the same
+workload, one 100-sample mini-batch per step.
+
+Multi-GPU (torchrun): every rank trains an independent replica (model seed +
+rank) on the same stream -- the paper's "realizations of the initial
+conditions" -- with no collective on the data path; the value is the sum over
+ranks (weak scaling) and the time the max over ranks.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import workloads as W  # noqa: E402
+
+CONFIG_KEY = "C5"
+SAMPLES_PER_STEP = 100_000
+STEPS_PER_EPOCH = 10
+EVAL_BATCH = 65_536
+
+# HBM traffic of k_update per launch from the committed ncu capture
+# (profiles/k_update_c5.md), valid while the kernel source hashes to
+# UPDATE_TRAFFIC_SRC_SHA; otherwise reported as null.
+UPDATE_TRAFFIC_BYTES = None
+UPDATE_TRAFFIC_SRC_SHA = None
+
+
+def bitpairs_per_sample(widths, classes):
+    """Forward XNOR bit-pairs per pattern: sum_l K_l (K_{l-1} + c) (Table 3)."""
+    return sum(widths[l] * (widths[l - 1] + classes) for l in range(1, len(widths)))
+
+
+def update_bytes_per_launch(widths):
+    """Algorithmic HBM bytes of one update launch (all layers active): int16 H
+    read + write of every row, packed W row written."""
+    b = 0
+    for l in range(1, len(widths)):
+        nw = (widths[l - 1] + 63) // 64
+        b += widths[l] * (nw * 64 * 2 * 2 + nw * 8)
+    return b
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return d.get("hbm_gbs", 6800.0), d.get("sm_max_mhz", 2070.0), "measured"
+    except OSError:
+        return 6800.0, 2070.0, "fallback"
+
+
+def popc_peak_bitpairs(sm_mhz, sms=152, popc_per_clk=16):
+    """CUDA-core popcount peak: SMs x 16 POPC results/clock/SM x 32 bit-pairs."""
+    return sms * popc_per_clk * 32 * sm_mhz * 1e6
+
+
+def src_sha(*names):
+    h = hashlib.sha256()
+    for n in names:
+        with open(os.path.join(ROOT, "paper_2412_00119_gb300", "csrc", n), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+# -- distributed helpers (also exercised by the gloo tests) ----------------------
+
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+def replica_seed(base_seed, rank):
+    return base_seed + rank
+
+
+def max_over_ranks(value, device=None):
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()):
+        return value
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def sum_over_ranks(value, device=None):
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()):
+        return value
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.SUM)
+    return float(t.item())
+
+
+def barrier():
+    import torch.distributed as dist
+    if dist.is_available() and dist.is_initialized():
+        dist.barrier()
+
+
+# -- clocks ------------------------------------------------------------------------
+
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.idx = gpu_index
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.idx), "--query-gpu=" + self.FIELDS,
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        self.lines = []
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                out, _ = self.proc.communicate(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+                out, _ = self.proc.communicate()
+            self.lines = [ln for ln in out.splitlines() if ln.strip()]
+        return False
+
+    def summary(self):
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in getattr(self, "lines", []):
+            p = [v.strip() for v in ln.split(",")]
+            if len(p) < 9:
+                continue
+            try:
+                sm.append(float(p[1]))
+                mx = float(p[2])
+            except ValueError:
+                continue
+            for name, v in zip(names, p[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(name)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": mx,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# -- workload ----------------------------------------------------------------------
+
+def make_stream(cfg, n, device):
+    import torch
+    xp = W.make_inputs(cfg, "train", n)
+    xd = torch.from_numpy(xp.view(np.int64)).to(device)
+    yd = W.teacher_labels_packed_torch(W.make_teacher(cfg), xd, cfg.widths[0], chunk=16384)
+    return xp, xd, yd
+
+
+def cpu_baseline(cfg, x_pm1, y, threads):
+    """The oracle, as it stands, on one 100-sample mini-batch of the stream."""
+    import oracle as O
+    cores = O.set_threads(threads)
+    m = O.OracleModel(list(cfg.widths), cfg.classes, seed=cfg.model_seed, bs=100)
+    t0 = time.perf_counter()
+    m.train(x_pm1[:100], y[:100])
+    dt = time.perf_counter() - t0
+    m.close()
+    return {"value": 100.0 / dt, "unit": "samples/s", "cores": cores, "kind": "oracle",
+            "sample": "1 mini-batch (100 samples) of the 8192->8192x4->10 stream, "
+                      "forward + local classifiers + selection + CP + R of all 4 layers",
+            "seconds": dt}
+
+
+def run_reference(args):
+    """--impl reference: the CPU oracle on the host cores, same config/metric."""
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return 0
+    import oracle as O
+    cfg = W.CONFIGS[CONFIG_KEY]
+    threads = os.cpu_count() or 1
+    cores = O.set_threads(threads)
+    n = 100 * (args.steps + args.warmup)
+    xp = W.make_inputs(cfg, "train", n)
+    xpm = W.unpack(xp, cfg.widths[0])
+    y = W.teacher_labels_pm1(W.make_teacher(cfg), xpm)
+    m = O.OracleModel(list(cfg.widths), cfg.classes, seed=cfg.model_seed, bs=100)
+    for s in range(args.warmup):
+        m.train(xpm[100 * s:100 * s + 100], y[100 * s:100 * s + 100])
+    t0 = time.perf_counter()
+    for s in range(args.warmup, args.warmup + args.steps):
+        m.train(xpm[100 * s:100 * s + 100], y[100 * s:100 * s + 100])
+    dt = time.perf_counter() - t0
+    value = 100.0 * args.steps / dt
+    line = {
+        "impl": "reference", "metric": "training samples/sec", "value": value,
+        "unit": "samples/s", "n_gpus": 0, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": 1000.0 * dt / args.steps, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "int8/int32", "data": "synthetic",
+        "config": {"workload": "C5 train 8192->8192x4->10, bs 100 (one mini-batch per step)",
+                   "model": cfg.name, "global_batch": 100, "seq_len": 0, "parallelism": "none"},
+        "cpu_baseline": {"value": value, "unit": "samples/s", "cores": cores, "kind": "oracle",
+                         "sample": "%d mini-batches of 100 samples" % args.steps},
+        "e2e": {"value": value, "unit": "samples/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def run_ours(args):
+    import torch
+    import torch.distributed as dist
+
+    from paper_2412_00119_gb300 import bmlp as B
+
+    rank, world, local = dist_env()
+    if world > 1 and not dist.is_initialized():
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    cfg = W.CONFIGS[CONFIG_KEY]
+    stream = torch.cuda.current_stream()
+    hbm_gbs, sm_max_mhz, peak_src = peaks()
+
+    n_stream = cfg.n_train
+    xp, xd, yd = make_stream(cfg, n_stream, dev)
+    seed = replica_seed(cfg.model_seed, rank)
+    model = B.BMLP(cfg.widths, cfg.classes, seed=seed, bs=100)
+    h = model.h
+    steps_total = args.warmup + args.steps
+
+    def train_step(i, x, y):
+        s0 = (i % STEPS_PER_EPOCH) * SAMPLES_PER_STEP
+        end = (i % STEPS_PER_EPOCH) == STEPS_PER_EPOCH - 1
+        B.bmlp_train(h, x[s0:s0 + SAMPLES_PER_STEP], y[s0:s0 + SAMPLES_PER_STEP], SAMPLES_PER_STEP,
+                     B.BMLP_EPOCH_END if end else 0, stream)
+
+    for i in range(args.warmup):
+        train_step(i, xd, yd)
+    torch.cuda.synchronize()
+
+    # timed region: every 10th mini-batch is launched with per-kernel events
+    B.bmlp_set_profiling(h, 10)
+    B.bmlp_reset_profile(h)
+    launches0 = B.bmlp_launch_count(h)
+    ev0 = torch.cuda.Event(enable_timing=True)
+    ev1 = torch.cuda.Event(enable_timing=True)
+    barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(local) as clk:
+        ev0.record(stream)
+        for i in range(args.warmup, steps_total):
+            train_step(i, xd, yd)
+        ev1.record(stream)
+        torch.cuda.synchronize()
+    barrier()
+    ms = ev0.elapsed_time(ev1)
+    launches = B.bmlp_launch_count(h) - launches0
+    prof = B.bmlp_get_profile(h)
+    B.bmlp_set_profiling(h, 0)
+    ms_max = max_over_ranks(ms, dev)
+    total_samples = sum_over_ranks(args.steps * SAMPLES_PER_STEP, dev)
+    value = total_samples / (ms_max / 1000.0)
+
+    # per-kernel device time per mini-batch, from the sampled launches
+    L = len(cfg.widths) - 1
+    per_mb = {}
+    for kind, (n, tot) in prof.items():
+        if n:
+            per_mb[kind] = tot / n * (L if kind == "train_forward" else 1)
+    dominant = max(per_mb, key=per_mb.get)
+    step_ms_mb = ms / (args.steps * SAMPLES_PER_STEP / 100)
+    upd_avg_s = prof["update"][1] / max(prof["update"][0], 1) / 1000.0
+    fwd_avg_s = prof["train_forward"][1] / max(prof["train_forward"][0], 1) / 1000.0
+    upd_bytes = update_bytes_per_launch(cfg.widths)
+    bp_layer = 100 * cfg.widths[1] * cfg.widths[0]  # bit-pairs of one 8192x8192 forward launch
+    popc_peak = popc_peak_bitpairs(sm_max_mhz)
+    traffic = None
+    if UPDATE_TRAFFIC_BYTES is not None and UPDATE_TRAFFIC_SRC_SHA == src_sha("kern_update.cu"):
+        traffic = UPDATE_TRAFFIC_BYTES
+    kernels = {
+        "update": {"bound": "hbm", "achieved": upd_bytes / upd_avg_s / 1e9, "peak": hbm_gbs,
+                   "unit": "GB/s", "frac": upd_bytes / upd_avg_s / 1e9 / hbm_gbs,
+                   "traffic": traffic, "avg_us": upd_avg_s * 1e6,
+                   "algorithmic_bytes": upd_bytes},
+        "train_forward": {"bound": "alu", "achieved": bp_layer / fwd_avg_s / 1e12,
+                          "peak": popc_peak / 1e12, "unit": "Tbitpair/s",
+                          "frac": bp_layer / fwd_avg_s / popc_peak, "traffic": None,
+                          "avg_us": fwd_avg_s * 1e6, "algorithmic_bitpairs": bp_layer},
+    }
+    dom_key = "update" if dominant == "update" else "train_forward"
+    roofline = {k: v for k, v in kernels[dom_key].items() if k in
+                ("bound", "achieved", "peak", "unit", "frac", "traffic")}
+    roofline["kernel"] = {"update": "k_update", "train_forward": "k_train_forward"}[dom_key]
+    roofline["peak_source"] = peak_src + (" (HBM copy)" if dom_key == "update" else
+                                          " SM max clock x 152 SMs x 16 POPC/clk x 32")
+
+    # end-to-end through the C-ABI with host (pinned) buffers
+    x_host = torch.from_numpy(xp.view(np.int64)).pin_memory()
+    y_host = yd.cpu().pin_memory()
+    n_e2e = max(1, min(args.steps, 5))
+    barrier()
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for i in range(n_e2e):
+        s0 = ((args.warmup + i) % STEPS_PER_EPOCH) * SAMPLES_PER_STEP
+        B.bmlp_train(h, x_host[s0:s0 + SAMPLES_PER_STEP], y_host[s0:s0 + SAMPLES_PER_STEP],
+                     SAMPLES_PER_STEP, 0, stream, count_errors=True)
+    torch.cuda.synchronize()
+    e2e_s = max_over_ranks(time.perf_counter() - t0, dev)
+    e2e_value = sum_over_ranks(n_e2e * SAMPLES_PER_STEP, dev) / e2e_s
+
+    # forward-only evaluation sweep: 65,536 samples at batch 65,536
+    xe = torch.from_numpy(W.make_inputs(cfg, "test", EVAL_BATCH).view(np.int64)).to(dev)
+    out = torch.empty(EVAL_BATCH, dtype=torch.int32, device=dev)
+    B.bmlp_predict(h, xe, out, EVAL_BATCH, stream)
+    B.bmlp_set_profiling(h, 1)
+    B.bmlp_reset_profile(h)
+    reps = 3
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(reps):
+        B.bmlp_predict(h, xe, out, EVAL_BATCH, stream)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    B.bmlp_set_profiling(h, 0)
+    eprof = B.bmlp_get_profile(h)
+    eval_ms = e0.elapsed_time(e1) / reps
+    eval_bp = EVAL_BATCH * bitpairs_per_sample(cfg.widths, cfg.classes)
+    efwd_s = eprof["eval_forward"][1] / max(eprof["eval_forward"][0], 1) / 1000.0
+    efwd_bp = EVAL_BATCH * cfg.widths[1] * cfg.widths[0]
+    eval_info = {
+        "samples_per_s": EVAL_BATCH / (eval_ms / 1000.0), "ms_per_sweep": eval_ms,
+        "gbops": 2 * eval_bp / (eval_ms / 1000.0) / 1e9,
+        "roofline": {"bound": "alu", "kernel": "k_forward_eval",
+                     "achieved": efwd_bp / efwd_s / 1e12, "peak": popc_peak / 1e12,
+                     "unit": "Tbitpair/s", "frac": efwd_bp / efwd_s / popc_peak, "traffic": None},
+    }
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = cpu_baseline(cfg, W.unpack(xp[:100], cfg.widths[0]),
+                           yd[:100].cpu().numpy().astype(np.int32), os.cpu_count() or 1)
+
+    bp = bitpairs_per_sample(cfg.widths, cfg.classes)
+    line = {
+        "metric": "training samples/sec", "value": value, "unit": "samples/s",
+        "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_max / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "b1 (u64-packed XOR/popcount) + int16 hidden weights", "data": "synthetic",
+        "config": {"workload": "C5 train: 8192->8192x4->10, bs 100, 1,000,000-sample i.i.d. "
+                               "stream, teacher 8192->1024->10; step = 100,000 samples",
+                   "model": cfg.name, "global_batch": 100 * world, "seq_len": 0,
+                   "parallelism": "replicas x%d (independent seeds)" % world,
+                   "l2": "inputs larger than L2 (1 GB stream, 512 MiB hidden weights)"},
+        "gbops": 2 * bp * value / 1e9,
+        "roofline": roofline,
+        "kernels": {k: {kk: vv for kk, vv in v.items()} for k, v in kernels.items()},
+        "kernel_ms_per_minibatch": per_mb, "ms_per_minibatch": step_ms_mb,
+        "cpu_baseline": cpu,
+        "e2e": {"value": e2e_value, "unit": "samples/s",
+                "h2d_bytes_per_step": SAMPLES_PER_STEP * (8 * xp.shape[1] + 4),
+                "d2h_bytes_per_step": 24},
+        "gpu_launches": launches,
+        "clocks": clk.summary(),
+        "eval": eval_info,
+    }
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    model.close()
+    if world > 1:
+        dist.destroy_process_group()
+    return 0
+
+
+def run_ncu_case(args):
+    """Small case for profiler captures: the 8192->8192x4->10 model trained on
+    N mini-batches twice (the second pass is the one to capture)."""
+    import torch
+
+    from paper_2412_00119_gb300 import bmlp as B
+
+    cfg = W.CONFIGS[CONFIG_KEY]
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    n = 100 * args.ncu_case
+    xp, xd, yd = make_stream(cfg, n, dev)
+    model = B.BMLP(cfg.widths, cfg.classes, seed=cfg.model_seed, bs=100)
+    for _ in range(2):
+        model.train(xd, yd)
+    out = torch.empty(n, dtype=torch.int32, device=dev)
+    model.predict(xd, out)
+    torch.cuda.synchronize()
+    print(json.dumps({"ncu_case_minibatches": args.ncu_case, "launches": B.bmlp_launch_count(model.h)}))
+    model.close()
+    return 0
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--ncu-case", type=int, default=0, metavar="N",
+                    help="run only a small N-mini-batch case (for profiler captures)")
+    args = ap.parse_args(argv)
+    if args.ncu_case:
+        return run_ncu_case(args)
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_ours(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

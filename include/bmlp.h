@@ -159,14 +159,17 @@ uint64_t bmlp_reinforce_threshold(double p_r, int32_t K);
 int bmlp_debug_last_step(const bmlp_t* h, int32_t layer, int16_t* Z, uint64_t* A,
                          uint8_t* mark, int16_t* sel);
 
-/* Per-kernel timing.  With profiling on, train/predict launch kernels one by
- * one with CUDA events around each (no CUDA graph) and accumulate, per kernel
- * kind, the launch count and the summed device time.  kinds: 0 forward
+/* Per-kernel timing.  every = 0: off.  every = S > 0: every S-th training
+ * mini-batch (counted by the step counter t) and every evaluation launch is
+ * enqueued kernel by kernel between two CUDA events on the caller's stream; the
+ * other mini-batches replay the captured step graph as usual.  Per kernel kind
+ * the library accumulates the launch count and the summed device time when
+ * the call ends (which then synchronises the stream).  kinds: 0 forward
  * (train), 1 local classifier + selection, 2 update (CP + R + repack),
  * 3 forward (predict), 4 predict output, 5 host-buffer copies.
  * bmlp_launch_count: kernels this handle has launched since creation (graph
  * replays count each node). */
-int bmlp_set_profiling(bmlp_t* h, int32_t on);
+int bmlp_set_profiling(bmlp_t* h, int32_t every);
 int bmlp_get_profile(const bmlp_t* h, int32_t kind, int64_t* launches, double* total_ms);
 int bmlp_reset_profile(bmlp_t* h);
 int64_t bmlp_launch_count(const bmlp_t* h);

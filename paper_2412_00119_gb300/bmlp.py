@@ -223,8 +223,9 @@ def bmlp_last_error(h=None):
     return m.decode() if m else ""
 
 
-def bmlp_set_profiling(h, on=True):
-    _check(lib().bmlp_set_profiling(h, 1 if on else 0), h)
+def bmlp_set_profiling(h, every=1):
+    """every: 0 off, 1 every mini-batch, S every S-th mini-batch (True = 1)."""
+    _check(lib().bmlp_set_profiling(h, int(every)), h)
 
 
 def bmlp_get_profile(h):

@@ -56,7 +56,8 @@ struct bmlp {
   int updCtas = 0;
   size_t updSmem = 0;
   // profiling
-  bool profiling = false;
+  bool profiling = false;       // events around the kernels being enqueued now
+  int32_t profEvery = 0;        // 0 off, 1 every mini-batch, S every S-th mini-batch
   std::vector<cudaEvent_t> evPool;
   size_t evUsed = 0;
   std::vector<std::pair<int, size_t>> evPairs;  // (kind, index of start event)
@@ -203,16 +204,21 @@ int run_steps(bmlp_t* h, const uint64_t* xd, const int32_t* yd, int64_t n, cudaS
                         sizeof(StepParams) - head, cudaMemcpyHostToDevice, st));
   CK(h, cudaMemsetAsync(&h->dCtrl->s, 0, sizeof(uint32_t), st));
   const int64_t steps = (n + h->bs - 1) / h->bs;
-  if (h->profiling) {
-    for (int64_t s = 0; s < steps; ++s) {
-      int rc = enqueue_step(h, st);
-      if (rc != BMLP_OK) return rc;
-    }
-  } else {
+  if (h->profEvery != 1) {
     int rc = ensure_graph(h);
     if (rc != BMLP_OK) return rc;
-    for (int64_t s = 0; s < steps; ++s) CK(h, cudaGraphLaunch(h->stepExec, st));
   }
+  for (int64_t s = 0; s < steps; ++s) {
+    // sampled mini-batches are launched kernel by kernel between CUDA events
+    h->profiling = h->profEvery > 0 && ((h->t_host + s) % h->profEvery) == 0;
+    if (h->profiling) {
+      int rc = enqueue_step(h, st);
+      if (rc != BMLP_OK) return rc;
+    } else {
+      CK(h, cudaGraphLaunch(h->stepExec, st));
+    }
+  }
+  h->profiling = h->profEvery > 0;
   h->launches += steps * (h->L + 2);
   h->t_host += steps;
   return BMLP_OK;
@@ -597,9 +603,10 @@ int bmlp_debug_last_step(const bmlp_t* hc, int32_t layer, int16_t* Z, uint64_t* 
   return BMLP_OK;
 }
 
-int bmlp_set_profiling(bmlp_t* h, int32_t on) {
-  if (!h) return BMLP_EINVAL;
-  h->profiling = on != 0;
+int bmlp_set_profiling(bmlp_t* h, int32_t every) {
+  if (!h || every < 0) return BMLP_EINVAL;
+  h->profEvery = every;
+  h->profiling = every > 0;
   return BMLP_OK;
 }
 
