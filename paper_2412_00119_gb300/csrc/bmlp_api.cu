@@ -160,7 +160,11 @@ int prof_collect(bmlp_t* h, cudaStream_t st) {
 int enqueue_step(bmlp_t* h, cudaStream_t st) {
   for (int l = 1; l <= h->L; ++l) {
     prof_begin(h, kProfTrainFwd, st);
-    k_train_forward<<<train_forward_grid(h->bs, h->K[l]), train_forward_block(), 0, st>>>(h->dP, l);
+    if (h->fwd_impl == BMLP_FWD_TCGEN05)
+      k_train_forward_tc<<<train_forward_tc_grid(h->K[l]), train_forward_tc_block(),
+                           train_forward_tc_smem(), st>>>(h->dP, l);
+    else
+      k_train_forward<<<train_forward_grid(h->bs, h->K[l]), train_forward_block(), 0, st>>>(h->dP, l);
     prof_end(h, st);
   }
   prof_begin(h, kProfCls, st);
@@ -289,8 +293,8 @@ int bmlp_create(const int32_t* widths, int32_t n_widths, int32_t classes, int16_
   if (n_widths < 2 || n_widths > BMLP_MAX_LAYERS + 1)
     return fail(nullptr, BMLP_EINVAL, "n_widths must be in 2..%d", BMLP_MAX_LAYERS + 1);
   for (int i = 0; i < n_widths; ++i)
-    if (widths[i] < 1 || widths[i] > (1 << 20))
-      return fail(nullptr, BMLP_EINVAL, "width %d out of range (1..2^20)", i);
+    if (widths[i] < 1 || widths[i] > 32767)  // |z| <= K_{l-1} must fit the int16 Z buffer
+      return fail(nullptr, BMLP_EINVAL, "width %d out of range (1..32767)", i);
   if (classes < 2 || classes > BMLP_MAX_CLASSES)
     return fail(nullptr, BMLP_EINVAL, "classes must be in 2..%d", BMLP_MAX_CLASSES);
   if (h_max < 1 || (h_max % 2) == 0) return fail(nullptr, BMLP_EINVAL, "h_max must be odd and >= 1");
@@ -303,8 +307,12 @@ int bmlp_create(const int32_t* widths, int32_t n_widths, int32_t classes, int16_
   if (r_den < 0 || r_num < 0) return fail(nullptr, BMLP_EINVAL, "r must be non-negative");
   const double p_r0 = hp.p_r0 < 0 ? 0.5 : hp.p_r0;
   if (!(p_r0 >= 0.0) || !std::isfinite(p_r0)) return fail(nullptr, BMLP_EINVAL, "p_r0 invalid");
-  int fwd = hp.fwd_impl == BMLP_FWD_AUTO ? BMLP_FWD_POPC : hp.fwd_impl;
-  if (fwd != BMLP_FWD_POPC) return fail(nullptr, BMLP_EINVAL, "fwd_impl %d not available", hp.fwd_impl);
+  int fwd = hp.fwd_impl;
+  if (fwd == BMLP_FWD_AUTO) fwd = bs <= 128 ? BMLP_FWD_TCGEN05 : BMLP_FWD_POPC;
+  if (fwd != BMLP_FWD_POPC && fwd != BMLP_FWD_TCGEN05)
+    return fail(nullptr, BMLP_EINVAL, "fwd_impl %d not available", hp.fwd_impl);
+  if (fwd == BMLP_FWD_TCGEN05 && bs > 128)
+    return fail(nullptr, BMLP_EINVAL, "fwd_impl TCGEN05 needs bs <= 128");
   const int L = n_widths - 1;
   std::vector<int> gam(L + 1, 0);
   for (int l = 1; l <= L; ++l) {
@@ -386,6 +394,10 @@ int bmlp_create(const int32_t* widths, int32_t n_widths, int32_t classes, int16_
   }
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return bail(cuda_fail(h, e, "init kernels"));
+  if (fwd == BMLP_FWD_TCGEN05 &&
+      (e = cudaFuncSetAttribute(k_train_forward_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                (int)train_forward_tc_smem())) != cudaSuccess)
+    return bail(cuda_fail(h, e, "tcgen05 forward smem attribute"));
   if ((e = cudaMemset(h->dCtrl, 0, sizeof(Ctrl))) != cudaSuccess) return bail(cuda_fail(h, e, "memset"));
   if ((e = cudaMemcpy(h->dP, &P, sizeof(P), cudaMemcpyHostToDevice)) != cudaSuccess)
     return bail(cuda_fail(h, e, "param upload"));
@@ -451,7 +463,14 @@ int bmlp_train(bmlp_t* h, const uint64_t* x, const int32_t* labels, int64_t n, u
                           cudaMemcpyDeviceToHost, st));
     CK(h, cudaMemcpyAsync(&h->hostPinned[2], &h->dCtrl->bad_labels, sizeof(unsigned long long),
                           cudaMemcpyDeviceToHost, st));
+    CK(h, cudaMemcpyAsync(&h->hostPinned[3], &h->dCtrl->timeouts, sizeof(uint32_t),
+                          cudaMemcpyDeviceToHost, st));
     CK(h, cudaStreamSynchronize(st));
+    if ((uint32_t)h->hostPinned[3] != 0) {
+      CK(h, cudaMemsetAsync(&h->dCtrl->timeouts, 0, sizeof(uint32_t), st));
+      h->hostPinned[3] = 0;
+      return fail(h, BMLP_ETIMEOUT, "a bounded device-side wait expired");
+    }
     if (h->hostPinned[2] != 0) {
       CK(h, cudaMemsetAsync(&h->dCtrl->bad_labels, 0, sizeof(unsigned long long), st));
       return fail(h, BMLP_EINVAL, "%llu labels outside 0..c-1", (unsigned long long)h->hostPinned[2]);
@@ -626,3 +645,4 @@ int bmlp_reset_profile(bmlp_t* h) {
 int64_t bmlp_launch_count(const bmlp_t* h) { return h ? h->launches : -1; }
 
 }  // extern "C"
+

@@ -44,6 +44,7 @@ struct Ctrl {
   unsigned long long bad_labels;// labels outside 0..c-1 seen by the kernels
   uint32_t s;                   // mini-batch index within the current train call
   uint32_t done;                // CTAs of the update kernel finished this step
+  uint32_t timeouts;            // bounded device waits that expired (BMLP_ETIMEOUT)
   uint32_t any_mark[BMLP_MAX_LAYERS];
 };
 
@@ -60,6 +61,7 @@ struct StepParams {
 
 // Rows of one group handled by one update CTA.
 constexpr int kUpdRowsPerCta = 16;
+constexpr int kUpdUnroll = 4;  // 16-byte H loads in flight per lane in k_update
 constexpr int kUpdThreads = 256;
 constexpr int kClsThreads = 256;
 
@@ -119,8 +121,12 @@ __global__ void k_init_rho(int8_t* rho, int Kout, int c, int l, uint32_t key0, u
 __global__ void k_pack_pt(const int8_t* rho, uint64_t* PT, int Kout, int c, int nw_out);
 // Re-derive W from H for one layer (after set_state).
 __global__ void k_repack_w(const int16_t* H, uint64_t* W, int Kin, int Kout, int ldh, int nw_in);
-// Tensor-core forward (tcgen05), training layer l.
+// Tensor-core forward (tcgen05, +-1 as e4m3, exact fp32 sums), training layer l;
+// needs bs <= 128.
 __global__ void k_train_forward_tc(const StepParams* P, int l);
+size_t train_forward_tc_smem();
+dim3 train_forward_tc_grid(int Kout);
+dim3 train_forward_tc_block();
 
 // Launch helpers implemented in the kernel files (grid shapes live next to the
 // kernels they describe).

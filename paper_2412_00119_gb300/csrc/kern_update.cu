@@ -111,21 +111,133 @@ __global__ void __launch_bounds__(kClsThreads) k_cls_select(const StepParams* __
 }
 
 // ---------------------------------------------------------------------------
-// Hidden-weight update, fused with the visible-weight repack (Alg. 3).
+// Hidden-weight update, fused with the visible-weight repack (Alg. 3, Sec. 3.1).
 // CTA = (layer, group g, slice of kUpdRowsPerCta neurons).  A warp owns one
 // neuron row k at a time: it collects, in ascending mu, the patterns whose
 // selection in group g is k (the CP tuples of k), then streams the row in
-// chunks of 8 hidden weights (one 16-byte vector per lane):
-//   CP: h_i <- clip(h_i + 2 a^mu_i rho_{k,y^mu}) per tuple, in mu order
+// chunks of 8 hidden weights (one 16-byte vector per lane, kUpdUnroll vectors
+// in flight per lane):
+//   CP: h_i <- clip(h_i + 2 a^mu_i rho_{k,y^mu}) per tuple, in mu order.  The
+//       8 weights stay packed as int16 pairs; a shared table turns the
+//       activation byte into four packed +-2 delta words and the DPX
+//       add-min / max3 instructions clip two weights per instruction.
 //   R : U = Philox draw (hi16 lane from purpose 3, lo16 from purpose 4);
-//       U < T  ->  h_i <- clip(h_i + 2 sign h_i).  The low half is computed only
-//       when a high half equals T's high half (probability 2^-16 per weight).
-//   W : bit i = (h_i > 0); one byte per chunk, written in place.
+//       U < T  ->  h_i <- clip(h_i + 2 sign h_i).  The 16-bit lanes of the
+//       Philox output line up with the int16 pairs; a SIMD-within-a-register
+//       test against T's high half finds the chunks with an event or a tie
+//       (about 4% of chunks at the paper's p_r), and only those take the
+//       per-weight path; the low half is drawn only on a tie.
+//   W : bit i = (h_i > 0) = NOT sign bit; one byte per chunk, in place.
+// Chunks that hold only padding (i >= K_{l-1}) are never touched; a chunk that
+// is partly padding takes the per-weight path with the padding masked.
 // Layers with an empty M_l are skipped (no CP, no R).  The last CTA to finish
 // advances the step counters and clears the per-step flags.
 // ---------------------------------------------------------------------------
-__global__ void __launch_bounds__(kUpdThreads) k_update(const StepParams* __restrict__ P) {
+namespace {
+
+struct UpdCtx {
+  const uint8_t* aprev;  // previous layer's packed activations, bytes
+  size_t arow_bytes;
+  const int32_t* list;   // CP tuples of the row: mu | (rho < 0) << 16
+  int n_t;
+  int h_max;
+  uint32_t Thi, Tlo, Tpair;
+  bool fast_r;           // Thi < 2^15: the SIMD test is exact
+  uint32_t key0, key1;
+  uint32_t k, c2_hi, c2_lo, t;
+  const uint4* delta;    // [2][256] packed +-2 deltas per activation byte and rho sign
+};
+
+__device__ __forceinline__ int lane_h(const uint32_t (&w)[4], int j) {
+  return (int)(int16_t)(uint16_t)(w[j >> 1] >> (16 * (j & 1)));
+}
+
+__device__ __forceinline__ void set_lane_h(uint32_t (&w)[4], int j, int h) {
+  const int sh = 16 * (j & 1);
+  w[j >> 1] = (w[j >> 1] & ~(0xFFFFu << sh)) | (((uint32_t)h & 0xFFFFu) << sh);
+}
+
+// Per-weight path: CP (already applied by the caller when `cp_done`), R and W
+// for the first `nvalid` weights of the chunk.
+__device__ __noinline__ uint32_t chunk_scalar(uint32_t (&w)[4], int ch, int nvalid, bool cp_done,
+                                              const UpdCtx& C, uint4 rh) {
+  if (!cp_done) {
+    for (int q = 0; q < C.n_t; ++q) {
+      const int e = C.list[q];
+      const int m = e & 0xFFFF;
+      const int rho = (e & 0x10000) ? -1 : 1;
+      const uint32_t byte = C.aprev[(size_t)m * C.arow_bytes + ch];
+      for (int j = 0; j < nvalid; ++j) {
+        const int step = ((byte >> j) & 1u) ? rho : -rho;
+        set_lane_h(w, j, clip_h(lane_h(w, j) + 2 * step, C.h_max));
+      }
+    }
+  }
+  uint32_t ties = 0;
+  for (int j = 0; j < 8; ++j) ties |= (lane16(rh, j) == C.Thi ? 1u : 0u) << j;
+  uint4 rl = make_uint4(0, 0, 0, 0);
+  if (ties)
+    rl = philox4x32_10(make_uint4((uint32_t)ch, C.k, C.c2_lo, C.t), C.key0, C.key1);
+  uint32_t wbyte = 0;
+  for (int j = 0; j < nvalid; ++j) {
+    const uint32_t u = lane16(rh, j);
+    const bool fire = (u < C.Thi) || (((ties >> j) & 1u) && lane16(rl, j) < C.Tlo);
+    int h = lane_h(w, j);
+    if (fire) {
+      h = clip_h(h + (h > 0 ? 2 : -2), C.h_max);
+      set_lane_h(w, j, h);
+    }
+    wbyte |= (h > 0 ? 1u : 0u) << j;
+  }
+  return wbyte;
+}
+
+// Sign bits of the 8 packed weights -> W byte (bit j = h_j > 0, h never 0).
+__device__ __forceinline__ uint32_t w_byte(const uint32_t (&w)[4]) {
+  const uint32_t p0 = __byte_perm(w[0], w[1], 0x7531) & 0x80808080u;
+  const uint32_t p1 = __byte_perm(w[2], w[3], 0x7531) & 0x80808080u;
+  const uint32_t neg = ((p0 * 0x00204081u) >> 28) | (((p1 * 0x00204081u) >> 28) << 4);
+  return ~neg & 0xFFu;
+}
+
+__device__ __forceinline__ uint32_t chunk_packed(uint32_t (&w)[4], int ch, const UpdCtx& C,
+                                                 uint32_t neg_pair, uint32_t pos_pair) {
+  // Clipped Perceptron, two weights per DPX instruction
+  for (int q = 0; q < C.n_t; ++q) {
+    const int e = C.list[q];
+    const int m = e & 0xFFFF;
+    const uint32_t byte = C.aprev[(size_t)m * C.arow_bytes + ch];
+    const uint4 d = C.delta[((e >> 16) & 1) * 256 + byte];
+    w[0] = __vimax3_s16x2(__viaddmin_s16x2(w[0], d.x, pos_pair), neg_pair, neg_pair);
+    w[1] = __vimax3_s16x2(__viaddmin_s16x2(w[1], d.y, pos_pair), neg_pair, neg_pair);
+    w[2] = __vimax3_s16x2(__viaddmin_s16x2(w[2], d.z, pos_pair), neg_pair, neg_pair);
+    w[3] = __vimax3_s16x2(__viaddmin_s16x2(w[3], d.w, pos_pair), neg_pair, neg_pair);
+  }
+  // Reinforcement draws for the 8 weights
+  const uint4 rh = philox4x32_10(make_uint4((uint32_t)ch, C.k, C.c2_hi, C.t), C.key0, C.key1);
+  uint32_t any = 1;
+  if (C.fast_r) {
+    // lane fires iff its 16-bit draw u < Thi (< 2^15): top bit clear and low 15
+    // bits below Thi; lane ties iff u == Thi (zero lane of u ^ Tpair)
+    const uint32_t H = 0x80008000u;
+    const uint32_t u[4] = {rh.x, rh.y, rh.z, rh.w};
+    any = 0;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const uint32_t d = ((u[i] & 0x7FFF7FFFu) | H) - C.Tpair;
+      const uint32_t x = u[i] ^ C.Tpair;
+      any |= (~(d | u[i]) & H) | ((x - 0x00010001u) & ~x & H);
+    }
+  }
+  if (any) return chunk_scalar(w, ch, 8, true, C, rh);
+  return w_byte(w);
+}
+
+}  // namespace
+
+__global__ void __launch_bounds__(kUpdThreads, 3) k_update(const StepParams* __restrict__ P) {
   extern __shared__ int32_t dyn[];
+  __shared__ uint4 s_delta[2 * 256];
   const int bid = blockIdx.x;
   int li = 0;
   while (li + 1 < P->L && bid >= P->layer[li + 1].upd_cta_base) ++li;
@@ -149,20 +261,45 @@ __global__ void __launch_bounds__(kUpdThreads) k_update(const StepParams* __rest
     int32_t* s_list = dyn + (P->bs + 1) / 2 + warp * P->bs;         // [nwarps][bs]
 
     for (int m = threadIdx.x; m < bsz; m += blockDim.x) s_sel[m] = Ly.sel[(int64_t)m * Ly.G + g];
+    // s_delta[r][b]: packed int16 pair p of entry = (+-2 for bit 2p, +-2 for
+    // bit 2p+1 of b), sign flipped for r = 1 (rho = -1)
+    for (int i = threadIdx.x; i < 512; i += blockDim.x) {
+      const int r = i >> 8, b = i & 255;
+      uint32_t v[4];
+#pragma unroll
+      for (int p = 0; p < 4; ++p) {
+        int lo = ((b >> (2 * p)) & 1) ? 2 : -2;
+        int hi = ((b >> (2 * p + 1)) & 1) ? 2 : -2;
+        if (r) { lo = -lo; hi = -hi; }
+        v[p] = ((uint32_t)lo & 0xFFFFu) | ((uint32_t)hi << 16);
+      }
+      s_delta[i] = make_uint4(v[0], v[1], v[2], v[3]);
+    }
     __syncthreads();
 
     const int l = li + 1;
     const int c = P->c;
-    const int h_max = P->h_max;
+    UpdCtx C;
+    C.h_max = P->h_max;
     const unsigned long long T = P->T[li];
-    const uint32_t Thi = (uint32_t)(T >> 16);   // 0..65536
-    const uint32_t Tlo = (uint32_t)(T & 0xFFFFu);
+    C.Thi = (uint32_t)(T >> 16);   // 0..65536
+    C.Tlo = (uint32_t)(T & 0xFFFFu);
+    C.fast_r = C.Thi < 0x8000u;
+    C.Tpair = C.Thi * 0x00010001u;
+    C.key0 = P->key0;
+    C.key1 = P->key1;
+    C.c2_hi = (3u << 16) + (uint32_t)l;
+    C.c2_lo = (4u << 16) + (uint32_t)l;
+    C.t = (uint32_t)t;
+    C.delta = s_delta;
     const int Kin = Ly.Kin;
-    const int nch = Ly.ldh >> 3;                 // chunks of 8 weights per row
-    const size_t arow_bytes = (size_t)Ly.nw_in * 8;
-    const uint8_t* aprev = (li == 0)
-        ? reinterpret_cast<const uint8_t*>(P->x + start * P->nw0)
-        : reinterpret_cast<const uint8_t*>(P->layer[li - 1].A);
+    const int nch = (Kin + 7) >> 3;             // chunks holding at least one input
+    const int full = Kin >> 3;                  // chunks of 8 real inputs
+    C.arow_bytes = (size_t)Ly.nw_in * 8;
+    C.aprev = (li == 0) ? reinterpret_cast<const uint8_t*>(P->x + start * P->nw0)
+                        : reinterpret_cast<const uint8_t*>(P->layer[li - 1].A);
+    const uint32_t neg_pair = (uint32_t)(-C.h_max & 0xFFFF) * 0x00010001u;
+    const uint32_t pos_pair = (uint32_t)C.h_max * 0x00010001u;
 
     for (int rr = r0 + warp; rr < r1; rr += nwarps) {
       const int k = g * gamma + rr;
@@ -176,59 +313,41 @@ __global__ void __launch_bounds__(kUpdThreads) k_update(const StepParams* __rest
           int yv = P->y[start + m];
           if (yv < 0 || yv >= c) yv = 0;
           const int rho = Ly.rho[(int64_t)k * c + yv];
-          s_list[n_t + __popc(bal & ((1u << lane) - 1u))] = m | ((rho > 0) ? 0x10000 : 0);
+          s_list[n_t + __popc(bal & ((1u << lane) - 1u))] = m | ((rho > 0) ? 0 : 0x10000);
         }
         n_t += __popc(bal);
       }
       __syncwarp();
+      C.list = s_list;
+      C.n_t = n_t;
+      C.k = (uint32_t)k;
 
       int16_t* hrow = Ly.H + (int64_t)k * Ly.ldh;
       uint8_t* wrow = reinterpret_cast<uint8_t*>(Ly.W + (int64_t)k * Ly.nw_in);
-      for (int ch = lane; ch < nch; ch += 32) {
-        int4 hv = *reinterpret_cast<const int4*>(hrow + 8 * ch);
-        int h[8];
-        h[0] = (int16_t)(hv.x & 0xFFFF); h[1] = (int16_t)((uint32_t)hv.x >> 16);
-        h[2] = (int16_t)(hv.y & 0xFFFF); h[3] = (int16_t)((uint32_t)hv.y >> 16);
-        h[4] = (int16_t)(hv.z & 0xFFFF); h[5] = (int16_t)((uint32_t)hv.z >> 16);
-        h[6] = (int16_t)(hv.w & 0xFFFF); h[7] = (int16_t)((uint32_t)hv.w >> 16);
-        const int nvalid = min(8, Kin - 8 * ch);  // >= 1 except in pure padding
-        // Clipped Perceptron (Alg. 3 l.2-4)
-        for (int q = 0; q < n_t; ++q) {
-          const int e = s_list[q];
-          const int m = e & 0xFFFF;
-          const int rho = (e & 0x10000) ? 1 : -1;
-          const uint32_t byte = aprev[(size_t)m * arow_bytes + ch];
+      // kUpdUnroll 16-byte loads in flight per lane before any is processed;
+      // H is streamed (read once, written once per step)
+      for (int base = lane; base < nch; base += 32 * kUpdUnroll) {
+        uint4 hbuf[kUpdUnroll];
 #pragma unroll
-          for (int j = 0; j < 8; ++j) {
-            const int step = ((byte >> j) & 1u) ? rho : -rho;
-            if (j < nvalid) h[j] = clip_h(h[j] + 2 * step, h_max);
-          }
+        for (int u = 0; u < kUpdUnroll; ++u) {
+          const int ch = base + 32 * u;
+          if (ch < nch) hbuf[u] = __ldcs(reinterpret_cast<const uint4*>(hrow + 8 * ch));
         }
-        // Reinforcement (Alg. 3 l.5-12)
-        const uint4 rh = philox4x32_10(make_uint4((uint32_t)ch, (uint32_t)k, (3u << 16) + (uint32_t)l,
-                                                  (uint32_t)t), P->key0, P->key1);
-        uint32_t ties = 0;
 #pragma unroll
-        for (int j = 0; j < 8; ++j) ties |= (lane16(rh, j) == Thi ? 1u : 0u) << j;
-        uint4 rl = make_uint4(0, 0, 0, 0);
-        if (ties) rl = philox4x32_10(make_uint4((uint32_t)ch, (uint32_t)k, (4u << 16) + (uint32_t)l,
-                                                (uint32_t)t), P->key0, P->key1);
-        uint32_t wbyte = 0;
-#pragma unroll
-        for (int j = 0; j < 8; ++j) {
-          const uint32_t u = lane16(rh, j);
-          const bool fire = (u < Thi) || (((ties >> j) & 1u) && lane16(rl, j) < Tlo);
-          if (j < nvalid) {
-            if (fire) h[j] = clip_h(h[j] + (h[j] > 0 ? 2 : -2), h_max);
-            wbyte |= (h[j] > 0 ? 1u : 0u) << j;
+        for (int u = 0; u < kUpdUnroll; ++u) {
+          const int ch = base + 32 * u;
+          if (ch >= nch) break;
+          uint32_t w[4] = {hbuf[u].x, hbuf[u].y, hbuf[u].z, hbuf[u].w};
+          uint32_t wbyte;
+          if (ch < full) {
+            wbyte = chunk_packed(w, ch, C, neg_pair, pos_pair);
+          } else {
+            const uint4 rh = philox4x32_10(make_uint4((uint32_t)ch, C.k, C.c2_hi, C.t), C.key0, C.key1);
+            wbyte = chunk_scalar(w, ch, Kin - 8 * ch, false, C, rh);
           }
+          __stcs(reinterpret_cast<uint4*>(hrow + 8 * ch), make_uint4(w[0], w[1], w[2], w[3]));
+          wrow[ch] = (uint8_t)wbyte;
         }
-        hv.x = (int)(((uint32_t)h[0] & 0xFFFFu) | ((uint32_t)h[1] << 16));
-        hv.y = (int)(((uint32_t)h[2] & 0xFFFFu) | ((uint32_t)h[3] << 16));
-        hv.z = (int)(((uint32_t)h[4] & 0xFFFFu) | ((uint32_t)h[5] << 16));
-        hv.w = (int)(((uint32_t)h[6] & 0xFFFFu) | ((uint32_t)h[7] << 16));
-        *reinterpret_cast<int4*>(hrow + 8 * ch) = hv;
-        wrow[ch] = (uint8_t)wbyte;
       }
       __syncwarp();
     }

@@ -53,11 +53,14 @@ def assert_same_state(gpu, ref, where=""):
 
 def run_pair(widths, classes, n_train, n_test=64, epochs=2, seed=5, bs=100, gamma=None, h_max=255,
              r=(1, 4), p_r0=0.5, gen="bias", host=False, profiling=False, teacher_hidden=16,
-             data_number=99):
+             data_number=99, fwd=B.BMLP_FWD_AUTO):
     cfg = W.small_config(widths, classes, n_train, n_test, gen=gen, teacher_hidden=teacher_hidden,
                          number=data_number)
     tr = W.make_split(cfg, "train")
-    gpu = B.BMLP(widths, classes, h_max=h_max, seed=seed, bs=bs, r=r, p_r0=p_r0, gamma=gamma)
+    gpu = B.BMLP(widths, classes, h_max=h_max, seed=seed, bs=bs, r=r, p_r0=p_r0, gamma=gamma,
+                 fwd_impl=fwd)
+    assert gpu.info["fwd_impl"] == (fwd if fwd else
+                                    (B.BMLP_FWD_TCGEN05 if bs <= 128 else B.BMLP_FWD_POPC))
     ref = O.OracleModel(list(widths), classes, h_max=h_max, seed=seed, bs=bs, r=r, p_r0=p_r0,
                         gamma=gamma)
     if profiling:
@@ -83,6 +86,27 @@ def run_pair(widths, classes, n_train, n_test=64, epochs=2, seed=5, bs=100, gamm
     return gpu, ref
 
 
+ENGINES = {"popc": B.BMLP_FWD_POPC, "tcgen05": B.BMLP_FWD_TCGEN05}
+
+
+@pytest.mark.parametrize("engine", sorted(ENGINES))
+def test_forward_single_tile(engine):
+    """One mini-batch through one 64-neuron tile, then a ragged multi-tile layer:
+    pre-activations and packed activations equal the oracle's Alg. 1 l.8-9."""
+    for widths, bs in (((128, 64), 100), ((200, 130), 37)):
+        cfg = W.small_config(widths, 4, bs, 0, teacher_hidden=8)
+        tr = W.make_split(cfg, "train")
+        gpu = B.BMLP(widths, 4, seed=2, bs=bs, fwd_impl=ENGINES[engine])
+        ref = O.OracleModel(list(widths), 4, seed=2, bs=bs)
+        H1 = ref.H(1)
+        gpu.train(dev_x(tr.xp), dev_y(tr.y))
+        z, a = O.layer_forward(tr.pm1(), H1)
+        Zg, Ag, _, _ = B.bmlp_debug_last_step(gpu.h, 1)
+        assert np.array_equal(Zg[:bs].astype(np.int32), z), engine
+        assert np.array_equal(Ag[:bs], W.pack(a)), engine
+        gpu.close()
+
+
 CASES = {
     "ragged_3layer": dict(widths=(200, 130, 70), classes=10, n_train=300, bs=50, gamma=[13, 7]),
     "tail_batch": dict(widths=(64, 64), classes=4, n_train=250),
@@ -102,9 +126,13 @@ CASES = {
 }
 
 
+@pytest.mark.parametrize("engine", sorted(ENGINES))
 @pytest.mark.parametrize("name", sorted(CASES))
-def test_small_case(name):
-    gpu, _ = run_pair(**CASES[name])
+def test_small_case(name, engine):
+    kw = dict(CASES[name])
+    if engine == "tcgen05" and kw.get("bs", 100) > 128:
+        pytest.skip("the tcgen05 forward takes mini-batches of at most 128")
+    gpu, _ = run_pair(fwd=ENGINES[engine], **kw)
     gpu.close()
 
 
@@ -202,13 +230,13 @@ def test_zero_patterns_is_a_noop():
 
 # -- the workload shapes at full width ------------------------------------------
 
-def _full_width(key, steps=None, n_test=None, sweep=False):
+def _full_width(key, steps=None, n_test=None, sweep=False, fwd=B.BMLP_FWD_AUTO):
     cfg = W.CONFIGS[key]
     n = cfg.n_train if steps is None else steps * 100
     xp = W.make_inputs(cfg, "train", n)
     teacher = W.make_teacher(cfg)
     y = W.teacher_labels_pm1(teacher, W.unpack(xp, cfg.widths[0]))
-    gpu = B.BMLP(cfg.widths, cfg.classes, seed=cfg.model_seed, bs=100)
+    gpu = B.BMLP(cfg.widths, cfg.classes, seed=cfg.model_seed, bs=100, fwd_impl=fwd)
     ref = O.OracleModel(list(cfg.widths), cfg.classes, seed=cfg.model_seed, bs=100)
     eg = gpu.train(dev_x(xp), dev_y(y), epoch_end=steps is None, count_errors=True)
     er = ref.train(W.unpack(xp, cfg.widths[0]), y, epoch_end=steps is None)
@@ -247,3 +275,11 @@ def test_c4_3072_4096x4_100cls_prefix():
 
 def test_c5_8192x5_prefix_and_sweep():
     _full_width("C5", steps=2, n_test=65536, sweep=True)
+
+
+def test_c1_784_256_full_epoch_popc_engine():
+    _full_width("C1", n_test=500, fwd=B.BMLP_FWD_POPC)
+
+
+def test_c5_8192x5_prefix_popc_engine():
+    _full_width("C5", steps=1, n_test=0, fwd=B.BMLP_FWD_POPC)
