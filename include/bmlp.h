@@ -174,6 +174,28 @@ int bmlp_get_profile(const bmlp_t* h, int32_t kind, int64_t* launches, double* t
 int bmlp_reset_profile(bmlp_t* h);
 int64_t bmlp_launch_count(const bmlp_t* h);
 
+/* Forward-only evaluation that allocates no memory.  The paper has no
+ * counterpart: this is bmlp_predict with its scratch moved into the library,
+ * for callers that cannot call cudaMalloc -- code running in a host callback,
+ * a real-time loop with a fixed memory plan, or a process whose device
+ * allocator belongs to another runtime.  bmlp_predict allocates its
+ * inter-layer activation buffers on first use; this call instead uses one
+ * fixed 16 MiB device array inside the library (two buffers of 2^20 64-bit
+ * words), which every GPU that loads the library holds until the process
+ * exits.  Results equal bmlp_predict's.
+ *   n * ceil(max_l K_l / 64) must not exceed 1,048,576 (n <= 8192 for
+ *   8192-wide layers); a larger n returns BMLP_EINVAL before any work.
+ *   x_packed and labels_out must be device pointers (staging host buffers
+ *   would allocate); host pointers return BMLP_EINVAL.
+ *   The first call on a device looks up the array's device address once
+ *   (cudaGetSymbolAddress); make that first call before any stream capture.
+ *   Every call shares the array and it keeps the last call's contents (each
+ *   call writes every word it reads); calls whose GPU work overlaps -- on
+ *   different streams, or from different handles -- race on it.
+ *   Calls no cudaMalloc, cudaFree or allocating library routine. */
+int bmlp_predict_noalloc(bmlp_t* h, const uint64_t* x_packed, int64_t n, int32_t* labels_out,
+                         void* cuda_stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -70,6 +70,7 @@ SIGNATURES = [
     ("bmlp_get_profile", C.c_int, [_vp, C.c_int32, _i64p, _f64p]),
     ("bmlp_reset_profile", C.c_int, [_vp]),
     ("bmlp_launch_count", C.c_int64, [_vp]),
+    ("bmlp_predict_noalloc", C.c_int, [_vp, _vp, C.c_int64, _vp, _vp]),
 ]
 
 
@@ -165,6 +166,13 @@ def bmlp_train(h, x_packed, labels, n=None, flags=0, stream=None, count_errors=F
 def bmlp_predict(h, x_packed, labels_out, n=None, stream=None):
     n = labels_out.shape[0] if n is None else n
     _check(lib().bmlp_predict(h, _ptr(x_packed), n, _ptr(labels_out), _stream(stream)), h)
+
+
+def bmlp_predict_noalloc(h, x_packed, labels_out, n=None, stream=None):
+    """Allocation-free bmlp_predict for callers that cannot allocate device
+    memory (device buffers only; n * ceil(max K_l / 64) <= 2^20)."""
+    n = labels_out.shape[0] if n is None else n
+    _check(lib().bmlp_predict_noalloc(h, _ptr(x_packed), n, _ptr(labels_out), _stream(stream)), h)
 
 
 def bmlp_get_info(h):

@@ -646,3 +646,17 @@ int64_t bmlp_launch_count(const bmlp_t* h) { return h ? h->launches : -1; }
 
 }  // extern "C"
 
+// ---------------------------------------------------------------------------
+// Internal accessors for bmlp_noalloc.cu (not part of the C-ABI).
+int bmlp_internal_eval_view(const bmlp_t* h, const bk::StepParams** params, int* nwmax) {
+  if (!h) return BMLP_EINVAL;
+  *params = &h->hp;
+  int m = 0;
+  for (int l = 1; l <= h->L; ++l) m = std::max(m, (h->K[l] + 63) / 64);
+  *nwmax = m;
+  return BMLP_OK;
+}
+
+int bmlp_internal_fail(bmlp_t* h, int code, const char* msg) { return fail(h, code, "%s", msg); }
+
+void bmlp_internal_count_launches(bmlp_t* h, int64_t n) { h->launches += n; }
