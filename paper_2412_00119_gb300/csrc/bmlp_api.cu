@@ -171,7 +171,7 @@ int enqueue_step(bmlp_t* h, cudaStream_t st) {
   k_cls_select<<<dim3((unsigned)h->bs, (unsigned)h->L), kClsThreads, 0, st>>>(h->dP);
   prof_end(h, st);
   prof_begin(h, kProfUpd, st);
-  k_update<<<h->updCtas, kUpdThreads, h->updSmem, st>>>(h->dP);
+  k_update<<<h->updCtas, kUpdThreads, h->updSmem, st>>>(h->dP, h->hp.key0, h->hp.key1);
   prof_end(h, st);
   CK(h, cudaGetLastError());
   return BMLP_OK;

@@ -61,7 +61,6 @@ struct StepParams {
 
 // Rows of one group handled by one update CTA.
 constexpr int kUpdRowsPerCta = 16;
-constexpr int kUpdUnroll = 4;  // 16-byte H loads in flight per lane in k_update
 constexpr int kUpdThreads = 256;
 constexpr int kClsThreads = 256;
 
@@ -77,13 +76,10 @@ constexpr int kClsThreads = 256;
 __device__ __forceinline__ uint4 philox4x32_10(uint4 ctr, uint32_t k0, uint32_t k1) {
 #pragma unroll
   for (int r = 0; r < 10; ++r) {
-    const uint32_t lo0 = 0xD2511F53u * ctr.x;
-    const uint32_t hi0 = __umulhi(0xD2511F53u, ctr.x);
-    const uint32_t lo1 = 0xCD9E8D57u * ctr.z;
-    const uint32_t hi1 = __umulhi(0xCD9E8D57u, ctr.z);
-    ctr = make_uint4(hi1 ^ ctr.y ^ k0, lo1, hi0 ^ ctr.w ^ k1, lo0);
-    k0 += 0x9E3779B9u;
-    k1 += 0xBB67AE85u;
+    const uint64_t p0 = (uint64_t)0xD2511F53u * ctr.x;  // one wide multiply each
+    const uint64_t p1 = (uint64_t)0xCD9E8D57u * ctr.z;
+    ctr = make_uint4((uint32_t)(p1 >> 32) ^ ctr.y ^ (k0 + (uint32_t)r * 0x9E3779B9u), (uint32_t)p1,
+                     (uint32_t)(p0 >> 32) ^ ctr.w ^ (k1 + (uint32_t)r * 0xBB67AE85u), (uint32_t)p0);
   }
   return ctr;
 }
@@ -105,7 +101,9 @@ __global__ void k_train_forward(const StepParams* P, int l);
 // Local classifier, 01-loss, margin, marks, and the group selection, all layers.
 __global__ void k_cls_select(const StepParams* P);
 // CP + R + repack of every layer with a non-empty M_l, then advance the step.
-__global__ void k_update(const StepParams* P);
+// (key0, key1) = the Philox key, passed by value so that the round keys are
+// kernel-uniform.
+__global__ void k_update(const StepParams* P, uint32_t key0, uint32_t key1);
 // Generic forward for evaluation: A (M x nw_in) against W -> Aout (M x nw_out).
 __global__ void k_forward_eval(const uint64_t* __restrict__ A, int64_t M, int nw_in,
                                const uint64_t* __restrict__ W, int N, int Kin,

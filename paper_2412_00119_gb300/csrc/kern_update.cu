@@ -115,127 +115,144 @@ __global__ void __launch_bounds__(kClsThreads) k_cls_select(const StepParams* __
 // CTA = (layer, group g, slice of kUpdRowsPerCta neurons).  A warp owns one
 // neuron row k at a time: it collects, in ascending mu, the patterns whose
 // selection in group g is k (the CP tuples of k), then streams the row in
-// chunks of 8 hidden weights (one 16-byte vector per lane, kUpdUnroll vectors
-// in flight per lane):
-//   CP: h_i <- clip(h_i + 2 a^mu_i rho_{k,y^mu}) per tuple, in mu order.  The
-//       8 weights stay packed as int16 pairs; a shared table turns the
-//       activation byte into four packed +-2 delta words and the DPX
-//       add-min / max3 instructions clip two weights per instruction.
-//   R : U = Philox draw (hi16 lane from purpose 3, lo16 from purpose 4);
-//       U < T  ->  h_i <- clip(h_i + 2 sign h_i).  The 16-bit lanes of the
-//       Philox output line up with the int16 pairs; a SIMD-within-a-register
-//       test against T's high half finds the chunks with an event or a tie
-//       (about 4% of chunks at the paper's p_r), and only those take the
-//       per-weight path; the low half is drawn only on a tie.
-//   W : bit i = (h_i > 0) = NOT sign bit; one byte per chunk, in place.
-// Chunks that hold only padding (i >= K_{l-1}) are never touched; a chunk that
-// is partly padding takes the per-weight path with the padding masked.
-// Layers with an empty M_l are skipped (no CP, no R).  The last CTA to finish
+// chunks of 8 hidden weights, one 16-byte vector per lane, with a rotating
+// queue of four vectors in flight per lane.
+// In registers a chunk is 4 words of two offset-binary 16-bit lanes
+// (u = h + 2^15 = h XOR 0x8000).  |h| <= h_max + 2 < 2^14 keeps every lane
+// inside (0, 2^16), so a packed pair of +-2 steps is one 32-bit add without
+// carries between lanes; bit 15 of a lane is (h > 0); a lane equal to a given
+// value is found exactly with a carry-free test.  All of the rule then runs on
+// packed lanes, with warp-uniform branches only:
+//   CP: per tuple (ascending mu) add the packed deltas 2 a^mu_i rho_{k,y^mu}
+//       from a shared byte -> delta table; when some lane may cross a bound
+//       (|h| > h_max - 2 n_k somewhere in the warp), lanes that reached
+//       +-(h_max + 2) are moved back by 2 after each tuple (the clip).
+//   R : the Philox draw's 16-bit lanes line up with the weight lanes; lanes
+//       whose high half is below T's high half (< 2^15) fire; a fired lane
+//       moves 2 away from 0 unless it sits at +-h_max.
+//   W : one byte per chunk from the lanes' bit 15, written in place.
+// A chunk with a tie (draw high half == T high half, probability 8 / 2^16),
+// the partly padded last chunk of a row, and every chunk when T >= 2^31 take
+// the per-weight path instead.  Chunks of padding only are never touched.
+// Layers with an empty M_l are skipped (no CP, no R).  The last warp to finish
 // advances the step counters and clears the per-step flags.
 // ---------------------------------------------------------------------------
 namespace {
 
-struct UpdCtx {
-  const uint8_t* aprev;  // previous layer's packed activations, bytes
-  size_t arow_bytes;
-  const int32_t* list;   // CP tuples of the row: mu | (rho < 0) << 16
-  int n_t;
-  int h_max;
-  uint32_t Thi, Tlo, Tpair;
-  bool fast_r;           // Thi < 2^15: the SIMD test is exact
-  uint32_t key0, key1;
-  uint32_t k, c2_hi, c2_lo, t;
-  const uint4* delta;    // [2][256] packed +-2 deltas per activation byte and rho sign
+constexpr uint32_t kLaneTop = 0x80008000u;
+constexpr unsigned kFull = 0xffffffffu;
+
+__device__ __forceinline__ int lane_h(const uint4& w, int j) {
+  const uint32_t word = (j < 2) ? w.x : (j < 4) ? w.y : (j < 6) ? w.z : w.w;
+  return (int)(int16_t)(uint16_t)(word >> (16 * (j & 1)));
+}
+
+__device__ __forceinline__ void set_lane_h(uint4& w, int j, int h) {
+  const int sh = 16 * (j & 1);
+  const uint32_t m = ~(0xFFFFu << sh), v = ((uint32_t)h & 0xFFFFu) << sh;
+  if (j < 2) w.x = (w.x & m) | v;
+  else if (j < 4) w.y = (w.y & m) | v;
+  else if (j < 6) w.z = (w.z & m) | v;
+  else w.w = (w.w & m) | v;
+}
+
+struct ChunkOut {
+  uint4 w;
+  uint32_t wbyte;
 };
 
-__device__ __forceinline__ int lane_h(const uint32_t (&w)[4], int j) {
-  return (int)(int16_t)(uint16_t)(w[j >> 1] >> (16 * (j & 1)));
-}
-
-__device__ __forceinline__ void set_lane_h(uint32_t (&w)[4], int j, int h) {
-  const int sh = 16 * (j & 1);
-  w[j >> 1] = (w[j >> 1] & ~(0xFFFFu << sh)) | (((uint32_t)h & 0xFFFFu) << sh);
-}
-
-// Per-weight path: CP (already applied by the caller when `cp_done`), R and W
-// for the first `nvalid` weights of the chunk.
-__device__ __noinline__ uint32_t chunk_scalar(uint32_t (&w)[4], int ch, int nvalid, bool cp_done,
-                                              const UpdCtx& C, uint4 rh) {
+// Per-weight path on two's-complement lanes: CP (unless `cp_done`), R and W for
+// the first `nvalid` weights of the chunk.  Loops stay rolled: rarely taken.
+__device__ __forceinline__ ChunkOut chunk_scalar(uint4 w, int ch, int nvalid, bool cp_done,
+                                                 const int32_t* list, int n_t, const uint8_t* aprev,
+                                                 uint32_t arow_bytes, int h_max, uint32_t Thi,
+                                                 uint32_t Tlo, uint32_t key0, uint32_t key1,
+                                                 uint32_t k, uint32_t c2_lo, uint32_t t, uint4 rh) {
   if (!cp_done) {
-    for (int q = 0; q < C.n_t; ++q) {
-      const int e = C.list[q];
+#pragma unroll 1
+    for (int q = 0; q < n_t; ++q) {
+      const int e = list[q];
       const int m = e & 0xFFFF;
       const int rho = (e & 0x10000) ? -1 : 1;
-      const uint32_t byte = C.aprev[(size_t)m * C.arow_bytes + ch];
+      const uint32_t byte = aprev[(size_t)m * arow_bytes + ch];
+#pragma unroll 1
       for (int j = 0; j < nvalid; ++j) {
         const int step = ((byte >> j) & 1u) ? rho : -rho;
-        set_lane_h(w, j, clip_h(lane_h(w, j) + 2 * step, C.h_max));
+        set_lane_h(w, j, clip_h(lane_h(w, j) + 2 * step, h_max));
       }
     }
   }
   uint32_t ties = 0;
-  for (int j = 0; j < 8; ++j) ties |= (lane16(rh, j) == C.Thi ? 1u : 0u) << j;
+  for (int j = 0; j < 8; ++j) ties |= (lane16(rh, j) == Thi ? 1u : 0u) << j;
   uint4 rl = make_uint4(0, 0, 0, 0);
-  if (ties)
-    rl = philox4x32_10(make_uint4((uint32_t)ch, C.k, C.c2_lo, C.t), C.key0, C.key1);
-  uint32_t wbyte = 0;
+  if (ties) rl = philox4x32_10(make_uint4((uint32_t)ch, k, c2_lo, t), key0, key1);
+  ChunkOut out;
+  out.wbyte = 0;
+#pragma unroll 1
   for (int j = 0; j < nvalid; ++j) {
     const uint32_t u = lane16(rh, j);
-    const bool fire = (u < C.Thi) || (((ties >> j) & 1u) && lane16(rl, j) < C.Tlo);
+    const bool fire = (u < Thi) || (((ties >> j) & 1u) && lane16(rl, j) < Tlo);
     int h = lane_h(w, j);
     if (fire) {
-      h = clip_h(h + (h > 0 ? 2 : -2), C.h_max);
+      h = clip_h(h + (h > 0 ? 2 : -2), h_max);
       set_lane_h(w, j, h);
     }
-    wbyte |= (h > 0 ? 1u : 0u) << j;
+    out.wbyte |= (h > 0 ? 1u : 0u) << j;
   }
-  return wbyte;
+  out.w = w;
+  return out;
 }
 
-// Sign bits of the 8 packed weights -> W byte (bit j = h_j > 0, h never 0).
-__device__ __forceinline__ uint32_t w_byte(const uint32_t (&w)[4]) {
-  const uint32_t p0 = __byte_perm(w[0], w[1], 0x7531) & 0x80808080u;
-  const uint32_t p1 = __byte_perm(w[2], w[3], 0x7531) & 0x80808080u;
-  const uint32_t neg = ((p0 * 0x00204081u) >> 28) | (((p1 * 0x00204081u) >> 28) << 4);
-  return ~neg & 0xFFu;
+// bit 15 of every lane of w equal to the lane value of cpair (exact, carry-free)
+__device__ __forceinline__ uint32_t eq_flags(uint32_t w, uint32_t cpair) {
+  const uint32_t x = w ^ cpair;
+  return ~(((x & 0x7FFF7FFFu) + 0x7FFF7FFFu) | x) & kLaneTop;
 }
 
-__device__ __forceinline__ uint32_t chunk_packed(uint32_t (&w)[4], int ch, const UpdCtx& C,
-                                                 uint32_t neg_pair, uint32_t pos_pair) {
-  // Clipped Perceptron, two weights per DPX instruction
-  for (int q = 0; q < C.n_t; ++q) {
-    const int e = C.list[q];
-    const int m = e & 0xFFFF;
-    const uint32_t byte = C.aprev[(size_t)m * C.arow_bytes + ch];
-    const uint4 d = C.delta[((e >> 16) & 1) * 256 + byte];
-    w[0] = __vimax3_s16x2(__viaddmin_s16x2(w[0], d.x, pos_pair), neg_pair, neg_pair);
-    w[1] = __vimax3_s16x2(__viaddmin_s16x2(w[1], d.y, pos_pair), neg_pair, neg_pair);
-    w[2] = __vimax3_s16x2(__viaddmin_s16x2(w[2], d.z, pos_pair), neg_pair, neg_pair);
-    w[3] = __vimax3_s16x2(__viaddmin_s16x2(w[3], d.w, pos_pair), neg_pair, neg_pair);
-  }
-  // Reinforcement draws for the 8 weights
-  const uint4 rh = philox4x32_10(make_uint4((uint32_t)ch, C.k, C.c2_hi, C.t), C.key0, C.key1);
-  uint32_t any = 1;
-  if (C.fast_r) {
-    // lane fires iff its 16-bit draw u < Thi (< 2^15): top bit clear and low 15
-    // bits below Thi; lane ties iff u == Thi (zero lane of u ^ Tpair)
-    const uint32_t H = 0x80008000u;
-    const uint32_t u[4] = {rh.x, rh.y, rh.z, rh.w};
-    any = 0;
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const uint32_t d = ((u[i] & 0x7FFF7FFFu) | H) - C.Tpair;
-      const uint32_t x = u[i] ^ C.Tpair;
-      any |= (~(d | u[i]) & H) | ((x - 0x00010001u) & ~x & H);
-    }
-  }
-  if (any) return chunk_scalar(w, ch, 8, true, C, rh);
-  return w_byte(w);
+// Bit 15 of each offset-binary lane (= h > 0) -> W byte.
+__device__ __forceinline__ uint32_t w_byte_ob(const uint4& w) {
+  const uint32_t p0 = __byte_perm(w.x, w.y, 0x7531) & 0x80808080u;
+  const uint32_t p1 = __byte_perm(w.z, w.w, 0x7531) & 0x80808080u;
+  return ((p0 * 0x00204081u) >> 28) | (((p1 * 0x00204081u) >> 28) << 4);
+}
+
+// lanes of a draw word whose high half u < Thi (< 2^15): top bit clear, low 15
+// bits below Thi (guard-bit subtraction, no borrow between lanes)
+__device__ __forceinline__ uint32_t fire_flags(uint32_t u, uint32_t Tpair) {
+  const uint32_t dd = ((u & 0x7FFF7FFFu) | kLaneTop) - Tpair;
+  return ~(dd | u) & kLaneTop;
+}
+
+// nonzero iff some lane of a draw word equals Thi
+__device__ __forceinline__ uint32_t tie_any(uint32_t u, uint32_t Tpair) {
+  const uint32_t x = u ^ Tpair;
+  return (x - 0x00010001u) & ~x & kLaneTop;
+}
+
+// lanes of an offset-binary word outside [lo, hi] after subtracting `base`
+__device__ __forceinline__ uint32_t range_flags(uint32_t w, uint32_t base_pair, uint32_t lo_pair,
+                                                uint32_t hi_pair) {
+  const uint32_t a = w - base_pair;
+  return ~(((a | kLaneTop) - lo_pair) & ((hi_pair | kLaneTop) - a)) & kLaneTop;
+}
+
+// clip after a +-2 step: lanes at +-(h_max + 2) move back by 2
+__device__ __forceinline__ uint32_t clip_step(uint32_t w, uint32_t over_pair, uint32_t under_pair) {
+  return w + (eq_flags(w, under_pair) >> 14) - (eq_flags(w, over_pair) >> 14);
+}
+
+// reinforcement of the fired lanes: 2 away from 0 unless at +-h_max
+__device__ __forceinline__ uint32_t reinforce(uint32_t w, uint32_t fire, uint32_t top_pair,
+                                              uint32_t bot_pair) {
+  const uint32_t inc = fire & w & ~eq_flags(w, top_pair);
+  const uint32_t dec = fire & ~w & ~eq_flags(w, bot_pair);
+  return w + (inc >> 14) - (dec >> 14);
 }
 
 }  // namespace
 
-__global__ void __launch_bounds__(kUpdThreads, 3) k_update(const StepParams* __restrict__ P) {
+__global__ void __launch_bounds__(kUpdThreads, 3) k_update(const StepParams* __restrict__ P,
+                                                           uint32_t key0, uint32_t key1) {
   extern __shared__ int32_t dyn[];
   __shared__ uint4 s_delta[2 * 256];
   const int bid = blockIdx.x;
@@ -246,6 +263,7 @@ __global__ void __launch_bounds__(kUpdThreads, 3) k_update(const StepParams* __r
   const unsigned long long t = ctrl->t;
   const uint32_t s = ctrl->s;
   const bool active = ctrl->any_mark[li] != 0u;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nwarps = blockDim.x >> 5;
 
   if (active) {
     const int gamma = Ly.gamma;
@@ -256,13 +274,13 @@ __global__ void __launch_bounds__(kUpdThreads, 3) k_update(const StepParams* __r
     const int r1 = min(r0 + kUpdRowsPerCta, gamma);
     const int64_t start = (int64_t)s * P->bs;
     const int bsz = (int)batch_size(P, start);
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nwarps = blockDim.x >> 5;
     int16_t* s_sel = reinterpret_cast<int16_t*>(dyn);               // [bs]
     int32_t* s_list = dyn + (P->bs + 1) / 2 + warp * P->bs;         // [nwarps][bs]
 
     for (int m = threadIdx.x; m < bsz; m += blockDim.x) s_sel[m] = Ly.sel[(int64_t)m * Ly.G + g];
-    // s_delta[r][b]: packed int16 pair p of entry = (+-2 for bit 2p, +-2 for
-    // bit 2p+1 of b), sign flipped for r = 1 (rho = -1)
+    // s_delta[r][b]: word p packs the steps of bits 2p and 2p+1 of b as
+    // d_lo + 2^16 d_hi (d = +-2, negated for r = 1, i.e. rho = -1); added to a
+    // word of two offset-binary lanes it moves each lane by its own step
     for (int i = threadIdx.x; i < 512; i += blockDim.x) {
       const int r = i >> 8, b = i & 255;
       uint32_t v[4];
@@ -271,35 +289,34 @@ __global__ void __launch_bounds__(kUpdThreads, 3) k_update(const StepParams* __r
         int lo = ((b >> (2 * p)) & 1) ? 2 : -2;
         int hi = ((b >> (2 * p + 1)) & 1) ? 2 : -2;
         if (r) { lo = -lo; hi = -hi; }
-        v[p] = ((uint32_t)lo & 0xFFFFu) | ((uint32_t)hi << 16);
+        v[p] = (uint32_t)(lo + 65536 * hi);
       }
       s_delta[i] = make_uint4(v[0], v[1], v[2], v[3]);
     }
     __syncthreads();
 
-    const int l = li + 1;
+    const uint32_t l = (uint32_t)li + 1u;
     const int c = P->c;
-    UpdCtx C;
-    C.h_max = P->h_max;
+    const int h_max = P->h_max;
     const unsigned long long T = P->T[li];
-    C.Thi = (uint32_t)(T >> 16);   // 0..65536
-    C.Tlo = (uint32_t)(T & 0xFFFFu);
-    C.fast_r = C.Thi < 0x8000u;
-    C.Tpair = C.Thi * 0x00010001u;
-    C.key0 = P->key0;
-    C.key1 = P->key1;
-    C.c2_hi = (3u << 16) + (uint32_t)l;
-    C.c2_lo = (4u << 16) + (uint32_t)l;
-    C.t = (uint32_t)t;
-    C.delta = s_delta;
+    const uint32_t Thi = (uint32_t)(T >> 16);   // 0..65536
+    const uint32_t Tlo = (uint32_t)(T & 0xFFFFu);
+    const uint32_t Tpair = Thi * 0x00010001u;
+    const uint32_t c2_hi = (3u << 16) + l, c2_lo = (4u << 16) + l;
+    const uint32_t tt = (uint32_t)t;
     const int Kin = Ly.Kin;
     const int nch = (Kin + 7) >> 3;             // chunks holding at least one input
     const int full = Kin >> 3;                  // chunks of 8 real inputs
-    C.arow_bytes = (size_t)Ly.nw_in * 8;
-    C.aprev = (li == 0) ? reinterpret_cast<const uint8_t*>(P->x + start * P->nw0)
-                        : reinterpret_cast<const uint8_t*>(P->layer[li - 1].A);
-    const uint32_t neg_pair = (uint32_t)(-C.h_max & 0xFFFF) * 0x00010001u;
-    const uint32_t pos_pair = (uint32_t)C.h_max * 0x00010001u;
+    const uint32_t arow_bytes = (uint32_t)Ly.nw_in * 8u;
+    const uint8_t* aprev = (li == 0) ? reinterpret_cast<const uint8_t*>(P->x + start * P->nw0)
+                                     : reinterpret_cast<const uint8_t*>(P->layer[li - 1].A);
+    // packed lanes on the rule's boundary values (offset binary)
+    const bool packed = h_max < 0x3FFF && Thi < 0x8000u;
+    const uint32_t top_pair = (uint32_t)(0x8000 + h_max) * 0x00010001u;
+    const uint32_t bot_pair = (uint32_t)(0x8000 - h_max) * 0x00010001u;
+    const uint32_t over_pair = (uint32_t)(0x8000 + h_max + 2) * 0x00010001u;
+    const uint32_t under_pair = (uint32_t)(0x8000 - h_max - 2) * 0x00010001u;
+    const int iters = (nch + 31) >> 5;
 
     for (int rr = r0 + warp; rr < r1; rr += nwarps) {
       const int k = g * gamma + rr;
@@ -308,7 +325,7 @@ __global__ void __launch_bounds__(kUpdThreads, 3) k_update(const StepParams* __r
       for (int base = 0; base < bsz; base += 32) {
         const int m = base + lane;
         const bool hit = (m < bsz) && (s_sel[m] == k);
-        const unsigned bal = __ballot_sync(0xffffffffu, hit);
+        const unsigned bal = __ballot_sync(kFull, hit);
         if (hit) {
           int yv = P->y[start + m];
           if (yv < 0 || yv >= c) yv = 0;
@@ -318,34 +335,82 @@ __global__ void __launch_bounds__(kUpdThreads, 3) k_update(const StepParams* __r
         n_t += __popc(bal);
       }
       __syncwarp();
-      C.list = s_list;
-      C.n_t = n_t;
-      C.k = (uint32_t)k;
+      // no clip can trigger in a chunk whose lanes all keep |h| <= h_max - 2 n_t
+      const bool range_test = 2 * n_t <= h_max;
+      const uint32_t lo_pair = (uint32_t)(2 * n_t) * 0x00010001u;
+      const uint32_t hi_pair = (uint32_t)(range_test ? 2 * h_max - 2 * n_t : 0) * 0x00010001u;
 
       int16_t* hrow = Ly.H + (int64_t)k * Ly.ldh;
       uint8_t* wrow = reinterpret_cast<uint8_t*>(Ly.W + (int64_t)k * Ly.nw_in);
-      // kUpdUnroll 16-byte loads in flight per lane before any is processed;
-      // H is streamed (read once, written once per step)
-      for (int base = lane; base < nch; base += 32 * kUpdUnroll) {
-        uint4 hbuf[kUpdUnroll];
-#pragma unroll
-        for (int u = 0; u < kUpdUnroll; ++u) {
-          const int ch = base + 32 * u;
-          if (ch < nch) hbuf[u] = __ldcs(reinterpret_cast<const uint4*>(hrow + 8 * ch));
-        }
-#pragma unroll
-        for (int u = 0; u < kUpdUnroll; ++u) {
-          const int ch = base + 32 * u;
-          if (ch >= nch) break;
-          uint32_t w[4] = {hbuf[u].x, hbuf[u].y, hbuf[u].z, hbuf[u].w};
-          uint32_t wbyte;
-          if (ch < full) {
-            wbyte = chunk_packed(w, ch, C, neg_pair, pos_pair);
-          } else {
-            const uint4 rh = philox4x32_10(make_uint4((uint32_t)ch, C.k, C.c2_hi, C.t), C.key0, C.key1);
-            wbyte = chunk_scalar(w, ch, Kin - 8 * ch, false, C, rh);
+      // rotating queue of H vectors (chunks ch, ch + 32, ch + 64, ch + 96);
+      // every lane runs the same number of iterations (warp votes below)
+      uint4 q0 = make_uint4(0, 0, 0, 0), q1 = q0, q2 = q0, q3 = q0;
+      if (lane < nch) q0 = __ldcs(reinterpret_cast<const uint4*>(hrow + 8 * lane));
+      if (lane + 32 < nch) q1 = __ldcs(reinterpret_cast<const uint4*>(hrow + 8 * (lane + 32)));
+      if (lane + 64 < nch) q2 = __ldcs(reinterpret_cast<const uint4*>(hrow + 8 * (lane + 64)));
+      if (lane + 96 < nch) q3 = __ldcs(reinterpret_cast<const uint4*>(hrow + 8 * (lane + 96)));
+#pragma unroll 1
+      for (int it = 0; it < iters; ++it) {
+        const int ch = 32 * it + lane;
+        const bool live = ch < nch;
+        const uint4 w_in = q0;   // two's complement, as loaded
+        uint4 w = q0;
+        q0 = q1;
+        q1 = q2;
+        q2 = q3;
+        if (ch + 128 < nch) q3 = __ldcs(reinterpret_cast<const uint4*>(hrow + 8 * (ch + 128)));
+        const uint4 rh = philox4x32_10(make_uint4((uint32_t)ch, (uint32_t)k, c2_hi, tt), key0, key1);
+        const bool simd = packed && ch < full;   // this lane's chunk runs on packed lanes
+        w.x ^= kLaneTop; w.y ^= kLaneTop; w.z ^= kLaneTop; w.w ^= kLaneTop;  // offset binary
+        // ---- Clipped Perceptron ----
+        if (n_t > 0) {
+          bool safe = true;
+          if (range_test && simd)
+            safe = (range_flags(w.x, bot_pair, lo_pair, hi_pair) | range_flags(w.y, bot_pair, lo_pair, hi_pair) |
+                    range_flags(w.z, bot_pair, lo_pair, hi_pair) | range_flags(w.w, bot_pair, lo_pair, hi_pair)) == 0u;
+          else if (!range_test)
+            safe = false;
+          const bool clip = !__all_sync(kFull, safe || !live);
+#pragma unroll 1
+          for (int q = 0; q < n_t; ++q) {
+            const int e = s_list[q];
+            const uint32_t byte = live ? aprev[(size_t)(e & 0xFFFF) * arow_bytes + ch] : 0u;
+            const uint4 d = s_delta[((e >> 16) & 1) * 256 + byte];
+            w.x += d.x; w.y += d.y; w.z += d.z; w.w += d.w;
+            if (clip) {
+              w.x = clip_step(w.x, over_pair, under_pair);
+              w.y = clip_step(w.y, over_pair, under_pair);
+              w.z = clip_step(w.z, over_pair, under_pair);
+              w.w = clip_step(w.w, over_pair, under_pair);
+            }
           }
-          __stcs(reinterpret_cast<uint4*>(hrow + 8 * ch), make_uint4(w[0], w[1], w[2], w[3]));
+        }
+        // ---- Reinforcement ----
+        const uint32_t tie = simd ? (tie_any(rh.x, Tpair) | tie_any(rh.y, Tpair) |
+                                     tie_any(rh.z, Tpair) | tie_any(rh.w, Tpair)) : 1u;
+        const bool slow = live && (tie != 0u);
+        const uint4 f = make_uint4(fire_flags(rh.x, Tpair), fire_flags(rh.y, Tpair),
+                                   fire_flags(rh.z, Tpair), fire_flags(rh.w, Tpair));
+        const bool fires = live && !slow && ((f.x | f.y | f.z | f.w) != 0u);
+        if (__any_sync(kFull, fires) && fires) {
+          w.x = reinforce(w.x, f.x, top_pair, bot_pair);
+          w.y = reinforce(w.y, f.y, top_pair, bot_pair);
+          w.z = reinforce(w.z, f.z, top_pair, bot_pair);
+          w.w = reinforce(w.w, f.w, top_pair, bot_pair);
+        }
+        uint32_t wbyte = w_byte_ob(w);
+        w.x ^= kLaneTop; w.y ^= kLaneTop; w.z ^= kLaneTop; w.w ^= kLaneTop;  // back to int16
+        if (slow) {
+          // a packed chunk with a tie keeps its packed CP result; any other chunk
+          // restarts from the loaded values and the per-weight path does it all
+          const ChunkOut o = chunk_scalar(simd ? w : w_in, ch, min(8, Kin - 8 * ch), simd, s_list, n_t, aprev,
+                                          arow_bytes, h_max, Thi, Tlo, key0, key1, (uint32_t)k,
+                                          c2_lo, tt, rh);
+          w = o.w;
+          wbyte = o.wbyte;
+        }
+        if (live) {
+          __stcs(reinterpret_cast<uint4*>(hrow + 8 * ch), w);
           wrow[ch] = (uint8_t)wbyte;
         }
       }
@@ -353,12 +418,12 @@ __global__ void __launch_bounds__(kUpdThreads, 3) k_update(const StepParams* __r
     }
   }
 
-  // step completion: the last CTA advances the counters
-  __syncthreads();
-  if (threadIdx.x == 0) {
+  // step completion: the last warp to finish advances the counters
+  __syncwarp();
+  if (lane == 0) {
     __threadfence();
     const unsigned prev = atomicAdd(&ctrl->done, 1u);
-    if (prev == gridDim.x - 1) {
+    if (prev == gridDim.x * nwarps - 1) {
       ctrl->t = t + 1;
       ctrl->s = s + 1;
       for (int i = 0; i < P->L; ++i) ctrl->any_mark[i] = 0u;

@@ -123,6 +123,8 @@ CASES = {
     "bs_max": dict(widths=(64, 128), classes=4, n_train=2048, bs=1024),
     "multi_tile_k": dict(widths=(1100, 320, 200), classes=10, n_train=300, bs=100),
     "field_inputs": dict(widths=(3072, 128), classes=10, n_train=200, gen="field", teacher_hidden=32),
+    "h_max_5_clipping": dict(widths=(96, 64, 64), classes=4, n_train=500, h_max=5, p_r0=1.0),
+    "q_above_half": dict(widths=(40, 8), classes=3, n_train=120, bs=20, p_r0=2.0, gamma=[4]),
 }
 
 
