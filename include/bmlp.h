@@ -98,7 +98,7 @@ typedef struct bmlp_hparams {
 
 /* Create a model and initialise H_l, P_l uniformly on {+-1} from `seed`
  * (Alg. 1 l.2).  widths: K_0..K_L (n_widths = L + 1, 2..BMLP_MAX_LAYERS + 1,
- * each 1..32767); classes: 2..BMLP_MAX_CLASSES; h_max: odd, 1..32767 (255 = 8-bit
+ * each 1..32767); classes: 2..BMLP_MAX_CLASSES; h_max: odd, 1..16383 (255 = 8-bit
  * hidden weights, Table 4); hp may be NULL (paper defaults).  Allocates the
  * model state on the current CUDA device.  On success *out owns it. */
 int bmlp_create(const int32_t* widths, int32_t n_widths, int32_t classes, int16_t h_max,

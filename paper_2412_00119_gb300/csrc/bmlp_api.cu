@@ -171,7 +171,8 @@ int enqueue_step(bmlp_t* h, cudaStream_t st) {
   k_cls_select<<<dim3((unsigned)h->bs, (unsigned)h->L), kClsThreads, 0, st>>>(h->dP);
   prof_end(h, st);
   prof_begin(h, kProfUpd, st);
-  k_update<<<h->updCtas, kUpdThreads, h->updSmem, st>>>(h->dP, h->hp.key0, h->hp.key1);
+  launch_update(((h->h_max + 1) & h->h_max) == 0, (unsigned)h->updCtas, h->updSmem, st, h->dP,
+                h->hp.key0, h->hp.key1);
   prof_end(h, st);
   CK(h, cudaGetLastError());
   return BMLP_OK;
@@ -297,7 +298,8 @@ int bmlp_create(const int32_t* widths, int32_t n_widths, int32_t classes, int16_
       return fail(nullptr, BMLP_EINVAL, "width %d out of range (1..32767)", i);
   if (classes < 2 || classes > BMLP_MAX_CLASSES)
     return fail(nullptr, BMLP_EINVAL, "classes must be in 2..%d", BMLP_MAX_CLASSES);
-  if (h_max < 1 || (h_max % 2) == 0) return fail(nullptr, BMLP_EINVAL, "h_max must be odd and >= 1");
+  if (h_max < 1 || h_max > 16383 || (h_max % 2) == 0)
+    return fail(nullptr, BMLP_EINVAL, "h_max must be odd and in 1..16383");
   bmlp_hparams hp{};
   if (hpin) hp = *hpin;
   const int bs = hp.bs == 0 ? 100 : hp.bs;
@@ -332,7 +334,7 @@ int bmlp_create(const int32_t* widths, int32_t n_widths, int32_t classes, int16_
   cudaDeviceProp prop;
   cudaFuncAttributes fa;
   if (cudaGetDeviceProperties(&prop, h->device) != cudaSuccess || prop.major != 10 ||
-      cudaFuncGetAttributes(&fa, k_update) != cudaSuccess) {
+      update_kernel_attributes(&fa) != cudaSuccess) {
     (void)cudaGetLastError();
     delete h;
     return fail(nullptr, BMLP_ENODEV, "device has no sm_103a kernel image (needs a GB300)");
@@ -348,6 +350,8 @@ int bmlp_create(const int32_t* widths, int32_t n_widths, int32_t classes, int16_
   std::memset(&P, 0, sizeof(P));
   P.L = L; P.c = classes; P.bs = bs; P.h_max = h_max; P.r_num = r_num; P.r_den = r_den;
   P.nw0 = words_of(widths[0]);
+  P.hb = 1;
+  while ((1 << P.hb) < h_max + 1) ++P.hb;
   P.key0 = (uint32_t)(seed & 0xffffffffu);
   P.key1 = (uint32_t)(seed >> 32);
   int cta = 0;
@@ -386,7 +390,7 @@ int bmlp_create(const int32_t* widths, int32_t n_widths, int32_t classes, int16_
     DevLayer& D = P.layer[l - 1];
     const int64_t n1 = (int64_t)D.Kout * (D.ldh >> 3);
     k_init_hw<<<(unsigned)((n1 + 255) / 256), 256>>>(D.H, D.W, D.Kin, D.Kout, D.ldh, D.nw_in, l,
-                                                       P.key0, P.key1);
+                                                       P.key0, P.key1, h_max, P.hb);
     const int64_t n2 = (int64_t)D.Kout * classes;
     k_init_rho<<<(unsigned)((n2 + 255) / 256), 256>>>(D.rho, D.Kout, classes, l, P.key0, P.key1);
     const int64_t n3 = (int64_t)classes * D.nw_out;
@@ -544,9 +548,14 @@ int bmlp_get_state(const bmlp_t* hc, int32_t layer, int16_t* H_out, uint64_t* W_
   if (layer < 1 || layer > h->L) return fail(h, BMLP_EINVAL, "layer must be in 1..%d", h->L);
   CK(h, cudaDeviceSynchronize());
   const DevLayer& D = h->hp.layer[layer - 1];
-  if (H_out)
+  if (H_out) {
     CK(h, cudaMemcpy2D(H_out, sizeof(int16_t) * D.Kin, D.H, sizeof(int16_t) * D.ldh,
                        sizeof(int16_t) * D.Kin, D.Kout, cudaMemcpyDeviceToHost));
+    // lattice index -> h
+    const int base = 1 << h->hp.hb;
+    const int64_t cnt = (int64_t)D.Kout * D.Kin;
+    for (int64_t i = 0; i < cnt; ++i) H_out[i] = (int16_t)(2 * ((int)H_out[i] - base) - h->h_max);
+  }
   if (W_out) CK(h, cudaMemcpy(W_out, D.W, sizeof(uint64_t) * D.Kout * D.nw_in, cudaMemcpyDeviceToHost));
   if (P_out) CK(h, cudaMemcpy(P_out, D.rho, (size_t)D.Kout * h->c, cudaMemcpyDeviceToHost));
   if (p_r_out) *p_r_out = h->p_r;
@@ -574,10 +583,16 @@ int bmlp_set_state(bmlp_t* h, int32_t layer, const int16_t* H_in, double p_r, in
   if (step >= 0 && (!(p_r >= 0.0) || !std::isfinite(p_r))) return fail(h, BMLP_ESTATE, "p_r invalid");
   CK(h, cudaDeviceSynchronize());
   if (H_in) {
-    CK(h, cudaMemcpy2D(D.H, sizeof(int16_t) * D.ldh, H_in, sizeof(int16_t) * D.Kin,
+    // h -> lattice index
+    const int base = 1 << h->hp.hb;
+    const int64_t cnt = (int64_t)D.Kout * D.Kin;
+    std::vector<int16_t> v((size_t)cnt);
+    for (int64_t i = 0; i < cnt; ++i) v[(size_t)i] = (int16_t)((H_in[i] + h->h_max) / 2 + base);
+    CK(h, cudaMemcpy2D(D.H, sizeof(int16_t) * D.ldh, v.data(), sizeof(int16_t) * D.Kin,
                        sizeof(int16_t) * D.Kin, D.Kout, cudaMemcpyHostToDevice));
     const int64_t nwt = (int64_t)D.Kout * D.nw_in;
-    k_repack_w<<<(unsigned)((nwt + 255) / 256), 256>>>(D.H, D.W, D.Kin, D.Kout, D.ldh, D.nw_in);
+    k_repack_w<<<(unsigned)((nwt + 255) / 256), 256>>>(D.H, D.W, D.Kin, D.Kout, D.ldh, D.nw_in,
+                                                       h->h_max, h->hp.hb);
     CK(h, cudaGetLastError());
     h->launches += 1;
   }

@@ -12,7 +12,12 @@ namespace bk {
 // ---------------------------------------------------------------------------
 // HBM layout of one layer l (K_in = K_{l-1}, K_out = K_l):
 //   H    int16 [K_out][ldh]      hidden weights, neuron-major; ldh = 64*nw_in;
-//                                 entries i >= K_in are padding (never read as weights)
+//                                 entries i >= K_in are padding (never read as weights).
+//                                 A weight h (odd, |h| <= h_max) is stored as its
+//                                 lattice index v = (h + h_max)/2 + 2^hb, where 2^hb
+//                                 is the least power of two >= h_max + 1 (hb >= 1), so
+//                                 v lies in [2^hb, 2^hb + h_max], h > 0 iff
+//                                 v >= 2^hb + (h_max + 1)/2, and an event moves v by 1
 //   W    uint64 [K_out][nw_in]    packed sign(H), bit (i%64) of word i/64 = (h_ik > 0)
 //   PT   uint64 [c][nw_out]       packed P_l^T, bit (k%64) of word k/64 = (rho_kj > 0)
 //   rho  int8  [K_out][c]         P_l itself, for the stability rho_{k,y}
@@ -56,6 +61,7 @@ struct StepParams {
   const unsigned long long* T;  // [L] reinforcement thresholds (Alg. 3 l.8)
   Ctrl* ctrl;
   int32_t L, c, bs, h_max, r_num, r_den, nw0, upd_ctas_total;
+  int32_t hb;                   // lattice-index offset exponent (see H above)
   uint32_t key0, key1;          // Philox key = (seed mod 2^32, seed div 2^32)
 };
 
@@ -102,8 +108,11 @@ __global__ void k_train_forward(const StepParams* P, int l);
 __global__ void k_cls_select(const StepParams* P);
 // CP + R + repack of every layer with a non-empty M_l, then advance the step.
 // (key0, key1) = the Philox key, passed by value so that the round keys are
-// kernel-uniform.
-__global__ void k_update(const StepParams* P, uint32_t key0, uint32_t key1);
+// kernel-uniform.  kPow2: h_max + 1 is a power of two (both clip bounds are bit
+// boundaries of the lattice index).
+void launch_update(bool pow2, unsigned grid, size_t smem, cudaStream_t st, const StepParams* P,
+                   uint32_t key0, uint32_t key1);
+cudaError_t update_kernel_attributes(cudaFuncAttributes* fa);
 // Generic forward for evaluation: A (M x nw_in) against W -> Aout (M x nw_out).
 __global__ void k_forward_eval(const uint64_t* __restrict__ A, int64_t M, int nw_in,
                                const uint64_t* __restrict__ W, int N, int Kin,
@@ -114,11 +123,12 @@ __global__ void k_predict_out(const uint64_t* __restrict__ A, int64_t M, int nw,
                               int32_t* __restrict__ out);
 // Initialisation of H, W of one layer and rho, PT.
 __global__ void k_init_hw(int16_t* H, uint64_t* W, int Kin, int Kout, int ldh, int nw_in,
-                          int l, uint32_t key0, uint32_t key1);
+                          int l, uint32_t key0, uint32_t key1, int h_max, int hb);
 __global__ void k_init_rho(int8_t* rho, int Kout, int c, int l, uint32_t key0, uint32_t key1);
 __global__ void k_pack_pt(const int8_t* rho, uint64_t* PT, int Kout, int c, int nw_out);
 // Re-derive W from H for one layer (after set_state).
-__global__ void k_repack_w(const int16_t* H, uint64_t* W, int Kin, int Kout, int ldh, int nw_in);
+__global__ void k_repack_w(const int16_t* H, uint64_t* W, int Kin, int Kout, int ldh, int nw_in,
+                           int h_max, int hb);
 // Tensor-core forward (tcgen05, +-1 as e4m3, exact fp32 sums), training layer l;
 // needs bs <= 128.
 __global__ void k_train_forward_tc(const StepParams* P, int l);

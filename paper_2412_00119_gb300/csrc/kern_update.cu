@@ -117,20 +117,21 @@ __global__ void __launch_bounds__(kClsThreads) k_cls_select(const StepParams* __
 // selection in group g is k (the CP tuples of k), then streams the row in
 // chunks of 8 hidden weights, one 16-byte vector per lane, with a rotating
 // queue of four vectors in flight per lane.
-// In registers a chunk is 4 words of two offset-binary 16-bit lanes
-// (u = h + 2^15 = h XOR 0x8000).  |h| <= h_max + 2 < 2^14 keeps every lane
-// inside (0, 2^16), so a packed pair of +-2 steps is one 32-bit add without
-// carries between lanes; bit 15 of a lane is (h > 0); a lane equal to a given
-// value is found exactly with a carry-free test.  All of the rule then runs on
-// packed lanes, with warp-uniform branches only:
-//   CP: per tuple (ascending mu) add the packed deltas 2 a^mu_i rho_{k,y^mu}
-//       from a shared byte -> delta table; when some lane may cross a bound
-//       (|h| > h_max - 2 n_k somewhere in the warp), lanes that reached
-//       +-(h_max + 2) are moved back by 2 after each tuple (the clip).
+// H holds each weight as its lattice index v = (h + h_max)/2 + 2^hb (see
+// DevLayer): a CP or R event is a step of +-1 in v, and v stays in
+// [2^hb, 2^hb + h_max] subset of (0, 2^15).  A 32-bit word holds two lanes, so a
+// packed pair of +-1 steps is one 32-bit add with no carry between lanes.
+// After a step a lane can only have left the range by one, to 2^hb - 1 (bit hb
+// clear) or to 2^hb + h_max + 1 (= 2^(hb+1) when h_max + 1 = 2^hb, kPow2); the
+// clip moves it back.  h > 0 is the lane's bit hb - 1 (kPow2) or v >= 2^hb +
+// (h_max + 1)/2.  All of the rule runs on packed lanes, warp-uniform branches
+// only:
+//   CP: per tuple (ascending mu) add the packed +-1 steps 2 a^mu_i rho_{k,y^mu}/2
+//       from a 16-entry shared nibble table, then clip.
 //   R : the Philox draw's 16-bit lanes line up with the weight lanes; lanes
-//       whose high half is below T's high half (< 2^15) fire; a fired lane
-//       moves 2 away from 0 unless it sits at +-h_max.
-//   W : one byte per chunk from the lanes' bit 15, written in place.
+//       whose high half is below T's high half (< 2^15) fire and step away
+//       from 0, then clip.
+//   W : one byte per chunk from the lanes' sign flags, written in place.
 // A chunk with a tie (draw high half == T high half, probability 8 / 2^16),
 // the partly padded last chunk of a row, and every chunk when T >= 2^31 take
 // the per-weight path instead.  Chunks of padding only are never touched.
@@ -140,20 +141,21 @@ __global__ void __launch_bounds__(kClsThreads) k_cls_select(const StepParams* __
 namespace {
 
 constexpr uint32_t kLaneTop = 0x80008000u;
+constexpr uint32_t kLaneOne = 0x00010001u;
 constexpr unsigned kFull = 0xffffffffu;
 
-__device__ __forceinline__ int lane_h(const uint4& w, int j) {
+__device__ __forceinline__ uint32_t lane_v(const uint4& w, int j) {
   const uint32_t word = (j < 2) ? w.x : (j < 4) ? w.y : (j < 6) ? w.z : w.w;
-  return (int)(int16_t)(uint16_t)(word >> (16 * (j & 1)));
+  return (word >> (16 * (j & 1))) & 0xFFFFu;
 }
 
-__device__ __forceinline__ void set_lane_h(uint4& w, int j, int h) {
+__device__ __forceinline__ void set_lane_v(uint4& w, int j, uint32_t v) {
   const int sh = 16 * (j & 1);
-  const uint32_t m = ~(0xFFFFu << sh), v = ((uint32_t)h & 0xFFFFu) << sh;
-  if (j < 2) w.x = (w.x & m) | v;
-  else if (j < 4) w.y = (w.y & m) | v;
-  else if (j < 6) w.z = (w.z & m) | v;
-  else w.w = (w.w & m) | v;
+  const uint32_t m = ~(0xFFFFu << sh), x = (v & 0xFFFFu) << sh;
+  if (j < 2) w.x = (w.x & m) | x;
+  else if (j < 4) w.y = (w.y & m) | x;
+  else if (j < 6) w.z = (w.z & m) | x;
+  else w.w = (w.w & m) | x;
 }
 
 struct ChunkOut {
@@ -161,11 +163,18 @@ struct ChunkOut {
   uint32_t wbyte;
 };
 
-// Per-weight path on two's-complement lanes: CP (unless `cp_done`), R and W for
-// the first `nvalid` weights of the chunk.  Loops stay rolled: rarely taken.
+struct Enc {
+  int h_max, hb, base;  // v = (h + h_max)/2 + base, base = 2^hb
+  __device__ __forceinline__ int dec(uint32_t v) const { return 2 * ((int)v - base) - h_max; }
+  __device__ __forceinline__ uint32_t enc(int h) const { return (uint32_t)((h + h_max) / 2 + base); }
+};
+
+// Per-weight path (rule as printed, on decoded h): CP (unless `cp_done`), R
+// and W for the first `nvalid` weights of the chunk.  Rarely taken; its loops
+// stay rolled.
 __device__ __forceinline__ ChunkOut chunk_scalar(uint4 w, int ch, int nvalid, bool cp_done,
                                                  const int32_t* list, int n_t, const uint8_t* aprev,
-                                                 uint32_t arow_bytes, int h_max, uint32_t Thi,
+                                                 uint32_t arow_bytes, Enc E, uint32_t Thi,
                                                  uint32_t Tlo, uint32_t key0, uint32_t key1,
                                                  uint32_t k, uint32_t c2_lo, uint32_t t, uint4 rh) {
   if (!cp_done) {
@@ -178,7 +187,7 @@ __device__ __forceinline__ ChunkOut chunk_scalar(uint4 w, int ch, int nvalid, bo
 #pragma unroll 1
       for (int j = 0; j < nvalid; ++j) {
         const int step = ((byte >> j) & 1u) ? rho : -rho;
-        set_lane_h(w, j, clip_h(lane_h(w, j) + 2 * step, h_max));
+        set_lane_v(w, j, E.enc(clip_h(E.dec(lane_v(w, j)) + 2 * step, E.h_max)));
       }
     }
   }
@@ -192,10 +201,10 @@ __device__ __forceinline__ ChunkOut chunk_scalar(uint4 w, int ch, int nvalid, bo
   for (int j = 0; j < nvalid; ++j) {
     const uint32_t u = lane16(rh, j);
     const bool fire = (u < Thi) || (((ties >> j) & 1u) && lane16(rl, j) < Tlo);
-    int h = lane_h(w, j);
+    int h = E.dec(lane_v(w, j));
     if (fire) {
-      h = clip_h(h + (h > 0 ? 2 : -2), h_max);
-      set_lane_h(w, j, h);
+      h = clip_h(h + (h > 0 ? 2 : -2), E.h_max);
+      set_lane_v(w, j, E.enc(h));
     }
     out.wbyte |= (h > 0 ? 1u : 0u) << j;
   }
@@ -209,10 +218,10 @@ __device__ __forceinline__ uint32_t eq_flags(uint32_t w, uint32_t cpair) {
   return ~(((x & 0x7FFF7FFFu) + 0x7FFF7FFFu) | x) & kLaneTop;
 }
 
-// Bit 15 of each offset-binary lane (= h > 0) -> W byte.
-__device__ __forceinline__ uint32_t w_byte_ob(const uint4& w) {
-  const uint32_t p0 = __byte_perm(w.x, w.y, 0x7531) & 0x80808080u;
-  const uint32_t p1 = __byte_perm(w.z, w.w, 0x7531) & 0x80808080u;
+// Gather bit 15 of the 8 lanes into a byte (lane j -> bit j).
+__device__ __forceinline__ uint32_t gather_top(uint32_t a, uint32_t b, uint32_t c, uint32_t d) {
+  const uint32_t p0 = __byte_perm(a, b, 0x7531) & 0x80808080u;
+  const uint32_t p1 = __byte_perm(c, d, 0x7531) & 0x80808080u;
   return ((p0 * 0x00204081u) >> 28) | (((p1 * 0x00204081u) >> 28) << 4);
 }
 
@@ -226,35 +235,44 @@ __device__ __forceinline__ uint32_t fire_flags(uint32_t u, uint32_t Tpair) {
 // nonzero iff some lane of a draw word equals Thi
 __device__ __forceinline__ uint32_t tie_any(uint32_t u, uint32_t Tpair) {
   const uint32_t x = u ^ Tpair;
-  return (x - 0x00010001u) & ~x & kLaneTop;
+  return (x - kLaneOne) & ~x & kLaneTop;
 }
 
-// lanes of an offset-binary word outside [lo, hi] after subtracting `base`
-__device__ __forceinline__ uint32_t range_flags(uint32_t w, uint32_t base_pair, uint32_t lo_pair,
-                                                uint32_t hi_pair) {
-  const uint32_t a = w - base_pair;
-  return ~(((a | kLaneTop) - lo_pair) & ((hi_pair | kLaneTop) - a)) & kLaneTop;
-}
-
-// clip after a +-2 step: lanes at +-(h_max + 2) move back by 2
-__device__ __forceinline__ uint32_t clip_step(uint32_t w, uint32_t over_pair, uint32_t under_pair) {
-  return w + (eq_flags(w, under_pair) >> 14) - (eq_flags(w, over_pair) >> 14);
-}
-
-// reinforcement of the fired lanes: 2 away from 0 unless at +-h_max
-__device__ __forceinline__ uint32_t reinforce(uint32_t w, uint32_t fire, uint32_t top_pair,
-                                              uint32_t bot_pair) {
-  const uint32_t inc = fire & w & ~eq_flags(w, top_pair);
-  const uint32_t dec = fire & ~w & ~eq_flags(w, bot_pair);
-  return w + (inc >> 14) - (dec >> 14);
-}
+template <bool kPow2>
+struct Lanes {
+  int hb;
+  uint32_t over_pair;  // pair(2^hb + h_max + 1), used when !kPow2
+  uint32_t pos_pair;   // pair(2^hb + (h_max + 1)/2), used when !kPow2
+  // lanes that left [2^hb, 2^hb + h_max] by one step go back
+  __device__ __forceinline__ uint32_t clip(uint32_t v) const {
+    if (kPow2) {
+      const uint32_t t = (v >> hb) & 0x00030003u;  // 0 under, 1 inside, 2 over
+      return v + kLaneOne - t;
+    } else {
+      const uint32_t under = (~v >> hb) & kLaneOne;
+      return v + under - (eq_flags(v, over_pair) >> 15);
+    }
+  }
+  // bit 15 of each lane = (h > 0)
+  __device__ __forceinline__ uint32_t pos_top(uint32_t v) const {
+    if (kPow2) return (v << (16 - hb)) & kLaneTop;
+    return ((v | kLaneTop) - pos_pair) & kLaneTop;
+  }
+  // fired lanes step away from 0 (then clip)
+  __device__ __forceinline__ uint32_t reinforce(uint32_t v, uint32_t fire_top) const {
+    const uint32_t f = fire_top >> 15;
+    const uint32_t p = pos_top(v) >> 15;
+    return clip(v + (f & p) - (f & ~p));
+  }
+};
 
 }  // namespace
 
+template <bool kPow2>
 __global__ void __launch_bounds__(kUpdThreads, 3) k_update(const StepParams* __restrict__ P,
                                                            uint32_t key0, uint32_t key1) {
   extern __shared__ int32_t dyn[];
-  __shared__ uint4 s_delta[2 * 256];
+  __shared__ uint2 s_dn[2][16];
   const int bid = blockIdx.x;
   int li = 0;
   while (li + 1 < P->L && bid >= P->layer[li + 1].upd_cta_base) ++li;
@@ -278,30 +296,33 @@ __global__ void __launch_bounds__(kUpdThreads, 3) k_update(const StepParams* __r
     int32_t* s_list = dyn + (P->bs + 1) / 2 + warp * P->bs;         // [nwarps][bs]
 
     for (int m = threadIdx.x; m < bsz; m += blockDim.x) s_sel[m] = Ly.sel[(int64_t)m * Ly.G + g];
-    // s_delta[r][b]: word p packs the steps of bits 2p and 2p+1 of b as
-    // d_lo + 2^16 d_hi (d = +-2, negated for r = 1, i.e. rho = -1); added to a
-    // word of two offset-binary lanes it moves each lane by its own step
-    for (int i = threadIdx.x; i < 512; i += blockDim.x) {
-      const int r = i >> 8, b = i & 255;
-      uint32_t v[4];
+    // s_dn[r][n]: the +-1 lattice steps of the 4 weights of nibble n, two lanes
+    // per word (d_lo + 2^16 d_hi), d = +1 for a set bit, negated for r = 1
+    // (rho = -1)
+    if (threadIdx.x < 32) {
+      const int r = threadIdx.x >> 4, n = threadIdx.x & 15;
+      int d[4];
 #pragma unroll
-      for (int p = 0; p < 4; ++p) {
-        int lo = ((b >> (2 * p)) & 1) ? 2 : -2;
-        int hi = ((b >> (2 * p + 1)) & 1) ? 2 : -2;
-        if (r) { lo = -lo; hi = -hi; }
-        v[p] = (uint32_t)(lo + 65536 * hi);
-      }
-      s_delta[i] = make_uint4(v[0], v[1], v[2], v[3]);
+      for (int j = 0; j < 4; ++j) d[j] = (((n >> j) & 1) ? 1 : -1) * (r ? -1 : 1);
+      s_dn[r][n] = make_uint2((uint32_t)(d[0] + 65536 * d[1]), (uint32_t)(d[2] + 65536 * d[3]));
     }
     __syncthreads();
 
     const uint32_t l = (uint32_t)li + 1u;
     const int c = P->c;
-    const int h_max = P->h_max;
+    Enc E;
+    E.h_max = P->h_max;
+    E.hb = P->hb;
+    E.base = 1 << P->hb;
+    Lanes<kPow2> LN;
+    LN.hb = P->hb;
+    LN.over_pair = (uint32_t)(E.base + E.h_max + 1) * kLaneOne;
+    LN.pos_pair = (uint32_t)(E.base + (E.h_max + 1) / 2) * kLaneOne;
     const unsigned long long T = P->T[li];
     const uint32_t Thi = (uint32_t)(T >> 16);   // 0..65536
     const uint32_t Tlo = (uint32_t)(T & 0xFFFFu);
-    const uint32_t Tpair = Thi * 0x00010001u;
+    const uint32_t Tpair = Thi * kLaneOne;
+    const bool packed = Thi < 0x8000u;           // the SIMD draw test is exact
     const uint32_t c2_hi = (3u << 16) + l, c2_lo = (4u << 16) + l;
     const uint32_t tt = (uint32_t)t;
     const int Kin = Ly.Kin;
@@ -310,12 +331,6 @@ __global__ void __launch_bounds__(kUpdThreads, 3) k_update(const StepParams* __r
     const uint32_t arow_bytes = (uint32_t)Ly.nw_in * 8u;
     const uint8_t* aprev = (li == 0) ? reinterpret_cast<const uint8_t*>(P->x + start * P->nw0)
                                      : reinterpret_cast<const uint8_t*>(P->layer[li - 1].A);
-    // packed lanes on the rule's boundary values (offset binary)
-    const bool packed = h_max < 0x3FFF && Thi < 0x8000u;
-    const uint32_t top_pair = (uint32_t)(0x8000 + h_max) * 0x00010001u;
-    const uint32_t bot_pair = (uint32_t)(0x8000 - h_max) * 0x00010001u;
-    const uint32_t over_pair = (uint32_t)(0x8000 + h_max + 2) * 0x00010001u;
-    const uint32_t under_pair = (uint32_t)(0x8000 - h_max - 2) * 0x00010001u;
     const int iters = (nch + 31) >> 5;
 
     for (int rr = r0 + warp; rr < r1; rr += nwarps) {
@@ -335,10 +350,6 @@ __global__ void __launch_bounds__(kUpdThreads, 3) k_update(const StepParams* __r
         n_t += __popc(bal);
       }
       __syncwarp();
-      // no clip can trigger in a chunk whose lanes all keep |h| <= h_max - 2 n_t
-      const bool range_test = 2 * n_t <= h_max;
-      const uint32_t lo_pair = (uint32_t)(2 * n_t) * 0x00010001u;
-      const uint32_t hi_pair = (uint32_t)(range_test ? 2 * h_max - 2 * n_t : 0) * 0x00010001u;
 
       int16_t* hrow = Ly.H + (int64_t)k * Ly.ldh;
       uint8_t* wrow = reinterpret_cast<uint8_t*>(Ly.W + (int64_t)k * Ly.nw_in);
@@ -353,7 +364,7 @@ __global__ void __launch_bounds__(kUpdThreads, 3) k_update(const StepParams* __r
       for (int it = 0; it < iters; ++it) {
         const int ch = 32 * it + lane;
         const bool live = ch < nch;
-        const uint4 w_in = q0;   // two's complement, as loaded
+        const uint4 w_in = q0;
         uint4 w = q0;
         q0 = q1;
         q1 = q2;
@@ -361,29 +372,17 @@ __global__ void __launch_bounds__(kUpdThreads, 3) k_update(const StepParams* __r
         if (ch + 128 < nch) q3 = __ldcs(reinterpret_cast<const uint4*>(hrow + 8 * (ch + 128)));
         const uint4 rh = philox4x32_10(make_uint4((uint32_t)ch, (uint32_t)k, c2_hi, tt), key0, key1);
         const bool simd = packed && ch < full;   // this lane's chunk runs on packed lanes
-        w.x ^= kLaneTop; w.y ^= kLaneTop; w.z ^= kLaneTop; w.w ^= kLaneTop;  // offset binary
         // ---- Clipped Perceptron ----
-        if (n_t > 0) {
-          bool safe = true;
-          if (range_test && simd)
-            safe = (range_flags(w.x, bot_pair, lo_pair, hi_pair) | range_flags(w.y, bot_pair, lo_pair, hi_pair) |
-                    range_flags(w.z, bot_pair, lo_pair, hi_pair) | range_flags(w.w, bot_pair, lo_pair, hi_pair)) == 0u;
-          else if (!range_test)
-            safe = false;
-          const bool clip = !__all_sync(kFull, safe || !live);
 #pragma unroll 1
-          for (int q = 0; q < n_t; ++q) {
-            const int e = s_list[q];
-            const uint32_t byte = live ? aprev[(size_t)(e & 0xFFFF) * arow_bytes + ch] : 0u;
-            const uint4 d = s_delta[((e >> 16) & 1) * 256 + byte];
-            w.x += d.x; w.y += d.y; w.z += d.z; w.w += d.w;
-            if (clip) {
-              w.x = clip_step(w.x, over_pair, under_pair);
-              w.y = clip_step(w.y, over_pair, under_pair);
-              w.z = clip_step(w.z, over_pair, under_pair);
-              w.w = clip_step(w.w, over_pair, under_pair);
-            }
-          }
+        for (int q = 0; q < n_t; ++q) {
+          const int e = s_list[q];
+          const uint32_t byte = live ? aprev[(size_t)(e & 0xFFFF) * arow_bytes + ch] : 0u;
+          const uint2* dn = s_dn[(e >> 16) & 1];
+          const uint2 dl = dn[byte & 15u], dh = dn[byte >> 4];
+          w.x = LN.clip(w.x + dl.x);
+          w.y = LN.clip(w.y + dl.y);
+          w.z = LN.clip(w.z + dh.x);
+          w.w = LN.clip(w.w + dh.y);
         }
         // ---- Reinforcement ----
         const uint32_t tie = simd ? (tie_any(rh.x, Tpair) | tie_any(rh.y, Tpair) |
@@ -393,19 +392,18 @@ __global__ void __launch_bounds__(kUpdThreads, 3) k_update(const StepParams* __r
                                    fire_flags(rh.z, Tpair), fire_flags(rh.w, Tpair));
         const bool fires = live && !slow && ((f.x | f.y | f.z | f.w) != 0u);
         if (__any_sync(kFull, fires) && fires) {
-          w.x = reinforce(w.x, f.x, top_pair, bot_pair);
-          w.y = reinforce(w.y, f.y, top_pair, bot_pair);
-          w.z = reinforce(w.z, f.z, top_pair, bot_pair);
-          w.w = reinforce(w.w, f.w, top_pair, bot_pair);
+          w.x = LN.reinforce(w.x, f.x);
+          w.y = LN.reinforce(w.y, f.y);
+          w.z = LN.reinforce(w.z, f.z);
+          w.w = LN.reinforce(w.w, f.w);
         }
-        uint32_t wbyte = w_byte_ob(w);
-        w.x ^= kLaneTop; w.y ^= kLaneTop; w.z ^= kLaneTop; w.w ^= kLaneTop;  // back to int16
+        uint32_t wbyte = gather_top(LN.pos_top(w.x), LN.pos_top(w.y), LN.pos_top(w.z), LN.pos_top(w.w));
         if (slow) {
           // a packed chunk with a tie keeps its packed CP result; any other chunk
           // restarts from the loaded values and the per-weight path does it all
-          const ChunkOut o = chunk_scalar(simd ? w : w_in, ch, min(8, Kin - 8 * ch), simd, s_list, n_t, aprev,
-                                          arow_bytes, h_max, Thi, Tlo, key0, key1, (uint32_t)k,
-                                          c2_lo, tt, rh);
+          const ChunkOut o = chunk_scalar(simd ? w : w_in, ch, min(8, Kin - 8 * ch), simd, s_list,
+                                          n_t, aprev, arow_bytes, E, Thi, Tlo, key0, key1,
+                                          (uint32_t)k, c2_lo, tt, rh);
           w = o.w;
           wbyte = o.wbyte;
         }
@@ -431,6 +429,18 @@ __global__ void __launch_bounds__(kUpdThreads, 3) k_update(const StepParams* __r
       __threadfence();
     }
   }
+}
+
+void launch_update(bool pow2, unsigned grid, size_t smem, cudaStream_t st, const StepParams* P,
+                   uint32_t key0, uint32_t key1) {
+  if (pow2)
+    k_update<true><<<grid, kUpdThreads, smem, st>>>(P, key0, key1);
+  else
+    k_update<false><<<grid, kUpdThreads, smem, st>>>(P, key0, key1);
+}
+
+cudaError_t update_kernel_attributes(cudaFuncAttributes* fa) {
+  return cudaFuncGetAttributes(fa, k_update<true>);
 }
 
 // ---------------------------------------------------------------------------
@@ -460,12 +470,13 @@ __global__ void __launch_bounds__(256) k_predict_out(const uint64_t* __restrict_
 }
 
 // ---------------------------------------------------------------------------
-// Initialisation (Alg. 1 l.2): h_ik = +-1 from Philox purpose 1, pad entries
-// -1 (never used; their W bits stay 0); W = packed sign(H).  One thread per
+// Initialisation (Alg. 1 l.2): h_ik = +-1 from Philox purpose 1, stored as the
+// lattice index v = (h + h_max)/2 + 2^hb; pad entries get 2^hb (never used;
+// their W bits stay 0); W = packed sign(H).  One thread per
 // chunk of 8 inputs of one neuron row.
 // ---------------------------------------------------------------------------
 __global__ void k_init_hw(int16_t* H, uint64_t* W, int Kin, int Kout, int ldh, int nw_in, int l,
-                          uint32_t key0, uint32_t key1) {
+                          uint32_t key0, uint32_t key1, int h_max, int hb) {
   const int nch = ldh >> 3;
   const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (idx >= (int64_t)Kout * nch) return;
@@ -479,8 +490,9 @@ __global__ void k_init_hw(int16_t* H, uint64_t* W, int Kin, int Kout, int ldh, i
 #pragma unroll
   for (int j = 0; j < 8; ++j) {
     const int i = 8 * ch + j;
-    h[j] = (i < Kin) ? ((w8[j] >> 31) ? (int16_t)1 : (int16_t)-1) : (int16_t)-1;
-    if (i < Kin && h[j] > 0) wbyte |= 1u << j;
+    const int hv = (w8[j] >> 31) ? 1 : -1;
+    h[j] = (int16_t)((i < Kin ? (hv + h_max) / 2 : 0) + (1 << hb));  // lattice index v
+    if (i < Kin && hv > 0) wbyte |= 1u << j;
   }
   int4 hv;
   hv.x = (int)(((uint32_t)(uint16_t)h[0]) | ((uint32_t)(uint16_t)h[1] << 16));
@@ -516,8 +528,10 @@ __global__ void k_pack_pt(const int8_t* rho, uint64_t* PT, int Kout, int c, int 
   PT[idx] = bits;
 }
 
-// W = packed sign(H) for one layer, pad bits 0.
-__global__ void k_repack_w(const int16_t* H, uint64_t* W, int Kin, int Kout, int ldh, int nw_in) {
+// W = packed sign(H) for one layer (H as lattice indices), pad bits 0.
+__global__ void k_repack_w(const int16_t* H, uint64_t* W, int Kin, int Kout, int ldh, int nw_in,
+                           int h_max, int hb) {
+  const int pos_from = (1 << hb) + (h_max + 1) / 2;  // lattice index of h = +1
   const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (idx >= (int64_t)Kout * nw_in) return;
   const int k = (int)(idx / nw_in);
@@ -525,7 +539,7 @@ __global__ void k_repack_w(const int16_t* H, uint64_t* W, int Kin, int Kout, int
   uint64_t bits = 0;
   for (int b = 0; b < 64; ++b) {
     const int i = 64 * w + b;
-    if (i < Kin && H[(int64_t)k * ldh + i] > 0) bits |= 1ull << b;
+    if (i < Kin && H[(int64_t)k * ldh + i] >= pos_from) bits |= 1ull << b;
   }
   W[idx] = bits;
 }

@@ -46,6 +46,7 @@ def test_threshold_matches_oracle(oracle_mod):
     (dict(widths=[10, 0], classes=2), "width"),
     (dict(widths=[10, 8], classes=1), "classes"),
     (dict(widths=[10, 8], classes=2, h_max=4), "h_max"),
+    (dict(widths=[10, 8], classes=2, h_max=16385), "h_max"),
     (dict(widths=[10, 8], classes=2, bs=2000), "bs"),
     (dict(widths=[10, 8], classes=2, gamma=[3]), "gamma"),
     (dict(widths=[10, 8], classes=2, r=(-1, 4)), "r must"),
