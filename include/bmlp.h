@@ -118,9 +118,22 @@ int bmlp_train(bmlp_t* h, const uint64_t* x_packed, const int32_t* labels, int64
                uint32_t flags, void* cuda_stream, int64_t* n_errors_out);
 
 /* Forward-only evaluation (Sec. 3.1): labels_out[mu] = argmax_j (a_L P_L)_{mu j}
- * (lowest index on ties) for n packed rows of K_0 bits.  Does not change state. */
+ * (lowest index on ties) for n packed rows of K_0 bits.  Does not change state.
+ * With device x_packed and labels_out the call does not synchronise, and an
+ * expired bounded device wait (tensor-core engine) is reported by the next
+ * call that does (BMLP_ETIMEOUT). */
 int bmlp_predict(bmlp_t* h, const uint64_t* x_packed, int64_t n, int32_t* labels_out,
                  void* cuda_stream);
+
+/* One layer of forward-only evaluation (Sec. 3.1; Alg. 1 l.8-9):
+ * a_out = sign(a_in W_l), sign(0) = +1, for n packed rows.  a_in: n rows of
+ * ceil(K_{l-1}/64) words (pad bits 0); a_out: n rows of ceil(K_l/64) words,
+ * written with pad bits 0.  Both must be device pointers (else BMLP_EINVAL).
+ * Runs the engine bmlp_predict uses for this handle; asynchronous on
+ * cuda_stream.  An expired bounded device wait (tensor-core engine) is
+ * reported by the next call that synchronises (BMLP_ETIMEOUT). */
+int bmlp_layer_forward(bmlp_t* h, int32_t layer, const uint64_t* a_in, int64_t n,
+                       uint64_t* a_out, void* cuda_stream);
 
 /* Copy layer `layer` (1..L) to host buffers (each may be NULL; formats above),
  * plus the current p_r and step counter t (mini-batches since creation). */

@@ -71,6 +71,7 @@ SIGNATURES = [
     ("bmlp_reset_profile", C.c_int, [_vp]),
     ("bmlp_launch_count", C.c_int64, [_vp]),
     ("bmlp_predict_noalloc", C.c_int, [_vp, _vp, C.c_int64, _vp, _vp]),
+    ("bmlp_layer_forward", C.c_int, [_vp, C.c_int32, _vp, C.c_int64, _vp, _vp]),
 ]
 
 
@@ -173,6 +174,12 @@ def bmlp_predict_noalloc(h, x_packed, labels_out, n=None, stream=None):
     memory (device buffers only; n * ceil(max K_l / 64) <= 2^20)."""
     n = labels_out.shape[0] if n is None else n
     _check(lib().bmlp_predict_noalloc(h, _ptr(x_packed), n, _ptr(labels_out), _stream(stream)), h)
+
+
+def bmlp_layer_forward(h, layer, a_in, a_out, n=None, stream=None):
+    """a_out = sign(a_in W_layer), packed rows on the device."""
+    n = a_out.shape[0] if n is None else n
+    _check(lib().bmlp_layer_forward(h, layer, _ptr(a_in), n, _ptr(a_out), _stream(stream)), h)
 
 
 def bmlp_get_info(h):

@@ -161,8 +161,7 @@ int enqueue_step(bmlp_t* h, cudaStream_t st) {
   for (int l = 1; l <= h->L; ++l) {
     prof_begin(h, kProfTrainFwd, st);
     if (h->fwd_impl == BMLP_FWD_TCGEN05)
-      k_train_forward_tc<<<train_forward_tc_grid(h->K[l]), train_forward_tc_block(),
-                           train_forward_tc_smem(), st>>>(h->dP, l);
+      launch_train_forward_tc(l > 1, h->K[l], st, h->dP, l);
     else
       k_train_forward<<<train_forward_grid(h->bs, h->K[l]), train_forward_block(), 0, st>>>(h->dP, l);
     prof_end(h, st);
@@ -372,6 +371,12 @@ int bmlp_create(const int32_t* widths, int32_t n_widths, int32_t classes, int16_
         (rc = dalloc(h, &D.mark, (size_t)bs)) ||
         (rc = dalloc(h, &D.sel, (size_t)bs * D.G)))
       return bail(rc);
+    D.AE = nullptr;
+    if (fwd == BMLP_FWD_TCGEN05 && l < L) {
+      if ((rc = dalloc(h, &D.AE, act_tile_bytes(D.Kout))) != BMLP_OK) return bail(rc);
+      cudaError_t ez = cudaMemset(D.AE, 0, act_tile_bytes(D.Kout));
+      if (ez != cudaSuccess) return bail(cuda_fail(h, ez, "cudaMemset"));
+    }
   }
   h->updCtas = cta;
   P.upd_ctas_total = cta;
@@ -399,8 +404,7 @@ int bmlp_create(const int32_t* widths, int32_t n_widths, int32_t classes, int16_
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return bail(cuda_fail(h, e, "init kernels"));
   if (fwd == BMLP_FWD_TCGEN05 &&
-      (e = cudaFuncSetAttribute(k_train_forward_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                (int)train_forward_tc_smem())) != cudaSuccess)
+      ((e = prepare_train_forward_tc()) != cudaSuccess || (e = prepare_forward_eval_tc()) != cudaSuccess))
     return bail(cuda_fail(h, e, "tcgen05 forward smem attribute"));
   if ((e = cudaMemset(h->dCtrl, 0, sizeof(Ctrl))) != cudaSuccess) return bail(cuda_fail(h, e, "memset"));
   if ((e = cudaMemcpy(h->dP, &P, sizeof(P), cudaMemcpyHostToDevice)) != cudaSuccess)
@@ -517,8 +521,12 @@ int bmlp_predict(bmlp_t* h, const uint64_t* x, int64_t n, int32_t* out, void* cu
     for (int l = 1; l <= h->L; ++l) {
       const DevLayer& D = h->hp.layer[l - 1];
       prof_begin(h, kProfEvalFwd, st);
-      k_forward_eval<<<eval_forward_grid(m, D.Kout), eval_forward_block(), 0, st>>>(
-          in, m, D.nw_in, D.W, D.Kout, D.Kin, h->evA[cur], D.nw_out);
+      if (h->fwd_impl == BMLP_FWD_TCGEN05)
+        launch_forward_eval_tc(in, m, D.nw_in, D.W, D.Kout, D.Kin, h->evA[cur], D.nw_out,
+                               &h->dCtrl->timeouts, st);
+      else
+        k_forward_eval<<<eval_forward_grid(m, D.Kout), eval_forward_block(), 0, st>>>(
+            in, m, D.nw_in, D.W, D.Kout, D.Kin, h->evA[cur], D.nw_out);
       prof_end(h, st);
       in = h->evA[cur];
       cur ^= 1;
@@ -536,7 +544,17 @@ int bmlp_predict(bmlp_t* h, const uint64_t* x, int64_t n, int32_t* out, void* cu
       prof_end(h, st);
     }
   }
-  if (!odev) CK(h, cudaStreamSynchronize(st));
+  if (!odev) {
+    if (h->fwd_impl == BMLP_FWD_TCGEN05)
+      CK(h, cudaMemcpyAsync(&h->hostPinned[3], &h->dCtrl->timeouts, sizeof(uint32_t),
+                            cudaMemcpyDeviceToHost, st));
+    CK(h, cudaStreamSynchronize(st));
+    if (h->fwd_impl == BMLP_FWD_TCGEN05 && (uint32_t)h->hostPinned[3] != 0) {
+      CK(h, cudaMemsetAsync(&h->dCtrl->timeouts, 0, sizeof(uint32_t), st));
+      h->hostPinned[3] = 0;
+      return fail(h, BMLP_ETIMEOUT, "a bounded device-side wait expired");
+    }
+  }
   return prof_collect(h, st);
 }
 
@@ -620,6 +638,35 @@ int bmlp_get_info(const bmlp_t* h, int32_t* n_layers, int32_t* widths_out, int32
   if (bs) *bs = h->bs;
   if (fwd_impl) *fwd_impl = h->fwd_impl;
   return BMLP_OK;
+}
+
+int bmlp_layer_forward(bmlp_t* h, int32_t layer, const uint64_t* a_in, int64_t n, uint64_t* a_out,
+                       void* cuda_stream) {
+  if (!h) return BMLP_EINVAL;
+  h->err.clear();
+  if (layer < 1 || layer > h->L) return fail(h, BMLP_EINVAL, "layer must be in 1..%d", h->L);
+  if (n < 0) return fail(h, BMLP_EINVAL, "n < 0");
+  if (n == 0) return BMLP_OK;
+  if (!a_in || !a_out || !is_device_ptr(a_in) || !is_device_ptr(a_out))
+    return fail(h, BMLP_EINVAL, "a_in and a_out must be device pointers");
+  cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
+  const DevLayer& D = h->hp.layer[layer - 1];
+  for (int64_t s0 = 0; s0 < n; s0 += kEvalChunk) {
+    const int64_t m = std::min(kEvalChunk, n - s0);
+    const uint64_t* in = a_in + s0 * D.nw_in;
+    uint64_t* out = a_out + s0 * D.nw_out;
+    prof_begin(h, kProfEvalFwd, st);
+    if (h->fwd_impl == BMLP_FWD_TCGEN05)
+      launch_forward_eval_tc(in, m, D.nw_in, D.W, D.Kout, D.Kin, out, D.nw_out,
+                             &h->dCtrl->timeouts, st);
+    else
+      k_forward_eval<<<eval_forward_grid(m, D.Kout), eval_forward_block(), 0, st>>>(
+          in, m, D.nw_in, D.W, D.Kout, D.Kin, out, D.nw_out);
+    prof_end(h, st);
+    CK(h, cudaGetLastError());
+    h->launches += 1;
+  }
+  return prof_collect(h, st);
 }
 
 int bmlp_debug_last_step(const bmlp_t* hc, int32_t layer, int16_t* Z, uint64_t* A, uint8_t* mark,

@@ -25,6 +25,11 @@ namespace bk {
 //   A    uint64 [bs][nw_out]      packed activations a_l of the current mini-batch
 //   mark uint8 [bs]               1 iff the pattern is in M_l
 //   sel  int16 [bs][G]            selected neuron per (pattern, group), -1 = none
+//   AE   uint8 [ceil(K_out/128)][128][128]  (tcgen05 engine, l < L) the
+//                                 activations of the mini-batch as e4m3 +-1 (0 past
+//                                 K_out), in the 128B-swizzled K-major image of
+//                                 128 patterns x 128 K-elements per tile that the
+//                                 next layer's MMA reads; rows >= bs are zero
 // ---------------------------------------------------------------------------
 struct DevLayer {
   int16_t* H;
@@ -35,6 +40,7 @@ struct DevLayer {
   uint64_t* A;
   uint8_t* mark;
   int16_t* sel;
+  uint8_t* AE;
   int32_t Kin, Kout, nw_in, nw_out, ldh, gamma, G;
   int32_t upd_cta_base;  // first CTA of this layer in the update grid
   int32_t upd_ctas;      // CTAs of this layer in the update grid
@@ -130,11 +136,18 @@ __global__ void k_pack_pt(const int8_t* rho, uint64_t* PT, int Kout, int c, int 
 __global__ void k_repack_w(const int16_t* H, uint64_t* W, int Kin, int Kout, int ldh, int nw_in,
                            int h_max, int hb);
 // Tensor-core forward (tcgen05, +-1 as e4m3, exact fp32 sums), training layer l;
-// needs bs <= 128.
-__global__ void k_train_forward_tc(const StepParams* P, int l);
+// needs bs <= 128.  tiles: take the A operand from layer l-1's AE image.
 size_t train_forward_tc_smem();
-dim3 train_forward_tc_grid(int Kout);
-dim3 train_forward_tc_block();
+cudaError_t prepare_train_forward_tc();
+void launch_train_forward_tc(bool tiles, int Kout, cudaStream_t st, const StepParams* P, int l);
+size_t act_tile_bytes(int K);  // bytes of an AE image for K activations
+// Tensor-core forward for evaluation: A (M x nw_in) against W -> Aout
+// (M x nw_out), 128-pattern x 256-neuron tiles; an expired bounded wait adds
+// one to *timeouts.
+cudaError_t prepare_forward_eval_tc();
+void launch_forward_eval_tc(const uint64_t* A, int64_t M, int nw_in, const uint64_t* W, int N,
+                            int Kin, uint64_t* Aout, int nw_out, unsigned int* timeouts,
+                            cudaStream_t st);
 
 // Launch helpers implemented in the kernel files (grid shapes live next to the
 // kernels they describe).

@@ -7,6 +7,12 @@
 // in e4m3 (0x38 / 0xB8), pad elements are 0x00, and every partial sum is an
 // integer of magnitude <= K_in < 2^24, exact in fp32 whatever the order.
 // One CTA owns TN = 64 neurons and all (<= 128) patterns of the mini-batch.
+// The A operand of layers l >= 2 arrives pre-expanded: the epilogue of layer
+// l - 1 also writes its activations as e4m3 in the swizzled stage image (one
+// 16 KB tile per 128 K-elements, DevLayer::AE), and one producer pulls each
+// tile into the stage with a single cp.async.bulk that completes on the
+// stage's "full" mbarrier.  For layer 1 (the caller's bit-packed input) and in
+// general:
 //   - 16 producer warps expand the bit-packed activations (A, patterns x
 //     words) and visible weights (W, neurons x words), 128 K-elements (two
 //     64-bit words) per row per stage, into the K-major SWIZZLE_128B layout the
@@ -25,14 +31,15 @@
 // Every mbarrier wait is bounded; the first expiry sets a shared flag that
 // stops every other wait, the kernel counts the failure in the control block
 // (host: BMLP_ETIMEOUT), releases its TMEM and returns.
-#include "bmlp_internal.cuh"
+#include "tc_common.cuh"
 
 namespace bk {
 namespace {
 
+using namespace tc;
+
 constexpr int TM = 128;           // MMA M: patterns (rows >= bsz are zero)
 constexpr int TN = 64;            // MMA N: neurons per CTA
-constexpr int KB = 128;           // K elements (bytes) per stage and row
 constexpr int kStages = 4;
 constexpr int kPrefetch = 8;      // stages of bit-words held in registers ahead
 constexpr int kProducers = 512;   // 16 warps: one (row, half) item per thread
@@ -41,7 +48,6 @@ constexpr int A_BYTES = TM * KB;  // 16 KB
 constexpr int B_BYTES = TN * KB;  // 8 KB
 constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
 constexpr int TMEM_COLS = 64;
-constexpr unsigned long long kWaitCycles = 4000000000ull;  // ~2 s at 2 GHz
 
 struct __align__(8) TcShared {
   unsigned long long full[kStages];   // the producers filled stage s
@@ -53,123 +59,36 @@ struct __align__(8) TcShared {
 
 constexpr size_t kSmemBytes = 1024 /*alignment slack*/ + kStages * STAGE_BYTES + sizeof(TcShared);
 
-__device__ __forceinline__ uint32_t smem_u32(const void* p) {
-  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
-}
+constexpr uint32_t kIdesc = tc::idesc_f8(TM, TN);
 
-__device__ __forceinline__ void mbar_init(unsigned long long* bar, uint32_t count) {
-  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count));
-}
-
-__device__ __forceinline__ void mbar_arrive(unsigned long long* bar) {
-  asm volatile("{\n .reg .b64 st;\n mbarrier.arrive.shared::cta.b64 st, [%0];\n}"
-               ::"r"(smem_u32(bar)) : "memory");
-}
-
-// Bounded wait for the phase with the given parity; false on expiry or when
-// another thread already recorded a failure.
-__device__ __forceinline__ bool mbar_wait(unsigned long long* bar, uint32_t parity,
-                                          volatile int* failed) {
-  const uint32_t a = smem_u32(bar);
-  const unsigned long long t0 = clock64();
-  while (true) {
-    uint32_t ok;
-    asm volatile(
-        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
-        " selp.u32 %0, 1, 0, p;\n}"
-        : "=r"(ok) : "r"(a), "r"(parity) : "memory");
-    if (ok) return true;
-    if (*failed) return false;
-    if (clock64() - t0 > kWaitCycles) {
-      *failed = 1;
-      return false;
-    }
-  }
-}
-
-// Shared-memory matrix descriptor: K-major, SWIZZLE_128B, 8-row groups 1024 B apart.
-__device__ __forceinline__ uint64_t smem_desc(uint32_t saddr) {
-  uint64_t d = 0;
-  d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);           // start address
-  d |= (uint64_t)1 << 16;                              // leading byte offset (unused for SW128 K-major)
-  d |= (uint64_t)(1024 >> 4) << 32;                    // stride byte offset
-  d |= (uint64_t)1 << 46;                              // descriptor version (sm_100 family)
-  d |= (uint64_t)2 << 61;                              // swizzle: 128B
-  return d;
-}
-
-// Instruction descriptor, kind::f8f6f4: D fp32, A = B = e4m3, both K-major.
-constexpr uint32_t kIdesc = (1u << 4)                  // D format: f32
-                            | (0u << 7) | (0u << 10)   // A, B format: e4m3
-                            | ((uint32_t)(TN >> 3) << 17)
-                            | ((uint32_t)(TM >> 4) << 24);
-
-__device__ __forceinline__ void mma_f8(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc,
-                                       uint32_t accumulate) {
-  asm volatile(
-      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
-      " tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], %1, %2, %3, p;\n}"
-      ::"r"(tmem_d), "l"(adesc), "l"(bdesc), "r"(kIdesc), "r"(accumulate));
-}
-
-__device__ __forceinline__ void mma_commit(unsigned long long* bar) {
-  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];"
-               ::"r"(smem_u32(bar)) : "memory");
-}
-
-// 8 bits -> 8 e4m3 bytes (+1 = 0x38, -1 = 0xB8) as two words.  Byte j of the
-// replicated value keeps bit j of b; adding (0x80 - 2^j) per byte moves it to
-// bit 7 without carries between bytes.
-__device__ __forceinline__ uint2 expand8(uint32_t b) {
-  const uint32_t rep = b * 0x01010101u;
-  const uint32_t lo = (rep & 0x08040201u) + 0x787C7E7Fu;
-  const uint32_t hi = (rep & 0x80402010u) + 0x00406070u;
-  return make_uint2((lo & 0x80808080u) ^ 0xB8B8B8B8u, (hi & 0x80808080u) ^ 0xB8B8B8B8u);
-}
-
-// Expand one 64-bit word (64 K-elements) into four 16-byte chunks of row r of
-// a swizzled stage, chunks chunk0 .. chunk0+3.  `valid` = real elements (0..64).
-__device__ __forceinline__ void expand_word(uint8_t* row_base, int r, int chunk0, uint64_t w,
-                                            int valid) {
-#pragma unroll
-  for (int q = 0; q < 4; ++q) {        // chunk q: elements 16q .. 16q+15
-    const uint32_t bits = (uint32_t)(w >> (16 * q)) & 0xFFFFu;
-    const uint2 e0 = expand8(bits & 0xFF);
-    const uint2 e1 = expand8(bits >> 8);
-    uint4 v = make_uint4(e0.x, e0.y, e1.x, e1.y);
-    if (valid < 64) {
-      uint32_t* vv = &v.x;
-#pragma unroll
-      for (int b = 0; b < 4; ++b) {
-        const int n_ok = valid - (16 * q + 4 * b);  // real elements in this 4-byte group
-        const uint32_t keep = n_ok >= 4 ? 0xFFFFFFFFu : (n_ok <= 0 ? 0u : ((1u << (8 * n_ok)) - 1u));
-        vv[b] &= keep;
-      }
-    }
-    const int c = chunk0 + q;
-    *reinterpret_cast<uint4*>(row_base + 16 * (c ^ (r & 7))) = v;
-  }
-}
-
-// A producer item: one (matrix, row, half) of the current tile.
-struct Item {
-  const uint64_t* src;  // row start (bit words), or null when the thread has no item
-  int soff;             // byte offset of the row inside a stage (A or B part)
-  int r;                // row index inside its matrix (for the swizzle)
-  int half;             // which of the stage's two words
-};
-
-__device__ __forceinline__ uint64_t load_word(const Item& it, int kb, int nw) {
-  const int wi = 2 * kb + it.half;
-  return (it.src != nullptr && wi < nw) ? __ldg(it.src + wi) : 0ull;
-}
+template <bool kTiles>
+__global__ void __launch_bounds__(THREADS, 1) k_train_forward_tc(const StepParams* __restrict__ P, int l);
 
 }  // namespace
 
 size_t train_forward_tc_smem() { return kSmemBytes; }
-dim3 train_forward_tc_grid(int Kout) { return dim3((unsigned)((Kout + TN - 1) / TN)); }
-dim3 train_forward_tc_block() { return dim3(THREADS); }
 
+cudaError_t prepare_train_forward_tc() {
+  cudaError_t e = cudaFuncSetAttribute(k_train_forward_tc<false>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
+  if (e != cudaSuccess) return e;
+  return cudaFuncSetAttribute(k_train_forward_tc<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              (int)kSmemBytes);
+}
+
+void launch_train_forward_tc(bool tiles, int Kout, cudaStream_t st, const StepParams* P, int l) {
+  const dim3 grid((unsigned)((Kout + TN - 1) / TN));
+  if (tiles)
+    k_train_forward_tc<true><<<grid, THREADS, kSmemBytes, st>>>(P, l);
+  else
+    k_train_forward_tc<false><<<grid, THREADS, kSmemBytes, st>>>(P, l);
+}
+
+size_t act_tile_bytes(int K) { return (size_t)((K + KB - 1) / KB) * A_BYTES; }
+
+namespace {
+
+template <bool kTiles>
 __global__ void __launch_bounds__(THREADS, 1) k_train_forward_tc(const StepParams* __restrict__ P, int l) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* base = reinterpret_cast<uint8_t*>(
@@ -199,7 +118,8 @@ __global__ void __launch_bounds__(THREADS, 1) k_train_forward_tc(const StepParam
   }
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
-      mbar_init(&sh->full[s], kProducers);
+      // kTiles: 2 NB B-producers arrive, plus the tile copy's expect_tx arrival
+      mbar_init(&sh->full[s], kTiles ? 2 * TN + 1 : kProducers);
       mbar_init(&sh->empty[s], 1);
     }
     mbar_init(&sh->done, 1);
@@ -217,10 +137,11 @@ __global__ void __launch_bounds__(THREADS, 1) k_train_forward_tc(const StepParam
   asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
   const uint32_t tmem = sh->tmem_base;
 
-  if (threadIdx.x < kProducers) {
+  if (threadIdx.x < (kTiles ? 2 * TN : kProducers)) {
     // ---------------- producers ----------------
-    // items: A rows [0, M) x 2 halves, then B rows [0, NB) x 2 halves
-    const int nA = 2 * M, nItems = nA + 2 * NB;
+    // items: A rows [0, M) x 2 halves (only without tiles), then B rows
+    // [0, NB) x 2 halves
+    const int nA = kTiles ? 0 : 2 * M, nItems = nA + 2 * NB;
     const int i = threadIdx.x;
     Item it;
     if (i < nA) {
@@ -244,6 +165,11 @@ __global__ void __launch_bounds__(THREADS, 1) k_train_forward_tc(const StepParam
         if (kb >= kStages && !mbar_wait(&sh->empty[s], (uint32_t)((kb / kStages - 1) & 1), failed))
           break;
         uint8_t* stage = base + s * STAGE_BYTES;
+        if (kTiles && threadIdx.x == 0) {
+          // A: the pre-expanded activation tile of this k-block
+          mbar_arrive_tx(&sh->full[s], A_BYTES);
+          bulk_g2s(stage, P->layer[l - 2].AE + (size_t)kb * A_BYTES, A_BYTES, &sh->full[s]);
+        }
         if (it.src != nullptr) {
           const int wi = 2 * kb + it.half;
           const int valid = min(64, max(0, Kin - 64 * wi));
@@ -255,8 +181,8 @@ __global__ void __launch_bounds__(THREADS, 1) k_train_forward_tc(const StepParam
       }
       if (*failed) break;
     }
-  } else if (lane == 0) {
-    // ---------------- MMA issuer ----------------
+  } else if (threadIdx.x == kProducers) {
+    // ---------------- MMA issuer (lane 0 of the last warp) ----------------
     for (int kb = 0; kb < nkb; ++kb) {
       const int s = kb % kStages;
       if (!mbar_wait(&sh->full[s], (uint32_t)((kb / kStages) & 1), failed)) break;
@@ -266,7 +192,7 @@ __global__ void __launch_bounds__(THREADS, 1) k_train_forward_tc(const StepParam
       const uint64_t bd = smem_desc(smem_u32(sa + A_BYTES));
 #pragma unroll
       for (int j = 0; j < KB / 32; ++j)   // K = 32 bytes per MMA: +2 in the address field
-        mma_f8(tmem, ad + 2 * j, bd + 2 * j, (kb > 0 || j > 0) ? 1u : 0u);
+        mma_f8<kIdesc>(tmem, ad + 2 * j, bd + 2 * j, (kb > 0 || j > 0) ? 1u : 0u);
       mma_commit(&sh->empty[s]);
     }
     if (!*failed) mma_commit(&sh->done);
@@ -305,6 +231,26 @@ __global__ void __launch_bounds__(THREADS, 1) k_train_forward_tc(const StepParam
         }
       }
       reinterpret_cast<uint16_t*>(Ly.A + (int64_t)m * Ly.nw_out + (n0 >> 6))[col0 >> 4] = (uint16_t)bits;
+      if (Ly.AE != nullptr) {
+        // the same 16 activations as e4m3 (+1 0x38, -1 0xB8, past N 0x00) in the
+        // swizzled tile image that the next layer's stages copy verbatim
+        const int nf = n0 + col0;
+        uint32_t q[4];
+#pragma unroll
+        for (int b = 0; b < 4; ++b) {
+          uint32_t word = 0;
+#pragma unroll
+          for (int j = 0; j < 4; ++j) {
+            const int jj = 4 * b + j;
+            const uint32_t e = (nf + jj < N) ? (((bits >> jj) & 1u) ? 0x38u : 0xB8u) : 0u;
+            word |= e << (8 * j);
+          }
+          q[b] = word;
+        }
+        const int c = (nf % KB) / 16;
+        uint8_t* dst = Ly.AE + (size_t)(nf / KB) * A_BYTES + (size_t)m * KB + 16 * (c ^ (m & 7));
+        *reinterpret_cast<uint4*>(dst) = make_uint4(q[0], q[1], q[2], q[3]);
+      }
     }
   }
   asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
@@ -314,4 +260,5 @@ __global__ void __launch_bounds__(THREADS, 1) k_train_forward_tc(const StepParam
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(TMEM_COLS) : "memory");
 }
 
+}  // namespace
 }  // namespace bk

@@ -115,8 +115,8 @@ __global__ void __launch_bounds__(kClsThreads) k_cls_select(const StepParams* __
 // CTA = (layer, group g, slice of kUpdRowsPerCta neurons).  A warp owns one
 // neuron row k at a time: it collects, in ascending mu, the patterns whose
 // selection in group g is k (the CP tuples of k), then streams the row in
-// chunks of 8 hidden weights, one 16-byte vector per lane, with a rotating
-// queue of four vectors in flight per lane.
+// chunks of 8 hidden weights, two chunks per lane per iteration, with a
+// rotating queue of four 16-byte vectors in flight per lane.
 // H holds each weight as its lattice index v = (h + h_max)/2 + 2^hb (see
 // DevLayer): a CP or R event is a step of +-1 in v, and v stays in
 // [2^hb, 2^hb + h_max] subset of (0, 2^15).  A 32-bit word holds two lanes, so a
@@ -258,6 +258,20 @@ struct Lanes {
     if (kPow2) return (v << (16 - hb)) & kLaneTop;
     return ((v | kLaneTop) - pos_pair) & kLaneTop;
   }
+  // W byte of a chunk (lane j -> bit j = h_j > 0)
+  __device__ __forceinline__ uint32_t w_byte(const uint4& w) const {
+    if (kPow2) {
+      // move each lane's sign bit (bit hb - 1) to bit 7 of the lane's low byte;
+      // the low bytes of the 8 lanes then hold the 8 sign bits at bit 7
+      const int sh = 8 - hb;
+      const uint32_t x = sh >= 0 ? w.x << sh : w.x >> -sh, y = sh >= 0 ? w.y << sh : w.y >> -sh;
+      const uint32_t z = sh >= 0 ? w.z << sh : w.z >> -sh, u = sh >= 0 ? w.w << sh : w.w >> -sh;
+      const uint32_t p0 = __byte_perm(x, y, 0x6420) & 0x80808080u;
+      const uint32_t p1 = __byte_perm(z, u, 0x6420) & 0x80808080u;
+      return ((p0 * 0x00204081u) >> 28) | (((p1 * 0x00204081u) >> 28) << 4);
+    }
+    return gather_top(pos_top(w.x), pos_top(w.y), pos_top(w.z), pos_top(w.w));
+  }
   // fired lanes step away from 0 (then clip)
   __device__ __forceinline__ uint32_t reinforce(uint32_t v, uint32_t fire_top) const {
     const uint32_t f = fire_top >> 15;
@@ -331,7 +345,6 @@ __global__ void __launch_bounds__(kUpdThreads, 3) k_update(const StepParams* __r
     const uint32_t arow_bytes = (uint32_t)Ly.nw_in * 8u;
     const uint8_t* aprev = (li == 0) ? reinterpret_cast<const uint8_t*>(P->x + start * P->nw0)
                                      : reinterpret_cast<const uint8_t*>(P->layer[li - 1].A);
-    const int iters = (nch + 31) >> 5;
 
     for (int rr = r0 + warp; rr < r1; rr += nwarps) {
       const int k = g * gamma + rr;
@@ -353,63 +366,93 @@ __global__ void __launch_bounds__(kUpdThreads, 3) k_update(const StepParams* __r
 
       int16_t* hrow = Ly.H + (int64_t)k * Ly.ldh;
       uint8_t* wrow = reinterpret_cast<uint8_t*>(Ly.W + (int64_t)k * Ly.nw_in);
-      // rotating queue of H vectors (chunks ch, ch + 32, ch + 64, ch + 96);
-      // every lane runs the same number of iterations (warp votes below)
+      // Each iteration handles two chunks per lane, ch and ch + 32 (64 chunks
+      // per warp), so the tuple loop and the loop control are shared and the
+      // two Philox chains run side by side.  A rotating queue keeps the H
+      // vectors of the next iteration in flight (4 per lane).  Every lane runs
+      // the same number of iterations (warp votes below).
       uint4 q0 = make_uint4(0, 0, 0, 0), q1 = q0, q2 = q0, q3 = q0;
       if (lane < nch) q0 = __ldcs(reinterpret_cast<const uint4*>(hrow + 8 * lane));
       if (lane + 32 < nch) q1 = __ldcs(reinterpret_cast<const uint4*>(hrow + 8 * (lane + 32)));
       if (lane + 64 < nch) q2 = __ldcs(reinterpret_cast<const uint4*>(hrow + 8 * (lane + 64)));
       if (lane + 96 < nch) q3 = __ldcs(reinterpret_cast<const uint4*>(hrow + 8 * (lane + 96)));
+      const int iters2 = (nch + 63) >> 6;
 #pragma unroll 1
-      for (int it = 0; it < iters; ++it) {
-        const int ch = 32 * it + lane;
-        const bool live = ch < nch;
-        const uint4 w_in = q0;
-        uint4 w = q0;
-        q0 = q1;
-        q1 = q2;
-        q2 = q3;
-        if (ch + 128 < nch) q3 = __ldcs(reinterpret_cast<const uint4*>(hrow + 8 * (ch + 128)));
-        const uint4 rh = philox4x32_10(make_uint4((uint32_t)ch, (uint32_t)k, c2_hi, tt), key0, key1);
-        const bool simd = packed && ch < full;   // this lane's chunk runs on packed lanes
+      for (int it = 0; it < iters2; ++it) {
+        int chv[2];
+        bool live[2], simd[2];
+        uint4 w_in[2], w[2], rh[2];
+        chv[0] = 64 * it + lane;
+        chv[1] = chv[0] + 32;
+        w_in[0] = q0;
+        w_in[1] = q1;
+        q0 = q2;
+        q1 = q3;
+        if (chv[0] + 128 < nch) q2 = __ldcs(reinterpret_cast<const uint4*>(hrow + 8 * (chv[0] + 128)));
+        if (chv[1] + 128 < nch) q3 = __ldcs(reinterpret_cast<const uint4*>(hrow + 8 * (chv[1] + 128)));
+#pragma unroll
+        for (int u = 0; u < 2; ++u) {
+          live[u] = chv[u] < nch;
+          simd[u] = packed && chv[u] < full;   // this chunk runs on packed lanes
+          w[u] = w_in[u];
+          rh[u] = philox4x32_10(make_uint4((uint32_t)chv[u], (uint32_t)k, c2_hi, tt), key0, key1);
+        }
         // ---- Clipped Perceptron ----
 #pragma unroll 1
         for (int q = 0; q < n_t; ++q) {
           const int e = s_list[q];
-          const uint32_t byte = live ? aprev[(size_t)(e & 0xFFFF) * arow_bytes + ch] : 0u;
           const uint2* dn = s_dn[(e >> 16) & 1];
-          const uint2 dl = dn[byte & 15u], dh = dn[byte >> 4];
-          w.x = LN.clip(w.x + dl.x);
-          w.y = LN.clip(w.y + dl.y);
-          w.z = LN.clip(w.z + dh.x);
-          w.w = LN.clip(w.w + dh.y);
+          const uint8_t* arow = aprev + (size_t)(e & 0xFFFF) * arow_bytes;
+#pragma unroll
+          for (int u = 0; u < 2; ++u) {
+            const uint32_t byte = live[u] ? arow[chv[u]] : 0u;
+            const uint2 dl = dn[byte & 15u], dh = dn[byte >> 4];
+            w[u].x = LN.clip(w[u].x + dl.x);
+            w[u].y = LN.clip(w[u].y + dl.y);
+            w[u].z = LN.clip(w[u].z + dh.x);
+            w[u].w = LN.clip(w[u].w + dh.y);
+          }
         }
-        // ---- Reinforcement ----
-        const uint32_t tie = simd ? (tie_any(rh.x, Tpair) | tie_any(rh.y, Tpair) |
-                                     tie_any(rh.z, Tpair) | tie_any(rh.w, Tpair)) : 1u;
-        const bool slow = live && (tie != 0u);
-        const uint4 f = make_uint4(fire_flags(rh.x, Tpair), fire_flags(rh.y, Tpair),
-                                   fire_flags(rh.z, Tpair), fire_flags(rh.w, Tpair));
-        const bool fires = live && !slow && ((f.x | f.y | f.z | f.w) != 0u);
-        if (__any_sync(kFull, fires) && fires) {
-          w.x = LN.reinforce(w.x, f.x);
-          w.y = LN.reinforce(w.y, f.y);
-          w.z = LN.reinforce(w.z, f.z);
-          w.w = LN.reinforce(w.w, f.w);
+        // ---- Reinforcement, W ----
+        uint4 f[2];
+        bool slow[2], fires[2];
+#pragma unroll
+        for (int u = 0; u < 2; ++u) {
+          const uint32_t tie = simd[u] ? (tie_any(rh[u].x, Tpair) | tie_any(rh[u].y, Tpair) |
+                                          tie_any(rh[u].z, Tpair) | tie_any(rh[u].w, Tpair)) : 1u;
+          slow[u] = live[u] && (tie != 0u);
+          f[u] = make_uint4(fire_flags(rh[u].x, Tpair), fire_flags(rh[u].y, Tpair),
+                            fire_flags(rh[u].z, Tpair), fire_flags(rh[u].w, Tpair));
+          fires[u] = live[u] && !slow[u] && ((f[u].x | f[u].y | f[u].z | f[u].w) != 0u);
         }
-        uint32_t wbyte = gather_top(LN.pos_top(w.x), LN.pos_top(w.y), LN.pos_top(w.z), LN.pos_top(w.w));
-        if (slow) {
-          // a packed chunk with a tie keeps its packed CP result; any other chunk
-          // restarts from the loaded values and the per-weight path does it all
-          const ChunkOut o = chunk_scalar(simd ? w : w_in, ch, min(8, Kin - 8 * ch), simd, s_list,
-                                          n_t, aprev, arow_bytes, E, Thi, Tlo, key0, key1,
-                                          (uint32_t)k, c2_lo, tt, rh);
-          w = o.w;
-          wbyte = o.wbyte;
+        if (__any_sync(kFull, fires[0] || fires[1])) {
+#pragma unroll
+          for (int u = 0; u < 2; ++u) {
+            if (fires[u]) {
+              w[u].x = LN.reinforce(w[u].x, f[u].x);
+              w[u].y = LN.reinforce(w[u].y, f[u].y);
+              w[u].z = LN.reinforce(w[u].z, f[u].z);
+              w[u].w = LN.reinforce(w[u].w, f[u].w);
+            }
+          }
         }
-        if (live) {
-          __stcs(reinterpret_cast<uint4*>(hrow + 8 * ch), w);
-          wrow[ch] = (uint8_t)wbyte;
+#pragma unroll
+        for (int u = 0; u < 2; ++u) {
+          uint32_t wbyte = LN.w_byte(w[u]);
+          if (slow[u]) {
+            // a packed chunk with a tie keeps its packed CP result; any other
+            // chunk restarts from the loaded values and the per-weight path
+            // does it all
+            const ChunkOut o = chunk_scalar(simd[u] ? w[u] : w_in[u], chv[u], min(8, Kin - 8 * chv[u]),
+                                            simd[u], s_list, n_t, aprev, arow_bytes, E, Thi, Tlo,
+                                            key0, key1, (uint32_t)k, c2_lo, tt, rh[u]);
+            w[u] = o.w;
+            wbyte = o.wbyte;
+          }
+          if (live[u]) {
+            __stcs(reinterpret_cast<uint4*>(hrow + 8 * chv[u]), w[u]);
+            wrow[chv[u]] = (uint8_t)wbyte;
+          }
         }
       }
       __syncwarp();

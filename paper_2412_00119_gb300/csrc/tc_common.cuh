@@ -1,0 +1,144 @@
+// tc_common.cuh -- device helpers shared by the tcgen05 forward kernels:
+// mbarrier waits (bounded), shared-memory matrix descriptors, the
+// tcgen05.mma kind::f8f6f4 issue and commit, and the expansion of bit-packed
+// +-1 vectors into e4m3 bytes in the 128B-swizzled K-major stage layout.
+#pragma once
+
+#include "bmlp_internal.cuh"
+
+namespace bk {
+namespace tc {
+
+constexpr int KB = 128;  // K elements (bytes of e4m3) per stage row
+constexpr unsigned long long kWaitCycles = 4000000000ull;  // ~2 s at 2 GHz
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ void mbar_init(unsigned long long* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count));
+}
+
+__device__ __forceinline__ void mbar_arrive(unsigned long long* bar) {
+  asm volatile("{\n .reg .b64 st;\n mbarrier.arrive.shared::cta.b64 st, [%0];\n}"
+               ::"r"(smem_u32(bar)) : "memory");
+}
+
+// Bounded wait for the phase with the given parity; false on expiry or when
+// another thread already recorded a failure.
+__device__ __forceinline__ bool mbar_wait(unsigned long long* bar, uint32_t parity,
+                                          volatile int* failed) {
+  const uint32_t a = smem_u32(bar);
+  const unsigned long long t0 = clock64();
+  while (true) {
+    uint32_t ok;
+    asm volatile(
+        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+        " selp.u32 %0, 1, 0, p;\n}"
+        : "=r"(ok) : "r"(a), "r"(parity) : "memory");
+    if (ok) return true;
+    if (*failed) return false;
+    if (clock64() - t0 > kWaitCycles) {
+      *failed = 1;
+      return false;
+    }
+  }
+}
+
+// Shared-memory matrix descriptor: K-major, SWIZZLE_128B, 8-row groups 1024 B apart.
+__device__ __forceinline__ uint64_t smem_desc(uint32_t saddr) {
+  uint64_t d = 0;
+  d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);           // start address
+  d |= (uint64_t)1 << 16;                              // leading byte offset (unused for SW128 K-major)
+  d |= (uint64_t)(1024 >> 4) << 32;                    // stride byte offset
+  d |= (uint64_t)1 << 46;                              // descriptor version (sm_100 family)
+  d |= (uint64_t)2 << 61;                              // swizzle: 128B
+  return d;
+}
+
+// Instruction descriptor, kind::f8f6f4: D fp32, A = B = e4m3, both K-major,
+// M x N per instruction (K = 32).
+constexpr uint32_t idesc_f8(int M, int N) {
+  return (1u << 4)                        // D format: f32
+         | (0u << 7) | (0u << 10)         // A, B format: e4m3
+         | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+}
+
+template <uint32_t kIdesc>
+__device__ __forceinline__ void mma_f8(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc,
+                                       uint32_t accumulate) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], %1, %2, %3, p;\n}"
+      ::"r"(tmem_d), "l"(adesc), "l"(bdesc), "r"(kIdesc), "r"(accumulate));
+}
+
+__device__ __forceinline__ void mma_commit(unsigned long long* bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];"
+               ::"r"(smem_u32(bar)) : "memory");
+}
+
+// 8 bits -> 8 e4m3 bytes (+1 = 0x38, -1 = 0xB8) as two words.  Byte j of the
+// replicated value keeps bit j of b; adding (0x80 - 2^j) per byte moves it to
+// bit 7 without carries between bytes.
+__device__ __forceinline__ uint2 expand8(uint32_t b) {
+  const uint32_t rep = b * 0x01010101u;
+  const uint32_t lo = (rep & 0x08040201u) + 0x787C7E7Fu;
+  const uint32_t hi = (rep & 0x80402010u) + 0x00406070u;
+  return make_uint2((lo & 0x80808080u) ^ 0xB8B8B8B8u, (hi & 0x80808080u) ^ 0xB8B8B8B8u);
+}
+
+// Expand one 64-bit word (64 K-elements) into four 16-byte chunks of row r of
+// a swizzled stage, chunks chunk0 .. chunk0+3.  `valid` = real elements (0..64).
+__device__ __forceinline__ void expand_word(uint8_t* row_base, int r, int chunk0, uint64_t w,
+                                            int valid) {
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {        // chunk q: elements 16q .. 16q+15
+    const uint32_t bits = (uint32_t)(w >> (16 * q)) & 0xFFFFu;
+    const uint2 e0 = expand8(bits & 0xFF);
+    const uint2 e1 = expand8(bits >> 8);
+    uint4 v = make_uint4(e0.x, e0.y, e1.x, e1.y);
+    if (valid < 64) {
+      uint32_t* vv = &v.x;
+#pragma unroll
+      for (int b = 0; b < 4; ++b) {
+        const int n_ok = valid - (16 * q + 4 * b);  // real elements in this 4-byte group
+        const uint32_t keep = n_ok >= 4 ? 0xFFFFFFFFu : (n_ok <= 0 ? 0u : ((1u << (8 * n_ok)) - 1u));
+        vv[b] &= keep;
+      }
+    }
+    const int c = chunk0 + q;
+    *reinterpret_cast<uint4*>(row_base + 16 * (c ^ (r & 7))) = v;
+  }
+}
+
+
+__device__ __forceinline__ void mbar_arrive_tx(unsigned long long* bar, uint32_t bytes) {
+  asm volatile("{\n .reg .b64 st;\n mbarrier.arrive.expect_tx.shared::cta.b64 st, [%0], %1;\n}"
+               ::"r"(smem_u32(bar)), "r"(bytes) : "memory");
+}
+
+// 1-D bulk copy global -> this CTA's shared memory, completing on `bar`
+__device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes,
+                                         unsigned long long* bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+      ::"r"(smem_u32(dst)), "l"(src), "r"(bytes), "r"(smem_u32(bar)) : "memory");
+}
+
+// A producer item: one (matrix, row, half) of the current tile.
+struct Item {
+  const uint64_t* src;  // row start (bit words), or null when the thread has no item
+  int soff;             // byte offset of the row inside a stage (A or B part)
+  int r;                // row index inside its matrix (for the swizzle)
+  int half;             // which of the stage's two words
+};
+
+__device__ __forceinline__ uint64_t load_word(const Item& it, int kb, int nw) {
+  const int wi = 2 * kb + it.half;
+  return (it.src != nullptr && wi < nw) ? __ldg(it.src + wi) : 0ull;
+}
+
+}  // namespace tc
+}  // namespace bk

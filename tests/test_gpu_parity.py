@@ -107,6 +107,29 @@ def test_forward_single_tile(engine):
         gpu.close()
 
 
+# (widths, n): one tile, exact tiles, ragged K / neurons / patterns over several
+# 128 x 256 evaluation tiles, and an 8192 -> 8192 layer.
+LAYER_CASES = [((1, 8), 5), ((64, 64), 128), ((130, 257, 129), 129), ((1100, 700, 300), 1000),
+               ((8192, 8192), 300)]
+
+
+@pytest.mark.parametrize("engine", sorted(ENGINES))
+@pytest.mark.parametrize("widths,n", LAYER_CASES)
+def test_layer_forward_eval(widths, n, engine):
+    """Forward-only layer evaluation: every packed activation bit (pads 0)
+    equals the oracle's sign(a_{l-1} W_l) of Alg. 1 l.8-9."""
+    gpu = B.BMLP(widths, 4, seed=9, bs=64, fwd_impl=ENGINES[engine])
+    ref = O.OracleModel(list(widths), 4, seed=9, bs=64)
+    for l in range(1, len(widths)):
+        xp = W.random_packed(100 * l + n, n, widths[l - 1])
+        out = torch.full((n, W.words(widths[l])), -1, dtype=torch.int64, device=DEV)
+        B.bmlp_layer_forward(gpu.h, l, dev_x(xp), out)
+        _, a = O.layer_forward(W.unpack(xp, widths[l - 1]), ref.H(l))
+        got = out.cpu().numpy().view(np.uint64)
+        assert np.array_equal(got, W.pack(a)), (engine, widths, l)
+    gpu.close()
+
+
 CASES = {
     "ragged_3layer": dict(widths=(200, 130, 70), classes=10, n_train=300, bs=50, gamma=[13, 7]),
     "tail_batch": dict(widths=(64, 64), classes=4, n_train=250),

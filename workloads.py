@@ -124,6 +124,11 @@ def _iid_packed(rng, n, K):
     return xp
 
 
+def random_packed(seed: int, n: int, K: int) -> np.ndarray:
+    """n packed rows of K i.i.d. fair +-1 values (pad bits 0), seeded."""
+    return _iid_packed(np.random.default_rng(seed), n, K)
+
+
 # -- teacher -------------------------------------------------------------------
 
 @dataclasses.dataclass
