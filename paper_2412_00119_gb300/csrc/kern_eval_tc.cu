@@ -70,7 +70,7 @@ __global__ void __launch_bounds__(THREADS, 1)
   }
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
-      mbar_init(&sh->full[s], kProducers);
+      mbar_init(&sh->full[s], kProducers / 32);  // one arrival per producer warp
       mbar_init(&sh->empty[s], 1);
     }
     mbar_init(&sh->done, 1);
@@ -116,7 +116,8 @@ __global__ void __launch_bounds__(THREADS, 1)
         const int kb = kb0 + d;
         if (kb >= nkb) break;
         const int s = kb % kStages;
-        if (kb >= kStages && !mbar_wait(&sh->empty[s], (uint32_t)((kb / kStages - 1) & 1), failed))
+        if (kb >= kStages &&
+            !__all_sync(kFull, mbar_wait(&sh->empty[s], (uint32_t)((kb / kStages - 1) & 1), failed)))
           break;
         uint8_t* stage = base + s * STAGE_BYTES;
 #pragma unroll
@@ -129,9 +130,10 @@ __global__ void __launch_bounds__(THREADS, 1)
           pre[d][j] = load_word(it[j], kb + kPrefetch, nw);
         }
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-        mbar_arrive(&sh->full[s]);
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&sh->full[s]);
       }
-      if (*failed) break;
+      if (__any_sync(kFull, *failed != 0)) break;
     }
   } else if (threadIdx.x == kProducers) {
     // MMA issuer: lane 0 of the last warp

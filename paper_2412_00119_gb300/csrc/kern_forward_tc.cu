@@ -19,7 +19,8 @@
 //     MMA reads (16-byte chunk c of row r stored at chunk c ^ (r % 8)).  Each
 //     thread owns at most one (row, half) item (2 x 128 + 2 x 64 <= 512); its
 //     64-bit words are loaded kPrefetch stages ahead into registers, so the
-//     L2 latency is off the critical path.  A producer arrives on the stage's "full" mbarrier.
+//     L2 latency is off the critical path.  Each producer warp arrives once on
+//     the stage's "full" mbarrier, after every lane's proxy fence.
 //   - 1 MMA warp waits on "full", issues tcgen05.mma.kind::f8f6f4 (M = 128,
 //     N = 64, K = 32) four times per stage into a 128-lane x 64-column fp32
 //     accumulator in TMEM, and commits to the stage's "empty" mbarrier, on
@@ -118,8 +119,9 @@ __global__ void __launch_bounds__(THREADS, 1) k_train_forward_tc(const StepParam
   }
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
-      // kTiles: 2 NB B-producers arrive, plus the tile copy's expect_tx arrival
-      mbar_init(&sh->full[s], kTiles ? 2 * TN + 1 : kProducers);
+      // one arrival per producer warp; kTiles: 4 B-producer warps plus the
+      // tile copy's expect_tx arrival
+      mbar_init(&sh->full[s], kTiles ? 2 * TN / 32 + 1 : kProducers / 32);
       mbar_init(&sh->empty[s], 1);
     }
     mbar_init(&sh->done, 1);
@@ -162,7 +164,8 @@ __global__ void __launch_bounds__(THREADS, 1) k_train_forward_tc(const StepParam
         const int kb = kb0 + d;
         if (kb >= nkb) break;
         const int s = kb % kStages;
-        if (kb >= kStages && !mbar_wait(&sh->empty[s], (uint32_t)((kb / kStages - 1) & 1), failed))
+        if (kb >= kStages &&
+            !__all_sync(kFull, mbar_wait(&sh->empty[s], (uint32_t)((kb / kStages - 1) & 1), failed)))
           break;
         uint8_t* stage = base + s * STAGE_BYTES;
         if (kTiles && threadIdx.x == 0) {
@@ -176,10 +179,12 @@ __global__ void __launch_bounds__(THREADS, 1) k_train_forward_tc(const StepParam
           expand_word(stage + it.soff, it.r, 4 * it.half, pre[d], valid);
         }
         pre[d] = load_word(it, kb + kPrefetch, nw);
+        // every writer orders its stores for the async proxy; one arrival per warp
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-        mbar_arrive(&sh->full[s]);
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&sh->full[s]);
       }
-      if (*failed) break;
+      if (__any_sync(kFull, *failed != 0)) break;
     }
   } else if (threadIdx.x == kProducers) {
     // ---------------- MMA issuer (lane 0 of the last warp) ----------------

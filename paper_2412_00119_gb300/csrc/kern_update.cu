@@ -143,6 +143,7 @@ namespace {
 constexpr uint32_t kLaneTop = 0x80008000u;
 constexpr uint32_t kLaneOne = 0x00010001u;
 constexpr unsigned kFull = 0xffffffffu;
+constexpr int kPre = 4;  // tuples per row whose activation bytes are prefetched
 
 __device__ __forceinline__ uint32_t lane_v(const uint4& w, int j) {
   const uint32_t word = (j < 2) ? w.x : (j < 4) ? w.y : (j < 6) ? w.z : w.w;
@@ -169,26 +170,24 @@ struct Enc {
   __device__ __forceinline__ uint32_t enc(int h) const { return (uint32_t)((h + h_max) / 2 + base); }
 };
 
-// Per-weight path (rule as printed, on decoded h): CP (unless `cp_done`), R
-// and W for the first `nvalid` weights of the chunk.  Rarely taken; its loops
-// stay rolled.
-__device__ __forceinline__ ChunkOut chunk_scalar(uint4 w, int ch, int nvalid, bool cp_done,
+// Per-weight path (rule as printed, on decoded h): CP, R and W for the first
+// `nvalid` weights of the chunk, from the loaded values.  Rarely taken; its
+// loops stay rolled.
+__device__ __forceinline__ ChunkOut chunk_scalar(uint4 w, int ch, int nvalid,
                                                  const int32_t* list, int n_t, const uint8_t* aprev,
                                                  uint32_t arow_bytes, Enc E, uint32_t Thi,
                                                  uint32_t Tlo, uint32_t key0, uint32_t key1,
                                                  uint32_t k, uint32_t c2_lo, uint32_t t, uint4 rh) {
-  if (!cp_done) {
 #pragma unroll 1
-    for (int q = 0; q < n_t; ++q) {
-      const int e = list[q];
-      const int m = e & 0xFFFF;
-      const int rho = (e & 0x10000) ? -1 : 1;
-      const uint32_t byte = aprev[(size_t)m * arow_bytes + ch];
+  for (int q = 0; q < n_t; ++q) {
+    const int e = list[q];
+    const int m = e & 0xFFFF;
+    const int rho = (e & 0x10000) ? -1 : 1;
+    const uint32_t byte = aprev[(size_t)m * arow_bytes + ch];
 #pragma unroll 1
-      for (int j = 0; j < nvalid; ++j) {
-        const int step = ((byte >> j) & 1u) ? rho : -rho;
-        set_lane_v(w, j, E.enc(clip_h(E.dec(lane_v(w, j)) + 2 * step, E.h_max)));
-      }
+    for (int j = 0; j < nvalid; ++j) {
+      const int step = ((byte >> j) & 1u) ? rho : -rho;
+      set_lane_v(w, j, E.enc(clip_h(E.dec(lane_v(w, j)) + 2 * step, E.h_max)));
     }
   }
   uint32_t ties = 0;
@@ -232,10 +231,10 @@ __device__ __forceinline__ uint32_t fire_flags(uint32_t u, uint32_t Tpair) {
   return ~(dd | u) & kLaneTop;
 }
 
-// nonzero iff some lane of a draw word equals Thi
-__device__ __forceinline__ uint32_t tie_any(uint32_t u, uint32_t Tpair) {
-  const uint32_t x = u ^ Tpair;
-  return (x - kLaneOne) & ~x & kLaneTop;
+// lanes of a draw word whose high half u <= Thi (< 2^15): the same test
+// against T1pair = pair(Thi + 1), Thi + 1 <= 2^15
+__device__ __forceinline__ uint32_t le_flags(uint32_t u, uint32_t T1pair) {
+  return fire_flags(u, T1pair);
 }
 
 template <bool kPow2>
@@ -336,6 +335,7 @@ __global__ void __launch_bounds__(kUpdThreads, 3) k_update(const StepParams* __r
     const uint32_t Thi = (uint32_t)(T >> 16);   // 0..65536
     const uint32_t Tlo = (uint32_t)(T & 0xFFFFu);
     const uint32_t Tpair = Thi * kLaneOne;
+    const uint32_t T1pair = (Thi + 1u) * kLaneOne;  // used only when packed
     const bool packed = Thi < 0x8000u;           // the SIMD draw test is exact
     const uint32_t c2_hi = (3u << 16) + l, c2_lo = (4u << 16) + l;
     const uint32_t tt = (uint32_t)t;
@@ -366,6 +366,9 @@ __global__ void __launch_bounds__(kUpdThreads, 3) k_update(const StepParams* __r
 
       int16_t* hrow = Ly.H + (int64_t)k * Ly.ldh;
       uint8_t* wrow = reinterpret_cast<uint8_t*>(Ly.W + (int64_t)k * Ly.nw_in);
+      // the activation bytes of the first kPre tuples are fetched at the top of
+      // each iteration, ahead of the Philox chains, so that their latency
+      // overlaps the draw
       // Each iteration handles two chunks per lane, ch and ch + 32 (64 chunks
       // per warp), so the tuple loop and the loop control are shared and the
       // two Philox chains run side by side.  A rotating queue keeps the H
@@ -380,26 +383,52 @@ __global__ void __launch_bounds__(kUpdThreads, 3) k_update(const StepParams* __r
 #pragma unroll 1
       for (int it = 0; it < iters2; ++it) {
         int chv[2];
-        bool live[2], simd[2];
-        uint4 w_in[2], w[2], rh[2];
+        bool live[2], simd[2], slow[2];
+        uint4 w[2], rh[2];
+        uint32_t pb[2] = {0u, 0u};  // activation bytes of tuples 0..kPre-1, one per byte
         chv[0] = 64 * it + lane;
         chv[1] = chv[0] + 32;
-        w_in[0] = q0;
-        w_in[1] = q1;
+        live[0] = chv[0] < nch;
+        live[1] = chv[1] < nch;
+#pragma unroll
+        for (int q = 0; q < kPre; ++q) {
+          if (q < n_t) {
+            const uint8_t* arow = aprev + (size_t)(s_list[q] & 0xFFFF) * arow_bytes;
+#pragma unroll
+            for (int u = 0; u < 2; ++u)
+              if (live[u]) pb[u] |= (uint32_t)__ldg(arow + chv[u]) << (8 * q);
+          }
+        }
+        w[0] = q0;
+        w[1] = q1;
         q0 = q2;
         q1 = q3;
         if (chv[0] + 128 < nch) q2 = __ldcs(reinterpret_cast<const uint4*>(hrow + 8 * (chv[0] + 128)));
         if (chv[1] + 128 < nch) q3 = __ldcs(reinterpret_cast<const uint4*>(hrow + 8 * (chv[1] + 128)));
 #pragma unroll
         for (int u = 0; u < 2; ++u) {
-          live[u] = chv[u] < nch;
           simd[u] = packed && chv[u] < full;   // this chunk runs on packed lanes
-          w[u] = w_in[u];
+          slow[u] = live[u] && !simd[u];
           rh[u] = philox4x32_10(make_uint4((uint32_t)chv[u], (uint32_t)k, c2_hi, tt), key0, key1);
         }
         // ---- Clipped Perceptron ----
+#pragma unroll
+        for (int q = 0; q < kPre; ++q) {
+          if (q < n_t) {
+            const uint2* dn = s_dn[(s_list[q] >> 16) & 1];
+#pragma unroll
+            for (int u = 0; u < 2; ++u) {
+              const uint32_t byte = (pb[u] >> (8 * q)) & 0xFFu;
+              const uint2 dl = dn[byte & 15u], dh = dn[byte >> 4];
+              w[u].x = LN.clip(w[u].x + dl.x);
+              w[u].y = LN.clip(w[u].y + dl.y);
+              w[u].z = LN.clip(w[u].z + dh.x);
+              w[u].w = LN.clip(w[u].w + dh.y);
+            }
+          }
+        }
 #pragma unroll 1
-        for (int q = 0; q < n_t; ++q) {
+        for (int q = kPre; q < n_t; ++q) {
           const int e = s_list[q];
           const uint2* dn = s_dn[(e >> 16) & 1];
           const uint8_t* arow = aprev + (size_t)(e & 0xFFFF) * arow_bytes;
@@ -413,39 +442,37 @@ __global__ void __launch_bounds__(kUpdThreads, 3) k_update(const StepParams* __r
             w[u].w = LN.clip(w[u].w + dh.y);
           }
         }
-        // ---- Reinforcement, W ----
-        uint4 f[2];
-        bool slow[2], fires[2];
+        // ---- Reinforcement: per draw word, only where some lane of the warp
+        // has a candidate (draw high half <= Thi); a tie (== Thi) sends the
+        // chunk to the per-weight path, which restarts from the loaded values.
 #pragma unroll
         for (int u = 0; u < 2; ++u) {
-          const uint32_t tie = simd[u] ? (tie_any(rh[u].x, Tpair) | tie_any(rh[u].y, Tpair) |
-                                          tie_any(rh[u].z, Tpair) | tie_any(rh[u].w, Tpair)) : 1u;
-          slow[u] = live[u] && (tie != 0u);
-          f[u] = make_uint4(fire_flags(rh[u].x, Tpair), fire_flags(rh[u].y, Tpair),
-                            fire_flags(rh[u].z, Tpair), fire_flags(rh[u].w, Tpair));
-          fires[u] = live[u] && !slow[u] && ((f[u].x | f[u].y | f[u].z | f[u].w) != 0u);
-        }
-        if (__any_sync(kFull, fires[0] || fires[1])) {
+          const bool on = live[u] && simd[u];
+          uint32_t* wv = reinterpret_cast<uint32_t*>(&w[u]);
+          const uint32_t* rv = reinterpret_cast<const uint32_t*>(&rh[u]);
 #pragma unroll
-          for (int u = 0; u < 2; ++u) {
-            if (fires[u]) {
-              w[u].x = LN.reinforce(w[u].x, f[u].x);
-              w[u].y = LN.reinforce(w[u].y, f[u].y);
-              w[u].z = LN.reinforce(w[u].z, f[u].z);
-              w[u].w = LN.reinforce(w[u].w, f[u].w);
+          for (int j = 0; j < 4; ++j) {
+            const uint32_t cand = on ? le_flags(rv[j], T1pair) : 0u;
+            if (__any_sync(kFull, cand != 0u)) {
+              if (cand != 0u) {
+                const uint32_t fire = fire_flags(rv[j], Tpair);
+                if (cand & ~fire) slow[u] = true;
+                else wv[j] = LN.reinforce(wv[j], fire);
+              }
             }
           }
         }
+        // ---- W, store ----
 #pragma unroll
         for (int u = 0; u < 2; ++u) {
           uint32_t wbyte = LN.w_byte(w[u]);
           if (slow[u]) {
-            // a packed chunk with a tie keeps its packed CP result; any other
-            // chunk restarts from the loaded values and the per-weight path
-            // does it all
-            const ChunkOut o = chunk_scalar(simd[u] ? w[u] : w_in[u], chv[u], min(8, Kin - 8 * chv[u]),
-                                            simd[u], s_list, n_t, aprev, arow_bytes, E, Thi, Tlo,
-                                            key0, key1, (uint32_t)k, c2_lo, tt, rh[u]);
+            // the per-weight path restarts from the row as loaded (H is
+            // written back only below)
+            const uint4 w0 = *reinterpret_cast<const uint4*>(hrow + 8 * chv[u]);
+            const ChunkOut o = chunk_scalar(w0, chv[u], min(8, Kin - 8 * chv[u]), s_list, n_t,
+                                            aprev, arow_bytes, E, Thi, Tlo, key0, key1, (uint32_t)k,
+                                            c2_lo, tt, rh[u]);
             w[u] = o.w;
             wbyte = o.wbyte;
           }

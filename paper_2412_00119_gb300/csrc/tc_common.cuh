@@ -9,6 +9,7 @@
 namespace bk {
 namespace tc {
 
+constexpr unsigned kFull = 0xffffffffu;
 constexpr int KB = 128;  // K elements (bytes of e4m3) per stage row
 constexpr unsigned long long kWaitCycles = 4000000000ull;  // ~2 s at 2 GHz
 
