@@ -51,8 +51,8 @@ EVAL_BATCH = 65_536
 # HBM traffic of k_update per launch from the committed ncu capture
 # (profiles/k_update_c5.md), valid while the kernel source hashes to
 # UPDATE_TRAFFIC_SRC_SHA; otherwise reported as null.
-UPDATE_TRAFFIC_BYTES = None
-UPDATE_TRAFFIC_SRC_SHA = None
+UPDATE_TRAFFIC_BYTES = 537_796_608 + 509_770_240  # dram read + write, one launch (profiles/k_update_c5.md)
+UPDATE_TRAFFIC_SRC_SHA = "64595062a208f6c7"
 
 
 def bitpairs_per_sample(widths, classes):
