@@ -5,8 +5,9 @@
 // pads 0, fp32 sums exact), tiled for large batches: a CTA computes 128
 // patterns x 256 neurons over the whole K range.
 //   - 16 producer warps expand bit-packed activations (128 rows) and visible
-//     weights (256 rows) into 128B-swizzled K-major stages of 48 KB, two
-//     (row, half) items per thread, bit words prefetched kPrefetch stages ahead;
+//     weights (256 rows) into 128B-swizzled K-major stages of 48 KB: every
+//     thread owns six 16-byte chunks of the stage (16 bits each), loaded
+//     kPrefetch stages ahead;
 //   - 1 MMA warp issues tcgen05.mma.kind::f8f6f4 M128 N256 K32 (four per stage)
 //     into a 128 x 256 fp32 accumulator in TMEM (256 columns) and commits to
 //     the stage's "empty" mbarrier (4-stage ring);
@@ -25,8 +26,9 @@ using namespace tc;
 constexpr int TM = 128;
 constexpr int TN = 256;
 constexpr int kStages = 4;
-constexpr int kPrefetch = 4;
+constexpr int kPrefetch = 3;
 constexpr int kProducers = 512;
+constexpr int kItems = 8 * (TM + TN) / kProducers;  // 16-byte chunks per producer thread
 constexpr int THREADS = kProducers + 32;
 constexpr int A_BYTES = TM * KB;   // 16 KB
 constexpr int B_BYTES = TN * KB;   // 32 KB
@@ -89,26 +91,27 @@ __global__ void __launch_bounds__(THREADS, 1)
   const uint32_t tmem = sh->tmem_base;
 
   if (threadIdx.x < kProducers) {
-    // items: A rows [0, MR) x 2 halves, then B rows [0, NB) x 2 halves
-    const int nA = 2 * MR, nItems = nA + 2 * NB;
-    Item it[2];
+    // items: the 16-byte chunks of A rows [0, MR), then of B rows [0, NB);
+    // item i belongs to thread i % kProducers
+    const int nA = 8 * MR, nItems = nA + 8 * NB;
+    Chunk ch[kItems];
 #pragma unroll
-    for (int j = 0; j < 2; ++j) {
+    for (int j = 0; j < kItems; ++j) {
       const int i = threadIdx.x + j * kProducers;
       if (i < nA) {
-        it[j] = Item{A + (m0 + (i >> 1)) * nw, (i >> 1) * KB, i >> 1, i & 1};
+        ch[j] = make_chunk(A + (m0 + (i >> 3)) * nw, 0, i >> 3, i & 7);
       } else if (i < nItems) {
         const int b = i - nA;
-        it[j] = Item{W + (int64_t)(n0 + (b >> 1)) * nw, A_BYTES + (b >> 1) * KB, b >> 1, b & 1};
+        ch[j] = make_chunk(W + (int64_t)(n0 + (b >> 3)) * nw, A_BYTES, b >> 3, b & 7);
       } else {
-        it[j] = Item{nullptr, 0, 0, 0};
+        ch[j] = Chunk{nullptr, 0u, 0};
       }
     }
-    uint64_t pre[kPrefetch][2];
+    uint32_t pre[kPrefetch][kItems];
 #pragma unroll
     for (int d = 0; d < kPrefetch; ++d)
 #pragma unroll
-      for (int j = 0; j < 2; ++j) pre[d][j] = load_word(it[j], d, nw);
+      for (int j = 0; j < kItems; ++j) pre[d][j] = load_chunk(ch[j], d, nw);
 
     for (int kb0 = 0; kb0 < nkb; kb0 += kPrefetch) {
 #pragma unroll
@@ -121,13 +124,9 @@ __global__ void __launch_bounds__(THREADS, 1)
           break;
         uint8_t* stage = base + s * STAGE_BYTES;
 #pragma unroll
-        for (int j = 0; j < 2; ++j) {
-          if (it[j].src != nullptr) {
-            const int wi = 2 * kb + it[j].half;
-            const int valid = min(64, max(0, Kin - 64 * wi));
-            expand_word(stage + it[j].soff, it[j].r, 4 * it[j].half, pre[d][j], valid);
-          }
-          pre[d][j] = load_word(it[j], kb + kPrefetch, nw);
+        for (int j = 0; j < kItems; ++j) {
+          if (ch[j].src != nullptr) store_chunk(stage, ch[j], pre[d][j], kb, Kin);
+          pre[d][j] = load_chunk(ch[j], kb + kPrefetch, nw);
         }
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
         __syncwarp();

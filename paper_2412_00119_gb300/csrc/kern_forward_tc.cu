@@ -14,13 +14,14 @@
 // stage's "full" mbarrier.  For layer 1 (the caller's bit-packed input) and in
 // general:
 //   - 16 producer warps expand the bit-packed activations (A, patterns x
-//     words) and visible weights (W, neurons x words), 128 K-elements (two
-//     64-bit words) per row per stage, into the K-major SWIZZLE_128B layout the
-//     MMA reads (16-byte chunk c of row r stored at chunk c ^ (r % 8)).  Each
-//     thread owns at most one (row, half) item (2 x 128 + 2 x 64 <= 512); its
-//     64-bit words are loaded kPrefetch stages ahead into registers, so the
-//     L2 latency is off the critical path.  Each producer warp arrives once on
-//     the stage's "full" mbarrier, after every lane's proxy fence.
+//     words) and visible weights (W, neurons x words), 128 K-elements per row
+//     per stage, into the K-major SWIZZLE_128B layout the MMA reads (16-byte
+//     chunk c of row r stored at chunk c ^ (r % 8)).  The stage's 16-byte
+//     chunks are dealt round-robin to the 512 producer threads (three per
+//     thread for A + B, one for B alone in tile mode); their 16-bit pieces of
+//     bits are loaded kPrefetch stages ahead into registers.  Each producer
+//     warp arrives once on the stage's "full" mbarrier, after every lane's
+//     proxy fence.
 //   - 1 MMA warp waits on "full", issues tcgen05.mma.kind::f8f6f4 (M = 128,
 //     N = 64, K = 32) four times per stage into a 128-lane x 64-column fp32
 //     accumulator in TMEM, and commits to the stage's "empty" mbarrier, on
@@ -119,9 +120,9 @@ __global__ void __launch_bounds__(THREADS, 1) k_train_forward_tc(const StepParam
   }
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
-      // one arrival per producer warp; kTiles: 4 B-producer warps plus the
-      // tile copy's expect_tx arrival
-      mbar_init(&sh->full[s], kTiles ? 2 * TN / 32 + 1 : kProducers / 32);
+      // one arrival per producer warp, plus (kTiles) the tile copy's
+      // expect_tx arrival
+      mbar_init(&sh->full[s], kProducers / 32 + (kTiles ? 1 : 0));
       mbar_init(&sh->empty[s], 1);
     }
     mbar_init(&sh->done, 1);
@@ -139,24 +140,30 @@ __global__ void __launch_bounds__(THREADS, 1) k_train_forward_tc(const StepParam
   asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
   const uint32_t tmem = sh->tmem_base;
 
-  if (threadIdx.x < (kTiles ? 2 * TN : kProducers)) {
+  if (threadIdx.x < kProducers) {
     // ---------------- producers ----------------
-    // items: A rows [0, M) x 2 halves (only without tiles), then B rows
-    // [0, NB) x 2 halves
-    const int nA = kTiles ? 0 : 2 * M, nItems = nA + 2 * NB;
-    const int i = threadIdx.x;
-    Item it;
-    if (i < nA) {
-      it = Item{A + (int64_t)(i >> 1) * nw, (i >> 1) * KB, i >> 1, i & 1};
-    } else if (i < nItems) {
-      const int b = i - nA;
-      it = Item{Ly.W + (int64_t)(n0 + (b >> 1)) * nw, A_BYTES + (b >> 1) * KB, b >> 1, b & 1};
-    } else {
-      it = Item{nullptr, 0, 0, 0};
-    }
-    uint64_t pre[kPrefetch];
+    // items: the 16-byte chunks of A rows [0, M) (only without tiles), then
+    // of B rows [0, NB); item i belongs to thread i % kProducers
+    constexpr int kItems = kTiles ? 8 * TN / kProducers : 8 * (TM + TN) / kProducers;
+    const int nA = kTiles ? 0 : 8 * M, nItems = nA + 8 * NB;
+    Chunk ch[kItems];
 #pragma unroll
-    for (int d = 0; d < kPrefetch; ++d) pre[d] = load_word(it, d, nw);
+    for (int j = 0; j < kItems; ++j) {
+      const int i = threadIdx.x + j * kProducers;
+      if (i < nA) {
+        ch[j] = make_chunk(A + (int64_t)(i >> 3) * nw, 0, i >> 3, i & 7);
+      } else if (i < nItems) {
+        const int b = i - nA;
+        ch[j] = make_chunk(Ly.W + (int64_t)(n0 + (b >> 3)) * nw, A_BYTES, b >> 3, b & 7);
+      } else {
+        ch[j] = Chunk{nullptr, 0u, 0};
+      }
+    }
+    uint32_t pre[kPrefetch][kItems];
+#pragma unroll
+    for (int d = 0; d < kPrefetch; ++d)
+#pragma unroll
+      for (int j = 0; j < kItems; ++j) pre[d][j] = load_chunk(ch[j], d, nw);
 
     for (int kb0 = 0; kb0 < nkb; kb0 += kPrefetch) {
 #pragma unroll
@@ -173,12 +180,11 @@ __global__ void __launch_bounds__(THREADS, 1) k_train_forward_tc(const StepParam
           mbar_arrive_tx(&sh->full[s], A_BYTES);
           bulk_g2s(stage, P->layer[l - 2].AE + (size_t)kb * A_BYTES, A_BYTES, &sh->full[s]);
         }
-        if (it.src != nullptr) {
-          const int wi = 2 * kb + it.half;
-          const int valid = min(64, max(0, Kin - 64 * wi));
-          expand_word(stage + it.soff, it.r, 4 * it.half, pre[d], valid);
+#pragma unroll
+        for (int j = 0; j < kItems; ++j) {
+          if (ch[j].src != nullptr) store_chunk(stage, ch[j], pre[d][j], kb, Kin);
+          pre[d][j] = load_chunk(ch[j], kb + kPrefetch, nw);
         }
-        pre[d] = load_word(it, kb + kPrefetch, nw);
         // every writer orders its stores for the async proxy; one arrival per warp
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
         __syncwarp();

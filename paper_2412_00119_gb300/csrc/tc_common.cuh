@@ -90,31 +90,6 @@ __device__ __forceinline__ uint2 expand8(uint32_t b) {
   return make_uint2((lo & 0x80808080u) ^ 0xB8B8B8B8u, (hi & 0x80808080u) ^ 0xB8B8B8B8u);
 }
 
-// Expand one 64-bit word (64 K-elements) into four 16-byte chunks of row r of
-// a swizzled stage, chunks chunk0 .. chunk0+3.  `valid` = real elements (0..64).
-__device__ __forceinline__ void expand_word(uint8_t* row_base, int r, int chunk0, uint64_t w,
-                                            int valid) {
-#pragma unroll
-  for (int q = 0; q < 4; ++q) {        // chunk q: elements 16q .. 16q+15
-    const uint32_t bits = (uint32_t)(w >> (16 * q)) & 0xFFFFu;
-    const uint2 e0 = expand8(bits & 0xFF);
-    const uint2 e1 = expand8(bits >> 8);
-    uint4 v = make_uint4(e0.x, e0.y, e1.x, e1.y);
-    if (valid < 64) {
-      uint32_t* vv = &v.x;
-#pragma unroll
-      for (int b = 0; b < 4; ++b) {
-        const int n_ok = valid - (16 * q + 4 * b);  // real elements in this 4-byte group
-        const uint32_t keep = n_ok >= 4 ? 0xFFFFFFFFu : (n_ok <= 0 ? 0u : ((1u << (8 * n_ok)) - 1u));
-        vv[b] &= keep;
-      }
-    }
-    const int c = chunk0 + q;
-    *reinterpret_cast<uint4*>(row_base + 16 * (c ^ (r & 7))) = v;
-  }
-}
-
-
 __device__ __forceinline__ void mbar_arrive_tx(unsigned long long* bar, uint32_t bytes) {
   asm volatile("{\n .reg .b64 st;\n mbarrier.arrive.expect_tx.shared::cta.b64 st, [%0], %1;\n}"
                ::"r"(smem_u32(bar)), "r"(bytes) : "memory");
@@ -128,17 +103,47 @@ __device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t by
       ::"r"(smem_u32(dst)), "l"(src), "r"(bytes), "r"(smem_u32(bar)) : "memory");
 }
 
-// A producer item: one (matrix, row, half) of the current tile.
-struct Item {
-  const uint64_t* src;  // row start (bit words), or null when the thread has no item
-  int soff;             // byte offset of the row inside a stage (A or B part)
-  int r;                // row index inside its matrix (for the swizzle)
-  int half;             // which of the stage's two words
+// A producer item: one 16-byte chunk of one row of a stage, i.e. 16
+// K-elements (two bytes of bits) -> 16 e4m3 bytes.  The chunk's logical index
+// c (K-elements 16c .. 16c + 15 of the stage's 128) is stored at physical
+// chunk c ^ (r % 8) of row r (SWIZZLE_128B).
+struct Chunk {
+  const uint16_t* src;  // the row's bits as 16-bit pieces; null: no item
+  uint32_t dst;         // byte offset of the chunk inside a stage
+  int c;                // logical chunk 0..7
 };
 
-__device__ __forceinline__ uint64_t load_word(const Item& it, int kb, int nw) {
-  const int wi = 2 * kb + it.half;
-  return (it.src != nullptr && wi < nw) ? __ldg(it.src + wi) : 0ull;
+// Item for row r (of a matrix whose rows start `soff` bytes into the stage).
+__device__ __forceinline__ Chunk make_chunk(const uint64_t* row, int soff, int r, int c) {
+  return Chunk{reinterpret_cast<const uint16_t*>(row),
+               (uint32_t)(soff + r * KB + 16 * (c ^ (r & 7))), c};
+}
+
+// The item's 16 bits for k-block kb (0 past the row's nw words).
+__device__ __forceinline__ uint32_t load_chunk(const Chunk& ch, int kb, int nw) {
+  const int pi = 8 * kb + ch.c;
+  return (ch.src != nullptr && pi < 4 * nw) ? (uint32_t)__ldg(ch.src + pi) : 0u;
+}
+
+// Bytes of a 4-byte group to keep when n_ok of its elements are real.
+__device__ __forceinline__ uint32_t keep_mask(int n_ok) {
+  return n_ok >= 4 ? 0xFFFFFFFFu : (n_ok <= 0 ? 0u : ((1u << (8 * n_ok)) - 1u));
+}
+
+// Expand the item's bits into its stage chunk; elements at K >= Kin are 0.
+__device__ __forceinline__ void store_chunk(uint8_t* stage, const Chunk& ch, uint32_t bits, int kb,
+                                            int Kin) {
+  const uint2 e0 = expand8(bits & 0xFFu);
+  const uint2 e1 = expand8(bits >> 8);
+  uint4 v = make_uint4(e0.x, e0.y, e1.x, e1.y);
+  const int valid = Kin - (KB * kb + 16 * ch.c);
+  if (valid < 16) {
+    v.x &= keep_mask(valid);
+    v.y &= keep_mask(valid - 4);
+    v.z &= keep_mask(valid - 8);
+    v.w &= keep_mask(valid - 12);
+  }
+  *reinterpret_cast<uint4*>(stage + ch.dst) = v;
 }
 
 }  // namespace tc
