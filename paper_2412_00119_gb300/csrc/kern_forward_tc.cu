@@ -6,33 +6,40 @@
 // is computed exactly as an e4m3 x e4m3 -> fp32 matrix product: +-1 are exact
 // in e4m3 (0x38 / 0xB8), pad elements are 0x00, and every partial sum is an
 // integer of magnitude <= K_in < 2^24, exact in fp32 whatever the order.
-// One CTA owns TN = 64 neurons and all (<= 128) patterns of the mini-batch.
-// The A operand of layers l >= 2 arrives pre-expanded: the epilogue of layer
-// l - 1 also writes its activations as e4m3 in the swizzled stage image (one
-// 16 KB tile per 128 K-elements, DevLayer::AE), and one producer pulls each
-// tile into the stage with a single cp.async.bulk that completes on the
-// stage's "full" mbarrier.  For layer 1 (the caller's bit-packed input) and in
-// general:
-//   - 16 producer warps expand the bit-packed activations (A, patterns x
-//     words) and visible weights (W, neurons x words), 128 K-elements per row
-//     per stage, into the K-major SWIZZLE_128B layout the MMA reads (16-byte
-//     chunk c of row r stored at chunk c ^ (r % 8)).  The stage's 16-byte
-//     chunks are dealt round-robin to the 512 producer threads (three per
-//     thread for A + B, one for B alone in tile mode); their 16-bit pieces of
-//     bits are loaded kPrefetch stages ahead into registers.  Each producer
-//     warp arrives once on the stage's "full" mbarrier, after every lane's
-//     proxy fence.
-//   - 1 MMA warp waits on "full", issues tcgen05.mma.kind::f8f6f4 (M = 128,
-//     N = 64, K = 32) four times per stage into a 128-lane x 64-column fp32
-//     accumulator in TMEM, and commits to the stage's "empty" mbarrier, on
-//     which producers wait before overwriting the stage (kStages-deep ring).
-//   - the epilogue reads the accumulator with tcgen05.ld (warp w % 4 owns TMEM
-//     lanes 32 (w % 4) .., 16 columns per warp), converts to int, stores z
-//     (int16) and packs the sign bits of 16 neurons per thread directly into
-//     the activation words.
+//
+// Tiling.  A tcgen05.mma of M = 128 rows costs about the same time for N = 64
+// as for N = 256, so the kernel uses the widest instruction: a tile is the
+// whole mini-batch (<= 128 patterns, rows >= bs unused) x TN = 256 neurons.
+// To keep every SM busy with only K_out / 256 tiles, the K range is split
+// across a cluster of kSplit = 4 CTAs: CTA r of the cluster accumulates
+// k-blocks [r nkb / 4, (r + 1) nkb / 4) in TMEM, writes its 128 x 256 fp32
+// partial to its own shared memory, and after a cluster barrier reduces the
+// four partials of its 64 columns through distributed shared memory
+// (mapa + ld.shared::cluster) and writes them out.
+//
+// Pipeline of a CTA (4-stage ring of 48 KB stages, 128 K-elements each):
+//   - 16 producer warps expand the bit-packed visible weights (W, neurons x
+//     words: 256 rows x 2 words = one 64-bit item per thread) into the K-major
+//     SWIZZLE_128B layout the MMA reads (16-byte chunk c of row r stored at
+//     chunk c ^ (r % 8)); for layer 1 they also expand the caller's packed
+//     inputs (A).  Bit words are loaded kPrefetch stages ahead into registers.
+//     Each producer warp arrives once on the stage's "full" mbarrier after
+//     every lane's proxy fence.
+//   - For layers l >= 2 the A operand arrives pre-expanded: the epilogue of
+//     layer l - 1 writes its activations as e4m3 in the swizzled stage image
+//     (one 16 KB tile per 128 K-elements, DevLayer::AE), and one thread pulls
+//     each tile with a bulk copy that completes on the same barrier.
+//   - 1 MMA thread waits on "full", issues tcgen05.mma.kind::f8f6f4 (M = 128,
+//     N = 256, K = 32) four times per stage into a 128 x 256 fp32 accumulator
+//     in TMEM, and commits to the stage's "empty" mbarrier.
+//   - Epilogue: tcgen05.ld -> shared partial; cluster barrier; reduction of
+//     this CTA's 64 columns over the 4 partials; z (int16), packed sign bits
+//     and, for the next layer, the e4m3 tile image; cluster barrier again so
+//     that no CTA leaves while a peer still reads its partial.
 // Every mbarrier wait is bounded; the first expiry sets a shared flag that
 // stops every other wait, the kernel counts the failure in the control block
-// (host: BMLP_ETIMEOUT), releases its TMEM and returns.
+// (host: BMLP_ETIMEOUT), still passes both cluster barriers, releases its TMEM
+// and returns.
 #include "tc_common.cuh"
 
 namespace bk {
@@ -40,16 +47,21 @@ namespace {
 
 using namespace tc;
 
-constexpr int TM = 128;           // MMA M: patterns (rows >= bsz are zero)
-constexpr int TN = 64;            // MMA N: neurons per CTA
+constexpr int TM = 128;           // MMA M: patterns (rows >= bsz unused)
+constexpr int TN = 256;           // MMA N: neurons per tile
+constexpr int kSplit = 4;         // CTAs per cluster, each a quarter of K
 constexpr int kStages = 4;
-constexpr int kPrefetch = 8;      // stages of bit-words held in registers ahead
-constexpr int kProducers = 512;   // 16 warps: one (row, half) item per thread
+constexpr int kPrefetch = 4;      // stages of bit-words held in registers ahead
+constexpr int kProducers = 512;   // 16 warps
 constexpr int THREADS = kProducers + 32;
 constexpr int A_BYTES = TM * KB;  // 16 KB
-constexpr int B_BYTES = TN * KB;  // 8 KB
+constexpr int B_BYTES = TN * KB;  // 32 KB
 constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-constexpr int TMEM_COLS = 64;
+constexpr int TMEM_COLS = TN;
+constexpr int PSTRIDE = TN + 4;   // floats per partial row (+16 B: no bank conflicts)
+constexpr int kCols = TN / kSplit;  // columns reduced by one CTA
+static_assert(TM * PSTRIDE * 4 <= kStages * STAGE_BYTES, "partial must fit in the stages");
+static_assert(kCols == 64, "one CTA writes one packed activation word per row");
 
 struct __align__(8) TcShared {
   unsigned long long full[kStages];   // the producers filled stage s
@@ -63,8 +75,29 @@ constexpr size_t kSmemBytes = 1024 /*alignment slack*/ + kStages * STAGE_BYTES +
 
 constexpr uint32_t kIdesc = tc::idesc_f8(TM, TN);
 
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+
+__device__ __forceinline__ void cluster_sync_all() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;"
+               ::: "memory");
+}
+
+__device__ __forceinline__ float4 ld_peer_f4(uint32_t local_addr, uint32_t rank) {
+  uint32_t a;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(a) : "r"(local_addr), "r"(rank));
+  float4 v;
+  asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];"
+               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w) : "r"(a) : "memory");
+  return v;
+}
+
 template <bool kTiles>
-__global__ void __launch_bounds__(THREADS, 1) k_train_forward_tc(const StepParams* __restrict__ P, int l);
+__global__ void __cluster_dims__(kSplit, 1, 1) __launch_bounds__(THREADS, 1)
+    k_train_forward_tc(const StepParams* __restrict__ P, int l);
 
 }  // namespace
 
@@ -79,7 +112,7 @@ cudaError_t prepare_train_forward_tc() {
 }
 
 void launch_train_forward_tc(bool tiles, int Kout, cudaStream_t st, const StepParams* P, int l) {
-  const dim3 grid((unsigned)((Kout + TN - 1) / TN));
+  const dim3 grid((unsigned)(((Kout + TN - 1) / TN) * kSplit));
   if (tiles)
     k_train_forward_tc<true><<<grid, THREADS, kSmemBytes, st>>>(P, l);
   else
@@ -91,7 +124,8 @@ size_t act_tile_bytes(int K) { return (size_t)((K + KB - 1) / KB) * A_BYTES; }
 namespace {
 
 template <bool kTiles>
-__global__ void __launch_bounds__(THREADS, 1) k_train_forward_tc(const StepParams* __restrict__ P, int l) {
+__global__ void __cluster_dims__(kSplit, 1, 1) __launch_bounds__(THREADS, 1)
+    k_train_forward_tc(const StepParams* __restrict__ P, int l) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* base = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
@@ -101,19 +135,24 @@ __global__ void __launch_bounds__(THREADS, 1) k_train_forward_tc(const StepParam
   const int64_t rem = P->n - start;
   const int M = (int)(rem < P->bs ? rem : P->bs);
   const uint64_t* A = (l == 1) ? P->x + start * P->nw0 : P->layer[l - 2].A;
-  const int n0 = blockIdx.x * TN;
+  const uint32_t rank = cluster_rank();
+  const int n0 = (int)(blockIdx.x / kSplit) * TN;
   const int N = Ly.Kout, Kin = Ly.Kin, nw = Ly.nw_in;
-  const int NB = min(TN, N - n0);   // neuron rows of this CTA
+  const int NB = min(TN, N - n0);   // neuron rows of this tile
   const int nkb = (Kin + KB - 1) / KB;
+  const int kb0 = (int)((nkb * rank) / kSplit);
+  const int nk = (int)((nkb * (rank + 1)) / kSplit) - kb0;  // k-blocks of this CTA (may be 0)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   volatile int* failed = &sh->failed;
 
   // zero the pattern rows >= M and neuron rows >= NB of every stage once; the
-  // producers never write them, so they stay zero (0 * anything = 0)
+  // producers never write them (their products land in unused rows/columns)
   for (int s = 0; s < kStages; ++s) {
-    uint4* a4 = reinterpret_cast<uint4*>(base + s * STAGE_BYTES);
-    for (int i = M * (KB / 16) + threadIdx.x; i < TM * (KB / 16); i += THREADS)
-      a4[i] = make_uint4(0, 0, 0, 0);
+    if (!kTiles) {
+      uint4* a4 = reinterpret_cast<uint4*>(base + s * STAGE_BYTES);
+      for (int i = M * (KB / 16) + threadIdx.x; i < TM * (KB / 16); i += THREADS)
+        a4[i] = make_uint4(0, 0, 0, 0);
+    }
     uint4* b4 = reinterpret_cast<uint4*>(base + s * STAGE_BYTES + A_BYTES);
     for (int i = NB * (KB / 16) + threadIdx.x; i < TN * (KB / 16); i += THREADS)
       b4[i] = make_uint4(0, 0, 0, 0);
@@ -142,37 +181,39 @@ __global__ void __launch_bounds__(THREADS, 1) k_train_forward_tc(const StepParam
 
   if (threadIdx.x < kProducers) {
     // ---------------- producers ----------------
-    // items: the 16-byte chunks of A rows [0, M) (only without tiles), then
-    // of B rows [0, NB); item i belongs to thread i % kProducers
-    constexpr int kItems = kTiles ? 8 * TN / kProducers : 8 * (TM + TN) / kProducers;
-    const int nA = kTiles ? 0 : 8 * M, nItems = nA + 8 * NB;
-    Chunk ch[kItems];
+    // items: W rows [0, NB) x 2 halves (item i: row i / 2, half i % 2), then
+    // (layer 1 only) input rows [0, M) x 2 halves; item i -> thread i % 512
+    constexpr int kItems = kTiles ? 1 : 2;
+    const int nB = 2 * NB, nItems = nB + (kTiles ? 0 : 2 * M);
+    Item it[kItems];
 #pragma unroll
     for (int j = 0; j < kItems; ++j) {
       const int i = threadIdx.x + j * kProducers;
-      if (i < nA) {
-        ch[j] = make_chunk(A + (int64_t)(i >> 3) * nw, 0, i >> 3, i & 7);
+      if (i < nB) {
+        it[j] = Item{Ly.W + (int64_t)(n0 + (i >> 1)) * nw, (uint32_t)(A_BYTES + (i >> 1) * KB), i >> 1,
+                     i & 1};
       } else if (i < nItems) {
-        const int b = i - nA;
-        ch[j] = make_chunk(Ly.W + (int64_t)(n0 + (b >> 3)) * nw, A_BYTES, b >> 3, b & 7);
+        const int a = i - nB;
+        it[j] = Item{A + (int64_t)(a >> 1) * nw, (uint32_t)((a >> 1) * KB), a >> 1, a & 1};
       } else {
-        ch[j] = Chunk{nullptr, 0u, 0};
+        it[j] = Item{nullptr, 0u, 0, 0};
       }
     }
-    uint32_t pre[kPrefetch][kItems];
+    uint64_t pre[kPrefetch][kItems];
 #pragma unroll
     for (int d = 0; d < kPrefetch; ++d)
 #pragma unroll
-      for (int j = 0; j < kItems; ++j) pre[d][j] = load_chunk(ch[j], d, nw);
+      for (int j = 0; j < kItems; ++j) pre[d][j] = load_word(it[j], kb0 + d, nw);
 
-    for (int kb0 = 0; kb0 < nkb; kb0 += kPrefetch) {
+    for (int k0 = 0; k0 < nk; k0 += kPrefetch) {
 #pragma unroll
       for (int d = 0; d < kPrefetch; ++d) {
-        const int kb = kb0 + d;
-        if (kb >= nkb) break;
-        const int s = kb % kStages;
-        if (kb >= kStages &&
-            !__all_sync(kFull, mbar_wait(&sh->empty[s], (uint32_t)((kb / kStages - 1) & 1), failed)))
+        const int k = k0 + d;
+        if (k >= nk) break;
+        const int kb = kb0 + k;
+        const int s = k % kStages;
+        if (k >= kStages &&
+            !__all_sync(kFull, mbar_wait(&sh->empty[s], (uint32_t)((k / kStages - 1) & 1), failed)))
           break;
         uint8_t* stage = base + s * STAGE_BYTES;
         if (kTiles && threadIdx.x == 0) {
@@ -182,8 +223,8 @@ __global__ void __launch_bounds__(THREADS, 1) k_train_forward_tc(const StepParam
         }
 #pragma unroll
         for (int j = 0; j < kItems; ++j) {
-          if (ch[j].src != nullptr) store_chunk(stage, ch[j], pre[d][j], kb, Kin);
-          pre[d][j] = load_chunk(ch[j], kb + kPrefetch, nw);
+          if (it[j].src != nullptr) store_word(stage, it[j], pre[d][j], kb, Kin);
+          pre[d][j] = load_word(it[j], kb + kPrefetch, nw);
         }
         // every writer orders its stores for the async proxy; one arrival per warp
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
@@ -194,59 +235,97 @@ __global__ void __launch_bounds__(THREADS, 1) k_train_forward_tc(const StepParam
     }
   } else if (threadIdx.x == kProducers) {
     // ---------------- MMA issuer (lane 0 of the last warp) ----------------
-    for (int kb = 0; kb < nkb; ++kb) {
-      const int s = kb % kStages;
-      if (!mbar_wait(&sh->full[s], (uint32_t)((kb / kStages) & 1), failed)) break;
+    for (int k = 0; k < nk; ++k) {
+      const int s = k % kStages;
+      if (!mbar_wait(&sh->full[s], (uint32_t)((k / kStages) & 1), failed)) break;
       asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
       const uint8_t* sa = base + s * STAGE_BYTES;
       const uint64_t ad = smem_desc(smem_u32(sa));
       const uint64_t bd = smem_desc(smem_u32(sa + A_BYTES));
 #pragma unroll
       for (int j = 0; j < KB / 32; ++j)   // K = 32 bytes per MMA: +2 in the address field
-        mma_f8<kIdesc>(tmem, ad + 2 * j, bd + 2 * j, (kb > 0 || j > 0) ? 1u : 0u);
+        mma_f8<kIdesc>(tmem, ad + 2 * j, bd + 2 * j, (k > 0 || j > 0) ? 1u : 0u);
       mma_commit(&sh->empty[s]);
     }
-    if (!*failed) mma_commit(&sh->done);
+    if (nk > 0 && !*failed) mma_commit(&sh->done);
   }
 
-  // ---------------- epilogue (producer warps) ----------------
-  // tcgen05.ld is warp-collective: the go / no-go decision is made per warp
-  bool go = false;
+  // ---------------- partial accumulator -> shared memory ----------------
+  // (the stages are free: every MMA that read them has completed)
+  float* part = reinterpret_cast<float*>(base);
   if (threadIdx.x < kProducers) {
-    go = !*failed && mbar_wait(&sh->done, 0, failed);
-    go = __all_sync(0xffffffffu, go);
-  }
-  if (go) {
-    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-    const int sub = warp & 3;            // TMEM lanes 32 sub .. 32 sub + 31
-    const int col0 = 16 * (warp >> 2);   // accumulator columns col0 .. col0 + 15
-    uint32_t v[16];
-    asm volatile(
-        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
-        : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]),
-          "=r"(v[7]), "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]),
-          "=r"(v[14]), "=r"(v[15])
-        : "r"(tmem + ((uint32_t)(32 * sub) << 16) + (uint32_t)col0));
-    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+    bool go = nk > 0 && !*failed && mbar_wait(&sh->done, 0, failed);
+    go = __all_sync(kFull, go);   // tcgen05.ld is warp-collective
+    if (go) asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+    const int sub = warp & 3;     // TMEM lanes 32 sub .. 32 sub + 31
     const int m = 32 * sub + lane;
+#pragma unroll
+    for (int half = 0; half < 2; ++half) {
+      const int col0 = 64 * (warp >> 2) + 32 * half;
+      uint32_t v[32];
+      if (go) {
+        asm volatile(
+            "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+            "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+            : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]),
+              "=r"(v[7]), "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]),
+              "=r"(v[13]), "=r"(v[14]), "=r"(v[15]), "=r"(v[16]), "=r"(v[17]), "=r"(v[18]),
+              "=r"(v[19]), "=r"(v[20]), "=r"(v[21]), "=r"(v[22]), "=r"(v[23]), "=r"(v[24]),
+              "=r"(v[25]), "=r"(v[26]), "=r"(v[27]), "=r"(v[28]), "=r"(v[29]), "=r"(v[30]),
+              "=r"(v[31])
+            : "r"(tmem + ((uint32_t)(32 * sub) << 16) + (uint32_t)col0));
+        asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+      } else {
+#pragma unroll
+        for (int j = 0; j < 32; ++j) v[j] = 0u;  // empty K range (or a failed wait): 0
+      }
+      float4* dst = reinterpret_cast<float4*>(part + m * PSTRIDE + col0);
+#pragma unroll
+      for (int q = 0; q < 8; ++q)
+        dst[q] = make_float4(__uint_as_float(v[4 * q]), __uint_as_float(v[4 * q + 1]),
+                             __uint_as_float(v[4 * q + 2]), __uint_as_float(v[4 * q + 3]));
+    }
+  }
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+  cluster_sync_all();
+
+  // ---------------- reduction of this CTA's 64 columns ----------------
+  if (threadIdx.x < kProducers) {
+    const int m = threadIdx.x >> 2;              // pattern row
+    const int c0 = kCols * (int)rank + 16 * (threadIdx.x & 3);  // column in the tile
+    const int nf = n0 + c0;                      // first neuron of the 16
     if (m < M) {
+      float acc[16];
+#pragma unroll
+      for (int j = 0; j < 16; ++j) acc[j] = 0.f;
+      const uint32_t local = smem_u32(part + m * PSTRIDE + c0);
+#pragma unroll
+      for (int q = 0; q < kSplit; ++q) {
+#pragma unroll
+        for (int h = 0; h < 4; ++h) {
+          const float4 v = ld_peer_f4(local + 16u * h, (uint32_t)q);
+          acc[4 * h] += v.x;
+          acc[4 * h + 1] += v.y;
+          acc[4 * h + 2] += v.z;
+          acc[4 * h + 3] += v.w;
+        }
+      }
       int16_t* zrow = Ly.Z + (int64_t)m * N;
       uint32_t bits = 0;
 #pragma unroll
       for (int j = 0; j < 16; ++j) {
-        const int n = n0 + col0 + j;
-        const int z = __float2int_rn(__uint_as_float(v[j]));
-        if (n < N) {
-          zrow[n] = (int16_t)z;
+        const int z = __float2int_rn(acc[j]);
+        if (nf + j < N) {
+          zrow[nf + j] = (int16_t)z;
           if (z >= 0) bits |= 1u << j;
         }
       }
-      reinterpret_cast<uint16_t*>(Ly.A + (int64_t)m * Ly.nw_out + (n0 >> 6))[col0 >> 4] = (uint16_t)bits;
-      if (Ly.AE != nullptr) {
+      if ((nf >> 4) < 4 * Ly.nw_out)   // pad groups of the last word get 0 bits
+        reinterpret_cast<uint16_t*>(Ly.A + (int64_t)m * Ly.nw_out)[nf >> 4] = (uint16_t)bits;
+      if (Ly.AE != nullptr && nf / KB < (N + KB - 1) / KB) {
         // the same 16 activations as e4m3 (+1 0x38, -1 0xB8, past N 0x00) in the
         // swizzled tile image that the next layer's stages copy verbatim
-        const int nf = n0 + col0;
-        uint32_t q[4];
+        uint32_t q4[4];
 #pragma unroll
         for (int b = 0; b < 4; ++b) {
           uint32_t word = 0;
@@ -256,16 +335,16 @@ __global__ void __launch_bounds__(THREADS, 1) k_train_forward_tc(const StepParam
             const uint32_t e = (nf + jj < N) ? (((bits >> jj) & 1u) ? 0x38u : 0xB8u) : 0u;
             word |= e << (8 * j);
           }
-          q[b] = word;
+          q4[b] = word;
         }
         const int c = (nf % KB) / 16;
         uint8_t* dst = Ly.AE + (size_t)(nf / KB) * A_BYTES + (size_t)m * KB + 16 * (c ^ (m & 7));
-        *reinterpret_cast<uint4*>(dst) = make_uint4(q[0], q[1], q[2], q[3]);
+        *reinterpret_cast<uint4*>(dst) = make_uint4(q4[0], q4[1], q4[2], q4[3]);
       }
     }
   }
-  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-  __syncthreads();
+  cluster_sync_all();   // no CTA leaves while a peer still reads its partial
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
   if (threadIdx.x == 0 && *failed) atomicAdd(&P->ctrl->timeouts, 1u);
   if (warp == 0)
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(TMEM_COLS) : "memory");

@@ -146,5 +146,42 @@ __device__ __forceinline__ void store_chunk(uint8_t* stage, const Chunk& ch, uin
   *reinterpret_cast<uint4*>(stage + ch.dst) = v;
 }
 
+// A producer item of 64 K-elements: one (row, half) of a stage row, i.e. one
+// 64-bit word of bits -> four 16-byte chunks (chunks 4 half .. 4 half + 3).
+struct Item {
+  const uint64_t* src;  // row start (bit words), or null when the thread has no item
+  uint32_t dst;         // byte offset of the row inside a stage
+  int r;                // row index inside its matrix (for the swizzle)
+  int half;             // which of the stage's two words
+};
+
+__device__ __forceinline__ uint64_t load_word(const Item& it, int kb, int nw) {
+  const int wi = 2 * kb + it.half;
+  return (it.src != nullptr && wi < nw) ? __ldg(it.src + wi) : 0ull;
+}
+
+// Expand the item's word for k-block kb into its four chunks; elements at
+// K >= Kin are 0.
+__device__ __forceinline__ void store_word(uint8_t* stage, const Item& it, uint64_t w, int kb,
+                                           int Kin) {
+  const int valid = Kin - (KB * kb + 64 * it.half);
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {  // chunk 4 half + q: elements 16 q .. 16 q + 15 of the word
+    const uint32_t bits = (uint32_t)(w >> (16 * q)) & 0xFFFFu;
+    const uint2 e0 = expand8(bits & 0xFFu);
+    const uint2 e1 = expand8(bits >> 8);
+    uint4 v = make_uint4(e0.x, e0.y, e1.x, e1.y);
+    if (valid < 64) {
+      const int n = valid - 16 * q;
+      v.x &= keep_mask(n);
+      v.y &= keep_mask(n - 4);
+      v.z &= keep_mask(n - 8);
+      v.w &= keep_mask(n - 12);
+    }
+    const int c = 4 * it.half + q;
+    *reinterpret_cast<uint4*>(stage + it.dst + 16 * (c ^ (it.r & 7))) = v;
+  }
+}
+
 }  // namespace tc
 }  // namespace bk
