@@ -311,14 +311,23 @@ __global__ void __cluster_dims__(kSplit, 1, 1) __launch_bounds__(THREADS, 1)
         }
       }
       int16_t* zrow = Ly.Z + (int64_t)m * N;
-      uint32_t bits = 0;
+      uint32_t bits = 0, zp[8];
 #pragma unroll
       for (int j = 0; j < 16; ++j) {
         const int z = __float2int_rn(acc[j]);
-        if (nf + j < N) {
-          zrow[nf + j] = (int16_t)z;
-          if (z >= 0) bits |= 1u << j;
-        }
+        if (nf + j < N && z >= 0) bits |= 1u << j;
+        if (j & 1) zp[j >> 1] |= (uint32_t)(z & 0xFFFF) << 16;
+        else zp[j >> 1] = (uint32_t)(z & 0xFFFF);
+      }
+      if ((N & 7) == 0 && nf + 16 <= N) {
+        // the 16 pre-activations are 32 contiguous, 16-byte aligned bytes
+        uint4* zv = reinterpret_cast<uint4*>(zrow + nf);
+        zv[0] = make_uint4(zp[0], zp[1], zp[2], zp[3]);
+        zv[1] = make_uint4(zp[4], zp[5], zp[6], zp[7]);
+      } else {
+#pragma unroll
+        for (int j = 0; j < 16; ++j)
+          if (nf + j < N) zrow[nf + j] = (int16_t)(zp[j >> 1] >> (16 * (j & 1)));
       }
       if ((nf >> 4) < 4 * Ly.nw_out)   // pad groups of the last word get 0 bits
         reinterpret_cast<uint16_t*>(Ly.A + (int64_t)m * Ly.nw_out)[nf >> 4] = (uint16_t)bits;
