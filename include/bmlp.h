@@ -21,9 +21,10 @@
  * Conventions where the paper is silent: sign(0) = +1; argmax ties go to the
  * lowest class; groups are contiguous (neuron k in group k / gamma); tuples are
  * applied in ascending pattern order with clipping after each; LayerUpdate runs
- * only when M_l is non-empty; Uniform(0,1) is a 32-bit Philox4x32-10 integer U
- * with p = U / 2^32 and "p < q" evaluated exactly.  Every result is an integer
- * or a bit and is reproducible bit for bit.
+ * only when M_l is non-empty; the reinforcement events are drawn per block
+ * of 64 inputs from 32-bit Philox4x32-10 draws against integer thresholds
+ * (bmlp_reinforce_tables).  Every result is an integer or a bit and is
+ * reproducible bit for bit.
  *
  * Data formats
  *   packed +-1 vectors: a vector of K values is ceil(K/64) little-endian uint64
@@ -159,10 +160,22 @@ const char* bmlp_last_error(const bmlp_t* h);
  * -1 for K < 1.  Host only. */
 int32_t bmlp_gamma_rule(int32_t K);
 
-/* Reinforcement threshold of Alg. 3 l.8 for the current p_r and layer width K:
- * q = p_r sqrt(2 / (pi K)) in IEEE double, returned as T = ceil(q 2^32)
- * clamped to [0, 2^32], so that a 32-bit U reinforces iff U < T.  Host only. */
-uint64_t bmlp_reinforce_threshold(double p_r, int32_t K);
+/* Thresholds of the reinforcement sampler (Alg. 3 l.5-12) for a block of n
+ * inputs (1 <= n <= 64) of a layer of width K at p_r.  Each hidden weight is
+ * reinforced independently with probability q = p_r sqrt(2 / (pi K)) (IEEE
+ * double; >= 1 taken as 1).  The events of a neuron row are drawn per block
+ * of 64 consecutive inputs (the last block shorter): the block has an event
+ * iff its 32-bit draw U < any_out; its first event is at the least j with
+ * V < first_out[j]; after an event at p the next is at p + 1 + g for the
+ * least g <= n - 2 - p with V < gap_out[g], none if there is no such g (V the
+ * block's successive 32-bit draws).  With thr(x) = ceil(x 2^32) (0 for
+ * x <= 0, 2^32 for x >= 1) and (1-q)^m a left-to-right IEEE product:
+ *   any_out = thr(1 - (1-q)^n), first_out[j] = thr((1 - (1-q)^(j+1)) /
+ *   (1 - (1-q)^n)) for j < n, gap_out[g] = thr(1 - (1-q)^(g+1)) for g < n - 1.
+ * first_out holds n values and gap_out n - 1 (caller-owned).  Host only;
+ * BMLP_EINVAL for K < 1, n outside 1..64 or a NULL output. */
+int bmlp_reinforce_tables(double p_r, int32_t K, int32_t n, uint64_t* any_out,
+                          uint64_t* first_out, uint64_t* gap_out);
 
 /* Debug view of the most recent training mini-batch (synchronises): for layer
  * `layer`, Z (bs x K_l int16 pre-activations), A (bs x ceil(K_l/64) packed

@@ -8,7 +8,8 @@ library and its Python binding never do.
 What each function follows (arXiv 2412.00119):
   ``philox4x32_10``            -- Salmon et al., SC'11 (the random stream)
   ``gamma_rule``               -- Sec. 4.3, choice of the group size
-  ``reinforce_threshold``      -- Alg. 3 l.7-8, exact "p < p_r sqrt(2/(pi K_l))"
+  ``reinforce_prob``           -- Alg. 3 l.8, q = p_r sqrt(2/(pi K_l))
+  ``r_block_tables``/``r_events`` -- Alg. 3 l.5-12, which weights are reinforced
   ``layer_forward``            -- Alg. 1 l.8-9
   ``local_output``/``local_loss`` -- Alg. 1 l.10-17 and Eq. 1
   ``select``                   -- Alg. 2
@@ -96,6 +97,7 @@ _i32p = C.POINTER(C.c_int32)
 _i8p = C.POINTER(C.c_int8)
 _u8p = C.POINTER(C.c_uint8)
 _u32p = C.POINTER(C.c_uint32)
+_u64p = C.POINTER(C.c_uint64)
 _i64p = C.POINTER(C.c_int64)
 
 
@@ -106,12 +108,13 @@ def _declare(L):
     L.or_init_h.restype = C.c_int32
     L.or_init_rho.argtypes = [C.c_uint64, C.c_int32, C.c_int32, C.c_int32]
     L.or_init_rho.restype = C.c_int32
-    L.or_uniform32.argtypes = [C.c_uint64, C.c_int32, C.c_int32, C.c_int32, C.c_uint32]
-    L.or_uniform32.restype = C.c_uint32
     L.or_reinforce_prob.argtypes = [C.c_double, C.c_int32]
     L.or_reinforce_prob.restype = C.c_double
-    L.or_reinforce_threshold.argtypes = [C.c_double, C.c_int32]
-    L.or_reinforce_threshold.restype = C.c_uint64
+    L.or_r_block_tables.argtypes = [C.c_double, C.c_int32, _u64p, _u64p, _u64p]
+    L.or_r_block_tables.restype = None
+    L.or_r_events.argtypes = [C.c_uint64, C.c_int32, C.c_int32, C.c_uint32, C.c_int32, C.c_double,
+                              _u8p]
+    L.or_r_events.restype = None
     L.or_gamma_rule.argtypes = [C.c_int32]
     L.or_gamma_rule.restype = C.c_int32
     L.or_layer_forward.argtypes = [_i8p, C.c_int32, C.c_int32, _i32p, C.c_int32, _i32p, _i8p]
@@ -126,7 +129,7 @@ def _declare(L):
     L.or_select.restype = None
     L.or_perceptron_update.argtypes = [_i32p, C.c_int32, C.c_int32, _i8p, _i32p, _i8p,
                                        C.c_int32, _i32p, C.c_int32, C.c_int32, C.c_int32,
-                                       C.c_uint64, C.c_uint64, C.c_int32, C.c_uint32]
+                                       C.c_double, C.c_uint64, C.c_int32, C.c_uint32]
     L.or_perceptron_update.restype = None
     L.or_create.argtypes = [_i32p, C.c_int32, C.c_int32, C.c_int32, C.c_uint64, C.c_int32,
                             C.c_int32, C.c_int32, C.c_double, _i32p, C.POINTER(C.c_void_p)]
@@ -188,16 +191,24 @@ def init_rho(seed, l, k, j):
     return lib().or_init_rho(seed, l, k, j)
 
 
-def uniform32(seed, l, k, i, t):
-    return lib().or_uniform32(seed, l, k, i, t & 0xFFFFFFFF)
-
-
 def reinforce_prob(p_r, K):
     return lib().or_reinforce_prob(p_r, K)
 
 
-def reinforce_threshold(p_r, K):
-    return int(lib().or_reinforce_threshold(p_r, K))
+def r_block_tables(q, n):
+    """Thresholds of a block of n inputs: (any, first[n], gap[n-1])."""
+    any_ = np.zeros(1, np.uint64)
+    first = np.zeros(64, np.uint64)
+    gap = np.zeros(64, np.uint64)
+    lib().or_r_block_tables(q, n, _p(any_, _u64p), _p(first, _u64p), _p(gap, _u64p))
+    return int(any_[0]), first[:n].copy(), gap[:max(n - 1, 0)].copy()
+
+
+def r_events(seed, l, k, t, K_prev, q):
+    """Reinforcement events of neuron k (uint8 per input, 1 = reinforced)."""
+    fire = np.zeros(max(K_prev, 1), np.uint8)
+    lib().or_r_events(seed, l, k, t & 0xFFFFFFFF, K_prev, q, _p(fire, _u8p))
+    return fire[:K_prev]
 
 
 def gamma_rule(K):
@@ -259,8 +270,9 @@ def select(z, P, y, mark, gamma):
     return sel
 
 
-def perceptron_update(H, a_prev, y, P, sel, h_max, T, seed, l, t):
-    """Alg. 3 on a copy of H (K_prev x K).  Returns the updated H."""
+def perceptron_update(H, a_prev, y, P, sel, h_max, q, seed, l, t):
+    """Alg. 3 on a copy of H (K_prev x K), reinforcement probability q.
+    Returns the updated H."""
     H = np.array(H, dtype=np.int32, order="C", copy=True)
     a_prev = _c(a_prev, np.int8)
     y = _c(y, np.int32)
@@ -269,7 +281,8 @@ def perceptron_update(H, a_prev, y, P, sel, h_max, T, seed, l, t):
     Kp, K = H.shape
     b, G = sel.shape
     lib().or_perceptron_update(_p(H, _i32p), Kp, K, _p(a_prev, _i8p), _p(y, _i32p), _p(P, _i8p),
-                               P.shape[1], _p(sel, _i32p), b, G, h_max, T, seed, l, t & 0xFFFFFFFF)
+                               P.shape[1], _p(sel, _i32p), b, G, h_max, float(q), seed, l,
+                               t & 0xFFFFFFFF)
     return H
 
 

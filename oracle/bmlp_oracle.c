@@ -39,9 +39,22 @@
  *       among equal largest negative deltas the lowest k wins (Alg. 2 l.7).
  *   O8  Tuples of U_l are applied in (mu ascending, g ascending) order, the
  *       order in which Alg. 2 builds U_l (Alg. 3 l.2-4).
- *   O9  Uniform(0,1) of Alg. 3 l.7 is p = U / 2^32, U a 32-bit integer drawn
- *       from Philox4x32-10 (stream layout below); "p < q" is evaluated exactly
- *       as U < ceil(q * 2^32) with q computed in IEEE double.
+ *   O9  Alg. 3 l.7-8 reinforces each hidden weight independently with
+ *       probability q = p_r sqrt(2 / (pi K_l)) (q in IEEE double, taken as 1
+ *       when larger).  The events of one neuron row are sampled block by
+ *       block (blocks of 64 consecutive inputs, the last one shorter) with
+ *       32-bit Philox draws compared against integer thresholds thr(x) =
+ *       ceil(x 2^32) (0 for x <= 0, 2^32 for x >= 1), where (1-q)^m is the
+ *       left-to-right IEEE product of m factors (1-q):
+ *         - a block of n inputs holds at least one event iff its draw
+ *           U < thr(1 - (1-q)^n);
+ *         - then its first event is at the least j with
+ *           V < thr((1 - (1-q)^(j+1)) / (1 - (1-q)^n)), and after an event at p
+ *           the next one is at p + 1 + g for the least g <= n - 2 - p with
+ *           V < thr(1 - (1-q)^(g+1)); there is none when no such g exists.
+ *       This is the law of n independent Bernoulli(q) events (first success
+ *       given at least one, then geometric gaps), up to the 2^-32 rounding of
+ *       the thresholds.
  *   O10 K in sqrt(2 / (pi K_l)) is the layer width K_l, as printed (Alg. 3 l.8).
  *   O11 E^e = (# training patterns of the epoch whose last-layer 01-loss was 1 in
  *       the training forward pass) / (# patterns of the epoch); p_r <- p_r *
@@ -59,10 +72,10 @@
  * seed div 2^32); counter words (c0, c1, c2, c3):
  *   initial h_{ik} of layer l : (i/4, k, 1*2^16 + l, 0); word i%4; h = +1 iff bit 31 set
  *   rho_{kj} of P_l           : (j/4, k, 2*2^16 + l, 0); word j%4; rho = +1 iff bit 31 set
- *   U for h_{ik}, step t      : hi16 = 16-bit lane i%8 of (i/8, k, 3*2^16 + l, t)
- *                               lo16 = 16-bit lane i%8 of (i/8, k, 4*2^16 + l, t)
- *                               U = hi16 * 2^16 + lo16
- *   16-bit lane j of a Philox output (w0, w1, w2, w3) is (w_{j/2} >> (16 (j%2))) & 0xffff.
+ *   block draw U of block b (inputs 64b .. 64b+63) of neuron k, step t:
+ *                               (b/4, k, 3*2^16 + l, t); word b%4
+ *   event draws V_0, V_1, ... of that block, in this order:
+ *                               words 0..3 of (b, k, (4 + r)*2^16 + l, t), r = 0, 1, ...
  *   Layers are numbered l = 1..L as in the paper.
  */
 #include <math.h>
@@ -111,10 +124,6 @@ static void philox_at(uint64_t seed, uint32_t c0, uint32_t c1, uint32_t c2, uint
   or_philox4x32_10(ctr, key, out);
 }
 
-static uint32_t lane16(const uint32_t w[4], int j) {
-  return (w[j / 2] >> (16 * (j % 2))) & 0xffffu;
-}
-
 /* Initial hidden weight h_{ik} of layer l (Alg. 1 l.2: uniform on {+-1}). */
 int32_t or_init_h(uint64_t seed, int32_t l, int32_t k, int32_t i) {
   uint32_t w[4];
@@ -129,26 +138,80 @@ int32_t or_init_rho(uint64_t seed, int32_t l, int32_t k, int32_t j) {
   return (w[j % 4] >> 31) ? +1 : -1;
 }
 
-/* The 32-bit integer U behind the Uniform(0,1) draw p = U / 2^32 for hidden
- * weight h_{ik} of layer l at step t (Alg. 3 l.7). */
-uint32_t or_uniform32(uint64_t seed, int32_t l, int32_t k, int32_t i, uint32_t t) {
-  uint32_t hi[4], lo[4];
-  philox_at(seed, (uint32_t)(i / 8), (uint32_t)k, (3u << 16) + (uint32_t)l, t, hi);
-  philox_at(seed, (uint32_t)(i / 8), (uint32_t)k, (4u << 16) + (uint32_t)l, t, lo);
-  return (lane16(hi, i % 8) << 16) | lane16(lo, i % 8);
-}
-
-/* Reinforcement threshold of Alg. 3 l.8: q = p_r sqrt(2 / (pi K_l)), and the
- * integer T with (U < T) <=> (U / 2^32 < q) for every 32-bit U (reading O9). */
+/* Reinforcement probability of Alg. 3 l.8: q = p_r sqrt(2 / (pi K_l)). */
 double or_reinforce_prob(double p_r, int32_t K_l) {
   return p_r * sqrt(2.0 / (M_PI * (double)K_l));
 }
 
-uint64_t or_reinforce_threshold(double p_r, int32_t K_l) {
-  double q = or_reinforce_prob(p_r, K_l);
-  if (!(q > 0.0)) return 0;
-  if (q >= 1.0) return (uint64_t)1 << 32;
-  return (uint64_t)ceil(q * 4294967296.0);
+/* thr(x) of reading O9: the integer T with (V < T) <=> (V / 2^32 < x) for
+ * every 32-bit V. */
+static uint64_t thr(double x) {
+  if (!(x > 0.0)) return 0;
+  if (x >= 1.0) return (uint64_t)1 << 32;
+  return (uint64_t)ceil(x * 4294967296.0);
+}
+
+/* The thresholds of reading O9 for a block of n inputs (1 <= n <= 64):
+ * any = thr(1 - (1-q)^n); first[j] = thr((1 - (1-q)^(j+1)) / (1 - (1-q)^n)),
+ * j < n; gap[g] = thr(1 - (1-q)^(g+1)), g < n - 1. */
+void or_r_block_tables(double q, int32_t n, uint64_t* any, uint64_t* first, uint64_t* gap) {
+  if (q > 1.0) q = 1.0;
+  const double s = 1.0 - q;
+  double pw[65];  /* pw[m] = (1-q)^m */
+  pw[0] = 1.0;
+  for (int32_t m = 1; m <= n; m++) pw[m] = pw[m - 1] * s;
+  const double p_any = 1.0 - pw[n];
+  *any = thr(p_any);
+  for (int32_t j = 0; j < n; j++) first[j] = thr((1.0 - pw[j + 1]) / p_any);
+  for (int32_t g = 0; g + 1 < n; g++) gap[g] = thr(1.0 - pw[g + 1]);
+}
+
+/* The sequence of event draws V_0, V_1, ... of one block (stream layout). */
+typedef struct {
+  uint64_t seed;
+  uint32_t b, k, l, t;
+  uint32_t w[4];
+  int32_t used;  /* draws taken so far */
+} ev_stream;
+
+static uint32_t next_draw(ev_stream* e) {
+  if (e->used % 4 == 0)
+    philox_at(e->seed, e->b, e->k, ((4u + (uint32_t)(e->used / 4)) << 16) + e->l, e->t, e->w);
+  return e->w[e->used++ % 4];
+}
+
+/* Reinforcement events of neuron k of layer l at step t (Alg. 3 l.5-12,
+ * reading O9): fire[i] = 1 iff h_{ik} is reinforced, i < K_prev. */
+void or_r_events(uint64_t seed, int32_t l, int32_t k, uint32_t t, int32_t K_prev, double q,
+                 uint8_t* fire) {
+  uint64_t any[2], first[2][64], gap[2][64];
+  const int32_t tail = K_prev % 64;
+  or_r_block_tables(q, 64, &any[0], first[0], gap[0]);
+  if (tail) or_r_block_tables(q, tail, &any[1], first[1], gap[1]);
+  memset(fire, 0, (size_t)K_prev);
+  for (int32_t b = 0; 64 * b < K_prev; b++) {
+    const int32_t n = (K_prev - 64 * b < 64) ? K_prev - 64 * b : 64;
+    const int32_t x = (n == 64) ? 0 : 1;
+    uint32_t w[4];
+    philox_at(seed, (uint32_t)(b / 4), (uint32_t)k, (3u << 16) + (uint32_t)l, t, w);
+    if (!((uint64_t)w[b % 4] < any[x])) continue;  /* no event in this block */
+    ev_stream e = {seed, (uint32_t)b, (uint32_t)k, (uint32_t)l, t, {0, 0, 0, 0}, 0};
+    /* first event: the least j with V < first[j] (first[n-1] = 2^32, so the
+     * scan stops inside the block) */
+    uint32_t V = next_draw(&e);
+    int32_t p = 0;
+    while (p < n - 1 && !((uint64_t)V < first[x][p])) p++;
+    fire[64 * b + p] = 1;
+    /* later events: geometric gaps, cut at the end of the block */
+    while (p < n - 1) {
+      V = next_draw(&e);
+      int32_t g = 0;
+      while (g <= n - 2 - p && !((uint64_t)V < gap[x][g])) g++;
+      if (g > n - 2 - p) break;
+      p = p + 1 + g;
+      fire[64 * b + p] = 1;
+    }
+  }
 }
 
 /* Sec. 4.3: gamma* = the divisor of K_l closest to the range [75, 105]
@@ -262,10 +325,10 @@ void or_select(const int32_t* z, int32_t b, int32_t K, const int8_t* P, int32_t 
 /* ------------------------------------------------------------------------ */
 
 /* Clipped perceptron over U_l, in (mu, g) order (O8), then reinforcement of
- * every h of the layer with threshold T at step t (O9, O10).  H: K_prev x K. */
+ * every h of the layer with probability q at step t (O9, O10).  H: K_prev x K. */
 void or_perceptron_update(int32_t* H, int32_t K_prev, int32_t K, const int8_t* a_prev,
                           const int32_t* y, const int8_t* P, int32_t c, const int32_t* sel,
-                          int32_t b, int32_t G, int32_t h_max, uint64_t T, uint64_t seed,
+                          int32_t b, int32_t G, int32_t h_max, double q, uint64_t seed,
                           int32_t l, uint32_t t) {
   /* Clipped Perceptron, Alg. 3 l.2-4 */
   for (int32_t mu = 0; mu < b; mu++)
@@ -279,15 +342,20 @@ void or_perceptron_update(int32_t* H, int32_t K_prev, int32_t K, const int8_t* a
       }
     }
   /* Reinforcement, Alg. 3 l.5-12 */
-#pragma omp parallel for schedule(static)
-  for (int32_t k = 0; k < K; k++)
-    for (int32_t i = 0; i < K_prev; i++) {
-      uint32_t U = or_uniform32(seed, l, k, i, t);
-      if ((uint64_t)U < T) {
-        int32_t* h = &H[(int64_t)i * K + k];
-        *h = clip(*h + 2 * (*h > 0 ? 1 : -1), h_max);
-      }
+#pragma omp parallel
+  {
+    uint8_t* fire = (uint8_t*)malloc((size_t)(K_prev > 0 ? K_prev : 1));
+#pragma omp for schedule(static)
+    for (int32_t k = 0; k < K; k++) {
+      or_r_events(seed, l, k, t, K_prev, q, fire);
+      for (int32_t i = 0; i < K_prev; i++)
+        if (fire[i]) {
+          int32_t* h = &H[(int64_t)i * K + k];
+          *h = clip(*h + 2 * (*h > 0 ? 1 : -1), h_max);
+        }
     }
+    free(fire);
+  }
 }
 
 /* ------------------------------------------------------------------------ */
@@ -429,7 +497,7 @@ int or_train(or_model* m, const int8_t* x, const int32_t* y, int64_t n, int32_t 
       const int32_t G = m->K[l] / m->gamma[l];
       or_select(z[l], b, m->K[l], m->P[l], c, yb, mark[l], m->gamma[l], sel);
       or_perceptron_update(m->H[l], m->K[l - 1], m->K[l], a[l - 1], yb, m->P[l], c, sel, b, G,
-                           m->h_max, or_reinforce_threshold(m->p_r, m->K[l]), m->seed, l,
+                           m->h_max, or_reinforce_prob(m->p_r, m->K[l]), m->seed, l,
                            (uint32_t)m->t);
     }
     m->t += 1;

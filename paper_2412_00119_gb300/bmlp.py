@@ -64,7 +64,7 @@ SIGNATURES = [
     ("bmlp_get_info", C.c_int, [_vp, _i32p, _i32p, _i32p, _i32p, _i32p, _i32p]),
     ("bmlp_last_error", C.c_char_p, [_vp]),
     ("bmlp_gamma_rule", C.c_int32, [C.c_int32]),
-    ("bmlp_reinforce_threshold", C.c_uint64, [C.c_double, C.c_int32]),
+    ("bmlp_reinforce_tables", C.c_int, [C.c_double, C.c_int32, C.c_int32, _vp, _vp, _vp]),
     ("bmlp_debug_last_step", C.c_int, [_vp, C.c_int32, _vp, _vp, _vp, _vp]),
     ("bmlp_set_profiling", C.c_int, [_vp, C.c_int32]),
     ("bmlp_get_profile", C.c_int, [_vp, C.c_int32, _i64p, _f64p]),
@@ -229,8 +229,14 @@ def bmlp_gamma_rule(K):
     return lib().bmlp_gamma_rule(K)
 
 
-def bmlp_reinforce_threshold(p_r, K):
-    return int(lib().bmlp_reinforce_threshold(p_r, K))
+def bmlp_reinforce_tables(p_r, K, n):
+    """Sampler thresholds of a block of n inputs: (any, first[n], gap[n-1])."""
+    any_ = np.zeros(1, np.uint64)
+    first = np.zeros(64, np.uint64)
+    gap = np.zeros(64, np.uint64)
+    _check(lib().bmlp_reinforce_tables(p_r, K, n, any_.ctypes.data, first.ctypes.data,
+                                       gap.ctypes.data), None)
+    return int(any_[0]), first[:n].copy(), gap[:max(n - 1, 0)].copy()
 
 
 def bmlp_last_error(h=None):

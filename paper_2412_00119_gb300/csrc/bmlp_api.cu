@@ -39,7 +39,7 @@ struct bmlp {
   StepParams hp{};      // host copy of the parameter block
   StepParams* dP = nullptr;
   Ctrl* dCtrl = nullptr;
-  unsigned long long* dT = nullptr;
+  RTables* dRT = nullptr;
   std::vector<void*> allocs;
   // evaluation scratch (grown on demand)
   uint64_t* evA[2] = {nullptr, nullptr};
@@ -111,10 +111,44 @@ bool is_device_ptr(const void* p) {
 
 int words_of(int K) { return (K + 63) / 64; }
 
+// thr(x) of the reinforcement sampler: the integer T with (V < T) <=> (V / 2^32 < x)
+// for every 32-bit V.
+uint64_t sampler_thr(double x) {
+  if (!(x > 0.0)) return 0;
+  if (x >= 1.0) return (uint64_t)1 << 32;
+  return (uint64_t)std::ceil(x * 4294967296.0);
+}
+
+// Sampler thresholds of a block of n (1..64) inputs at probability q.
+void block_tables(double q, int n, unsigned long long* any, unsigned long long* first,
+                  unsigned long long* gap) {
+  if (q > 1.0) q = 1.0;
+  const double s = 1.0 - q;
+  double pw[65];
+  pw[0] = 1.0;
+  for (int m = 1; m <= n; ++m) pw[m] = pw[m - 1] * s;
+  const double p_any = 1.0 - pw[n];
+  *any = sampler_thr(p_any);
+  for (int j = 0; j < n; ++j) first[j] = sampler_thr((1.0 - pw[j + 1]) / p_any);
+  if (gap)
+    for (int g = 0; g + 1 < n; ++g) gap[g] = sampler_thr(1.0 - pw[g + 1]);
+}
+
+double reinforce_q(double p_r, int K) { return p_r * std::sqrt(2.0 / (M_PI * (double)K)); }
+
 int upload_thresholds(bmlp_t* h, cudaStream_t st) {
-  unsigned long long T[BMLP_MAX_LAYERS];
-  for (int l = 1; l <= h->L; ++l) T[l - 1] = bmlp_reinforce_threshold(h->p_r, h->K[l]);
-  CK(h, cudaMemcpyAsync(h->dT, T, sizeof(unsigned long long) * h->L, cudaMemcpyHostToDevice, st));
+  std::vector<RTables> rt((size_t)h->L);
+  for (int l = 1; l <= h->L; ++l) {
+    RTables& R = rt[(size_t)l - 1];
+    std::memset(&R, 0, sizeof(R));
+    const double q = reinforce_q(h->p_r, h->K[l]);
+    block_tables(q, 64, &R.any[0], R.first[0], R.gap);
+    const int tail = h->K[l - 1] % 64;
+    if (tail) block_tables(q, tail, &R.any[1], R.first[1], nullptr);
+  }
+  CK(h, cudaMemcpyAsync(h->dRT, rt.data(), sizeof(RTables) * (size_t)h->L, cudaMemcpyHostToDevice,
+                        st));
+  CK(h, cudaStreamSynchronize(st));  // rt is a host temporary
   return BMLP_OK;
 }
 
@@ -271,13 +305,15 @@ int32_t bmlp_gamma_rule(int32_t K) {
   return best;
 }
 
-uint64_t bmlp_reinforce_threshold(double p_r, int32_t K) {
-  if (K < 1) return 0;
-  const double pi = 3.14159265358979323846;
-  const double q = p_r * std::sqrt(2.0 / (pi * (double)K));
-  if (!(q > 0.0)) return 0;
-  if (q >= 1.0) return 1ull << 32;
-  return (uint64_t)std::ceil(q * 4294967296.0);
+int bmlp_reinforce_tables(double p_r, int32_t K, int32_t n, uint64_t* any_out,
+                          uint64_t* first_out, uint64_t* gap_out) {
+  if (K < 1 || n < 1 || n > 64 || !any_out || !first_out || !gap_out) return BMLP_EINVAL;
+  unsigned long long a = 0, f[64], g[64];
+  block_tables(reinforce_q(p_r, K), n, &a, f, g);
+  *any_out = a;
+  for (int j = 0; j < n; ++j) first_out[j] = f[j];
+  for (int j = 0; j + 1 < n; ++j) gap_out[j] = g[j];
+  return BMLP_OK;
 }
 
 const char* bmlp_last_error(const bmlp_t* h) {
@@ -333,7 +369,7 @@ int bmlp_create(const int32_t* widths, int32_t n_widths, int32_t classes, int16_
   cudaDeviceProp prop;
   cudaFuncAttributes fa;
   if (cudaGetDeviceProperties(&prop, h->device) != cudaSuccess || prop.major != 10 ||
-      update_kernel_attributes(&fa) != cudaSuccess) {
+      update_kernel_attributes(&fa, 0) != cudaSuccess) {
     (void)cudaGetLastError();
     delete h;
     return fail(nullptr, BMLP_ENODEV, "device has no sm_103a kernel image (needs a GB300)");
@@ -380,12 +416,18 @@ int bmlp_create(const int32_t* widths, int32_t n_widths, int32_t classes, int16_
   }
   h->updCtas = cta;
   P.upd_ctas_total = cta;
-  h->updSmem = sizeof(int32_t) * ((size_t)(bs + 1) / 2 + (size_t)(kUpdThreads / 32) * bs);
+  P.nblk_max = 0;
+  for (int l = 1; l <= L; ++l) P.nblk_max = std::max(P.nblk_max, (widths[l - 1] + 63) / 64);
+  h->updSmem = update_smem_bytes(bs, P.nblk_max);
+  {
+    cudaError_t ea = update_kernel_attributes(&fa, h->updSmem);
+    if (ea != cudaSuccess) return bail(cuda_fail(h, ea, "update kernel shared memory attribute"));
+  }
   if ((rc = dalloc(h, &h->dP, 1)) || (rc = dalloc(h, &h->dCtrl, 1)) ||
-      (rc = dalloc(h, &h->dT, BMLP_MAX_LAYERS)))
+      (rc = dalloc(h, &h->dRT, BMLP_MAX_LAYERS)))
     return bail(rc);
   P.ctrl = h->dCtrl;
-  P.T = h->dT;
+  P.rt = h->dRT;
   if (cudaMallocHost(&h->hostPinned, 4 * sizeof(unsigned long long)) != cudaSuccess) {
     h->hostPinned = nullptr;
     return bail(fail(h, BMLP_ENOMEM, "cudaMallocHost failed"));

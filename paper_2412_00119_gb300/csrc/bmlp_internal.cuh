@@ -59,12 +59,27 @@ struct Ctrl {
   uint32_t any_mark[BMLP_MAX_LAYERS];
 };
 
+// Thresholds of the reinforcement sampler of one layer (Alg. 3 l.5-12): the
+// events of a neuron row are drawn per block of 64 inputs (the last block
+// holds K_in mod 64 when that is not 0).  For a block of n inputs:
+//   any      = thr(1 - (1-q)^n)        at least one event iff the block draw < any
+//   first[j] = thr((1 - (1-q)^(j+1)) / (1 - (1-q)^n))   first event: least j with V < first[j]
+//   gap[g]   = thr(1 - (1-q)^(g+1))    next event p + 1 + g: least g <= n-2-p with V < gap[g]
+// thr(x) = ceil(x 2^32) (0 for x <= 0, 2^32 for x >= 1); (1-q)^m a left-to-right
+// IEEE product.  Index [0]: n = 64, [1]: the last, shorter block.
+struct RTables {
+  unsigned long long any[2];
+  unsigned long long first[2][64];
+  unsigned long long gap[64];       // entries g < 63 (independent of n)
+};
+
 struct StepParams {
   DevLayer layer[BMLP_MAX_LAYERS];
   const uint64_t* x;            // packed inputs of the current train call
   const int32_t* y;             // labels of the current train call
   int64_t n;                    // patterns in the current train call
-  const unsigned long long* T;  // [L] reinforcement thresholds (Alg. 3 l.8)
+  const RTables* rt;            // [L] reinforcement sampler thresholds
+  int32_t nblk_max;             // max over layers of ceil(K_in / 64)
   Ctrl* ctrl;
   int32_t L, c, bs, h_max, r_num, r_den, nw0, upd_ctas_total;
   int32_t hb;                   // lattice-index offset exponent (see H above)
@@ -118,7 +133,12 @@ __global__ void k_cls_select(const StepParams* P);
 // boundaries of the lattice index).
 void launch_update(bool pow2, unsigned grid, size_t smem, cudaStream_t st, const StepParams* P,
                    uint32_t key0, uint32_t key1);
-cudaError_t update_kernel_attributes(cudaFuncAttributes* fa);
+// Attributes of the update kernel; smem > 0 also raises its dynamic shared
+// memory limit to smem bytes.
+cudaError_t update_kernel_attributes(cudaFuncAttributes* fa, size_t smem);
+// Dynamic shared memory of the update kernel for mini-batches of bs and rows
+// of at most nblk_max blocks of 64 inputs.
+size_t update_smem_bytes(int bs, int nblk_max);
 // Generic forward for evaluation: A (M x nw_in) against W -> Aout (M x nw_out).
 __global__ void k_forward_eval(const uint64_t* __restrict__ A, int64_t M, int nw_in,
                                const uint64_t* __restrict__ W, int N, int Kin,

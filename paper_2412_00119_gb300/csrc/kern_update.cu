@@ -113,10 +113,19 @@ __global__ void __launch_bounds__(kClsThreads) k_cls_select(const StepParams* __
 // ---------------------------------------------------------------------------
 // Hidden-weight update, fused with the visible-weight repack (Alg. 3, Sec. 3.1).
 // CTA = (layer, group g, slice of kUpdRowsPerCta neurons).  A warp owns one
-// neuron row k at a time: it collects, in ascending mu, the patterns whose
-// selection in group g is k (the CP tuples of k), then streams the row in
-// chunks of 8 hidden weights, two chunks per lane per iteration, with a
-// rotating queue of four 16-byte vectors in flight per lane.
+// neuron row k at a time:
+//   1. it collects, in ascending mu, the patterns whose selection in group g
+//      is k (the CP tuples of k);
+//   2. it draws the row's reinforcement events into a shared bitmap, one
+//      64-bit word per block of 64 inputs: lane j draws the block draws of
+//      blocks 4j .. 4j+3 (one Philox call) and, for each block that holds an
+//      event, the event draws (binary searches in the layer's monotone
+//      threshold tables, staged in shared memory);
+//   3. it streams the row in chunks of 8 hidden weights, two chunks per lane
+//      per iteration, with a rotating queue of four 16-byte vectors in flight
+//      per lane: the CP tuples, then the chunk's reinforcement events (its byte
+//      of the bitmap; lanes with an event step away from 0, as Alg. 3 orders
+//      CP before R), then H and the W byte are written.
 // H holds each weight as its lattice index v = (h + h_max)/2 + 2^hb (see
 // DevLayer): a CP or R event is a step of +-1 in v, and v stays in
 // [2^hb, 2^hb + h_max] subset of (0, 2^15).  A 32-bit word holds two lanes, so a
@@ -124,19 +133,11 @@ __global__ void __launch_bounds__(kClsThreads) k_cls_select(const StepParams* __
 // After a step a lane can only have left the range by one, to 2^hb - 1 (bit hb
 // clear) or to 2^hb + h_max + 1 (= 2^(hb+1) when h_max + 1 = 2^hb, kPow2); the
 // clip moves it back.  h > 0 is the lane's bit hb - 1 (kPow2) or v >= 2^hb +
-// (h_max + 1)/2.  All of the rule runs on packed lanes, warp-uniform branches
-// only:
-//   CP: per tuple (ascending mu) add the packed +-1 steps 2 a^mu_i rho_{k,y^mu}/2
-//       from a 16-entry shared nibble table, then clip.
-//   R : the Philox draw's 16-bit lanes line up with the weight lanes; lanes
-//       whose high half is below T's high half (< 2^15) fire and step away
-//       from 0, then clip.
-//   W : one byte per chunk from the lanes' sign flags, written in place.
-// A chunk with a tie (draw high half == T high half, probability 8 / 2^16),
-// the partly padded last chunk of a row, and every chunk when T >= 2^31 take
-// the per-weight path instead.  Chunks of padding only are never touched.
-// Layers with an empty M_l are skipped (no CP, no R).  The last warp to finish
-// advances the step counters and clears the per-step flags.
+// (h_max + 1)/2.  The CP step per tuple adds the packed +-1 steps
+// 2 a^mu_i rho_{k,y^mu}/2 from a 16-entry shared nibble table, then clips.
+// The partly padded last chunk of a row runs per weight.  Layers with an
+// empty M_l are skipped (no CP, no R).  The last warp to finish advances the
+// step counters and clears the per-step flags.
 // ---------------------------------------------------------------------------
 namespace {
 
@@ -170,14 +171,12 @@ struct Enc {
   __device__ __forceinline__ uint32_t enc(int h) const { return (uint32_t)((h + h_max) / 2 + base); }
 };
 
-// Per-weight path (rule as printed, on decoded h): CP, R and W for the first
-// `nvalid` weights of the chunk, from the loaded values.  Rarely taken; its
-// loops stay rolled.
-__device__ __forceinline__ ChunkOut chunk_scalar(uint4 w, int ch, int nvalid,
-                                                 const int32_t* list, int n_t, const uint8_t* aprev,
-                                                 uint32_t arow_bytes, Enc E, uint32_t Thi,
-                                                 uint32_t Tlo, uint32_t key0, uint32_t key1,
-                                                 uint32_t k, uint32_t c2_lo, uint32_t t, uint4 rh) {
+// Per-weight path (rule as printed, on decoded h): CP, then R for the inputs
+// whose bit of `fire` is set, and W, for the first `nvalid` weights of the
+// chunk.  Taken only by the ragged last chunk of a row; its loops stay rolled.
+__device__ __forceinline__ ChunkOut chunk_scalar(uint4 w, int ch, int nvalid, const int32_t* list,
+                                                 int n_t, const uint8_t* aprev, uint32_t arow_bytes,
+                                                 Enc E, uint32_t fire) {
 #pragma unroll 1
   for (int q = 0; q < n_t; ++q) {
     const int e = list[q];
@@ -190,18 +189,12 @@ __device__ __forceinline__ ChunkOut chunk_scalar(uint4 w, int ch, int nvalid,
       set_lane_v(w, j, E.enc(clip_h(E.dec(lane_v(w, j)) + 2 * step, E.h_max)));
     }
   }
-  uint32_t ties = 0;
-  for (int j = 0; j < 8; ++j) ties |= (lane16(rh, j) == Thi ? 1u : 0u) << j;
-  uint4 rl = make_uint4(0, 0, 0, 0);
-  if (ties) rl = philox4x32_10(make_uint4((uint32_t)ch, k, c2_lo, t), key0, key1);
   ChunkOut out;
   out.wbyte = 0;
 #pragma unroll 1
   for (int j = 0; j < nvalid; ++j) {
-    const uint32_t u = lane16(rh, j);
-    const bool fire = (u < Thi) || (((ties >> j) & 1u) && lane16(rl, j) < Tlo);
     int h = E.dec(lane_v(w, j));
-    if (fire) {
+    if ((fire >> j) & 1u) {
       h = clip_h(h + (h > 0 ? 2 : -2), E.h_max);
       set_lane_v(w, j, E.enc(h));
     }
@@ -224,19 +217,6 @@ __device__ __forceinline__ uint32_t gather_top(uint32_t a, uint32_t b, uint32_t 
   return ((p0 * 0x00204081u) >> 28) | (((p1 * 0x00204081u) >> 28) << 4);
 }
 
-// lanes of a draw word whose high half u < Thi (< 2^15): top bit clear, low 15
-// bits below Thi (guard-bit subtraction, no borrow between lanes)
-__device__ __forceinline__ uint32_t fire_flags(uint32_t u, uint32_t Tpair) {
-  const uint32_t dd = ((u & 0x7FFF7FFFu) | kLaneTop) - Tpair;
-  return ~(dd | u) & kLaneTop;
-}
-
-// lanes of a draw word whose high half u <= Thi (< 2^15): the same test
-// against T1pair = pair(Thi + 1), Thi + 1 <= 2^15
-__device__ __forceinline__ uint32_t le_flags(uint32_t u, uint32_t T1pair) {
-  return fire_flags(u, T1pair);
-}
-
 template <bool kPow2>
 struct Lanes {
   int hb;
@@ -257,6 +237,11 @@ struct Lanes {
     if (kPow2) return (v << (16 - hb)) & kLaneTop;
     return ((v | kLaneTop) - pos_pair) & kLaneTop;
   }
+  // lanes with f = 1 (f: 0 or 1 per lane) step away from 0, then clip
+  __device__ __forceinline__ uint32_t reinforce(uint32_t v, uint32_t f) const {
+    const uint32_t p = pos_top(v) >> 15;
+    return clip(v + (f & p) - (f & ~p));
+  }
   // W byte of a chunk (lane j -> bit j = h_j > 0)
   __device__ __forceinline__ uint32_t w_byte(const uint4& w) const {
     if (kPow2) {
@@ -271,21 +256,67 @@ struct Lanes {
     }
     return gather_top(pos_top(w.x), pos_top(w.y), pos_top(w.z), pos_top(w.w));
   }
-  // fired lanes step away from 0 (then clip)
-  __device__ __forceinline__ uint32_t reinforce(uint32_t v, uint32_t fire_top) const {
-    const uint32_t f = fire_top >> 15;
-    const uint32_t p = pos_top(v) >> 15;
-    return clip(v + (f & p) - (f & ~p));
-  }
 };
 
+__device__ __forceinline__ uint32_t word_of(const uint4& v, int i) {
+  return i == 0 ? v.x : (i == 1 ? v.y : (i == 2 ? v.z : v.w));
+}
+
+// Least j in [0, hi] with V < tab[j], or hi when there is none (tab
+// nondecreasing).
+__device__ __forceinline__ int least_below(uint32_t V, const unsigned long long* tab, int hi) {
+  int lo = 0;
+  while (lo < hi) {
+    const int mid = (lo + hi) >> 1;
+    if ((unsigned long long)V < tab[mid]) hi = mid;
+    else lo = mid + 1;
+  }
+  return lo;
+}
+
+// The events of block b (n inputs, tables index x) of neuron k at step t,
+// given that the block holds at least one: the first from the first-event
+// table, the next ones by geometric gaps cut at the block's end; the draws
+// are the words of Philox((b, k, (4 + r) 2^16 + l, t)), r = 0, 1, ... in order.
+__device__ __forceinline__ uint64_t block_events(const RTables& R, int x, int n, uint32_t b,
+                                                 uint32_t k, uint32_t l, uint32_t t, uint32_t key0,
+                                                 uint32_t key1) {
+  uint32_t r = 0;
+  uint4 v = philox4x32_10(make_uint4(b, k, (4u << 16) + l, t), key0, key1);
+  int used = 1;
+  int p = least_below(v.x, R.first[x], n - 1);
+  uint64_t mask = 1ull << p;
+#pragma unroll 1
+  while (p < n - 1) {
+    if (used == 4) {
+      ++r;
+      v = philox4x32_10(make_uint4(b, k, ((4u + r) << 16) + l, t), key0, key1);
+      used = 0;
+    }
+    const uint32_t V = word_of(v, used++);
+    const int gmax = n - 2 - p;
+    if (!((unsigned long long)V < R.gap[gmax])) break;  // no further event in the block
+    p += 1 + least_below(V, R.gap, gmax);
+    mask |= 1ull << p;
+  }
+  return mask;
+}
+
 }  // namespace
+
+size_t update_smem_bytes(int bs, int nblk_max) {
+  const int nwarps = kUpdThreads / 32;
+  size_t words = (size_t)(bs + 1) / 2 + (size_t)nwarps * bs;  // s_sel (int16), s_list (int32)
+  words = (words + 1) & ~(size_t)1;                           // 8-byte alignment
+  return sizeof(int32_t) * words + sizeof(uint64_t) * (size_t)nwarps * nblk_max + sizeof(RTables);
+}
 
 template <bool kPow2>
 __global__ void __launch_bounds__(kUpdThreads, 3) k_update(const StepParams* __restrict__ P,
                                                            uint32_t key0, uint32_t key1) {
   extern __shared__ int32_t dyn[];
   __shared__ uint2 s_dn[2][16];
+  __shared__ uint2 s_fire[16];
   const int bid = blockIdx.x;
   int li = 0;
   while (li + 1 < P->L && bid >= P->layer[li + 1].upd_cta_base) ++li;
@@ -305,10 +336,22 @@ __global__ void __launch_bounds__(kUpdThreads, 3) k_update(const StepParams* __r
     const int r1 = min(r0 + kUpdRowsPerCta, gamma);
     const int64_t start = (int64_t)s * P->bs;
     const int bsz = (int)batch_size(P, start);
-    int16_t* s_sel = reinterpret_cast<int16_t*>(dyn);               // [bs]
-    int32_t* s_list = dyn + (P->bs + 1) / 2 + warp * P->bs;         // [nwarps][bs]
+    // dynamic shared memory: s_sel [bs] int16 | s_list [nwarps][bs] int32 |
+    // (8-byte aligned) s_ev [nwarps][nblk_max] uint64 | s_rt (this layer's tables)
+    int16_t* s_sel = reinterpret_cast<int16_t*>(dyn);
+    int32_t* s_list = dyn + (P->bs + 1) / 2 + warp * P->bs;
+    size_t words = (size_t)(P->bs + 1) / 2 + (size_t)nwarps * P->bs;
+    words = (words + 1) & ~(size_t)1;
+    uint64_t* s_ev_all = reinterpret_cast<uint64_t*>(dyn + words);
+    uint64_t* s_ev = s_ev_all + (size_t)warp * P->nblk_max;
+    RTables* s_rt = reinterpret_cast<RTables*>(s_ev_all + (size_t)nwarps * P->nblk_max);
 
     for (int m = threadIdx.x; m < bsz; m += blockDim.x) s_sel[m] = Ly.sel[(int64_t)m * Ly.G + g];
+    {
+      const unsigned long long* src = reinterpret_cast<const unsigned long long*>(P->rt + li);
+      unsigned long long* dst = reinterpret_cast<unsigned long long*>(s_rt);
+      for (int i = threadIdx.x; i < (int)(sizeof(RTables) / 8); i += blockDim.x) dst[i] = src[i];
+    }
     // s_dn[r][n]: the +-1 lattice steps of the 4 weights of nibble n, two lanes
     // per word (d_lo + 2^16 d_hi), d = +1 for a set bit, negated for r = 1
     // (rho = -1)
@@ -318,6 +361,10 @@ __global__ void __launch_bounds__(kUpdThreads, 3) k_update(const StepParams* __r
 #pragma unroll
       for (int j = 0; j < 4; ++j) d[j] = (((n >> j) & 1) ? 1 : -1) * (r ? -1 : 1);
       s_dn[r][n] = make_uint2((uint32_t)(d[0] + 65536 * d[1]), (uint32_t)(d[2] + 65536 * d[3]));
+      // s_fire[n]: 1 in each lane of nibble n whose bit is set, two lanes per word
+      if (r == 0)
+        s_fire[n] = make_uint2((uint32_t)((n & 1) | ((n >> 1) & 1) << 16),
+                               (uint32_t)(((n >> 2) & 1) | ((n >> 3) & 1) << 16));
     }
     __syncthreads();
 
@@ -331,24 +378,18 @@ __global__ void __launch_bounds__(kUpdThreads, 3) k_update(const StepParams* __r
     LN.hb = P->hb;
     LN.over_pair = (uint32_t)(E.base + E.h_max + 1) * kLaneOne;
     LN.pos_pair = (uint32_t)(E.base + (E.h_max + 1) / 2) * kLaneOne;
-    const unsigned long long T = P->T[li];
-    const uint32_t Thi = (uint32_t)(T >> 16);   // 0..65536
-    const uint32_t Tlo = (uint32_t)(T & 0xFFFFu);
-    const uint32_t Tpair = Thi * kLaneOne;
-    const uint32_t T1pair = (Thi + 1u) * kLaneOne;  // used only when packed
-    const bool packed = Thi < 0x8000u;           // the SIMD draw test is exact
-    const uint32_t c2_hi = (3u << 16) + l, c2_lo = (4u << 16) + l;
     const uint32_t tt = (uint32_t)t;
     const int Kin = Ly.Kin;
     const int nch = (Kin + 7) >> 3;             // chunks holding at least one input
     const int full = Kin >> 3;                  // chunks of 8 real inputs
+    const int nblk = (Kin + 63) >> 6;           // blocks of the reinforcement sampler
     const uint32_t arow_bytes = (uint32_t)Ly.nw_in * 8u;
     const uint8_t* aprev = (li == 0) ? reinterpret_cast<const uint8_t*>(P->x + start * P->nw0)
                                      : reinterpret_cast<const uint8_t*>(P->layer[li - 1].A);
 
     for (int rr = r0 + warp; rr < r1; rr += nwarps) {
       const int k = g * gamma + rr;
-      // CP tuples of neuron k, ascending mu
+      // ---- 1. CP tuples of neuron k, ascending mu ----
       int n_t = 0;
       for (int base = 0; base < bsz; base += 32) {
         const int m = base + lane;
@@ -362,18 +403,35 @@ __global__ void __launch_bounds__(kUpdThreads, 3) k_update(const StepParams* __r
         }
         n_t += __popc(bal);
       }
+      // ---- 2. reinforcement events of the row, one bitmap word per block ----
+#pragma unroll 1
+      for (int gq = lane; 4 * gq < nblk; gq += 32) {
+        const uint4 u = philox4x32_10(make_uint4((uint32_t)gq, (uint32_t)k, (3u << 16) + l, tt),
+                                      key0, key1);
+#pragma unroll
+        for (int wq = 0; wq < 4; ++wq) {
+          const int b = 4 * gq + wq;
+          if (b < nblk) {
+            const int n = min(64, Kin - 64 * b);
+            const int x = (n == 64) ? 0 : 1;
+            uint64_t mask = 0;
+            if ((unsigned long long)word_of(u, wq) < s_rt->any[x])
+              mask = block_events(*s_rt, x, n, (uint32_t)b, (uint32_t)k, l, tt, key0, key1);
+            s_ev[b] = mask;
+          }
+        }
+      }
       __syncwarp();
 
+      // ---- 3. CP and W over the row ----
       int16_t* hrow = Ly.H + (int64_t)k * Ly.ldh;
       uint8_t* wrow = reinterpret_cast<uint8_t*>(Ly.W + (int64_t)k * Ly.nw_in);
-      // the activation bytes of the first kPre tuples are fetched at the top of
-      // each iteration, ahead of the Philox chains, so that their latency
-      // overlaps the draw
       // Each iteration handles two chunks per lane, ch and ch + 32 (64 chunks
-      // per warp), so the tuple loop and the loop control are shared and the
-      // two Philox chains run side by side.  A rotating queue keeps the H
-      // vectors of the next iteration in flight (4 per lane).  Every lane runs
-      // the same number of iterations (warp votes below).
+      // per warp), so the tuple loop and the loop control are shared.  A
+      // rotating queue keeps the H vectors of the next iteration in flight (4
+      // per lane); the activation bytes of the first kPre tuples are fetched at
+      // the top of each iteration.  Every lane runs the same number of
+      // iterations.
       uint4 q0 = make_uint4(0, 0, 0, 0), q1 = q0, q2 = q0, q3 = q0;
       if (lane < nch) q0 = __ldcs(reinterpret_cast<const uint4*>(hrow + 8 * lane));
       if (lane + 32 < nch) q1 = __ldcs(reinterpret_cast<const uint4*>(hrow + 8 * (lane + 32)));
@@ -383,8 +441,8 @@ __global__ void __launch_bounds__(kUpdThreads, 3) k_update(const StepParams* __r
 #pragma unroll 1
       for (int it = 0; it < iters2; ++it) {
         int chv[2];
-        bool live[2], simd[2], slow[2];
-        uint4 w[2], rh[2];
+        bool live[2];
+        uint4 w[2];
         uint32_t pb[2] = {0u, 0u};  // activation bytes of tuples 0..kPre-1, one per byte
         chv[0] = 64 * it + lane;
         chv[1] = chv[0] + 32;
@@ -405,13 +463,6 @@ __global__ void __launch_bounds__(kUpdThreads, 3) k_update(const StepParams* __r
         q1 = q3;
         if (chv[0] + 128 < nch) q2 = __ldcs(reinterpret_cast<const uint4*>(hrow + 8 * (chv[0] + 128)));
         if (chv[1] + 128 < nch) q3 = __ldcs(reinterpret_cast<const uint4*>(hrow + 8 * (chv[1] + 128)));
-#pragma unroll
-        for (int u = 0; u < 2; ++u) {
-          simd[u] = packed && chv[u] < full;   // this chunk runs on packed lanes
-          slow[u] = live[u] && !simd[u];
-          rh[u] = philox4x32_10(make_uint4((uint32_t)chv[u], (uint32_t)k, c2_hi, tt), key0, key1);
-        }
-        // ---- Clipped Perceptron ----
 #pragma unroll
         for (int q = 0; q < kPre; ++q) {
           if (q < n_t) {
@@ -442,37 +493,32 @@ __global__ void __launch_bounds__(kUpdThreads, 3) k_update(const StepParams* __r
             w[u].w = LN.clip(w[u].w + dh.y);
           }
         }
-        // ---- Reinforcement: per draw word, only where some lane of the warp
-        // has a candidate (draw high half <= Thi); a tie (== Thi) sends the
-        // chunk to the per-weight path, which restarts from the loaded values.
+        // ---- R: the chunks' bytes of the row's event bitmap ----
+        uint32_t fb[2];
 #pragma unroll
-        for (int u = 0; u < 2; ++u) {
-          const bool on = live[u] && simd[u];
-          uint32_t* wv = reinterpret_cast<uint32_t*>(&w[u]);
-          const uint32_t* rv = reinterpret_cast<const uint32_t*>(&rh[u]);
+        for (int u = 0; u < 2; ++u)
+          fb[u] = live[u] ? (uint32_t)reinterpret_cast<const uint8_t*>(s_ev)[chv[u]] : 0u;
+        if (__any_sync(kFull, (fb[0] | fb[1]) != 0u)) {
 #pragma unroll
-          for (int j = 0; j < 4; ++j) {
-            const uint32_t cand = on ? le_flags(rv[j], T1pair) : 0u;
-            if (__any_sync(kFull, cand != 0u)) {
-              if (cand != 0u) {
-                const uint32_t fire = fire_flags(rv[j], Tpair);
-                if (cand & ~fire) slow[u] = true;
-                else wv[j] = LN.reinforce(wv[j], fire);
-              }
+          for (int u = 0; u < 2; ++u) {
+            if (fb[u] != 0u) {
+              const uint2 fl = s_fire[fb[u] & 15u], fh = s_fire[fb[u] >> 4];
+              w[u].x = LN.reinforce(w[u].x, fl.x);
+              w[u].y = LN.reinforce(w[u].y, fl.y);
+              w[u].z = LN.reinforce(w[u].z, fh.x);
+              w[u].w = LN.reinforce(w[u].w, fh.y);
             }
           }
         }
-        // ---- W, store ----
 #pragma unroll
         for (int u = 0; u < 2; ++u) {
           uint32_t wbyte = LN.w_byte(w[u]);
-          if (slow[u]) {
-            // the per-weight path restarts from the row as loaded (H is
-            // written back only below)
+          if (live[u] && chv[u] >= full) {
+            // the partly padded last chunk: per weight, from the row as
+            // loaded (H is written back only below)
             const uint4 w0 = *reinterpret_cast<const uint4*>(hrow + 8 * chv[u]);
-            const ChunkOut o = chunk_scalar(w0, chv[u], min(8, Kin - 8 * chv[u]), s_list, n_t,
-                                            aprev, arow_bytes, E, Thi, Tlo, key0, key1, (uint32_t)k,
-                                            c2_lo, tt, rh[u]);
+            const ChunkOut o = chunk_scalar(w0, chv[u], Kin - 8 * chv[u], s_list, n_t, aprev,
+                                            arow_bytes, E, fb[u]);
             w[u] = o.w;
             wbyte = o.wbyte;
           }
@@ -482,7 +528,7 @@ __global__ void __launch_bounds__(kUpdThreads, 3) k_update(const StepParams* __r
           }
         }
       }
-      __syncwarp();
+      __syncwarp();   // s_ev and s_list are reused by the next row
     }
   }
 
@@ -509,8 +555,14 @@ void launch_update(bool pow2, unsigned grid, size_t smem, cudaStream_t st, const
     k_update<false><<<grid, kUpdThreads, smem, st>>>(P, key0, key1);
 }
 
-cudaError_t update_kernel_attributes(cudaFuncAttributes* fa) {
-  return cudaFuncGetAttributes(fa, k_update<true>);
+cudaError_t update_kernel_attributes(cudaFuncAttributes* fa, size_t smem) {
+  cudaError_t e = cudaFuncGetAttributes(fa, k_update<true>);
+  if (e != cudaSuccess || smem == 0) return e;
+  if ((e = cudaFuncSetAttribute(k_update<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                (int)smem)) != cudaSuccess)
+    return e;
+  return cudaFuncSetAttribute(k_update<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              (int)smem);
 }
 
 // ---------------------------------------------------------------------------

@@ -10,8 +10,10 @@ Sources of the expected values:
   * hand-worked cases of Eq. 1 / Alg. 1 l.13-15, Alg. 2 and Alg. 3
     (``tests/golden/*.txt``, each derived in its comment header);
   * exhaustive brute force of the +-1 dot product, N - 2 popcount(a XOR w);
-  * exact rational arithmetic for the reinforcement threshold, a binomial
-    bound on the reinforcement rate, and the closed form of Alg. 1 l.21;
+  * exact rational arithmetic for the reinforcement probability and the
+    sampler's thresholds, the law of independent Bernoulli(q) events (marginal
+    rate, pair independence, per-block binomial counts), a binomial bound on
+    the reinforcement rate, and the closed form of Alg. 1 l.21;
   * invariants of Alg. 3 (odd h, |h| <= h_max, one lattice unit per event,
     reinforcement moves away from 0) and the learnability of a separable task.
 """
@@ -180,15 +182,20 @@ def check_perceptron_golden():
     y = np.array(d["y"][0], np.int32)
     rho = np.array(d["rho"], np.int8)
     sel = np.array(d["sel"], np.int32)
-    cp = O.perceptron_update(H, a, y, rho, sel, 3, 0, 7, 1, 0)
+    cp = O.perceptron_update(H, a, y, rho, sel, 3, 0.0, 7, 1, 0)
     assert cp.tolist() == d["cp"], cp.tolist()
-    cpr = O.perceptron_update(H, a, y, rho, sel, 3, 1 << 32, 7, 1, 0)
+    cpr = O.perceptron_update(H, a, y, rho, sel, 3, 1.0, 7, 1, 0)
     assert cpr.tolist() == d["cpr"], cpr.tolist()
 
 
+def _ceil_frac(x: Fraction) -> int:
+    return -((-x.numerator) // x.denominator)
+
+
 def check_threshold_exact():
-    """U < T  <=>  U / 2^32 < q, checked in exact rational arithmetic, and q is
-    p_r sqrt(2 / (pi K)) to within 2 ulp (40-digit decimal evaluation)."""
+    """q is p_r sqrt(2 / (pi K)) to within 2 ulp (40-digit decimal evaluation);
+    every threshold of the block sampler is ceil(x 2^32) of its double x (exact
+    rational check), and x is within 1e-12 of the exact (1-q)^m expression."""
     getcontext().prec = 40
     pi = Decimal("3.141592653589793238462643383279502884197")
     for p_r in (0.5, 0.25, 0.1234567, 1e-3, 0.9):
@@ -196,13 +203,37 @@ def check_threshold_exact():
             q = O.reinforce_prob(p_r, K)
             qd = Decimal(p_r) * (Decimal(2) / (pi * K)).sqrt()
             assert abs(Decimal(q) - qd) <= 2 * Decimal(math.ulp(q)), (p_r, K)
-            T = O.reinforce_threshold(p_r, K)
-            if q >= 1:
-                assert T == 1 << 32
-                continue
-            qf = Fraction(q)
-            assert Fraction(T - 1, 1 << 32) < qf <= Fraction(T, 1 << 32), (p_r, K, T)
-    assert O.reinforce_threshold(0.0, 100) == 0
+    two32 = 1 << 32
+    for q in (0.0044077, 0.0285, 0.05, 0.3, 0.77):
+        qf = Fraction(q)
+        for n in (1, 2, 7, 64):
+            any_, first, gap = O.r_block_tables(q, n)
+            s = 1.0 - q
+            pw = [1.0]
+            for _ in range(n):
+                pw.append(pw[-1] * s)
+            p_any = 1.0 - pw[n]
+            exact_any = 1 - (1 - qf) ** n
+            assert abs(Fraction(p_any) - exact_any) < Fraction(1, 10 ** 12), (q, n)
+            assert any_ == _ceil_frac(Fraction(p_any) * two32), (q, n, any_)
+            for j in range(n):
+                x = (1.0 - pw[j + 1]) / p_any
+                ex = (1 - (1 - qf) ** (j + 1)) / exact_any
+                assert abs(Fraction(x) - ex) < Fraction(1, 10 ** 12), (q, n, j)
+                want = two32 if x >= 1.0 else _ceil_frac(Fraction(x) * two32)
+                assert int(first[j]) == want, (q, n, j, int(first[j]), want)
+            assert int(first[n - 1]) == two32
+            for g in range(n - 1):
+                x = 1.0 - pw[g + 1]
+                assert abs(Fraction(x) - (1 - (1 - qf) ** (g + 1))) < Fraction(1, 10 ** 12)
+                assert int(gap[g]) == _ceil_frac(Fraction(x) * two32), (q, n, g)
+            assert np.all(np.diff(first.astype(np.float64)) >= 0)
+            assert np.all(np.diff(gap.astype(np.float64)) >= 0)
+    any0, first0, gap0 = O.r_block_tables(0.0, 64)
+    assert any0 == 0 and np.all(gap0 == 0)
+    for q in (1.0, 3.5):
+        a1, f1, g1 = O.r_block_tables(q, 64)
+        assert a1 == two32 and np.all(f1 == two32) and np.all(g1 == two32)
 
 
 def check_reinforce_rate():
@@ -218,33 +249,59 @@ def check_reinforce_rate():
     rho = np.ones((K, 2), np.int8)
     y = np.zeros(1, np.int32)
     q = 0.02
-    T = math.ceil(q * 2 ** 32)
-    H1 = O.perceptron_update(H, a, y, rho, sel, 255, T, 11, 2, 5)
+    H1 = O.perceptron_update(H, a, y, rho, sel, 255, q, 11, 2, 5)
     d = H1 - H
     moved = d != 0
     n = moved.sum()
     mean, sd = q * H.size, math.sqrt(q * (1 - q) * H.size)
     assert abs(n - mean) < 5 * sd, (n, mean, sd)
     assert np.array_equal(d[moved], 2 * np.sign(H[moved]))
-    H1b = O.perceptron_update(H, a, y, rho, sel, 255, T, 11, 2, 5)
+    H1b = O.perceptron_update(H, a, y, rho, sel, 255, q, 11, 2, 5)
     assert np.array_equal(H1, H1b)
-    H2 = O.perceptron_update(H, a, y, rho, sel, 255, T, 11, 2, 6)
+    H2 = O.perceptron_update(H, a, y, rho, sel, 255, q, 11, 2, 6)
     overlap = ((H2 - H) != 0) & moved
     assert overlap.sum() < 5 * q * n + 10
 
 
-def check_uniform_bits(n=40000):
-    """The 32-bit draws are uniform: each bit is set with frequency 1/2 and the
-    top 4 bits are uniform over 16 bins (chi-square, 15 dof, p ~ 1e-6 cut)."""
-    vals = np.array([O.uniform32(5, 1, k, i, 3) for k in range(n // 200) for i in range(200)],
-                    np.uint64)
-    for bit in range(32):
-        f = ((vals >> np.uint64(bit)) & np.uint64(1)).mean()
-        assert abs(f - 0.5) < 5 * math.sqrt(0.25 / vals.size), bit
-    counts = np.bincount((vals >> np.uint64(28)).astype(np.int64), minlength=16)
-    e = vals.size / 16
-    chi2 = ((counts - e) ** 2 / e).sum()
-    assert chi2 < 50, chi2
+def _events(q, K_prev, rows, seed=5, l=1, t=3):
+    return np.array([O.r_events(seed, l, k, t, K_prev, q) for k in range(rows)], np.float64)
+
+
+def check_event_law():
+    """The reinforcement events of a row are independent Bernoulli(q): every
+    input fires with frequency q (whole blocks and a ragged last block), pairs
+    inside a block and across a block boundary fire together with frequency
+    q^2, and the number of events of a 64-input block follows Binomial(64, q)
+    (chi-square).  q = 0 and q >= 1 give no event / every input."""
+    for q, rows in ((0.01, 4000), (0.05, 3000), (0.3, 1500)):
+        K_prev = 200                                   # blocks of 64, 64, 64, 8
+        ev = _events(q, K_prev, rows)
+        n = ev.shape[0]
+        # marginal rate per input position (pooled over rows)
+        f = ev.mean(axis=0)
+        sd = math.sqrt(q * (1 - q) / n)
+        assert np.all(np.abs(f - q) < 5.5 * sd), (q, float(np.abs(f - q).max() / sd))
+        assert abs(ev.mean() - q) < 5 * math.sqrt(q * (1 - q) / ev.size), (q, ev.mean())
+        # pairs: neighbours, a block boundary, the ragged block, far apart
+        for i, j in ((0, 1), (30, 31), (62, 63), (63, 64), (127, 128), (191, 192), (195, 199),
+                     (5, 70)):
+            both = (ev[:, i] * ev[:, j]).mean()
+            sd2 = math.sqrt(q * q * (1 - q * q) / n)
+            assert abs(both - q * q) < 5.5 * sd2 + 1e-12, (q, i, j, both)
+        # events per full block: Binomial(64, q)
+        counts = ev[:, :192].reshape(n * 3, 64).sum(axis=1).astype(np.int64)
+        lam = 64 * q
+        kmax = int(lam + 4 * math.sqrt(lam) + 2)
+        pmf = [math.comb(64, c) * q ** c * (1 - q) ** (64 - c) for c in range(kmax)]
+        obs = np.bincount(np.minimum(counts, kmax), minlength=kmax + 1)
+        exp = np.array(pmf + [1 - sum(pmf)]) * counts.size
+        keep = exp >= 5
+        chi2 = float((((obs - exp) ** 2 / np.maximum(exp, 1e-300))[keep]).sum())
+        dof = int(keep.sum()) - 1
+        assert chi2 < dof + 6 * math.sqrt(2 * dof) + 10, (q, chi2, dof)
+    assert _events(0.0, 130, 50).sum() == 0
+    for q in (1.0, 2.0):
+        assert np.all(_events(q, 130, 20) == 1)
 
 
 def check_update_invariants(seed=4):
@@ -259,7 +316,7 @@ def check_update_invariants(seed=4):
     rho = np.where(rng.random((K, c)) < 0.5, 1, -1).astype(np.int8)
     sel = -np.ones((3, 1), np.int32)
     sel[1, 0] = 7                       # one tuple: (mu=1, k=7), gamma = K
-    H1 = O.perceptron_update(H, a, y, rho, sel, h_max, 0, 1, 1, 0)
+    H1 = O.perceptron_update(H, a, y, rho, sel, h_max, 0.0, 1, 1, 0)
     d = H1 - H
     assert np.all(d[:, [k for k in range(K) if k != 7]] == 0)
     step = 2 * a[1] * rho[7, y[1]]
@@ -268,7 +325,7 @@ def check_update_invariants(seed=4):
     assert np.all(np.abs(d[:, 7]) <= 2)
     assert np.all((d[:, 7] == 0) == (np.abs(H[:, 7] + step) > h_max))
     # reinforcement only, probability 1
-    H2 = O.perceptron_update(H, a, y, rho, -np.ones((3, 1), np.int32), h_max, 1 << 32, 1, 1, 0)
+    H2 = O.perceptron_update(H, a, y, rho, -np.ones((3, 1), np.int32), h_max, 1.0, 1, 1, 0)
     assert np.array_equal(np.sign(H2), np.sign(H))
     assert np.array_equal(H2, np.clip(H + 2 * np.sign(H), -h_max, h_max))
     for M in (H1, H2):
@@ -402,7 +459,7 @@ ALL_CHECKS = [
     check_perceptron_golden,
     check_threshold_exact,
     check_reinforce_rate,
-    check_uniform_bits,
+    check_event_law,
     check_update_invariants,
     check_training_invariants,
     check_no_mark_no_update,

@@ -5,6 +5,7 @@ import ctypes as C
 import os
 import re
 
+import numpy as np
 import pytest
 
 from conftest import ROOT
@@ -35,10 +36,20 @@ def test_gamma_rule_matches_oracle(oracle_mod):
     assert B.bmlp_gamma_rule(0) == -1
 
 
-def test_threshold_matches_oracle(oracle_mod):
+def test_sampler_tables_match_oracle(oracle_mod):
+    """The library's reinforcement-sampler thresholds (host code) equal the
+    oracle's, entry for entry, for every block length."""
     for p_r in (0.0, 1e-9, 0.01, 0.1234567, 0.25, 0.5, 0.9, 1.0, 3.0):
         for K in (1, 2, 3, 10, 64, 100, 256, 784, 1024, 4096, 8192, 65536):
-            assert B.bmlp_reinforce_threshold(p_r, K) == oracle_mod.reinforce_threshold(p_r, K), (p_r, K)
+            q = oracle_mod.reinforce_prob(p_r, K)
+            for n in (1, 2, 5, 17, 63, 64):
+                a, f, g = B.bmlp_reinforce_tables(p_r, K, n)
+                ao, fo, go = oracle_mod.r_block_tables(q, n)
+                assert a == ao and np.array_equal(f, fo) and np.array_equal(g, go), (p_r, K, n)
+    with pytest.raises(B.BmlpError):
+        B.bmlp_reinforce_tables(0.5, 10, 65)
+    with pytest.raises(B.BmlpError):
+        B.bmlp_reinforce_tables(0.5, 0, 8)
 
 
 @pytest.mark.parametrize("kw,msg", [

@@ -36,7 +36,12 @@ MUTANTS = [
      "  for (int32_t mu = b - 1; mu >= 0; mu--)\n    for (int32_t g = 0; g < G; g++) {\n      int32_t k = sel"),
     ("reinforce_toward_zero", "*h = clip(*h + 2 * (*h > 0 ? 1 : -1), h_max);",
      "*h = clip(*h - 2 * (*h > 0 ? 1 : -1), h_max);"),
-    ("threshold_floor", "return (uint64_t)ceil(q * 4294967296.0);", "return (uint64_t)floor(q * 4294967296.0);"),
+    ("threshold_floor", "return (uint64_t)ceil(x * 4294967296.0);", "return (uint64_t)floor(x * 4294967296.0);"),
+    ("r_first_exponent", "first[j] = thr((1.0 - pw[j + 1]) / p_any);", "first[j] = thr((1.0 - pw[j]) / p_any);"),
+    ("r_gap_exponent", "gap[g] = thr(1.0 - pw[g + 1]);", "gap[g] = thr(1.0 - pw[g]);"),
+    ("r_block_gate_ignored", "if (!((uint64_t)w[b % 4] < any[x])) continue;", "(void)any;"),
+    ("r_one_event_per_block", "      if (g > n - 2 - p) break;", "      break;"),
+    ("r_tail_uses_full_tables", "const int32_t x = (n == 64) ? 0 : 1;", "const int32_t x = 0;"),
     ("philox_7_rounds", "for (int round = 0; round < 10; round++)", "for (int round = 0; round < 7; round++)"),
     ("update_without_marks", "if (!any) continue; /* O6 */", "(void)any;"),
     ("gamma_ties_small", "(dist == best_dist && g > best)", "(dist == best_dist && g < best)"),
