@@ -32,7 +32,8 @@
 //   - 1 MMA thread waits on "full", issues tcgen05.mma.kind::f8f6f4 (M = 128,
 //     N = 256, K = 32) four times per stage into a 128 x 256 fp32 accumulator
 //     in TMEM, and commits to the stage's "empty" mbarrier.
-//   - Epilogue: tcgen05.ld -> shared partial; cluster barrier; reduction of
+//   - Epilogue: tcgen05.ld -> shared partial (int16: a partial sum is an
+//     integer of magnitude <= K_in <= 32767), rows < bs only; cluster barrier; reduction of
 //     this CTA's 64 columns over the 4 partials; z (int16), packed sign bits
 //     and, for the next layer, the e4m3 tile image; cluster barrier again so
 //     that no CTA leaves while a peer still reads its partial.
@@ -58,9 +59,9 @@ constexpr int A_BYTES = TM * KB;  // 16 KB
 constexpr int B_BYTES = TN * KB;  // 32 KB
 constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
 constexpr int TMEM_COLS = TN;
-constexpr int PSTRIDE = TN + 4;   // floats per partial row (+16 B: no bank conflicts)
+constexpr int PSTRIDE = TN + 8;   // int16 per partial row (+16 B: no bank conflicts)
 constexpr int kCols = TN / kSplit;  // columns reduced by one CTA
-static_assert(TM * PSTRIDE * 4 <= kStages * STAGE_BYTES, "partial must fit in the stages");
+static_assert(TM * PSTRIDE * 2 <= kStages * STAGE_BYTES, "partial must fit in the stages");
 static_assert(kCols == 64, "one CTA writes one packed activation word per row");
 
 struct __align__(8) TcShared {
@@ -86,14 +87,18 @@ __device__ __forceinline__ void cluster_sync_all() {
                ::: "memory");
 }
 
-__device__ __forceinline__ float4 ld_peer_f4(uint32_t local_addr, uint32_t rank) {
+__device__ __forceinline__ uint4 ld_peer_u4(uint32_t local_addr, uint32_t rank) {
   uint32_t a;
   asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(a) : "r"(local_addr), "r"(rank));
-  float4 v;
-  asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];"
-               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w) : "r"(a) : "memory");
+  uint4 v;
+  asm volatile("ld.shared::cluster.v4.u32 {%0, %1, %2, %3}, [%4];"
+               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(a) : "memory");
   return v;
 }
+
+// z of a packed int16 pair (low half first)
+__device__ __forceinline__ int lo16(uint32_t p) { return (int)(int16_t)(p & 0xFFFFu); }
+__device__ __forceinline__ int hi16(uint32_t p) { return (int)(int16_t)(p >> 16); }
 
 template <bool kTiles>
 __global__ void __cluster_dims__(kSplit, 1, 1) __launch_bounds__(THREADS, 1)
@@ -252,7 +257,7 @@ __global__ void __cluster_dims__(kSplit, 1, 1) __launch_bounds__(THREADS, 1)
 
   // ---------------- partial accumulator -> shared memory ----------------
   // (the stages are free: every MMA that read them has completed)
-  float* part = reinterpret_cast<float*>(base);
+  int16_t* part = reinterpret_cast<int16_t*>(base);
   if (threadIdx.x < kProducers) {
     bool go = nk > 0 && !*failed && mbar_wait(&sh->done, 0, failed);
     go = __all_sync(kFull, go);   // tcgen05.ld is warp-collective
@@ -279,11 +284,16 @@ __global__ void __cluster_dims__(kSplit, 1, 1) __launch_bounds__(THREADS, 1)
 #pragma unroll
         for (int j = 0; j < 32; ++j) v[j] = 0u;  // empty K range (or a failed wait): 0
       }
-      float4* dst = reinterpret_cast<float4*>(part + m * PSTRIDE + col0);
+      if (m < M) {
+        uint32_t pk[16];
 #pragma unroll
-      for (int q = 0; q < 8; ++q)
-        dst[q] = make_float4(__uint_as_float(v[4 * q]), __uint_as_float(v[4 * q + 1]),
-                             __uint_as_float(v[4 * q + 2]), __uint_as_float(v[4 * q + 3]));
+        for (int j = 0; j < 16; ++j)
+          pk[j] = ((uint32_t)__float2int_rn(__uint_as_float(v[2 * j])) & 0xFFFFu) |
+                  ((uint32_t)__float2int_rn(__uint_as_float(v[2 * j + 1])) << 16);
+        uint4* dst = reinterpret_cast<uint4*>(part + m * PSTRIDE + col0);
+#pragma unroll
+        for (int q = 0; q < 4; ++q) dst[q] = make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]);
+      }
     }
   }
   asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
@@ -295,26 +305,30 @@ __global__ void __cluster_dims__(kSplit, 1, 1) __launch_bounds__(THREADS, 1)
     const int c0 = kCols * (int)rank + 16 * (threadIdx.x & 3);  // column in the tile
     const int nf = n0 + c0;                      // first neuron of the 16
     if (m < M) {
-      float acc[16];
+      int acc[16];
 #pragma unroll
-      for (int j = 0; j < 16; ++j) acc[j] = 0.f;
+      for (int j = 0; j < 16; ++j) acc[j] = 0;
       const uint32_t local = smem_u32(part + m * PSTRIDE + c0);
 #pragma unroll
       for (int q = 0; q < kSplit; ++q) {
 #pragma unroll
-        for (int h = 0; h < 4; ++h) {
-          const float4 v = ld_peer_f4(local + 16u * h, (uint32_t)q);
-          acc[4 * h] += v.x;
-          acc[4 * h + 1] += v.y;
-          acc[4 * h + 2] += v.z;
-          acc[4 * h + 3] += v.w;
+        for (int h = 0; h < 2; ++h) {
+          const uint4 v = ld_peer_u4(local + 16u * h, (uint32_t)q);
+          acc[8 * h + 0] += lo16(v.x);
+          acc[8 * h + 1] += hi16(v.x);
+          acc[8 * h + 2] += lo16(v.y);
+          acc[8 * h + 3] += hi16(v.y);
+          acc[8 * h + 4] += lo16(v.z);
+          acc[8 * h + 5] += hi16(v.z);
+          acc[8 * h + 6] += lo16(v.w);
+          acc[8 * h + 7] += hi16(v.w);
         }
       }
       int16_t* zrow = Ly.Z + (int64_t)m * N;
       uint32_t bits = 0, zp[8];
 #pragma unroll
       for (int j = 0; j < 16; ++j) {
-        const int z = __float2int_rn(acc[j]);
+        const int z = acc[j];
         if (nf + j < N && z >= 0) bits |= 1u << j;
         if (j & 1) zp[j >> 1] |= (uint32_t)(z & 0xFFFF) << 16;
         else zp[j >> 1] = (uint32_t)(z & 0xFFFF);

@@ -312,7 +312,7 @@ size_t update_smem_bytes(int bs, int nblk_max) {
 }
 
 template <bool kPow2>
-__global__ void __launch_bounds__(kUpdThreads, 3) k_update(const StepParams* __restrict__ P,
+__global__ void __launch_bounds__(kUpdThreads, 4) k_update(const StepParams* __restrict__ P,
                                                            uint32_t key0, uint32_t key1) {
   extern __shared__ int32_t dyn[];
   __shared__ uint2 s_dn[2][16];
