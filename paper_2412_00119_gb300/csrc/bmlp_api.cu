@@ -402,6 +402,7 @@ int bmlp_create(const int32_t* widths, int32_t n_widths, int32_t classes, int16_
         (rc = dalloc(h, &D.W, (size_t)D.Kout * D.nw_in)) ||
         (rc = dalloc(h, &D.PT, (size_t)classes * D.nw_out)) ||
         (rc = dalloc(h, &D.rho, (size_t)D.Kout * classes)) ||
+        (rc = dalloc(h, &D.rhoT, (size_t)D.Kout * classes)) ||
         (rc = dalloc(h, &D.Z, (size_t)bs * D.Kout)) ||
         (rc = dalloc(h, &D.A, (size_t)bs * D.nw_out)) ||
         (rc = dalloc(h, &D.mark, (size_t)bs)) ||
@@ -442,6 +443,7 @@ int bmlp_create(const int32_t* widths, int32_t n_widths, int32_t classes, int16_
     k_init_rho<<<(unsigned)((n2 + 255) / 256), 256>>>(D.rho, D.Kout, classes, l, P.key0, P.key1);
     const int64_t n3 = (int64_t)classes * D.nw_out;
     k_pack_pt<<<(unsigned)((n3 + 255) / 256), 256>>>(D.rho, D.PT, D.Kout, classes, D.nw_out);
+    k_transpose_rho<<<(unsigned)((n2 + 255) / 256), 256>>>(D.rho, D.rhoT, D.Kout, classes);
   }
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return bail(cuda_fail(h, e, "init kernels"));
@@ -453,7 +455,7 @@ int bmlp_create(const int32_t* widths, int32_t n_widths, int32_t classes, int16_
     return bail(cuda_fail(h, e, "param upload"));
   if ((rc = upload_thresholds(h, 0)) != BMLP_OK) return bail(rc);
   if ((e = cudaDeviceSynchronize()) != cudaSuccess) return bail(cuda_fail(h, e, "init"));
-  h->launches += 3 * L;
+  h->launches += 4 * L;
   *out = h;
   return BMLP_OK;
 }

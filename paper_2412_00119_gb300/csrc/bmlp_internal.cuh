@@ -21,6 +21,7 @@ namespace bk {
 //   W    uint64 [K_out][nw_in]    packed sign(H), bit (i%64) of word i/64 = (h_ik > 0)
 //   PT   uint64 [c][nw_out]       packed P_l^T, bit (k%64) of word k/64 = (rho_kj > 0)
 //   rho  int8  [K_out][c]         P_l itself, for the stability rho_{k,y}
+//   rhoT int8  [c][K_out]         the same, class-major
 //   Z    int16 [bs][K_out]        pre-activations of the current mini-batch
 //   A    uint64 [bs][nw_out]      packed activations a_l of the current mini-batch
 //   mark uint8 [bs]               1 iff the pattern is in M_l
@@ -36,6 +37,7 @@ struct DevLayer {
   uint64_t* W;
   uint64_t* PT;
   int8_t* rho;
+  int8_t* rhoT;       // [c][K_out]: rho transposed (class-major), for the selection
   int16_t* Z;
   uint64_t* A;
   uint8_t* mark;
@@ -152,6 +154,7 @@ __global__ void k_init_hw(int16_t* H, uint64_t* W, int Kin, int Kout, int ldh, i
                           int l, uint32_t key0, uint32_t key1, int h_max, int hb);
 __global__ void k_init_rho(int8_t* rho, int Kout, int c, int l, uint32_t key0, uint32_t key1);
 __global__ void k_pack_pt(const int8_t* rho, uint64_t* PT, int Kout, int c, int nw_out);
+__global__ void k_transpose_rho(const int8_t* rho, int8_t* rhoT, int Kout, int c);
 // Re-derive W from H for one layer (after set_state).
 __global__ void k_repack_w(const int16_t* H, uint64_t* W, int Kin, int Kout, int ldh, int nw_in,
                            int h_max, int hb);

@@ -87,6 +87,44 @@ __global__ void __launch_bounds__(kClsThreads) k_cls_select(const StepParams* __
   const int y = s_y;
   const int16_t* z = Ly.Z + (int64_t)mu * Ly.Kout;
   const int gamma = Ly.gamma;
+  const int per = gamma >> 3;  // 8-neuron chunks per group
+  if ((gamma & 7) == 0 && per <= 32 && (per & (per - 1)) == 0) {
+    // one thread per 8 neurons: 16-byte z loads, 8 bytes of rho^T, then the
+    // group's per lanes (consecutive, aligned) reduce with shuffles
+    const int8_t* rt = Ly.rhoT + (int64_t)y * Ly.Kout;
+    const int nchunk = Ly.Kout >> 3;
+    for (int base = 0; base < nchunk; base += blockDim.x) {
+      const int ci = base + threadIdx.x;
+      int bestd = INT_MIN, bestk = INT_MAX;
+      if (ci < nchunk) {
+        const uint4 zv = *reinterpret_cast<const uint4*>(z + 8 * ci);
+        const uint2 rv = *reinterpret_cast<const uint2*>(rt + 8 * ci);
+        const uint32_t zw[4] = {zv.x, zv.y, zv.z, zv.w};
+        const uint32_t rw[2] = {rv.x, rv.y};
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          const int zj = (int)(int16_t)(zw[j >> 1] >> (16 * (j & 1)));
+          const int rj = (int)(int8_t)(rw[j >> 2] >> (8 * (j & 3)));
+          const int d = zj * rj;
+          if (d < 0 && d > bestd) {  // ascending k: strict '>' keeps the lowest
+            bestd = d;
+            bestk = 8 * ci + j;
+          }
+        }
+      }
+      for (int off = per >> 1; off > 0; off >>= 1) {
+        const int od = __shfl_xor_sync(0xffffffffu, bestd, off);
+        const int ok = __shfl_xor_sync(0xffffffffu, bestk, off);
+        if (od > bestd || (od == bestd && ok < bestk)) {
+          bestd = od;
+          bestk = ok;
+        }
+      }
+      if (ci < nchunk && (ci & (per - 1)) == 0)
+        sel[ci / per] = (bestd == INT_MIN) ? (int16_t)-1 : (int16_t)bestk;
+    }
+    return;
+  }
   for (int g = warp; g < Ly.G; g += nwarps) {
     int bestd = INT_MIN, bestk = INT_MAX;
     for (int kk = lane; kk < gamma; kk += 32) {
@@ -648,6 +686,15 @@ __global__ void k_pack_pt(const int8_t* rho, uint64_t* PT, int Kout, int c, int 
     if (k < Kout && rho[(int64_t)k * c + j] > 0) bits |= 1ull << b;
   }
   PT[idx] = bits;
+}
+
+// rhoT[j][k] = rho[k][j].
+__global__ void k_transpose_rho(const int8_t* rho, int8_t* rhoT, int Kout, int c) {
+  const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (idx >= (int64_t)Kout * c) return;
+  const int j = (int)(idx / Kout);
+  const int k = (int)(idx % Kout);
+  rhoT[idx] = rho[(int64_t)k * c + j];
 }
 
 // W = packed sign(H) for one layer (H as lattice indices), pad bits 0.
