@@ -476,25 +476,36 @@ __global__ void __launch_bounds__(kUpdThreads, 4) k_update(const StepParams* __r
       if (lane + 64 < nch) q2 = __ldcs(reinterpret_cast<const uint4*>(hrow + 8 * (lane + 64)));
       if (lane + 96 < nch) q3 = __ldcs(reinterpret_cast<const uint4*>(hrow + 8 * (lane + 96)));
       const int iters2 = (nch + 63) >> 6;
-#pragma unroll 1
-      for (int it = 0; it < iters2; ++it) {
-        int chv[2];
-        bool live[2];
-        uint4 w[2];
-        uint32_t pb[2] = {0u, 0u};  // activation bytes of tuples 0..kPre-1, one per byte
-        chv[0] = 64 * it + lane;
-        chv[1] = chv[0] + 32;
-        live[0] = chv[0] < nch;
-        live[1] = chv[1] < nch;
+      // activation bytes of tuples 0..kPre-1 (one per byte) for the next
+      // iteration's two chunks, loaded one iteration ahead
+      auto tuple_bytes = [&](int it_next, uint32_t (&pbo)[2]) {
+        pbo[0] = 0u;
+        pbo[1] = 0u;
 #pragma unroll
         for (int q = 0; q < kPre; ++q) {
           if (q < n_t) {
             const uint8_t* arow = aprev + (size_t)(s_list[q] & 0xFFFF) * arow_bytes;
 #pragma unroll
-            for (int u = 0; u < 2; ++u)
-              if (live[u]) pb[u] |= (uint32_t)__ldg(arow + chv[u]) << (8 * q);
+            for (int u = 0; u < 2; ++u) {
+              const int ch = 64 * it_next + 32 * u + lane;
+              if (ch < nch) pbo[u] |= (uint32_t)__ldg(arow + ch) << (8 * q);
+            }
           }
         }
+      };
+      uint32_t pbn[2];
+      tuple_bytes(0, pbn);
+#pragma unroll 1
+      for (int it = 0; it < iters2; ++it) {
+        int chv[2];
+        bool live[2];
+        uint4 w[2];
+        uint32_t pb[2] = {pbn[0], pbn[1]};  // this iteration's tuple bytes
+        chv[0] = 64 * it + lane;
+        chv[1] = chv[0] + 32;
+        live[0] = chv[0] < nch;
+        live[1] = chv[1] < nch;
+        if (it + 1 < iters2) tuple_bytes(it + 1, pbn);
         w[0] = q0;
         w[1] = q1;
         q0 = q2;
