@@ -288,6 +288,7 @@ def run_ours(args):
     # timed region: every 10th mini-batch is launched with per-kernel events
     B.bmlp_set_profiling(h, 10)
     B.bmlp_reset_profile(h)
+    B.bmlp_update_stats(h, reset=True)
     launches0 = B.bmlp_launch_count(h)
     ev0 = torch.cuda.Event(enable_timing=True)
     ev1 = torch.cuda.Event(enable_timing=True)
@@ -302,6 +303,7 @@ def run_ours(args):
     barrier()
     ms = ev0.elapsed_time(ev1)
     launches = B.bmlp_launch_count(h) - launches0
+    upd_rows, upd_streamed, upd_bytes_total = B.bmlp_update_stats(h, reset=True)
     prof = B.bmlp_get_profile(h)
     B.bmlp_set_profiling(h, 0)
     ms_max = max_over_ranks(ms, dev)
@@ -318,7 +320,11 @@ def run_ours(args):
     step_ms_mb = ms / (args.steps * SAMPLES_PER_STEP / 100)
     upd_avg_s = prof["update"][1] / max(prof["update"][0], 1) / 1000.0
     fwd_avg_s = prof["train_forward"][1] / max(prof["train_forward"][0], 1) / 1000.0
-    upd_bytes = update_bytes_per_launch(cfg.widths)
+    # algorithmic bytes per update launch: what the rule touched in the timed
+    # region (rows with CP tuples streamed, sparse reinforcement elsewhere),
+    # averaged over its mini-batches; update_bytes_per_launch is the all-rows bound
+    n_mb = args.steps * SAMPLES_PER_STEP // 100
+    upd_bytes = upd_bytes_total / n_mb if upd_bytes_total > 0 else update_bytes_per_launch(cfg.widths)
     bp_layer = 100 * cfg.widths[1] * cfg.widths[0]  # bit-pairs of one 8192x8192 forward launch
     popc_peak = popc_peak_bitpairs(sm_max_mhz)
     traffic = None
@@ -328,7 +334,9 @@ def run_ours(args):
         "update": {"bound": "hbm", "achieved": upd_bytes / upd_avg_s / 1e9, "peak": hbm_gbs,
                    "unit": "GB/s", "frac": upd_bytes / upd_avg_s / 1e9 / hbm_gbs,
                    "traffic": traffic, "avg_us": upd_avg_s * 1e6,
-                   "algorithmic_bytes": upd_bytes},
+                   "algorithmic_bytes": upd_bytes,
+                   "all_rows_bytes": update_bytes_per_launch(cfg.widths),
+                   "rows_streamed_frac": upd_streamed / max(upd_rows, 1)},
     }
     if tc:
         fp8_sus = FP8_PER_BF16 * bf16_tf_sus

@@ -200,6 +200,17 @@ int bmlp_get_profile(const bmlp_t* h, int32_t kind, int64_t* launches, double* t
 int bmlp_reset_profile(bmlp_t* h);
 int64_t bmlp_launch_count(const bmlp_t* h);
 
+/* Update-kernel statistics accumulated since creation or the last reset
+ * (synchronises): neuron rows visited (layers with a non-empty M_l), rows
+ * streamed (rows with at least one CP tuple; a row without tuple changes only
+ * at its reinforcement events and keeps its W), and the algorithmic bytes the
+ * rule touched: per streamed row its H read and written (int16) and its W row
+ * written, per reinforcement event of a row without tuple 2 bytes read and 2
+ * written.  Any output may be NULL; reset != 0 zeroes the counters after
+ * reading them. */
+int bmlp_update_stats(bmlp_t* h, int64_t* rows_out, int64_t* streamed_out, int64_t* bytes_out,
+                      int32_t reset);
+
 /* Forward-only evaluation that allocates no memory.  The paper has no
  * counterpart: this is bmlp_predict with its scratch moved into the library,
  * for callers that cannot call cudaMalloc -- code running in a host callback,

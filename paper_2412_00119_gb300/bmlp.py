@@ -72,6 +72,7 @@ SIGNATURES = [
     ("bmlp_launch_count", C.c_int64, [_vp]),
     ("bmlp_predict_noalloc", C.c_int, [_vp, _vp, C.c_int64, _vp, _vp]),
     ("bmlp_layer_forward", C.c_int, [_vp, C.c_int32, _vp, C.c_int64, _vp, _vp]),
+    ("bmlp_update_stats", C.c_int, [_vp, _vp, _vp, _vp, C.c_int32]),
 ]
 
 
@@ -180,6 +181,13 @@ def bmlp_layer_forward(h, layer, a_in, a_out, n=None, stream=None):
     """a_out = sign(a_in W_layer), packed rows on the device."""
     n = a_out.shape[0] if n is None else n
     _check(lib().bmlp_layer_forward(h, layer, _ptr(a_in), n, _ptr(a_out), _stream(stream)), h)
+
+
+def bmlp_update_stats(h, reset=False):
+    """(rows visited, rows streamed, algorithmic bytes) of the update kernel."""
+    r, st, by = C.c_int64(), C.c_int64(), C.c_int64()
+    _check(lib().bmlp_update_stats(h, C.byref(r), C.byref(st), C.byref(by), 1 if reset else 0), h)
+    return r.value, st.value, by.value
 
 
 def bmlp_get_info(h):

@@ -750,6 +750,20 @@ int bmlp_reset_profile(bmlp_t* h) {
 
 int64_t bmlp_launch_count(const bmlp_t* h) { return h ? h->launches : -1; }
 
+int bmlp_update_stats(bmlp_t* h, int64_t* rows_out, int64_t* streamed_out, int64_t* bytes_out,
+                      int32_t reset) {
+  if (!h) return BMLP_EINVAL;
+  h->err.clear();
+  unsigned long long v[3];
+  CK(h, cudaDeviceSynchronize());
+  CK(h, cudaMemcpy(v, &h->dCtrl->upd_rows, sizeof(v), cudaMemcpyDeviceToHost));
+  if (rows_out) *rows_out = (int64_t)v[0];
+  if (streamed_out) *streamed_out = (int64_t)v[1];
+  if (bytes_out) *bytes_out = (int64_t)v[2];
+  if (reset) CK(h, cudaMemset(&h->dCtrl->upd_rows, 0, sizeof(v)));
+  return BMLP_OK;
+}
+
 }  // extern "C"
 
 // ---------------------------------------------------------------------------

@@ -59,6 +59,11 @@ struct Ctrl {
   uint32_t done;                // CTAs of the update kernel finished this step
   uint32_t timeouts;            // bounded device waits that expired (BMLP_ETIMEOUT)
   uint32_t any_mark[BMLP_MAX_LAYERS];
+  // update-kernel statistics, accumulated until read with reset
+  unsigned long long upd_rows;       // neuron rows visited (layers with M_l non-empty)
+  unsigned long long upd_streamed;   // rows streamed (at least one CP tuple)
+  unsigned long long upd_bytes;      // algorithmic bytes: H read + write and W write of the
+                                     // streamed rows, int16 read + write per sparse event
 };
 
 // Thresholds of the reinforcement sampler of one layer (Alg. 3 l.5-12): the

@@ -159,6 +159,10 @@ __global__ void __launch_bounds__(kClsThreads) k_cls_select(const StepParams* __
 //      blocks 4j .. 4j+3 (one Philox call) and, for each block that holds an
 //      event, the event draws (binary searches in the layer's monotone
 //      threshold tables, staged in shared memory);
+//   (a row without CP tuple is not streamed: its H changes only at its
+//   reinforcement events, applied as single-weight read-modify-writes, and
+//   its W is unchanged because reinforcement never flips a sign; rows are
+//   taken from a per-CTA counter so that such rows rebalance the warps)
 //   3. it streams the row in chunks of 8 hidden weights, two chunks per lane
 //      per iteration, with a rotating queue of four 16-byte vectors in flight
 //      per lane: the CP tuples, then the chunk's reinforcement events (its byte
@@ -355,6 +359,8 @@ __global__ void __launch_bounds__(kUpdThreads, 4) k_update(const StepParams* __r
   extern __shared__ int32_t dyn[];
   __shared__ uint2 s_dn[2][16];
   __shared__ uint2 s_fire[16];
+  __shared__ int s_next[1];
+  __shared__ unsigned long long s_stats[3];
   const int bid = blockIdx.x;
   int li = 0;
   while (li + 1 < P->L && bid >= P->layer[li + 1].upd_cta_base) ++li;
@@ -385,6 +391,10 @@ __global__ void __launch_bounds__(kUpdThreads, 4) k_update(const StepParams* __r
     RTables* s_rt = reinterpret_cast<RTables*>(s_ev_all + (size_t)nwarps * P->nblk_max);
 
     for (int m = threadIdx.x; m < bsz; m += blockDim.x) s_sel[m] = Ly.sel[(int64_t)m * Ly.G + g];
+    if (threadIdx.x == 0) {
+      s_next[0] = 0;
+      s_stats[0] = s_stats[1] = s_stats[2] = 0ull;
+    }
     {
       const unsigned long long* src = reinterpret_cast<const unsigned long long*>(P->rt + li);
       unsigned long long* dst = reinterpret_cast<unsigned long long*>(s_rt);
@@ -417,6 +427,8 @@ __global__ void __launch_bounds__(kUpdThreads, 4) k_update(const StepParams* __r
     LN.over_pair = (uint32_t)(E.base + E.h_max + 1) * kLaneOne;
     LN.pos_pair = (uint32_t)(E.base + (E.h_max + 1) / 2) * kLaneOne;
     const uint32_t tt = (uint32_t)t;
+    const uint32_t pos_from = (uint32_t)(E.base + (E.h_max + 1) / 2);  // lattice index of h = +1
+    const uint32_t v_top = (uint32_t)(E.base + E.h_max);
     const int Kin = Ly.Kin;
     const int nch = (Kin + 7) >> 3;             // chunks holding at least one input
     const int full = Kin >> 3;                  // chunks of 8 real inputs
@@ -425,7 +437,14 @@ __global__ void __launch_bounds__(kUpdThreads, 4) k_update(const StepParams* __r
     const uint8_t* aprev = (li == 0) ? reinterpret_cast<const uint8_t*>(P->x + start * P->nw0)
                                      : reinterpret_cast<const uint8_t*>(P->layer[li - 1].A);
 
-    for (int rr = r0 + warp; rr < r1; rr += nwarps) {
+    // rows are taken dynamically (rows without tuples finish early)
+    uint32_t st_rows = 0, st_streamed = 0, st_bytes = 0;  // statistics (per warp)
+#pragma unroll 1
+    while (true) {
+      int rr = 0;
+      if (lane == 0) rr = r0 + atomicAdd(s_next, 1);
+      rr = __shfl_sync(kFull, rr, 0);
+      if (rr >= r1) break;
       const int k = g * gamma + rr;
       // ---- 1. CP tuples of neuron k, ascending mu ----
       int n_t = 0;
@@ -461,8 +480,35 @@ __global__ void __launch_bounds__(kUpdThreads, 4) k_update(const StepParams* __r
       }
       __syncwarp();
 
-      // ---- 3. CP and W over the row ----
       int16_t* hrow = Ly.H + (int64_t)k * Ly.ldh;
+      if (n_t == 0) {
+        // no tuple: H changes only at the reinforcement events, which never
+        // flip a sign, so W stays; single-weight read-modify-writes
+        int nev = 0;
+#pragma unroll 1
+        for (int b = lane; b < nblk; b += 32) {
+          uint64_t mask = s_ev[b];
+          nev += __popcll(mask);
+#pragma unroll 1
+          while (mask != 0ull) {
+            const int bit = __ffsll((long long)mask) - 1;
+            mask &= mask - 1ull;
+            int16_t* hp = hrow + 64 * b + bit;
+            const uint32_t v = (uint16_t)*hp;
+            *hp = (int16_t)((v >= pos_from) ? min(v + 1u, v_top) : max(v - 1u, (uint32_t)E.base));
+          }
+        }
+        nev = warp_sum(nev);
+        st_rows += 1u;
+        st_bytes += 4u * (uint32_t)nev;
+        __syncwarp();   // s_ev and s_list are reused by the next row
+        continue;
+      }
+      st_rows += 1u;
+      st_streamed += 1u;
+      st_bytes += 4u * (uint32_t)Ly.ldh + 8u * (uint32_t)Ly.nw_in;
+
+      // ---- 3. CP and W over the row ----
       uint8_t* wrow = reinterpret_cast<uint8_t*>(Ly.W + (int64_t)k * Ly.nw_in);
       // Each iteration handles two chunks per lane, ch and ch + 32 (64 chunks
       // per warp), so the tuple loop and the loop control are shared.  A
@@ -578,6 +624,18 @@ __global__ void __launch_bounds__(kUpdThreads, 4) k_update(const StepParams* __r
         }
       }
       __syncwarp();   // s_ev and s_list are reused by the next row
+    }
+    // statistics: per CTA, one atomic per counter
+    if (lane == 0) {
+      atomicAdd(&s_stats[0], (unsigned long long)st_rows);
+      atomicAdd(&s_stats[1], (unsigned long long)st_streamed);
+      atomicAdd(&s_stats[2], (unsigned long long)st_bytes);
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      atomicAdd(&ctrl->upd_rows, s_stats[0]);
+      atomicAdd(&ctrl->upd_streamed, s_stats[1]);
+      atomicAdd(&ctrl->upd_bytes, s_stats[2]);
     }
   }
 
