@@ -308,3 +308,28 @@ def test_c1_784_256_full_epoch_popc_engine():
 
 def test_c5_8192x5_prefix_popc_engine():
     _full_width("C5", steps=1, n_test=0, fwd=B.BMLP_FWD_POPC)
+
+
+def test_update_stats_count_rows_and_bytes():
+    """bmlp_update_stats: every neuron row of a layer with a non-empty M_l is
+    visited once per mini-batch; the rows streamed are exactly the rows that
+    received a CP tuple (bmlp_debug_last_step's selections); the bytes follow
+    from those counts and the reinforcement events of the other rows."""
+    widths, c, bs = (200, 130, 70), 10, 50
+    cfg = W.small_config(widths, c, bs, 0, teacher_hidden=16)
+    tr = W.make_split(cfg, "train")
+    gpu = B.BMLP(widths, c, seed=11, bs=bs, gamma=[13, 7])
+    B.bmlp_update_stats(gpu.h, reset=True)
+    gpu.train(dev_x(tr.xp), dev_y(tr.y))
+    rows, streamed, nbytes = B.bmlp_update_stats(gpu.h, reset=True)
+    want_rows = want_streamed = 0
+    for l in (1, 2):
+        _, _, mark, sel = B.bmlp_debug_last_step(gpu.h, l)
+        if mark.any():
+            want_rows += widths[l]
+            want_streamed += np.unique(sel[sel >= 0]).size
+    assert rows == want_rows and streamed == want_streamed, (rows, want_rows, streamed, want_streamed)
+    row_bytes = [4 * 64 * ((widths[l - 1] + 63) // 64) + 8 * ((widths[l - 1] + 63) // 64) for l in (1, 2)]
+    assert nbytes >= streamed * min(row_bytes) and (nbytes - streamed * min(row_bytes)) % 4 == 0
+    assert B.bmlp_update_stats(gpu.h) == (0, 0, 0)
+    gpu.close()
