@@ -192,7 +192,9 @@ int bmlp_debug_last_step(const bmlp_t* h, int32_t layer, int16_t* Z, uint64_t* A
  * the library accumulates the launch count and the summed device time when
  * the call ends (which then synchronises the stream).  kinds: 0 forward
  * (train), 1 local classifier + selection, 2 update (CP + R + repack),
- * 3 forward (predict), 4 predict output, 5 host-buffer copies.
+ * 3 forward (predict), 4 predict output, 5 host-buffer copies, 6 drawing of
+ * the reinforcement events (in the replayed step graph this kernel runs beside
+ * the forward passes; in a sampled mini-batch it runs first, alone).
  * bmlp_launch_count: kernels this handle has launched since creation (graph
  * replays count each node). */
 int bmlp_set_profiling(bmlp_t* h, int32_t every);

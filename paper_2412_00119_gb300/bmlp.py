@@ -29,7 +29,8 @@ BMLP_ESTATE = -5
 BMLP_ENODEV = -6
 BMLP_EPOCH_END = 1
 BMLP_FWD_AUTO, BMLP_FWD_POPC, BMLP_FWD_TCGEN05 = 0, 1, 2
-PROFILE_KINDS = ("train_forward", "cls_select", "update", "eval_forward", "eval_out", "copy")
+PROFILE_KINDS = ("train_forward", "cls_select", "update", "eval_forward", "eval_out", "copy",
+                 "r_events")
 
 _ERRNAMES = {-1: "EINVAL", -2: "ENOMEM", -3: "ECUDA", -4: "ETIMEOUT", -5: "ESTATE", -6: "ENODEV"}
 

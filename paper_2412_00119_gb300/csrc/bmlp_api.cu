@@ -24,7 +24,7 @@ namespace {
 thread_local std::string g_create_error;
 
 enum ProfKind { kProfTrainFwd = 0, kProfCls = 1, kProfUpd = 2, kProfEvalFwd = 3, kProfOut = 4,
-                kProfCopy = 5, kProfKinds = 6 };
+                kProfCopy = 5, kProfEvents = 6, kProfKinds = 7 };
 
 }  // namespace
 
@@ -53,6 +53,8 @@ struct bmlp {
   // graph of one training step
   cudaGraphExec_t stepExec = nullptr;
   cudaStream_t capStream = nullptr;
+  cudaStream_t sideStream = nullptr;  // the event-draw branch of the step graph
+  cudaEvent_t evFork = nullptr, evJoin = nullptr;
   int updCtas = 0;
   size_t updSmem = 0;
   // profiling
@@ -190,9 +192,26 @@ int prof_collect(bmlp_t* h, cudaStream_t st) {
   return BMLP_OK;
 }
 
-// Enqueue the kernels of one training mini-batch on `st`.
-int enqueue_step(bmlp_t* h, cudaStream_t st) {
+// Enqueue the kernels of one training mini-batch on `st`.  The reinforcement
+// events depend only on (seed, layer, neuron, step, p_r): when `fork` is set
+// (graph capture) their kernel runs on a side stream next to the forward
+// passes, which leave most of every SM idle, and joins before the update;
+// otherwise it runs first on `st`.
+int enqueue_step(bmlp_t* h, cudaStream_t st, bool fork) {
+  if (!fork) {
+    prof_begin(h, kProfEvents, st);
+    launch_r_events((unsigned)h->hp.ev_ctas_total, st, h->dP, h->hp.key0, h->hp.key1);
+    prof_end(h, st);
+  }
   for (int l = 1; l <= h->L; ++l) {
+    if (fork && l == 2) {
+      // fork after the first forward pass: its CTAs hold the SMs, and the
+      // event draws and the second pass become ready together
+      CK(h, cudaEventRecord(h->evFork, st));
+      CK(h, cudaStreamWaitEvent(h->sideStream, h->evFork, 0));
+      launch_r_events((unsigned)h->hp.ev_ctas_total, h->sideStream, h->dP, h->hp.key0, h->hp.key1);
+      CK(h, cudaEventRecord(h->evJoin, h->sideStream));
+    }
     prof_begin(h, kProfTrainFwd, st);
     if (h->fwd_impl == BMLP_FWD_TCGEN05)
       launch_train_forward_tc(l > 1, h->K[l], st, h->dP, l);
@@ -203,6 +222,13 @@ int enqueue_step(bmlp_t* h, cudaStream_t st) {
   prof_begin(h, kProfCls, st);
   k_cls_select<<<dim3((unsigned)h->bs, (unsigned)h->L), kClsThreads, 0, st>>>(h->dP);
   prof_end(h, st);
+  if (fork && h->L == 1) {
+    CK(h, cudaEventRecord(h->evFork, st));
+    CK(h, cudaStreamWaitEvent(h->sideStream, h->evFork, 0));
+    launch_r_events((unsigned)h->hp.ev_ctas_total, h->sideStream, h->dP, h->hp.key0, h->hp.key1);
+    CK(h, cudaEventRecord(h->evJoin, h->sideStream));
+  }
+  if (fork) CK(h, cudaStreamWaitEvent(st, h->evJoin, 0));
   prof_begin(h, kProfUpd, st);
   launch_update(((h->h_max + 1) & h->h_max) == 0, (unsigned)h->updCtas, h->updSmem, st, h->dP,
                 h->hp.key0, h->hp.key1);
@@ -213,12 +239,22 @@ int enqueue_step(bmlp_t* h, cudaStream_t st) {
 
 int ensure_graph(bmlp_t* h) {
   if (h->stepExec) return BMLP_OK;
-  if (!h->capStream) CK(h, cudaStreamCreateWithFlags(&h->capStream, cudaStreamNonBlocking));
+  // the forward chain is captured at the highest stream priority and the
+  // event-draw branch at the lowest, so that the block scheduler places
+  // forward CTAs first and the event draws fill the remaining room
+  int prio_low = 0, prio_high = 0;
+  CK(h, cudaDeviceGetStreamPriorityRange(&prio_low, &prio_high));
+  if (!h->capStream)
+    CK(h, cudaStreamCreateWithPriority(&h->capStream, cudaStreamNonBlocking, prio_high));
+  if (!h->sideStream)
+    CK(h, cudaStreamCreateWithPriority(&h->sideStream, cudaStreamNonBlocking, prio_low));
+  if (!h->evFork) CK(h, cudaEventCreateWithFlags(&h->evFork, cudaEventDisableTiming));
+  if (!h->evJoin) CK(h, cudaEventCreateWithFlags(&h->evJoin, cudaEventDisableTiming));
   cudaGraph_t g = nullptr;
   CK(h, cudaStreamBeginCapture(h->capStream, cudaStreamCaptureModeThreadLocal));
   const bool prof = h->profiling;
   h->profiling = false;
-  int rc = enqueue_step(h, h->capStream);
+  int rc = enqueue_step(h, h->capStream, true);
   h->profiling = prof;
   cudaError_t e = cudaStreamEndCapture(h->capStream, &g);
   if (rc != BMLP_OK) {
@@ -226,7 +262,7 @@ int ensure_graph(bmlp_t* h) {
     return rc;
   }
   if (e != cudaSuccess) return cuda_fail(h, e, "cudaStreamEndCapture");
-  e = cudaGraphInstantiate(&h->stepExec, g, 0);
+  e = cudaGraphInstantiate(&h->stepExec, g, cudaGraphInstantiateFlagUseNodePriority);
   cudaGraphDestroy(g);
   if (e != cudaSuccess) return cuda_fail(h, e, "cudaGraphInstantiate");
   return BMLP_OK;
@@ -250,14 +286,14 @@ int run_steps(bmlp_t* h, const uint64_t* xd, const int32_t* yd, int64_t n, cudaS
     // sampled mini-batches are launched kernel by kernel between CUDA events
     h->profiling = h->profEvery > 0 && ((h->t_host + s) % h->profEvery) == 0;
     if (h->profiling) {
-      int rc = enqueue_step(h, st);
+      int rc = enqueue_step(h, st, false);
       if (rc != BMLP_OK) return rc;
     } else {
       CK(h, cudaGraphLaunch(h->stepExec, st));
     }
   }
   h->profiling = h->profEvery > 0;
-  h->launches += steps * (h->L + 2);
+  h->launches += steps * (h->L + 3);
   h->t_host += steps;
   return BMLP_OK;
 }
@@ -389,7 +425,7 @@ int bmlp_create(const int32_t* widths, int32_t n_widths, int32_t classes, int16_
   while ((1 << P.hb) < h_max + 1) ++P.hb;
   P.key0 = (uint32_t)(seed & 0xffffffffu);
   P.key1 = (uint32_t)(seed >> 32);
-  int cta = 0;
+  int cta = 0, ev_cta = 0;
   for (int l = 1; l <= L; ++l) {
     DevLayer& D = P.layer[l - 1];
     D.Kin = h->K[l - 1]; D.Kout = h->K[l];
@@ -398,6 +434,9 @@ int bmlp_create(const int32_t* widths, int32_t n_widths, int32_t classes, int16_
     D.upd_cta_base = cta;
     D.upd_ctas = D.G * ((D.gamma + kUpdRowsPerCta - 1) / kUpdRowsPerCta);
     cta += D.upd_ctas;
+    D.ev_cta_base = ev_cta;
+    ev_cta += (D.Kout + kEvRowsPerCta - 1) / kEvRowsPerCta;
+    D.nblk = (D.Kin + 63) / 64;
     if ((rc = dalloc(h, &D.H, (size_t)D.Kout * D.ldh)) ||
         (rc = dalloc(h, &D.W, (size_t)D.Kout * D.nw_in)) ||
         (rc = dalloc(h, &D.PT, (size_t)classes * D.nw_out)) ||
@@ -406,7 +445,8 @@ int bmlp_create(const int32_t* widths, int32_t n_widths, int32_t classes, int16_
         (rc = dalloc(h, &D.Z, (size_t)bs * D.Kout)) ||
         (rc = dalloc(h, &D.A, (size_t)bs * D.nw_out)) ||
         (rc = dalloc(h, &D.mark, (size_t)bs)) ||
-        (rc = dalloc(h, &D.sel, (size_t)bs * D.G)))
+        (rc = dalloc(h, &D.sel, (size_t)bs * D.G)) ||
+        (rc = dalloc(h, &D.EV, (size_t)D.Kout * D.nblk)))
       return bail(rc);
     D.AE = nullptr;
     if (fwd == BMLP_FWD_TCGEN05 && l < L) {
@@ -417,6 +457,7 @@ int bmlp_create(const int32_t* widths, int32_t n_widths, int32_t classes, int16_
   }
   h->updCtas = cta;
   P.upd_ctas_total = cta;
+  P.ev_ctas_total = ev_cta;
   P.nblk_max = 0;
   for (int l = 1; l <= L; ++l) P.nblk_max = std::max(P.nblk_max, (widths[l - 1] + 63) / 64);
   h->updSmem = update_smem_bytes(bs, P.nblk_max);
@@ -465,6 +506,9 @@ void bmlp_destroy(bmlp_t* h) {
   cudaDeviceSynchronize();
   if (h->stepExec) cudaGraphExecDestroy(h->stepExec);
   if (h->capStream) cudaStreamDestroy(h->capStream);
+  if (h->sideStream) cudaStreamDestroy(h->sideStream);
+  if (h->evFork) cudaEventDestroy(h->evFork);
+  if (h->evJoin) cudaEventDestroy(h->evJoin);
   for (auto e : h->evPool) cudaEventDestroy(e);
   for (void* p : h->allocs) cudaFree(p);
   if (h->hostPinned) cudaFreeHost(h->hostPinned);

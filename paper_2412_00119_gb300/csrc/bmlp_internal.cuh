@@ -46,6 +46,10 @@ struct DevLayer {
   int32_t Kin, Kout, nw_in, nw_out, ldh, gamma, G;
   int32_t upd_cta_base;  // first CTA of this layer in the update grid
   int32_t upd_ctas;      // CTAs of this layer in the update grid
+  int32_t ev_cta_base;   // first CTA of this layer in the event-draw grid
+  int32_t nblk;          // blocks of 64 inputs per neuron row (ceil(K_in / 64))
+  uint64_t* EV;          // [K_out][nblk] reinforcement events of the current step,
+                         // bit i % 64 of word i / 64 = input i reinforced
 };
 
 // Device-resident step control.  The update kernel's last CTA advances t and s
@@ -88,7 +92,7 @@ struct StepParams {
   const RTables* rt;            // [L] reinforcement sampler thresholds
   int32_t nblk_max;             // max over layers of ceil(K_in / 64)
   Ctrl* ctrl;
-  int32_t L, c, bs, h_max, r_num, r_den, nw0, upd_ctas_total;
+  int32_t L, c, bs, h_max, r_num, r_den, nw0, upd_ctas_total, ev_ctas_total;
   int32_t hb;                   // lattice-index offset exponent (see H above)
   uint32_t key0, key1;          // Philox key = (seed mod 2^32, seed div 2^32)
 };
@@ -140,6 +144,12 @@ __global__ void k_cls_select(const StepParams* P);
 // boundaries of the lattice index).
 void launch_update(bool pow2, unsigned grid, size_t smem, cudaStream_t st, const StepParams* P,
                    uint32_t key0, uint32_t key1);
+// Reinforcement events of every neuron row of every layer for the current
+// step into DevLayer::EV (Alg. 3 l.5-12); grid = P->ev_ctas_total CTAs.
+void launch_r_events(unsigned grid, cudaStream_t st, const StepParams* P, uint32_t key0,
+                     uint32_t key1);
+constexpr int kEvRowsPerCta = 4;   // one warp per row
+constexpr int kEvThreads = 32 * kEvRowsPerCta;
 // Attributes of the update kernel; smem > 0 also raises its dynamic shared
 // memory limit to smem bytes.
 cudaError_t update_kernel_attributes(cudaFuncAttributes* fa, size_t smem);

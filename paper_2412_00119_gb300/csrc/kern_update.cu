@@ -154,11 +154,9 @@ __global__ void __launch_bounds__(kClsThreads) k_cls_select(const StepParams* __
 // neuron row k at a time:
 //   1. it collects, in ascending mu, the patterns whose selection in group g
 //      is k (the CP tuples of k);
-//   2. it draws the row's reinforcement events into a shared bitmap, one
-//      64-bit word per block of 64 inputs: lane j draws the block draws of
-//      blocks 4j .. 4j+3 (one Philox call) and, for each block that holds an
-//      event, the event draws (binary searches in the layer's monotone
-//      threshold tables, staged in shared memory);
+//   2. it copies the row's reinforcement-event bitmap (one 64-bit word per
+//      block of 64 inputs, drawn by k_r_events) into shared memory with
+//      cp.async, overlapping step 1;
 //   (a row without CP tuple is not streamed: its H changes only at its
 //   reinforcement events, applied as single-weight read-modify-writes, and
 //   its W is unchanged because reinforcement never flips a sign; rows are
@@ -187,6 +185,20 @@ constexpr uint32_t kLaneTop = 0x80008000u;
 constexpr uint32_t kLaneOne = 0x00010001u;
 constexpr unsigned kFull = 0xffffffffu;
 constexpr int kPre = 4;  // tuples per row whose activation bytes are prefetched
+
+__device__ __forceinline__ void cp_async8(void* smem, const void* gmem) {
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 8;"
+               ::"r"(static_cast<uint32_t>(__cvta_generic_to_shared(smem))), "l"(gmem) : "memory");
+}
+
+__device__ __forceinline__ void cp_async_commit() {
+  asm volatile("cp.async.commit_group;" ::: "memory");
+}
+
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
 
 __device__ __forceinline__ uint32_t lane_v(const uint4& w, int j) {
   const uint32_t word = (j < 2) ? w.x : (j < 4) ? w.y : (j < 6) ? w.z : w.w;
@@ -350,7 +362,7 @@ size_t update_smem_bytes(int bs, int nblk_max) {
   const int nwarps = kUpdThreads / 32;
   size_t words = (size_t)(bs + 1) / 2 + (size_t)nwarps * bs;  // s_sel (int16), s_list (int32)
   words = (words + 1) & ~(size_t)1;                           // 8-byte alignment
-  return sizeof(int32_t) * words + sizeof(uint64_t) * (size_t)nwarps * nblk_max + sizeof(RTables);
+  return sizeof(int32_t) * words + sizeof(uint64_t) * (size_t)nwarps * nblk_max;
 }
 
 template <bool kPow2>
@@ -381,24 +393,18 @@ __global__ void __launch_bounds__(kUpdThreads, 4) k_update(const StepParams* __r
     const int64_t start = (int64_t)s * P->bs;
     const int bsz = (int)batch_size(P, start);
     // dynamic shared memory: s_sel [bs] int16 | s_list [nwarps][bs] int32 |
-    // (8-byte aligned) s_ev [nwarps][nblk_max] uint64 | s_rt (this layer's tables)
+    // (8-byte aligned) s_ev [nwarps][nblk_max] uint64
     int16_t* s_sel = reinterpret_cast<int16_t*>(dyn);
     int32_t* s_list = dyn + (P->bs + 1) / 2 + warp * P->bs;
     size_t words = (size_t)(P->bs + 1) / 2 + (size_t)nwarps * P->bs;
     words = (words + 1) & ~(size_t)1;
     uint64_t* s_ev_all = reinterpret_cast<uint64_t*>(dyn + words);
     uint64_t* s_ev = s_ev_all + (size_t)warp * P->nblk_max;
-    RTables* s_rt = reinterpret_cast<RTables*>(s_ev_all + (size_t)nwarps * P->nblk_max);
 
     for (int m = threadIdx.x; m < bsz; m += blockDim.x) s_sel[m] = Ly.sel[(int64_t)m * Ly.G + g];
     if (threadIdx.x == 0) {
       s_next[0] = 0;
       s_stats[0] = s_stats[1] = s_stats[2] = 0ull;
-    }
-    {
-      const unsigned long long* src = reinterpret_cast<const unsigned long long*>(P->rt + li);
-      unsigned long long* dst = reinterpret_cast<unsigned long long*>(s_rt);
-      for (int i = threadIdx.x; i < (int)(sizeof(RTables) / 8); i += blockDim.x) dst[i] = src[i];
     }
     // s_dn[r][n]: the +-1 lattice steps of the 4 weights of nibble n, two lanes
     // per word (d_lo + 2^16 d_hi), d = +1 for a set bit, negated for r = 1
@@ -416,7 +422,6 @@ __global__ void __launch_bounds__(kUpdThreads, 4) k_update(const StepParams* __r
     }
     __syncthreads();
 
-    const uint32_t l = (uint32_t)li + 1u;
     const int c = P->c;
     Enc E;
     E.h_max = P->h_max;
@@ -426,7 +431,6 @@ __global__ void __launch_bounds__(kUpdThreads, 4) k_update(const StepParams* __r
     LN.hb = P->hb;
     LN.over_pair = (uint32_t)(E.base + E.h_max + 1) * kLaneOne;
     LN.pos_pair = (uint32_t)(E.base + (E.h_max + 1) / 2) * kLaneOne;
-    const uint32_t tt = (uint32_t)t;
     const uint32_t pos_from = (uint32_t)(E.base + (E.h_max + 1) / 2);  // lattice index of h = +1
     const uint32_t v_top = (uint32_t)(E.base + E.h_max);
     const int Kin = Ly.Kin;
@@ -446,6 +450,12 @@ __global__ void __launch_bounds__(kUpdThreads, 4) k_update(const StepParams* __r
       rr = __shfl_sync(kFull, rr, 0);
       if (rr >= r1) break;
       const int k = g * gamma + rr;
+      {
+        // the row's event bitmap -> shared memory, overlapping the tuple scan
+        const uint64_t* evrow = Ly.EV + (int64_t)k * nblk;
+        for (int b = lane; b < nblk; b += 32) cp_async8(s_ev + b, evrow + b);
+        cp_async_commit();
+      }
       // ---- 1. CP tuples of neuron k, ascending mu ----
       int n_t = 0;
       for (int base = 0; base < bsz; base += 32) {
@@ -460,24 +470,8 @@ __global__ void __launch_bounds__(kUpdThreads, 4) k_update(const StepParams* __r
         }
         n_t += __popc(bal);
       }
-      // ---- 2. reinforcement events of the row, one bitmap word per block ----
-#pragma unroll 1
-      for (int gq = lane; 4 * gq < nblk; gq += 32) {
-        const uint4 u = philox4x32_10(make_uint4((uint32_t)gq, (uint32_t)k, (3u << 16) + l, tt),
-                                      key0, key1);
-#pragma unroll
-        for (int wq = 0; wq < 4; ++wq) {
-          const int b = 4 * gq + wq;
-          if (b < nblk) {
-            const int n = min(64, Kin - 64 * b);
-            const int x = (n == 64) ? 0 : 1;
-            uint64_t mask = 0;
-            if ((unsigned long long)word_of(u, wq) < s_rt->any[x])
-              mask = block_events(*s_rt, x, n, (uint32_t)b, (uint32_t)k, l, tt, key0, key1);
-            s_ev[b] = mask;
-          }
-        }
-      }
+      // ---- 2. the row's reinforcement events (drawn by k_r_events) ----
+      cp_async_wait<0>();
       __syncwarp();
 
       int16_t* hrow = Ly.H + (int64_t)k * Ly.ldh;
@@ -652,6 +646,56 @@ __global__ void __launch_bounds__(kUpdThreads, 4) k_update(const StepParams* __r
       __threadfence();
     }
   }
+}
+
+// Reinforcement events of the current step (Alg. 3 l.5-12): warp per neuron
+// row; lane j draws the block draws of blocks 4j .. 4j+3 (one Philox call) and,
+// for each block that holds an event, its event draws (binary searches in the
+// layer's threshold tables, staged in shared memory); the row's bitmap goes to
+// DevLayer::EV.  It depends only on (seed, layer, neuron, step, p_r), so it
+// runs beside the forward passes.
+__global__ void __launch_bounds__(kEvThreads) k_r_events(const StepParams* __restrict__ P,
+                                                         uint32_t key0, uint32_t key1) {
+  __shared__ RTables s_rt;
+  const int bid = blockIdx.x;
+  int li = 0;
+  while (li + 1 < P->L && bid >= P->layer[li + 1].ev_cta_base) ++li;
+  const DevLayer& Ly = P->layer[li];
+  {
+    const unsigned long long* src = reinterpret_cast<const unsigned long long*>(P->rt + li);
+    unsigned long long* dst = reinterpret_cast<unsigned long long*>(&s_rt);
+    for (int i = threadIdx.x; i < (int)(sizeof(RTables) / 8); i += blockDim.x) dst[i] = src[i];
+  }
+  __syncthreads();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int k = (bid - Ly.ev_cta_base) * kEvRowsPerCta + warp;
+  if (k >= Ly.Kout) return;
+  const uint32_t l = (uint32_t)li + 1u;
+  const uint32_t tt = (uint32_t)P->ctrl->t;
+  const int Kin = Ly.Kin, nblk = Ly.nblk;
+  uint64_t* ev = Ly.EV + (int64_t)k * nblk;
+#pragma unroll 1
+  for (int gq = lane; 4 * gq < nblk; gq += 32) {
+    const uint4 u = philox4x32_10(make_uint4((uint32_t)gq, (uint32_t)k, (3u << 16) + l, tt), key0,
+                                  key1);
+#pragma unroll
+    for (int wq = 0; wq < 4; ++wq) {
+      const int b = 4 * gq + wq;
+      if (b < nblk) {
+        const int n = min(64, Kin - 64 * b);
+        const int x = (n == 64) ? 0 : 1;
+        uint64_t mask = 0;
+        if ((unsigned long long)word_of(u, wq) < s_rt.any[x])
+          mask = block_events(s_rt, x, n, (uint32_t)b, (uint32_t)k, l, tt, key0, key1);
+        ev[b] = mask;
+      }
+    }
+  }
+}
+
+void launch_r_events(unsigned grid, cudaStream_t st, const StepParams* P, uint32_t key0,
+                     uint32_t key1) {
+  k_r_events<<<grid, kEvThreads, 0, st>>>(P, key0, key1);
 }
 
 void launch_update(bool pow2, unsigned grid, size_t smem, cudaStream_t st, const StepParams* P,
