@@ -425,15 +425,14 @@ int bmlp_create(const int32_t* widths, int32_t n_widths, int32_t classes, int16_
   while ((1 << P.hb) < h_max + 1) ++P.hb;
   P.key0 = (uint32_t)(seed & 0xffffffffu);
   P.key1 = (uint32_t)(seed >> 32);
-  int cta = 0, ev_cta = 0;
+  int ev_cta = 0, rows_total = 0;
   for (int l = 1; l <= L; ++l) {
     DevLayer& D = P.layer[l - 1];
     D.Kin = h->K[l - 1]; D.Kout = h->K[l];
     D.nw_in = words_of(D.Kin); D.nw_out = words_of(D.Kout);
     D.ldh = 64 * D.nw_in; D.gamma = gam[l]; D.G = D.Kout / D.gamma;
-    D.upd_cta_base = cta;
-    D.upd_ctas = D.G * ((D.gamma + kUpdRowsPerCta - 1) / kUpdRowsPerCta);
-    cta += D.upd_ctas;
+    D.row_base = rows_total;
+    rows_total += D.Kout;
     D.ev_cta_base = ev_cta;
     ev_cta += (D.Kout + kEvRowsPerCta - 1) / kEvRowsPerCta;
     D.nblk = (D.Kin + 63) / 64;
@@ -455,8 +454,7 @@ int bmlp_create(const int32_t* widths, int32_t n_widths, int32_t classes, int16_
       if (ez != cudaSuccess) return bail(cuda_fail(h, ez, "cudaMemset"));
     }
   }
-  h->updCtas = cta;
-  P.upd_ctas_total = cta;
+  P.rows_total = rows_total;
   P.ev_ctas_total = ev_cta;
   P.nblk_max = 0;
   for (int l = 1; l <= L; ++l) P.nblk_max = std::max(P.nblk_max, (widths[l - 1] + 63) / 64);
@@ -464,6 +462,14 @@ int bmlp_create(const int32_t* widths, int32_t n_widths, int32_t classes, int16_
   {
     cudaError_t ea = update_kernel_attributes(&fa, h->updSmem);
     if (ea != cudaSuccess) return bail(cuda_fail(h, ea, "update kernel shared memory attribute"));
+    // the update grid is persistent: as many CTAs as fit on the device at once
+    int per_sm = 0;
+    ea = update_kernel_occupancy(((h_max + 1) & h_max) == 0, h->updSmem, &per_sm);
+    if (ea != cudaSuccess || per_sm < 1)
+      return bail(cuda_fail(h, ea != cudaSuccess ? ea : cudaErrorInvalidConfiguration,
+                            "update kernel occupancy"));
+    h->updCtas = per_sm * prop.multiProcessorCount;
+    P.upd_ctas_total = h->updCtas;
   }
   if ((rc = dalloc(h, &h->dP, 1)) || (rc = dalloc(h, &h->dCtrl, 1)) ||
       (rc = dalloc(h, &h->dRT, BMLP_MAX_LAYERS)))

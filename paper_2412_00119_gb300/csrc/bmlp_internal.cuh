@@ -44,9 +44,8 @@ struct DevLayer {
   int16_t* sel;
   uint8_t* AE;
   int32_t Kin, Kout, nw_in, nw_out, ldh, gamma, G;
-  int32_t upd_cta_base;  // first CTA of this layer in the update grid
-  int32_t upd_ctas;      // CTAs of this layer in the update grid
   int32_t ev_cta_base;   // first CTA of this layer in the event-draw grid
+  int32_t row_base;      // first row of this layer in the update's row numbering
   int32_t nblk;          // blocks of 64 inputs per neuron row (ceil(K_in / 64))
   uint64_t* EV;          // [K_out][nblk] reinforcement events of the current step,
                          // bit i % 64 of word i / 64 = input i reinforced
@@ -62,6 +61,7 @@ struct Ctrl {
   uint32_t s;                   // mini-batch index within the current train call
   uint32_t done;                // CTAs of the update kernel finished this step
   uint32_t timeouts;            // bounded device waits that expired (BMLP_ETIMEOUT)
+  uint32_t upd_next;            // next row for the update kernel's warps this step
   uint32_t any_mark[BMLP_MAX_LAYERS];
   // update-kernel statistics, accumulated until read with reset
   unsigned long long upd_rows;       // neuron rows visited (layers with M_l non-empty)
@@ -93,12 +93,11 @@ struct StepParams {
   int32_t nblk_max;             // max over layers of ceil(K_in / 64)
   Ctrl* ctrl;
   int32_t L, c, bs, h_max, r_num, r_den, nw0, upd_ctas_total, ev_ctas_total;
+  int32_t rows_total;           // sum of K_l over the layers (update rows)
   int32_t hb;                   // lattice-index offset exponent (see H above)
   uint32_t key0, key1;          // Philox key = (seed mod 2^32, seed div 2^32)
 };
 
-// Rows of one group handled by one update CTA.
-constexpr int kUpdRowsPerCta = 16;
 constexpr int kUpdThreads = 256;
 constexpr int kClsThreads = 256;
 
@@ -156,6 +155,8 @@ cudaError_t update_kernel_attributes(cudaFuncAttributes* fa, size_t smem);
 // Dynamic shared memory of the update kernel for mini-batches of bs and rows
 // of at most nblk_max blocks of 64 inputs.
 size_t update_smem_bytes(int bs, int nblk_max);
+// CTAs of the update kernel that fit on one SM at once.
+cudaError_t update_kernel_occupancy(bool pow2, size_t smem, int* per_sm);
 // Generic forward for evaluation: A (M x nw_in) against W -> Aout (M x nw_out).
 __global__ void k_forward_eval(const uint64_t* __restrict__ A, int64_t M, int nw_in,
                                const uint64_t* __restrict__ W, int N, int Kin,

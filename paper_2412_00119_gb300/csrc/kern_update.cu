@@ -150,8 +150,9 @@ __global__ void __launch_bounds__(kClsThreads) k_cls_select(const StepParams* __
 
 // ---------------------------------------------------------------------------
 // Hidden-weight update, fused with the visible-weight repack (Alg. 3, Sec. 3.1).
-// CTA = (layer, group g, slice of kUpdRowsPerCta neurons).  A warp owns one
-// neuron row k at a time:
+// The grid is persistent (as many CTAs as fit on the device); every warp takes
+// rows -- all layers' neuron rows in one numbering -- from the step's row
+// counter, kRowChunk at a time, and owns one neuron row k at a time:
 //   1. it collects, in ascending mu, the patterns whose selection in group g
 //      is k (the CP tuples of k);
 //   2. it copies the row's reinforcement-event bitmap (one 64-bit word per
@@ -159,8 +160,7 @@ __global__ void __launch_bounds__(kClsThreads) k_cls_select(const StepParams* __
 //      cp.async, overlapping step 1;
 //   (a row without CP tuple is not streamed: its H changes only at its
 //   reinforcement events, applied as single-weight read-modify-writes, and
-//   its W is unchanged because reinforcement never flips a sign; rows are
-//   taken from a per-CTA counter so that such rows rebalance the warps)
+//   its W is unchanged because reinforcement never flips a sign)
 //   3. it streams the row in chunks of 8 hidden weights, two chunks per lane
 //      per iteration, with a rotating queue of four 16-byte vectors in flight
 //      per lane: the CP tuples, then the chunk's reinforcement events (its byte
@@ -185,6 +185,12 @@ constexpr uint32_t kLaneTop = 0x80008000u;
 constexpr uint32_t kLaneOne = 0x00010001u;
 constexpr unsigned kFull = 0xffffffffu;
 constexpr int kPre = 4;  // tuples per row whose activation bytes are prefetched
+constexpr int kRowChunk = 2;  // rows a warp takes from the row counter at a time
+
+// shared memory of one update warp: s_list [bs] int32, s_ev [nblk_max] uint64
+__host__ __device__ __forceinline__ size_t update_warp_smem(int bs, int nblk_max) {
+  return ((sizeof(int32_t) * (size_t)bs + 7) & ~(size_t)7) + sizeof(uint64_t) * (size_t)nblk_max;
+}
 
 __device__ __forceinline__ void cp_async8(void* smem, const void* gmem) {
   asm volatile("cp.async.ca.shared.global [%0], [%1], 8;"
@@ -359,10 +365,7 @@ __device__ __forceinline__ uint64_t block_events(const RTables& R, int x, int n,
 }  // namespace
 
 size_t update_smem_bytes(int bs, int nblk_max) {
-  const int nwarps = kUpdThreads / 32;
-  size_t words = (size_t)(bs + 1) / 2 + (size_t)nwarps * bs;  // s_sel (int16), s_list (int32)
-  words = (words + 1) & ~(size_t)1;                           // 8-byte alignment
-  return sizeof(int32_t) * words + sizeof(uint64_t) * (size_t)nwarps * nblk_max;
+  return (size_t)(kUpdThreads / 32) * update_warp_smem(bs, nblk_max);
 }
 
 template <bool kPow2>
@@ -371,85 +374,75 @@ __global__ void __launch_bounds__(kUpdThreads, 4) k_update(const StepParams* __r
   extern __shared__ int32_t dyn[];
   __shared__ uint2 s_dn[2][16];
   __shared__ uint2 s_fire[16];
-  __shared__ int s_next[1];
   __shared__ unsigned long long s_stats[3];
-  const int bid = blockIdx.x;
-  int li = 0;
-  while (li + 1 < P->L && bid >= P->layer[li + 1].upd_cta_base) ++li;
-  const DevLayer& Ly = P->layer[li];
   Ctrl* ctrl = P->ctrl;
   const unsigned long long t = ctrl->t;
   const uint32_t s = ctrl->s;
-  const bool active = ctrl->any_mark[li] != 0u;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nwarps = blockDim.x >> 5;
+  const int64_t start = (int64_t)s * P->bs;
+  const int bsz = (int)batch_size(P, start);
+  // dynamic shared memory, per warp: s_list [bs] int32 | (8-byte aligned)
+  // s_ev [nblk_max] uint64
+  const size_t wbytes = update_warp_smem(P->bs, P->nblk_max);
+  uint8_t* wbase = reinterpret_cast<uint8_t*>(dyn) + (size_t)warp * wbytes;
+  int32_t* s_list = reinterpret_cast<int32_t*>(wbase);
+  uint64_t* s_ev = reinterpret_cast<uint64_t*>(wbase + ((sizeof(int32_t) * P->bs + 7) & ~(size_t)7));
 
-  if (active) {
-    const int gamma = Ly.gamma;
-    const int slices = (gamma + kUpdRowsPerCta - 1) / kUpdRowsPerCta;
-    const int local = bid - Ly.upd_cta_base;
-    const int g = local / slices;
-    const int r0 = (local % slices) * kUpdRowsPerCta;
-    const int r1 = min(r0 + kUpdRowsPerCta, gamma);
-    const int64_t start = (int64_t)s * P->bs;
-    const int bsz = (int)batch_size(P, start);
-    // dynamic shared memory: s_sel [bs] int16 | s_list [nwarps][bs] int32 |
-    // (8-byte aligned) s_ev [nwarps][nblk_max] uint64
-    int16_t* s_sel = reinterpret_cast<int16_t*>(dyn);
-    int32_t* s_list = dyn + (P->bs + 1) / 2 + warp * P->bs;
-    size_t words = (size_t)(P->bs + 1) / 2 + (size_t)nwarps * P->bs;
-    words = (words + 1) & ~(size_t)1;
-    uint64_t* s_ev_all = reinterpret_cast<uint64_t*>(dyn + words);
-    uint64_t* s_ev = s_ev_all + (size_t)warp * P->nblk_max;
-
-    for (int m = threadIdx.x; m < bsz; m += blockDim.x) s_sel[m] = Ly.sel[(int64_t)m * Ly.G + g];
-    if (threadIdx.x == 0) {
-      s_next[0] = 0;
-      s_stats[0] = s_stats[1] = s_stats[2] = 0ull;
-    }
-    // s_dn[r][n]: the +-1 lattice steps of the 4 weights of nibble n, two lanes
-    // per word (d_lo + 2^16 d_hi), d = +1 for a set bit, negated for r = 1
-    // (rho = -1)
-    if (threadIdx.x < 32) {
-      const int r = threadIdx.x >> 4, n = threadIdx.x & 15;
-      int d[4];
+  if (threadIdx.x == 0) s_stats[0] = s_stats[1] = s_stats[2] = 0ull;
+  // s_dn[r][n]: the +-1 lattice steps of the 4 weights of nibble n, two lanes
+  // per word (d_lo + 2^16 d_hi), d = +1 for a set bit, negated for r = 1
+  // (rho = -1)
+  if (threadIdx.x < 32) {
+    const int r = threadIdx.x >> 4, n = threadIdx.x & 15;
+    int d[4];
 #pragma unroll
-      for (int j = 0; j < 4; ++j) d[j] = (((n >> j) & 1) ? 1 : -1) * (r ? -1 : 1);
-      s_dn[r][n] = make_uint2((uint32_t)(d[0] + 65536 * d[1]), (uint32_t)(d[2] + 65536 * d[3]));
-      // s_fire[n]: 1 in each lane of nibble n whose bit is set, two lanes per word
-      if (r == 0)
-        s_fire[n] = make_uint2((uint32_t)((n & 1) | ((n >> 1) & 1) << 16),
-                               (uint32_t)(((n >> 2) & 1) | ((n >> 3) & 1) << 16));
-    }
-    __syncthreads();
+    for (int j = 0; j < 4; ++j) d[j] = (((n >> j) & 1) ? 1 : -1) * (r ? -1 : 1);
+    s_dn[r][n] = make_uint2((uint32_t)(d[0] + 65536 * d[1]), (uint32_t)(d[2] + 65536 * d[3]));
+    // s_fire[n]: 1 in each lane of nibble n whose bit is set, two lanes per word
+    if (r == 0)
+      s_fire[n] = make_uint2((uint32_t)((n & 1) | ((n >> 1) & 1) << 16),
+                             (uint32_t)(((n >> 2) & 1) | ((n >> 3) & 1) << 16));
+  }
+  __syncthreads();
 
-    const int c = P->c;
-    Enc E;
-    E.h_max = P->h_max;
-    E.hb = P->hb;
-    E.base = 1 << P->hb;
-    Lanes<kPow2> LN;
-    LN.hb = P->hb;
-    LN.over_pair = (uint32_t)(E.base + E.h_max + 1) * kLaneOne;
-    LN.pos_pair = (uint32_t)(E.base + (E.h_max + 1) / 2) * kLaneOne;
-    const uint32_t pos_from = (uint32_t)(E.base + (E.h_max + 1) / 2);  // lattice index of h = +1
-    const uint32_t v_top = (uint32_t)(E.base + E.h_max);
-    const int Kin = Ly.Kin;
-    const int nch = (Kin + 7) >> 3;             // chunks holding at least one input
-    const int full = Kin >> 3;                  // chunks of 8 real inputs
-    const int nblk = (Kin + 63) >> 6;           // blocks of the reinforcement sampler
-    const uint32_t arow_bytes = (uint32_t)Ly.nw_in * 8u;
-    const uint8_t* aprev = (li == 0) ? reinterpret_cast<const uint8_t*>(P->x + start * P->nw0)
-                                     : reinterpret_cast<const uint8_t*>(P->layer[li - 1].A);
+  const int c = P->c;
+  Enc E;
+  E.h_max = P->h_max;
+  E.hb = P->hb;
+  E.base = 1 << P->hb;
+  Lanes<kPow2> LN;
+  LN.hb = P->hb;
+  LN.over_pair = (uint32_t)(E.base + E.h_max + 1) * kLaneOne;
+  LN.pos_pair = (uint32_t)(E.base + (E.h_max + 1) / 2) * kLaneOne;
+  const uint32_t pos_from = (uint32_t)(E.base + (E.h_max + 1) / 2);  // lattice index of h = +1
+  const uint32_t v_top = (uint32_t)(E.base + E.h_max);
+  const int rows_total = P->rows_total;
 
-    // rows are taken dynamically (rows without tuples finish early)
-    uint32_t st_rows = 0, st_streamed = 0, st_bytes = 0;  // statistics (per warp)
+  // every warp takes chunks of kRowChunk rows (all layers, in order) from the
+  // step's row counter until the rows run out
+  uint32_t st_rows = 0, st_streamed = 0, st_bytes = 0;  // statistics (per warp)
 #pragma unroll 1
-    while (true) {
-      int rr = 0;
-      if (lane == 0) rr = r0 + atomicAdd(s_next, 1);
-      rr = __shfl_sync(kFull, rr, 0);
-      if (rr >= r1) break;
-      const int k = g * gamma + rr;
+  while (true) {
+    int base = 0;
+    if (lane == 0) base = (int)atomicAdd(&ctrl->upd_next, (unsigned)kRowChunk);
+    base = __shfl_sync(kFull, base, 0);
+    if (base >= rows_total) break;
+#pragma unroll 1
+    for (int gr = base; gr < min(base + kRowChunk, rows_total); ++gr) {
+      int li = 0;
+      while (li + 1 < P->L && gr >= P->layer[li + 1].row_base) ++li;
+      if (ctrl->any_mark[li] == 0u) continue;   // M_l empty: no CP, no R
+      const DevLayer& Ly = P->layer[li];
+      const int k = gr - Ly.row_base;
+      const int gamma = Ly.gamma;
+      const int g = k / gamma;
+      const int Kin = Ly.Kin;
+      const int nch = (Kin + 7) >> 3;             // chunks holding at least one input
+      const int full = Kin >> 3;                  // chunks of 8 real inputs
+      const int nblk = Ly.nblk;
+      const uint32_t arow_bytes = (uint32_t)Ly.nw_in * 8u;
+      const uint8_t* aprev = (li == 0) ? reinterpret_cast<const uint8_t*>(P->x + start * P->nw0)
+                                       : reinterpret_cast<const uint8_t*>(P->layer[li - 1].A);
       {
         // the row's event bitmap -> shared memory, overlapping the tuple scan
         const uint64_t* evrow = Ly.EV + (int64_t)k * nblk;
@@ -458,9 +451,9 @@ __global__ void __launch_bounds__(kUpdThreads, 4) k_update(const StepParams* __r
       }
       // ---- 1. CP tuples of neuron k, ascending mu ----
       int n_t = 0;
-      for (int base = 0; base < bsz; base += 32) {
-        const int m = base + lane;
-        const bool hit = (m < bsz) && (s_sel[m] == k);
+      for (int mb = 0; mb < bsz; mb += 32) {
+        const int m = mb + lane;
+        const bool hit = (m < bsz) && (Ly.sel[(int64_t)m * Ly.G + g] == k);
         const unsigned bal = __ballot_sync(kFull, hit);
         if (hit) {
           int yv = P->y[start + m];
@@ -474,91 +467,107 @@ __global__ void __launch_bounds__(kUpdThreads, 4) k_update(const StepParams* __r
       cp_async_wait<0>();
       __syncwarp();
 
-      int16_t* hrow = Ly.H + (int64_t)k * Ly.ldh;
-      if (n_t == 0) {
-        // no tuple: H changes only at the reinforcement events, which never
-        // flip a sign, so W stays; single-weight read-modify-writes
-        int nev = 0;
-#pragma unroll 1
-        for (int b = lane; b < nblk; b += 32) {
-          uint64_t mask = s_ev[b];
-          nev += __popcll(mask);
-#pragma unroll 1
-          while (mask != 0ull) {
-            const int bit = __ffsll((long long)mask) - 1;
-            mask &= mask - 1ull;
-            int16_t* hp = hrow + 64 * b + bit;
-            const uint32_t v = (uint16_t)*hp;
-            *hp = (int16_t)((v >= pos_from) ? min(v + 1u, v_top) : max(v - 1u, (uint32_t)E.base));
-          }
-        }
-        nev = warp_sum(nev);
-        st_rows += 1u;
-        st_bytes += 4u * (uint32_t)nev;
-        __syncwarp();   // s_ev and s_list are reused by the next row
-        continue;
-      }
-      st_rows += 1u;
-      st_streamed += 1u;
-      st_bytes += 4u * (uint32_t)Ly.ldh + 8u * (uint32_t)Ly.nw_in;
-
-      // ---- 3. CP and W over the row ----
-      uint8_t* wrow = reinterpret_cast<uint8_t*>(Ly.W + (int64_t)k * Ly.nw_in);
-      // Each iteration handles two chunks per lane, ch and ch + 32 (64 chunks
-      // per warp), so the tuple loop and the loop control are shared.  A
-      // rotating queue keeps the H vectors of the next iteration in flight (4
-      // per lane); the activation bytes of the first kPre tuples are fetched at
-      // the top of each iteration.  Every lane runs the same number of
-      // iterations.
-      uint4 q0 = make_uint4(0, 0, 0, 0), q1 = q0, q2 = q0, q3 = q0;
-      if (lane < nch) q0 = __ldcs(reinterpret_cast<const uint4*>(hrow + 8 * lane));
-      if (lane + 32 < nch) q1 = __ldcs(reinterpret_cast<const uint4*>(hrow + 8 * (lane + 32)));
-      if (lane + 64 < nch) q2 = __ldcs(reinterpret_cast<const uint4*>(hrow + 8 * (lane + 64)));
-      if (lane + 96 < nch) q3 = __ldcs(reinterpret_cast<const uint4*>(hrow + 8 * (lane + 96)));
-      const int iters2 = (nch + 63) >> 6;
-      // activation bytes of tuples 0..kPre-1 (one per byte) for the next
-      // iteration's two chunks, loaded one iteration ahead
-      auto tuple_bytes = [&](int it_next, uint32_t (&pbo)[2]) {
-        pbo[0] = 0u;
-        pbo[1] = 0u;
-#pragma unroll
-        for (int q = 0; q < kPre; ++q) {
-          if (q < n_t) {
-            const uint8_t* arow = aprev + (size_t)(s_list[q] & 0xFFFF) * arow_bytes;
-#pragma unroll
-            for (int u = 0; u < 2; ++u) {
-              const int ch = 64 * it_next + 32 * u + lane;
-              if (ch < nch) pbo[u] |= (uint32_t)__ldg(arow + ch) << (8 * q);
+        int16_t* hrow = Ly.H + (int64_t)k * Ly.ldh;
+        if (n_t == 0) {
+          // no tuple: H changes only at the reinforcement events, which never
+          // flip a sign, so W stays; single-weight read-modify-writes
+          int nev = 0;
+  #pragma unroll 1
+          for (int b = lane; b < nblk; b += 32) {
+            uint64_t mask = s_ev[b];
+            nev += __popcll(mask);
+  #pragma unroll 1
+            while (mask != 0ull) {
+              const int bit = __ffsll((long long)mask) - 1;
+              mask &= mask - 1ull;
+              int16_t* hp = hrow + 64 * b + bit;
+              const uint32_t v = (uint16_t)*hp;
+              *hp = (int16_t)((v >= pos_from) ? min(v + 1u, v_top) : max(v - 1u, (uint32_t)E.base));
             }
           }
+          nev = warp_sum(nev);
+          st_rows += 1u;
+          st_bytes += 4u * (uint32_t)nev;
+          __syncwarp();   // s_ev and s_list are reused by the next row
+          continue;
         }
-      };
-      uint32_t pbn[2];
-      tuple_bytes(0, pbn);
-#pragma unroll 1
-      for (int it = 0; it < iters2; ++it) {
-        int chv[2];
-        bool live[2];
-        uint4 w[2];
-        uint32_t pb[2] = {pbn[0], pbn[1]};  // this iteration's tuple bytes
-        chv[0] = 64 * it + lane;
-        chv[1] = chv[0] + 32;
-        live[0] = chv[0] < nch;
-        live[1] = chv[1] < nch;
-        if (it + 1 < iters2) tuple_bytes(it + 1, pbn);
-        w[0] = q0;
-        w[1] = q1;
-        q0 = q2;
-        q1 = q3;
-        if (chv[0] + 128 < nch) q2 = __ldcs(reinterpret_cast<const uint4*>(hrow + 8 * (chv[0] + 128)));
-        if (chv[1] + 128 < nch) q3 = __ldcs(reinterpret_cast<const uint4*>(hrow + 8 * (chv[1] + 128)));
-#pragma unroll
-        for (int q = 0; q < kPre; ++q) {
-          if (q < n_t) {
-            const uint2* dn = s_dn[(s_list[q] >> 16) & 1];
-#pragma unroll
+        st_rows += 1u;
+        st_streamed += 1u;
+        st_bytes += 4u * (uint32_t)Ly.ldh + 8u * (uint32_t)Ly.nw_in;
+
+        // ---- 3. CP and W over the row ----
+        uint8_t* wrow = reinterpret_cast<uint8_t*>(Ly.W + (int64_t)k * Ly.nw_in);
+        // Each iteration handles two chunks per lane, ch and ch + 32 (64 chunks
+        // per warp), so the tuple loop and the loop control are shared.  A
+        // rotating queue keeps the H vectors of the next iteration in flight (4
+        // per lane); the activation bytes of the first kPre tuples are fetched at
+        // the top of each iteration.  Every lane runs the same number of
+        // iterations.
+        uint4 q0 = make_uint4(0, 0, 0, 0), q1 = q0, q2 = q0, q3 = q0;
+        if (lane < nch) q0 = __ldcs(reinterpret_cast<const uint4*>(hrow + 8 * lane));
+        if (lane + 32 < nch) q1 = __ldcs(reinterpret_cast<const uint4*>(hrow + 8 * (lane + 32)));
+        if (lane + 64 < nch) q2 = __ldcs(reinterpret_cast<const uint4*>(hrow + 8 * (lane + 64)));
+        if (lane + 96 < nch) q3 = __ldcs(reinterpret_cast<const uint4*>(hrow + 8 * (lane + 96)));
+        const int iters2 = (nch + 63) >> 6;
+        // activation bytes of tuples 0..kPre-1 (one per byte) for the next
+        // iteration's two chunks, loaded one iteration ahead
+        auto tuple_bytes = [&](int it_next, uint32_t (&pbo)[2]) {
+          pbo[0] = 0u;
+          pbo[1] = 0u;
+  #pragma unroll
+          for (int q = 0; q < kPre; ++q) {
+            if (q < n_t) {
+              const uint8_t* arow = aprev + (size_t)(s_list[q] & 0xFFFF) * arow_bytes;
+  #pragma unroll
+              for (int u = 0; u < 2; ++u) {
+                const int ch = 64 * it_next + 32 * u + lane;
+                if (ch < nch) pbo[u] |= (uint32_t)__ldg(arow + ch) << (8 * q);
+              }
+            }
+          }
+        };
+        uint32_t pbn[2];
+        tuple_bytes(0, pbn);
+  #pragma unroll 1
+        for (int it = 0; it < iters2; ++it) {
+          int chv[2];
+          bool live[2];
+          uint4 w[2];
+          uint32_t pb[2] = {pbn[0], pbn[1]};  // this iteration's tuple bytes
+          chv[0] = 64 * it + lane;
+          chv[1] = chv[0] + 32;
+          live[0] = chv[0] < nch;
+          live[1] = chv[1] < nch;
+          if (it + 1 < iters2) tuple_bytes(it + 1, pbn);
+          w[0] = q0;
+          w[1] = q1;
+          q0 = q2;
+          q1 = q3;
+          if (chv[0] + 128 < nch) q2 = __ldcs(reinterpret_cast<const uint4*>(hrow + 8 * (chv[0] + 128)));
+          if (chv[1] + 128 < nch) q3 = __ldcs(reinterpret_cast<const uint4*>(hrow + 8 * (chv[1] + 128)));
+  #pragma unroll
+          for (int q = 0; q < kPre; ++q) {
+            if (q < n_t) {
+              const uint2* dn = s_dn[(s_list[q] >> 16) & 1];
+  #pragma unroll
+              for (int u = 0; u < 2; ++u) {
+                const uint32_t byte = (pb[u] >> (8 * q)) & 0xFFu;
+                const uint2 dl = dn[byte & 15u], dh = dn[byte >> 4];
+                w[u].x = LN.clip(w[u].x + dl.x);
+                w[u].y = LN.clip(w[u].y + dl.y);
+                w[u].z = LN.clip(w[u].z + dh.x);
+                w[u].w = LN.clip(w[u].w + dh.y);
+              }
+            }
+          }
+  #pragma unroll 1
+          for (int q = kPre; q < n_t; ++q) {
+            const int e = s_list[q];
+            const uint2* dn = s_dn[(e >> 16) & 1];
+            const uint8_t* arow = aprev + (size_t)(e & 0xFFFF) * arow_bytes;
+  #pragma unroll
             for (int u = 0; u < 2; ++u) {
-              const uint32_t byte = (pb[u] >> (8 * q)) & 0xFFu;
+              const uint32_t byte = live[u] ? arow[chv[u]] : 0u;
               const uint2 dl = dn[byte & 15u], dh = dn[byte >> 4];
               w[u].x = LN.clip(w[u].x + dl.x);
               w[u].y = LN.clip(w[u].y + dl.y);
@@ -566,71 +575,55 @@ __global__ void __launch_bounds__(kUpdThreads, 4) k_update(const StepParams* __r
               w[u].w = LN.clip(w[u].w + dh.y);
             }
           }
-        }
-#pragma unroll 1
-        for (int q = kPre; q < n_t; ++q) {
-          const int e = s_list[q];
-          const uint2* dn = s_dn[(e >> 16) & 1];
-          const uint8_t* arow = aprev + (size_t)(e & 0xFFFF) * arow_bytes;
-#pragma unroll
-          for (int u = 0; u < 2; ++u) {
-            const uint32_t byte = live[u] ? arow[chv[u]] : 0u;
-            const uint2 dl = dn[byte & 15u], dh = dn[byte >> 4];
-            w[u].x = LN.clip(w[u].x + dl.x);
-            w[u].y = LN.clip(w[u].y + dl.y);
-            w[u].z = LN.clip(w[u].z + dh.x);
-            w[u].w = LN.clip(w[u].w + dh.y);
+          // ---- R: the chunks' bytes of the row's event bitmap ----
+          uint32_t fb[2];
+  #pragma unroll
+          for (int u = 0; u < 2; ++u)
+            fb[u] = live[u] ? (uint32_t)reinterpret_cast<const uint8_t*>(s_ev)[chv[u]] : 0u;
+          if (__any_sync(kFull, (fb[0] | fb[1]) != 0u)) {
+  #pragma unroll
+            for (int u = 0; u < 2; ++u) {
+              if (fb[u] != 0u) {
+                const uint2 fl = s_fire[fb[u] & 15u], fh = s_fire[fb[u] >> 4];
+                w[u].x = LN.reinforce(w[u].x, fl.x);
+                w[u].y = LN.reinforce(w[u].y, fl.y);
+                w[u].z = LN.reinforce(w[u].z, fh.x);
+                w[u].w = LN.reinforce(w[u].w, fh.y);
+              }
+            }
           }
-        }
-        // ---- R: the chunks' bytes of the row's event bitmap ----
-        uint32_t fb[2];
-#pragma unroll
-        for (int u = 0; u < 2; ++u)
-          fb[u] = live[u] ? (uint32_t)reinterpret_cast<const uint8_t*>(s_ev)[chv[u]] : 0u;
-        if (__any_sync(kFull, (fb[0] | fb[1]) != 0u)) {
-#pragma unroll
+  #pragma unroll
           for (int u = 0; u < 2; ++u) {
-            if (fb[u] != 0u) {
-              const uint2 fl = s_fire[fb[u] & 15u], fh = s_fire[fb[u] >> 4];
-              w[u].x = LN.reinforce(w[u].x, fl.x);
-              w[u].y = LN.reinforce(w[u].y, fl.y);
-              w[u].z = LN.reinforce(w[u].z, fh.x);
-              w[u].w = LN.reinforce(w[u].w, fh.y);
+            uint32_t wbyte = LN.w_byte(w[u]);
+            if (live[u] && chv[u] >= full) {
+              // the partly padded last chunk: per weight, from the row as
+              // loaded (H is written back only below)
+              const uint4 w0 = *reinterpret_cast<const uint4*>(hrow + 8 * chv[u]);
+              const ChunkOut o = chunk_scalar(w0, chv[u], Kin - 8 * chv[u], s_list, n_t, aprev,
+                                              arow_bytes, E, fb[u]);
+              w[u] = o.w;
+              wbyte = o.wbyte;
+            }
+            if (live[u]) {
+              __stcs(reinterpret_cast<uint4*>(hrow + 8 * chv[u]), w[u]);
+              wrow[chv[u]] = (uint8_t)wbyte;
             }
           }
         }
-#pragma unroll
-        for (int u = 0; u < 2; ++u) {
-          uint32_t wbyte = LN.w_byte(w[u]);
-          if (live[u] && chv[u] >= full) {
-            // the partly padded last chunk: per weight, from the row as
-            // loaded (H is written back only below)
-            const uint4 w0 = *reinterpret_cast<const uint4*>(hrow + 8 * chv[u]);
-            const ChunkOut o = chunk_scalar(w0, chv[u], Kin - 8 * chv[u], s_list, n_t, aprev,
-                                            arow_bytes, E, fb[u]);
-            w[u] = o.w;
-            wbyte = o.wbyte;
-          }
-          if (live[u]) {
-            __stcs(reinterpret_cast<uint4*>(hrow + 8 * chv[u]), w[u]);
-            wrow[chv[u]] = (uint8_t)wbyte;
-          }
-        }
-      }
       __syncwarp();   // s_ev and s_list are reused by the next row
     }
-    // statistics: per CTA, one atomic per counter
-    if (lane == 0) {
-      atomicAdd(&s_stats[0], (unsigned long long)st_rows);
-      atomicAdd(&s_stats[1], (unsigned long long)st_streamed);
-      atomicAdd(&s_stats[2], (unsigned long long)st_bytes);
-    }
-    __syncthreads();
-    if (threadIdx.x == 0) {
-      atomicAdd(&ctrl->upd_rows, s_stats[0]);
-      atomicAdd(&ctrl->upd_streamed, s_stats[1]);
-      atomicAdd(&ctrl->upd_bytes, s_stats[2]);
-    }
+  }
+  // statistics: per CTA, one atomic per counter
+  if (lane == 0) {
+    atomicAdd(&s_stats[0], (unsigned long long)st_rows);
+    atomicAdd(&s_stats[1], (unsigned long long)st_streamed);
+    atomicAdd(&s_stats[2], (unsigned long long)st_bytes);
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    atomicAdd(&ctrl->upd_rows, s_stats[0]);
+    atomicAdd(&ctrl->upd_streamed, s_stats[1]);
+    atomicAdd(&ctrl->upd_bytes, s_stats[2]);
   }
 
   // step completion: the last warp to finish advances the counters
@@ -642,6 +635,7 @@ __global__ void __launch_bounds__(kUpdThreads, 4) k_update(const StepParams* __r
       ctrl->t = t + 1;
       ctrl->s = s + 1;
       for (int i = 0; i < P->L; ++i) ctrl->any_mark[i] = 0u;
+      ctrl->upd_next = 0u;
       ctrl->done = 0u;
       __threadfence();
     }
@@ -704,6 +698,11 @@ void launch_update(bool pow2, unsigned grid, size_t smem, cudaStream_t st, const
     k_update<true><<<grid, kUpdThreads, smem, st>>>(P, key0, key1);
   else
     k_update<false><<<grid, kUpdThreads, smem, st>>>(P, key0, key1);
+}
+
+cudaError_t update_kernel_occupancy(bool pow2, size_t smem, int* per_sm) {
+  return pow2 ? cudaOccupancyMaxActiveBlocksPerMultiprocessor(per_sm, k_update<true>, kUpdThreads, smem)
+              : cudaOccupancyMaxActiveBlocksPerMultiprocessor(per_sm, k_update<false>, kUpdThreads, smem);
 }
 
 cudaError_t update_kernel_attributes(cudaFuncAttributes* fa, size_t smem) {
