@@ -185,7 +185,10 @@ constexpr uint32_t kLaneTop = 0x80008000u;
 constexpr uint32_t kLaneOne = 0x00010001u;
 constexpr unsigned kFull = 0xffffffffu;
 constexpr int kPre = 4;  // tuples per row whose activation bytes are prefetched
-constexpr int kRowChunk = 2;  // rows a warp takes from the row counter at a time
+// the prefetched activation bytes of one chunk, one byte per tuple
+using TupleBytes = uint32_t;
+static_assert(kPre <= (int)sizeof(TupleBytes), "one byte per prefetched tuple");
+constexpr int kRowChunk = 1;  // rows a warp takes from the row counter at a time
 
 // shared memory of one update warp: s_list [bs] int32, s_ev [nblk_max] uint64
 __host__ __device__ __forceinline__ size_t update_warp_smem(int bs, int nblk_max) {
@@ -511,7 +514,7 @@ __global__ void __launch_bounds__(kUpdThreads, 4) k_update(const StepParams* __r
         const int iters2 = (nch + 63) >> 6;
         // activation bytes of tuples 0..kPre-1 (one per byte) for the next
         // iteration's two chunks, loaded one iteration ahead
-        auto tuple_bytes = [&](int it_next, uint32_t (&pbo)[2]) {
+        auto tuple_bytes = [&](int it_next, TupleBytes (&pbo)[2]) {
           pbo[0] = 0u;
           pbo[1] = 0u;
   #pragma unroll
@@ -521,19 +524,19 @@ __global__ void __launch_bounds__(kUpdThreads, 4) k_update(const StepParams* __r
   #pragma unroll
               for (int u = 0; u < 2; ++u) {
                 const int ch = 64 * it_next + 32 * u + lane;
-                if (ch < nch) pbo[u] |= (uint32_t)__ldg(arow + ch) << (8 * q);
+                if (ch < nch) pbo[u] |= (TupleBytes)__ldg(arow + ch) << (8 * q);
               }
             }
           }
         };
-        uint32_t pbn[2];
+        TupleBytes pbn[2];
         tuple_bytes(0, pbn);
   #pragma unroll 1
         for (int it = 0; it < iters2; ++it) {
           int chv[2];
           bool live[2];
           uint4 w[2];
-          uint32_t pb[2] = {pbn[0], pbn[1]};  // this iteration's tuple bytes
+          TupleBytes pb[2] = {pbn[0], pbn[1]};  // this iteration's tuple bytes
           chv[0] = 64 * it + lane;
           chv[1] = chv[0] + 32;
           live[0] = chv[0] < nch;
@@ -551,7 +554,7 @@ __global__ void __launch_bounds__(kUpdThreads, 4) k_update(const StepParams* __r
               const uint2* dn = s_dn[(s_list[q] >> 16) & 1];
   #pragma unroll
               for (int u = 0; u < 2; ++u) {
-                const uint32_t byte = (pb[u] >> (8 * q)) & 0xFFu;
+                const uint32_t byte = (uint32_t)(pb[u] >> (8 * q)) & 0xFFu;
                 const uint2 dl = dn[byte & 15u], dh = dn[byte >> 4];
                 w[u].x = LN.clip(w[u].x + dl.x);
                 w[u].y = LN.clip(w[u].y + dl.y);
