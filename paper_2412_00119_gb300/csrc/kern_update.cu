@@ -174,7 +174,7 @@ __global__ void __launch_bounds__(kClsThreads) k_cls_select(const StepParams* __
 // clear) or to 2^hb + h_max + 1 (= 2^(hb+1) when h_max + 1 = 2^hb, kPow2); the
 // clip moves it back.  h > 0 is the lane's bit hb - 1 (kPow2) or v >= 2^hb +
 // (h_max + 1)/2.  The CP step per tuple adds the packed +-1 steps
-// 2 a^mu_i rho_{k,y^mu}/2 from a 16-entry shared nibble table, then clips.
+// 2 a^mu_i rho_{k,y^mu}/2 from a 256-entry shared byte table, then clips.
 // The partly padded last chunk of a row runs per weight.  Layers with an
 // empty M_l are skipped (no CP, no R).  The last warp to finish advances the
 // step counters and clears the per-step flags.
@@ -375,7 +375,7 @@ template <bool kPow2>
 __global__ void __launch_bounds__(kUpdThreads, 4) k_update(const StepParams* __restrict__ P,
                                                            uint32_t key0, uint32_t key1) {
   extern __shared__ int32_t dyn[];
-  __shared__ uint2 s_dn[2][16];
+  __shared__ uint4 s_db[256];
   __shared__ uint2 s_fire[16];
   __shared__ unsigned long long s_stats[3];
   Ctrl* ctrl = P->ctrl;
@@ -392,15 +392,21 @@ __global__ void __launch_bounds__(kUpdThreads, 4) k_update(const StepParams* __r
   uint64_t* s_ev = reinterpret_cast<uint64_t*>(wbase + ((sizeof(int32_t) * P->bs + 7) & ~(size_t)7));
 
   if (threadIdx.x == 0) s_stats[0] = s_stats[1] = s_stats[2] = 0ull;
-  // s_dn[r][n]: the +-1 lattice steps of the 4 weights of nibble n, two lanes
-  // per word (d_lo + 2^16 d_hi), d = +1 for a set bit, negated for r = 1
-  // (rho = -1)
+  // s_db[b]: the +-1 lattice steps of the 8 weights of a chunk whose
+  // activation byte is b, for rho = +1 (rho = -1 indexes with ~b): d = +1 for
+  // a set bit, two lanes per word (d_lo + 2^16 d_hi)
+  {
+    const int b = threadIdx.x & 255;
+    uint32_t wv[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const int d0 = ((b >> (2 * j)) & 1) ? 1 : -1, d1 = ((b >> (2 * j + 1)) & 1) ? 1 : -1;
+      wv[j] = (uint32_t)(d0 + 65536 * d1);
+    }
+    if (threadIdx.x < 256) s_db[b] = make_uint4(wv[0], wv[1], wv[2], wv[3]);
+  }
   if (threadIdx.x < 32) {
     const int r = threadIdx.x >> 4, n = threadIdx.x & 15;
-    int d[4];
-#pragma unroll
-    for (int j = 0; j < 4; ++j) d[j] = (((n >> j) & 1) ? 1 : -1) * (r ? -1 : 1);
-    s_dn[r][n] = make_uint2((uint32_t)(d[0] + 65536 * d[1]), (uint32_t)(d[2] + 65536 * d[3]));
     // s_fire[n]: 1 in each lane of nibble n whose bit is set, two lanes per word
     if (r == 0)
       s_fire[n] = make_uint2((uint32_t)((n & 1) | ((n >> 1) & 1) << 16),
@@ -551,31 +557,30 @@ __global__ void __launch_bounds__(kUpdThreads, 4) k_update(const StepParams* __r
   #pragma unroll
           for (int q = 0; q < kPre; ++q) {
             if (q < n_t) {
-              const uint2* dn = s_dn[(s_list[q] >> 16) & 1];
+              const uint32_t xm = (s_list[q] & 0x10000) ? 0xFFu : 0u;  // rho = -1: ~byte
   #pragma unroll
               for (int u = 0; u < 2; ++u) {
-                const uint32_t byte = (uint32_t)(pb[u] >> (8 * q)) & 0xFFu;
-                const uint2 dl = dn[byte & 15u], dh = dn[byte >> 4];
-                w[u].x = LN.clip(w[u].x + dl.x);
-                w[u].y = LN.clip(w[u].y + dl.y);
-                w[u].z = LN.clip(w[u].z + dh.x);
-                w[u].w = LN.clip(w[u].w + dh.y);
+                const uint4 d = s_db[((uint32_t)(pb[u] >> (8 * q)) ^ xm) & 0xFFu];
+                w[u].x = LN.clip(w[u].x + d.x);
+                w[u].y = LN.clip(w[u].y + d.y);
+                w[u].z = LN.clip(w[u].z + d.z);
+                w[u].w = LN.clip(w[u].w + d.w);
               }
             }
           }
   #pragma unroll 1
           for (int q = kPre; q < n_t; ++q) {
             const int e = s_list[q];
-            const uint2* dn = s_dn[(e >> 16) & 1];
+            const uint32_t xm = (e & 0x10000) ? 0xFFu : 0u;
             const uint8_t* arow = aprev + (size_t)(e & 0xFFFF) * arow_bytes;
   #pragma unroll
             for (int u = 0; u < 2; ++u) {
               const uint32_t byte = live[u] ? arow[chv[u]] : 0u;
-              const uint2 dl = dn[byte & 15u], dh = dn[byte >> 4];
-              w[u].x = LN.clip(w[u].x + dl.x);
-              w[u].y = LN.clip(w[u].y + dl.y);
-              w[u].z = LN.clip(w[u].z + dh.x);
-              w[u].w = LN.clip(w[u].w + dh.y);
+              const uint4 d = s_db[(byte ^ xm) & 0xFFu];
+              w[u].x = LN.clip(w[u].x + d.x);
+              w[u].y = LN.clip(w[u].y + d.y);
+              w[u].z = LN.clip(w[u].z + d.z);
+              w[u].w = LN.clip(w[u].w + d.w);
             }
           }
           // ---- R: the chunks' bytes of the row's event bitmap ----
