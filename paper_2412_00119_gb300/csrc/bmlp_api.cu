@@ -230,7 +230,7 @@ int enqueue_step(bmlp_t* h, cudaStream_t st, bool fork) {
   }
   if (fork) CK(h, cudaStreamWaitEvent(st, h->evJoin, 0));
   prof_begin(h, kProfUpd, st);
-  launch_update(((h->h_max + 1) & h->h_max) == 0, (unsigned)h->updCtas, h->updSmem, st, h->dP,
+  launch_update(update_hb_mode(h->h_max, h->hp.hb), (unsigned)h->updCtas, h->updSmem, st, h->dP,
                 h->hp.key0, h->hp.key1);
   prof_end(h, st);
   CK(h, cudaGetLastError());
@@ -464,7 +464,7 @@ int bmlp_create(const int32_t* widths, int32_t n_widths, int32_t classes, int16_
     if (ea != cudaSuccess) return bail(cuda_fail(h, ea, "update kernel shared memory attribute"));
     // the update grid is persistent: as many CTAs as fit on the device at once
     int per_sm = 0;
-    ea = update_kernel_occupancy(((h_max + 1) & h_max) == 0, h->updSmem, &per_sm);
+    ea = update_kernel_occupancy(update_hb_mode(h_max, P.hb), h->updSmem, &per_sm);
     if (ea != cudaSuccess || per_sm < 1)
       return bail(cuda_fail(h, ea != cudaSuccess ? ea : cudaErrorInvalidConfiguration,
                             "update kernel occupancy"));

@@ -141,8 +141,13 @@ __global__ void k_cls_select(const StepParams* P);
 // (key0, key1) = the Philox key, passed by value so that the round keys are
 // kernel-uniform.  kPow2: h_max + 1 is a power of two (both clip bounds are bit
 // boundaries of the lattice index).
-void launch_update(bool pow2, unsigned grid, size_t smem, cudaStream_t st, const StepParams* P,
+// hb_mode: 8 when h_max = 255 (compile-time lattice exponent), -1 for another
+// h_max + 1 that is a power of two, 0 otherwise (update_hb_mode).
+void launch_update(int hb_mode, unsigned grid, size_t smem, cudaStream_t st, const StepParams* P,
                    uint32_t key0, uint32_t key1);
+inline int update_hb_mode(int h_max, int hb) {
+  return ((h_max + 1) & h_max) != 0 ? 0 : (hb == 8 ? 8 : -1);
+}
 // Reinforcement events of every neuron row of every layer for the current
 // step into DevLayer::EV (Alg. 3 l.5-12); grid = P->ev_ctas_total CTAs.
 void launch_r_events(unsigned grid, cudaStream_t st, const StepParams* P, uint32_t key0,
@@ -156,7 +161,7 @@ cudaError_t update_kernel_attributes(cudaFuncAttributes* fa, size_t smem);
 // of at most nblk_max blocks of 64 inputs.
 size_t update_smem_bytes(int bs, int nblk_max);
 // CTAs of the update kernel that fit on one SM at once.
-cudaError_t update_kernel_occupancy(bool pow2, size_t smem, int* per_sm);
+cudaError_t update_kernel_occupancy(int hb_mode, size_t smem, int* per_sm);
 // Generic forward for evaluation: A (M x nw_in) against W -> Aout (M x nw_out).
 __global__ void k_forward_eval(const uint64_t* __restrict__ A, int64_t M, int nw_in,
                                const uint64_t* __restrict__ W, int N, int Kin,

@@ -280,24 +280,28 @@ __device__ __forceinline__ uint32_t gather_top(uint32_t a, uint32_t b, uint32_t 
   return ((p0 * 0x00204081u) >> 28) | (((p1 * 0x00204081u) >> 28) << 4);
 }
 
-template <bool kPow2>
+// kHb > 0: h_max + 1 = 2^kHb, a compile-time exponent; kHb = -1: h_max + 1 a
+// power of two given at run time; kHb = 0: any odd h_max.
+template <int kHb>
 struct Lanes {
-  int hb;
+  static constexpr bool kPow2 = kHb != 0;
+  int hb_rt;
+  __device__ __forceinline__ int hb() const { return kHb > 0 ? kHb : hb_rt; }
   uint32_t over_pair;  // pair(2^hb + h_max + 1), used when !kPow2
   uint32_t pos_pair;   // pair(2^hb + (h_max + 1)/2), used when !kPow2
   // lanes that left [2^hb, 2^hb + h_max] by one step go back
   __device__ __forceinline__ uint32_t clip(uint32_t v) const {
     if (kPow2) {
-      const uint32_t t = (v >> hb) & 0x00030003u;  // 0 under, 1 inside, 2 over
+      const uint32_t t = (v >> hb()) & 0x00030003u;  // 0 under, 1 inside, 2 over
       return v + kLaneOne - t;
     } else {
-      const uint32_t under = (~v >> hb) & kLaneOne;
+      const uint32_t under = (~v >> hb()) & kLaneOne;
       return v + under - (eq_flags(v, over_pair) >> 15);
     }
   }
   // bit 15 of each lane = (h > 0)
   __device__ __forceinline__ uint32_t pos_top(uint32_t v) const {
-    if (kPow2) return (v << (16 - hb)) & kLaneTop;
+    if (kPow2) return (v << (16 - hb())) & kLaneTop;
     return ((v | kLaneTop) - pos_pair) & kLaneTop;
   }
   // lanes with f = 1 (f: 0 or 1 per lane) step away from 0, then clip
@@ -310,7 +314,7 @@ struct Lanes {
     if (kPow2) {
       // move each lane's sign bit (bit hb - 1) to bit 7 of the lane's low byte;
       // the low bytes of the 8 lanes then hold the 8 sign bits at bit 7
-      const int sh = 8 - hb;
+      const int sh = 8 - hb();
       const uint32_t x = sh >= 0 ? w.x << sh : w.x >> -sh, y = sh >= 0 ? w.y << sh : w.y >> -sh;
       const uint32_t z = sh >= 0 ? w.z << sh : w.z >> -sh, u = sh >= 0 ? w.w << sh : w.w >> -sh;
       const uint32_t p0 = __byte_perm(x, y, 0x6420) & 0x80808080u;
@@ -371,7 +375,7 @@ size_t update_smem_bytes(int bs, int nblk_max) {
   return (size_t)(kUpdThreads / 32) * update_warp_smem(bs, nblk_max);
 }
 
-template <bool kPow2>
+template <int kHb>
 __global__ void __launch_bounds__(kUpdThreads, 4) k_update(const StepParams* __restrict__ P,
                                                            uint32_t key0, uint32_t key1) {
   extern __shared__ int32_t dyn[];
@@ -419,8 +423,8 @@ __global__ void __launch_bounds__(kUpdThreads, 4) k_update(const StepParams* __r
   E.h_max = P->h_max;
   E.hb = P->hb;
   E.base = 1 << P->hb;
-  Lanes<kPow2> LN;
-  LN.hb = P->hb;
+  Lanes<kHb> LN;
+  LN.hb_rt = P->hb;
   LN.over_pair = (uint32_t)(E.base + E.h_max + 1) * kLaneOne;
   LN.pos_pair = (uint32_t)(E.base + (E.h_max + 1) / 2) * kLaneOne;
   const uint32_t pos_from = (uint32_t)(E.base + (E.h_max + 1) / 2);  // lattice index of h = +1
@@ -700,27 +704,33 @@ void launch_r_events(unsigned grid, cudaStream_t st, const StepParams* P, uint32
   k_r_events<<<grid, kEvThreads, 0, st>>>(P, key0, key1);
 }
 
-void launch_update(bool pow2, unsigned grid, size_t smem, cudaStream_t st, const StepParams* P,
+void launch_update(int hb_mode, unsigned grid, size_t smem, cudaStream_t st, const StepParams* P,
                    uint32_t key0, uint32_t key1) {
-  if (pow2)
-    k_update<true><<<grid, kUpdThreads, smem, st>>>(P, key0, key1);
+  if (hb_mode == 8)
+    k_update<8><<<grid, kUpdThreads, smem, st>>>(P, key0, key1);
+  else if (hb_mode != 0)
+    k_update<-1><<<grid, kUpdThreads, smem, st>>>(P, key0, key1);
   else
-    k_update<false><<<grid, kUpdThreads, smem, st>>>(P, key0, key1);
+    k_update<0><<<grid, kUpdThreads, smem, st>>>(P, key0, key1);
 }
 
-cudaError_t update_kernel_occupancy(bool pow2, size_t smem, int* per_sm) {
-  return pow2 ? cudaOccupancyMaxActiveBlocksPerMultiprocessor(per_sm, k_update<true>, kUpdThreads, smem)
-              : cudaOccupancyMaxActiveBlocksPerMultiprocessor(per_sm, k_update<false>, kUpdThreads, smem);
+cudaError_t update_kernel_occupancy(int hb_mode, size_t smem, int* per_sm) {
+  if (hb_mode == 8)
+    return cudaOccupancyMaxActiveBlocksPerMultiprocessor(per_sm, k_update<8>, kUpdThreads, smem);
+  if (hb_mode != 0)
+    return cudaOccupancyMaxActiveBlocksPerMultiprocessor(per_sm, k_update<-1>, kUpdThreads, smem);
+  return cudaOccupancyMaxActiveBlocksPerMultiprocessor(per_sm, k_update<0>, kUpdThreads, smem);
 }
 
 cudaError_t update_kernel_attributes(cudaFuncAttributes* fa, size_t smem) {
-  cudaError_t e = cudaFuncGetAttributes(fa, k_update<true>);
+  cudaError_t e = cudaFuncGetAttributes(fa, k_update<8>);
   if (e != cudaSuccess || smem == 0) return e;
-  if ((e = cudaFuncSetAttribute(k_update<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  if ((e = cudaFuncSetAttribute(k_update<8>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                (int)smem)) != cudaSuccess ||
+      (e = cudaFuncSetAttribute(k_update<-1>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 (int)smem)) != cudaSuccess)
     return e;
-  return cudaFuncSetAttribute(k_update<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              (int)smem);
+  return cudaFuncSetAttribute(k_update<0>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
 }
 
 // ---------------------------------------------------------------------------
