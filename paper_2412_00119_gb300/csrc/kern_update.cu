@@ -655,14 +655,16 @@ __global__ void __launch_bounds__(kUpdThreads, 4) k_update(const StepParams* __r
 }
 
 // Reinforcement events of the current step (Alg. 3 l.5-12): warp per neuron
-// row; lane j draws the block draws of blocks 4j .. 4j+3 (one Philox call) and,
-// for each block that holds an event, its event draws (binary searches in the
-// layer's threshold tables, staged in shared memory); the row's bitmap goes to
+// row; lane j draws the block draws of blocks 4j .. 4j+3 (one Philox call), the
+// blocks that hold an event are compacted into a per-warp list, and the lanes
+// share that list for the event draws (binary searches in the layer's
+// threshold tables, staged in shared memory); the row's bitmap goes to
 // DevLayer::EV.  It depends only on (seed, layer, neuron, step, p_r), so it
 // runs beside the forward passes.
 __global__ void __launch_bounds__(kEvThreads) k_r_events(const StepParams* __restrict__ P,
                                                          uint32_t key0, uint32_t key1) {
   __shared__ RTables s_rt;
+  __shared__ uint16_t s_cand[kEvRowsPerCta][128];  // blocks with an event, per warp
   const int bid = blockIdx.x;
   int li = 0;
   while (li + 1 < P->L && bid >= P->layer[li + 1].ev_cta_base) ++li;
@@ -680,22 +682,48 @@ __global__ void __launch_bounds__(kEvThreads) k_r_events(const StepParams* __res
   const uint32_t tt = (uint32_t)P->ctrl->t;
   const int Kin = Ly.Kin, nblk = Ly.nblk;
   uint64_t* ev = Ly.EV + (int64_t)k * nblk;
+  uint16_t* cand = s_cand[warp];
+  // rounds of 32 block groups (128 blocks): the block draws, one Philox call per
+  // lane; the blocks that hold an event are compacted into a list that the
+  // lanes then share, one block each, for the event draws
 #pragma unroll 1
-  for (int gq = lane; 4 * gq < nblk; gq += 32) {
-    const uint4 u = philox4x32_10(make_uint4((uint32_t)gq, (uint32_t)k, (3u << 16) + l, tt), key0,
-                                  key1);
+  for (int g0 = 0; 4 * g0 < nblk; g0 += 32) {
+    const int gq = g0 + lane;
+    uint32_t cmask = 0;
+    if (4 * gq < nblk) {
+      const uint4 u = philox4x32_10(make_uint4((uint32_t)gq, (uint32_t)k, (3u << 16) + l, tt), key0,
+                                    key1);
 #pragma unroll
-    for (int wq = 0; wq < 4; ++wq) {
-      const int b = 4 * gq + wq;
-      if (b < nblk) {
-        const int n = min(64, Kin - 64 * b);
-        const int x = (n == 64) ? 0 : 1;
-        uint64_t mask = 0;
-        if ((unsigned long long)word_of(u, wq) < s_rt.any[x])
-          mask = block_events(s_rt, x, n, (uint32_t)b, (uint32_t)k, l, tt, key0, key1);
-        ev[b] = mask;
+      for (int wq = 0; wq < 4; ++wq) {
+        const int b = 4 * gq + wq;
+        if (b < nblk) {
+          const int x = (Kin - 64 * b >= 64) ? 0 : 1;
+          if ((unsigned long long)word_of(u, wq) < s_rt.any[x]) cmask |= 1u << wq;
+          else ev[b] = 0ull;
+        }
       }
     }
+    // exclusive prefix of the candidate counts over the lanes
+    const int cnt = __popc(cmask);
+    int incl = cnt;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+      const int v = __shfl_up_sync(kFull, incl, off);
+      if (lane >= off) incl += v;
+    }
+    const int total = __shfl_sync(kFull, incl, 31);
+    int pos = incl - cnt;
+#pragma unroll
+    for (int wq = 0; wq < 4; ++wq)
+      if ((cmask >> wq) & 1u) cand[pos++] = (uint16_t)(4 * gq + wq);
+    __syncwarp();
+#pragma unroll 1
+    for (int i = lane; i < total; i += 32) {
+      const int b = cand[i];
+      const int n = min(64, Kin - 64 * b);
+      ev[b] = block_events(s_rt, (n == 64) ? 0 : 1, n, (uint32_t)b, (uint32_t)k, l, tt, key0, key1);
+    }
+    __syncwarp();
   }
 }
 
