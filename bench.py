@@ -48,11 +48,12 @@ SAMPLES_PER_STEP = 100_000
 STEPS_PER_EPOCH = 10
 EVAL_BATCH = 65_536
 
-# HBM traffic of k_update per launch from the committed ncu capture
-# (profiles/k_update_c5.md), valid while the kernel source hashes to
+# HBM traffic of one k_update launch of the timed region, from an ncu capture
+# of this bench (dram__bytes_read.sum + dram__bytes_write.sum, one pass; see
+# profiles/k_update_c5.md), valid while the kernel source hashes to
 # UPDATE_TRAFFIC_SRC_SHA; otherwise reported as null.
-UPDATE_TRAFFIC_BYTES = 537_796_608 + 509_770_240  # dram read + write, one launch (profiles/k_update_c5.md)
-UPDATE_TRAFFIC_SRC_SHA = "64595062a208f6c7"
+UPDATE_TRAFFIC_BYTES = 463_745_792 + 384_608_768  # dram read + write of one timed-region launch (ncu)
+UPDATE_TRAFFIC_SRC_SHA = "b7ea3673207a5b76"
 
 
 def bitpairs_per_sample(widths, classes):

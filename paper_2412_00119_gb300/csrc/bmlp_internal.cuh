@@ -99,7 +99,7 @@ struct StepParams {
 };
 
 constexpr int kUpdThreads = 256;
-constexpr int kClsThreads = 256;
+constexpr int kClsThreads = 512;
 
 // ---------------------------------------------------------------------------
 // Philox4x32-10 (Salmon, Moraes, Dror, Shaw, SC'11), device version.
