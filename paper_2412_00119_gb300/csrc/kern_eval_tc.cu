@@ -4,16 +4,17 @@
 // Same exact e4m3 formulation as the training forward (+-1 -> 0x38 / 0xB8,
 // pads 0, fp32 sums exact), tiled for large batches: a CTA computes 128
 // patterns x 256 neurons over the whole K range.
-//   - 16 producer warps expand bit-packed activations (128 rows) and visible
-//     weights (256 rows) into 128B-swizzled K-major stages of 48 KB: every
-//     thread owns six 16-byte chunks of the stage (16 bits each), loaded
-//     kPrefetch stages ahead;
+//   - 12 producer warps, one thread per stage row (128 activation rows, then
+//     256 weight rows): per 128-element k-block the thread loads the row's
+//     two bit words (one 16-byte load when the rows are 16-byte aligned),
+//     kPrefetch blocks ahead, and expands them into the row's eight 16-byte
+//     chunks of the 128B-swizzled K-major stage (48 KB, 4-stage ring);
 //   - 1 MMA warp issues tcgen05.mma.kind::f8f6f4 M128 N256 K32 (four per stage)
 //     into a 128 x 256 fp32 accumulator in TMEM (256 columns) and commits to
-//     the stage's "empty" mbarrier (4-stage ring);
-//   - the epilogue: warp w reads TMEM lanes 32 (w % 4) .., columns
-//     64 (w / 4) .. + 63, and writes the sign bits of each pattern as two
-//     32-bit halves of one packed word (pad bits 0).
+//     the stage's "empty" mbarrier;
+//   - the epilogue: the producer warps read TMEM (warp w: lanes 32 (w % 4) ..,
+//     column blocks w / 4, w / 4 + 3, ..) and write the sign bits of each
+//     pattern as 32-bit pieces of its packed row (pad bits 0).
 // Every mbarrier wait is bounded; the first expiry stops every other wait and
 // the kernel counts it in *timeouts, releases TMEM and returns.
 #include "tc_common.cuh"
@@ -26,15 +27,16 @@ using namespace tc;
 constexpr int TM = 128;
 constexpr int TN = 256;
 constexpr int kStages = 4;
-constexpr int kPrefetch = 3;
-constexpr int kProducers = 512;
-constexpr int kItems = 8 * (TM + TN) / kProducers;  // 16-byte chunks per producer thread
+constexpr int kPrefetch = 4;  // == kStages: the stage of k-block kb0 + d is d
+constexpr int kProducers = TM + TN;  // one stage row per producer thread
+constexpr int kProdWarps = kProducers / 32;
 constexpr int THREADS = kProducers + 32;
 constexpr int A_BYTES = TM * KB;   // 16 KB
 constexpr int B_BYTES = TN * KB;   // 32 KB
 constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
 constexpr int TMEM_COLS = 256;
 constexpr uint32_t kIdesc = idesc_f8(TM, TN);
+static_assert(kPrefetch == kStages, "stage index is the unrolled prefetch slot");
 
 struct __align__(8) EvShared {
   unsigned long long full[kStages];
@@ -46,6 +48,51 @@ struct __align__(8) EvShared {
 
 constexpr size_t kSmemBytes = 1024 + kStages * STAGE_BYTES + sizeof(EvShared);
 
+// Four K-elements, bits P .. P + 3 of x (P = 0 or 4), as four e4m3 bytes
+// (bit 1 -> 0x38 = +1, bit 0 -> 0xB8 = -1): the product places bit P + j at
+// bit 8 j + 7; its four shifted copies of the masked nibble do not overlap,
+// so it carries nothing.
+template <int P>
+__device__ __forceinline__ uint32_t e4m3_quad(uint32_t x) {
+  static_assert(P == 0 || P == 4, "nibble position");
+  constexpr uint32_t kMul = P == 0 ? 0x10204080u : 0x01020408u;
+  return ((x & (0xFu << P)) * kMul & 0x80808080u) ^ 0xB8B8B8B8u;
+}
+
+// The row's 128 K-elements of one k-block (four 32-bit words, element e =
+// bit e % 32 of word e / 32) -> its eight chunks; chunk c (elements 16 c ..
+// 16 c + 15) goes to physical chunk c ^ swz.  Elements at index >= valid are
+// written 0 (valid < 128 only in the last k-block of a ragged K).
+__device__ __forceinline__ void expand_row(uint8_t* row, int swz, uint4 w, int valid) {
+  const uint32_t x[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+  for (int c = 0; c < 8; ++c) {
+    const uint32_t h = x[c >> 1] >> (16 * (c & 1));
+    uint4 v = make_uint4(e4m3_quad<0>(h), e4m3_quad<4>(h), e4m3_quad<0>(h >> 8),
+                         e4m3_quad<4>(h >> 8));
+    if (valid < KB) {
+      const int n = valid - 16 * c;
+      v.x &= keep_mask(n);
+      v.y &= keep_mask(n - 4);
+      v.z &= keep_mask(n - 8);
+      v.w &= keep_mask(n - 12);
+    }
+    *reinterpret_cast<uint4*>(row + 16 * (c ^ swz)) = v;
+  }
+}
+
+// Bits of k-block kb of a row (words 2 kb, 2 kb + 1; 0 past the nw words).
+template <bool kVec>
+__device__ __forceinline__ uint4 load_block(const uint64_t* src, int kb, int nkb, int nw) {
+  if (src == nullptr || kb >= nkb) return make_uint4(0, 0, 0, 0);
+  if (kVec) return __ldg(reinterpret_cast<const uint4*>(src) + kb);
+  const uint64_t lo = __ldg(src + 2 * kb);
+  const uint64_t hi = 2 * kb + 1 < nw ? __ldg(src + 2 * kb + 1) : 0ull;
+  return make_uint4((uint32_t)lo, (uint32_t)(lo >> 32), (uint32_t)hi, (uint32_t)(hi >> 32));
+}
+
+// kVec: nw even and both operands 16-byte aligned (every row then is)
+template <bool kVec>
 __global__ void __launch_bounds__(THREADS, 1)
     k_forward_eval_tc(const uint64_t* __restrict__ A, int64_t M, int nw, const uint64_t* __restrict__ W,
                       int N, int Kin, uint64_t* __restrict__ Aout, int nw_out,
@@ -59,6 +106,7 @@ __global__ void __launch_bounds__(THREADS, 1)
   const int n0 = blockIdx.x * TN;
   const int NB = min(TN, N - n0);                 // neuron rows of this CTA
   const int nkb = (Kin + KB - 1) / KB;
+  const int tail = Kin - KB * (nkb - 1);          // valid elements of the last k-block
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   volatile int* failed = &sh->failed;
 
@@ -72,7 +120,7 @@ __global__ void __launch_bounds__(THREADS, 1)
   }
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
-      mbar_init(&sh->full[s], kProducers / 32);  // one arrival per producer warp
+      mbar_init(&sh->full[s], kProdWarps);  // one arrival per producer warp
       mbar_init(&sh->empty[s], 1);
     }
     mbar_init(&sh->done, 1);
@@ -91,46 +139,34 @@ __global__ void __launch_bounds__(THREADS, 1)
   const uint32_t tmem = sh->tmem_base;
 
   if (threadIdx.x < kProducers) {
-    // items: the 16-byte chunks of A rows [0, MR), then of B rows [0, NB);
-    // item i belongs to thread i % kProducers
-    const int nA = 8 * MR, nItems = nA + 8 * NB;
-    Chunk ch[kItems];
+    // this thread's stage row: activation row p (p < TM) or weight row p - TM
+    const int p = threadIdx.x;
+    const bool isA = p < TM;
+    const int r = isA ? p : p - TM;
+    const uint64_t* src = nullptr;
+    if (isA && r < MR) src = A + (m0 + r) * nw;
+    if (!isA && r < NB) src = W + (int64_t)(n0 + r) * nw;
+    const uint32_t row_off = (isA ? 0u : (uint32_t)A_BYTES) + (uint32_t)(r * KB);
+    const int swz = r & 7;
+
+    uint4 pre[kPrefetch];
 #pragma unroll
-    for (int j = 0; j < kItems; ++j) {
-      const int i = threadIdx.x + j * kProducers;
-      if (i < nA) {
-        ch[j] = make_chunk(A + (m0 + (i >> 3)) * nw, 0, i >> 3, i & 7);
-      } else if (i < nItems) {
-        const int b = i - nA;
-        ch[j] = make_chunk(W + (int64_t)(n0 + (b >> 3)) * nw, A_BYTES, b >> 3, b & 7);
-      } else {
-        ch[j] = Chunk{nullptr, 0u, 0};
-      }
-    }
-    uint32_t pre[kPrefetch][kItems];
-#pragma unroll
-    for (int d = 0; d < kPrefetch; ++d)
-#pragma unroll
-      for (int j = 0; j < kItems; ++j) pre[d][j] = load_chunk(ch[j], d, nw);
+    for (int d = 0; d < kPrefetch; ++d) pre[d] = load_block<kVec>(src, d, nkb, nw);
 
     for (int kb0 = 0; kb0 < nkb; kb0 += kPrefetch) {
 #pragma unroll
       for (int d = 0; d < kPrefetch; ++d) {
         const int kb = kb0 + d;
         if (kb >= nkb) break;
-        const int s = kb % kStages;
-        if (kb >= kStages &&
-            !__all_sync(kFull, mbar_wait(&sh->empty[s], (uint32_t)((kb / kStages - 1) & 1), failed)))
+        if (kb0 > 0 &&
+            !__all_sync(kFull, mbar_wait(&sh->empty[d], (uint32_t)((kb0 / kStages - 1) & 1), failed)))
           break;
-        uint8_t* stage = base + s * STAGE_BYTES;
-#pragma unroll
-        for (int j = 0; j < kItems; ++j) {
-          if (ch[j].src != nullptr) store_chunk(stage, ch[j], pre[d][j], kb, Kin);
-          pre[d][j] = load_chunk(ch[j], kb + kPrefetch, nw);
-        }
+        if (src != nullptr)
+          expand_row(base + d * STAGE_BYTES + row_off, swz, pre[d], kb == nkb - 1 ? tail : KB);
+        pre[d] = load_block<kVec>(src, kb + kPrefetch, nkb, nw);
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
         __syncwarp();
-        if (lane == 0) mbar_arrive(&sh->full[s]);
+        if (lane == 0) mbar_arrive(&sh->full[d]);
       }
       if (__any_sync(kFull, *failed != 0)) break;
     }
@@ -161,9 +197,8 @@ __global__ void __launch_bounds__(THREADS, 1)
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
     const int sub = warp & 3;
     const int m = 32 * sub + lane;
-#pragma unroll
-    for (int half = 0; half < 2; ++half) {
-      const int col0 = 64 * (warp >> 2) + 32 * half;
+    for (int cb = warp >> 2; cb < TN / 32; cb += kProdWarps / 4) {
+      const int col0 = 32 * cb;
       uint32_t v[32];
       asm volatile(
           "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
@@ -197,7 +232,10 @@ __global__ void __launch_bounds__(THREADS, 1)
 }  // namespace
 
 cudaError_t prepare_forward_eval_tc() {
-  return cudaFuncSetAttribute(k_forward_eval_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  cudaError_t e = cudaFuncSetAttribute(k_forward_eval_tc<true>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
+  if (e != cudaSuccess) return e;
+  return cudaFuncSetAttribute(k_forward_eval_tc<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                               (int)kSmemBytes);
 }
 
@@ -205,8 +243,14 @@ void launch_forward_eval_tc(const uint64_t* A, int64_t M, int nw_in, const uint6
                             int Kin, uint64_t* Aout, int nw_out, unsigned int* timeouts,
                             cudaStream_t st) {
   const dim3 grid((unsigned)((N + TN - 1) / TN), (unsigned)((M + TM - 1) / TM));
-  k_forward_eval_tc<<<grid, THREADS, kSmemBytes, st>>>(A, M, nw_in, W, N, Kin, Aout, nw_out,
-                                                      timeouts);
+  const bool vec = (nw_in % 2 == 0) && (reinterpret_cast<uintptr_t>(A) % 16 == 0) &&
+                   (reinterpret_cast<uintptr_t>(W) % 16 == 0);
+  if (vec)
+    k_forward_eval_tc<true><<<grid, THREADS, kSmemBytes, st>>>(A, M, nw_in, W, N, Kin, Aout,
+                                                                nw_out, timeouts);
+  else
+    k_forward_eval_tc<false><<<grid, THREADS, kSmemBytes, st>>>(A, M, nw_in, W, N, Kin, Aout,
+                                                                 nw_out, timeouts);
 }
 
 }  // namespace bk

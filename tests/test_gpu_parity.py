@@ -130,6 +130,25 @@ def test_layer_forward_eval(widths, n, engine):
     gpu.close()
 
 
+@pytest.mark.parametrize("widths,n", [((1100, 700), 300), ((8192, 512), 130)])
+def test_layer_forward_eval_8byte_aligned_input(widths, n):
+    """Input rows that start on an 8-byte (not 16-byte) boundary take the
+    word-by-word load path of the evaluation kernel; the bits are the same."""
+    gpu = B.BMLP(widths, 4, seed=9, bs=64, fwd_impl=B.BMLP_FWD_TCGEN05)
+    ref = O.OracleModel(list(widths), 4, seed=9, bs=64)
+    nw = W.words(widths[0])
+    xp = W.random_packed(77 + n, n, widths[0])
+    flat = torch.zeros(n * nw + 1, dtype=torch.int64, device=DEV)
+    flat[1:] = dev_x(xp).reshape(-1)
+    x = flat[1:].view(n, nw)
+    assert x.data_ptr() % 16 == 8
+    out = torch.full((n, W.words(widths[1])), -1, dtype=torch.int64, device=DEV)
+    B.bmlp_layer_forward(gpu.h, 1, x, out)
+    _, a = O.layer_forward(W.unpack(xp, widths[0]), ref.H(1))
+    assert np.array_equal(out.cpu().numpy().view(np.uint64), W.pack(a))
+    gpu.close()
+
+
 CASES = {
     "ragged_3layer": dict(widths=(200, 130, 70), classes=10, n_train=300, bs=50, gamma=[13, 7]),
     "tail_batch": dict(widths=(64, 64), classes=4, n_train=250),
