@@ -140,6 +140,12 @@ def _declare(L):
     L.or_train.restype = C.c_int
     L.or_predict.argtypes = [C.c_void_p, _i8p, C.c_int64, _i32p]
     L.or_predict.restype = C.c_int
+    L.or_predict_layers.argtypes = [C.c_void_p, _i8p, C.c_int64, _i32p]
+    L.or_predict_layers.restype = C.c_int
+    L.or_layer_errors.argtypes = [C.c_void_p, _i64p, C.c_int32]
+    L.or_layer_errors.restype = C.c_int
+    L.or_binarize_median.argtypes = [C.POINTER(C.c_float), C.c_int64, C.c_int32, _i8p]
+    L.or_binarize_median.restype = C.c_int
     L.or_num_layers.argtypes = [C.c_void_p]
     L.or_num_layers.restype = C.c_int32
     L.or_width.argtypes = [C.c_void_p, C.c_int32]
@@ -286,6 +292,17 @@ def perceptron_update(H, a_prev, y, P, sel, h_max, q, seed, l, t):
     return H
 
 
+def binarize_median(x):
+    """MedianBinarization (Alg. 1 l.5, O16): n x K fp32 -> n x K +-1 int8."""
+    x = _c(x, np.float32)
+    n, K = x.shape
+    a = np.zeros((n, K), np.int8)
+    rc = lib().or_binarize_median(x.ctypes.data_as(C.POINTER(C.c_float)), n, K, _p(a, _i8p))
+    if rc != 0:
+        raise ValueError("or_binarize_median failed: %d" % rc)
+    return a
+
+
 # -- the whole rule -------------------------------------------------------------
 
 class OracleModel:
@@ -337,6 +354,22 @@ class OracleModel:
         if rc != 0:
             raise ValueError("or_predict failed: %d" % rc)
         return out
+
+    def predict_layers(self, x):
+        """Early-exit predictions (O17): (L, n), row l-1 = argmax of a_l P_l."""
+        x = _c(x, np.int8)
+        n = x.shape[0]
+        out = np.zeros((self.L, n), np.int32)
+        rc = lib().or_predict_layers(self._h, _p(x, _i8p), n, _p(out, _i32p))
+        if rc != 0:
+            raise ValueError("or_predict_layers failed: %d" % rc)
+        return out
+
+    def layer_errors(self, reset=False):
+        """Local 01-loss counts of layers 1..L since creation or the last reset."""
+        out = np.zeros(self.L, np.int64)
+        lib().or_layer_errors(self._h, _p(out, _i64p), 1 if reset else 0)
+        return [int(v) for v in out]
 
     def gamma(self, l):
         return lib().or_gamma(self._h, l)

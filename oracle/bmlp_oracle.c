@@ -59,13 +59,25 @@
  *   O11 E^e = (# training patterns of the epoch whose last-layer 01-loss was 1 in
  *       the training forward pass) / (# patterns of the epoch); p_r <- p_r *
  *       sqrt(E^e) compounds over epochs (Alg. 1 l.21).
- *   O12 Inputs are already +-1, so MedianBinarization (Alg. 1 l.5) is the
- *       identity and is not applied.
+ *   O12 The training and evaluation entry points take inputs that are already
+ *       +-1, so MedianBinarization (Alg. 1 l.5) is the identity there; the
+ *       front end for real-valued patterns is a separate step (O16).
  *   O13 A last mini-batch shorter than bs is processed as a batch of its own
  *       size; the step counter t counts mini-batches since creation.
  *   O14 gamma rule of Sec. 4.3: among the divisors of K_l, the one whose distance
  *       to the interval [75, 105] is smallest; among equally distant divisors the
  *       largest (the paper's examples: 525 -> 105, 2025 -> 81).
+ *   O16 MedianBinarization of a real-valued pattern x in R^K (Alg. 1 l.5,
+ *       Sec. 3.2: the median value is the threshold): the median of the
+ *       pattern's own K values, taken as the lower median m = the
+ *       ceil(K/2)-th smallest; a_i = +1 iff x_i > m (strict, compared in
+ *       fp32), else -1.  With distinct values exactly floor(K/2) inputs are
+ *       +1; a constant pattern is all -1.
+ *   O17 Early exit (Sec. 3.1: the intermediate P_l may serve early-exit
+ *       strategies): the prediction of layer l is argmax_j of
+ *       yhat_l = a_l P_l, ties to the lowest class (O2); the local error
+ *       count of layer l is the number of training patterns whose 01-loss
+ *       l_l of Eq. 1 was 1 in their training forward pass.
  *
  * Philox stream layout (counter-based; Salmon, Moraes, Dror, Shaw, "Parallel
  * random numbers: as easy as 1, 2, 3", SC'11).  key = (seed mod 2^32,
@@ -373,6 +385,7 @@ typedef struct {
   int32_t* gamma;   /* gamma[1..L] */
   int64_t t;        /* mini-batches processed since creation */
   int64_t epoch_err, epoch_n;
+  int64_t* layer_err; /* layer_err[l]: local 01-loss count of layer l (O17) */
   int32_t** H;      /* H[l]: K[l-1] x K[l] */
   int8_t** P;       /* P[l]: K[l] x c */
 } or_model;
@@ -387,6 +400,7 @@ void or_destroy(or_model* m) {
   free(m->P);
   free(m->K);
   free(m->gamma);
+  free(m->layer_err);
   free(m);
 }
 
@@ -413,7 +427,8 @@ int or_create(const int32_t* widths, int32_t n_widths, int32_t classes, int32_t 
   m->gamma = (int32_t*)calloc((size_t)n_widths, sizeof(int32_t));
   m->H = (int32_t**)calloc((size_t)n_widths, sizeof(int32_t*));
   m->P = (int8_t**)calloc((size_t)n_widths, sizeof(int8_t*));
-  if (!m->K || !m->gamma || !m->H || !m->P) {
+  m->layer_err = (int64_t*)calloc((size_t)n_widths, sizeof(int64_t));
+  if (!m->K || !m->gamma || !m->H || !m->P || !m->layer_err) {
     or_destroy(m);
     return OR_ENOMEM;
   }
@@ -486,6 +501,7 @@ int or_train(or_model* m, const int8_t* x, const int32_t* y, int64_t n, int32_t 
       or_layer_forward(a[l - 1], b, m->K[l - 1], m->H[l], m->K[l], z[l], a[l]);
       or_local_output(a[l], b, m->K[l], m->P[l], c, yhat);
       or_local_loss(yhat, b, c, yb, m->K[l], m->r_num, m->r_den, NULL, ell, NULL, mark[l]);
+      for (int32_t mu = 0; mu < b; mu++) m->layer_err[l] += ell[mu]; /* O17 */
       if (l == L)
         for (int32_t mu = 0; mu < b; mu++) n_err += ell[mu];
     }
@@ -562,6 +578,83 @@ int or_predict(const or_model* m, const int8_t* x, int64_t n, int32_t* pred) {
   free(a1);
   free(z);
   free(yhat);
+  return rc;
+}
+
+/* Early-exit evaluation (Sec. 3.1, O17): pred[(l-1) n + mu] = argmax_j of
+ * a_l P_l for pattern mu, every layer l = 1..L. */
+int or_predict_layers(const or_model* m, const int8_t* x, int64_t n, int32_t* pred) {
+  if (!m || n < 0 || (n > 0 && (!x || !pred))) return OR_EINVAL;
+  const int32_t L = m->L, c = m->c;
+  int32_t Kmax = 0;
+  for (int32_t l = 0; l <= L; l++)
+    if (m->K[l] > Kmax) Kmax = m->K[l];
+  const int32_t chunk = 256;
+  int8_t* a0 = (int8_t*)malloc((size_t)chunk * (size_t)Kmax);
+  int8_t* a1 = (int8_t*)malloc((size_t)chunk * (size_t)Kmax);
+  int32_t* z = (int32_t*)malloc(sizeof(int32_t) * (size_t)chunk * (size_t)Kmax);
+  int32_t* yhat = (int32_t*)malloc(sizeof(int32_t) * (size_t)chunk * (size_t)c);
+  int rc = (a0 && a1 && z && yhat) ? OR_OK : OR_ENOMEM;
+  for (int64_t start = 0; rc == OR_OK && start < n; start += chunk) {
+    const int32_t b = (int32_t)((n - start) < chunk ? (n - start) : chunk);
+    const int8_t* in = x + start * m->K[0];
+    int8_t* cur = a0;
+    for (int32_t l = 1; l <= L; l++) {
+      or_layer_forward(in, b, m->K[l - 1], m->H[l], m->K[l], z, cur);
+      or_local_output(cur, b, m->K[l], m->P[l], c, yhat);
+      for (int32_t mu = 0; mu < b; mu++) {
+        int32_t jmax = 0;
+        for (int32_t j = 1; j < c; j++)
+          if (yhat[(int64_t)mu * c + j] > yhat[(int64_t)mu * c + jmax]) jmax = j;
+        pred[(int64_t)(l - 1) * n + start + mu] = jmax;
+      }
+      in = cur;
+      cur = (cur == a0) ? a1 : a0;
+    }
+  }
+  free(a0);
+  free(a1);
+  free(z);
+  free(yhat);
+  return rc;
+}
+
+/* Local 01-loss counts of every layer since creation or the last reset (O17):
+ * out[l-1] for l = 1..L. */
+int or_layer_errors(or_model* m, int64_t* out, int32_t reset) {
+  if (!m || !out) return OR_EINVAL;
+  for (int32_t l = 1; l <= m->L; l++) {
+    out[l - 1] = m->layer_err[l];
+    if (reset) m->layer_err[l] = 0;
+  }
+  return OR_OK;
+}
+
+static int or_cmp_float(const void* pa, const void* pb) {
+  const float a = *(const float*)pa, b = *(const float*)pb;
+  return (a < b) ? -1 : (a > b) ? 1 : 0;
+}
+
+/* MedianBinarization (Alg. 1 l.5, O16): x is n x K fp32 (finite), a is n x K
+ * +-1.  Each pattern is sorted (library sort) to find its lower median. */
+int or_binarize_median(const float* x, int64_t n, int32_t K, int8_t* a) {
+  if (n < 0 || K < 1 || (n > 0 && (!x || !a))) return OR_EINVAL;
+  int rc = OR_OK;
+#pragma omp parallel for schedule(static)
+  for (int64_t mu = 0; mu < n; mu++) {
+    float* s = (float*)malloc(sizeof(float) * (size_t)K);
+    if (!s) {
+#pragma omp atomic write
+      rc = OR_ENOMEM;
+      continue;
+    }
+    const float* row = x + mu * K;
+    memcpy(s, row, sizeof(float) * (size_t)K);
+    qsort(s, (size_t)K, sizeof(float), or_cmp_float);
+    const float med = s[(K + 1) / 2 - 1];
+    for (int32_t i = 0; i < K; i++) a[mu * K + i] = (int8_t)(row[i] > med ? 1 : -1);
+    free(s);
+  }
   return rc;
 }
 

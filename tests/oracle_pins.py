@@ -15,7 +15,10 @@ Sources of the expected values:
     rate, pair independence, per-block binomial counts), a binomial bound on
     the reinforcement rate, and the closed form of Alg. 1 l.21;
   * invariants of Alg. 3 (odd h, |h| <= h_max, one lattice unit per event,
-    reinforcement moves away from 0) and the learnability of a separable task.
+    reinforcement moves away from 0) and the learnability of a separable task;
+  * the rank form of the lower median (brute force), the truncated network
+    for early-exit predictions, and the evaluation path for the local error
+    counts.
 """
 from __future__ import annotations
 
@@ -446,6 +449,67 @@ def check_resume_equivalence(seed=8):
     assert a.step == b.step == c.step == 6
 
 
+# -- front end and early exit (O16, O17) -----------------------------------------
+
+def check_binarize_median_rank(seed=9):
+    """MedianBinarization (O16) against its rank form: x_i > m, m the
+    ceil(K/2)-th smallest value, holds iff at least ceil(K/2) values of the
+    pattern are strictly below x_i.  Exhaustive over small K with many ties,
+    negative values and signed zeros; distinct values give floor(K/2) ones; a
+    constant pattern gives none."""
+    rng = np.random.default_rng(seed)
+    for K in range(1, 12):
+        pool = np.array([-2.0, -1.0, -0.0, 0.0, 0.5, 1.0, 3.0], np.float32)
+        x = pool[rng.integers(0, len(pool), (200, K))]
+        a = O.binarize_median(x)
+        below = (x[:, None, :] < x[:, :, None]).sum(axis=2)   # below[mu, i] = #{j: x_j < x_i}
+        want = np.where(below >= (K + 1) // 2, 1, -1)
+        assert np.array_equal(a, want), K
+        d = np.stack([rng.permutation(K) for _ in range(20)]).astype(np.float32) - K / 3.0
+        assert np.all((O.binarize_median(d) == 1).sum(axis=1) == K // 2), K
+        assert np.all(O.binarize_median(np.full((3, K), 1.5, np.float32)) == -1)
+
+
+def check_early_exit_truncation(seed=10):
+    """The early-exit prediction of layer l (O17) is the prediction of the same
+    network cut after layer l: H_1..H_l and P_l depend only on (seed, l), so
+    the truncated model is that network."""
+    rng = np.random.default_rng(seed)
+    widths, c = [40, 24, 16, 12], 5
+    x, y = _bias_data(rng, 90, widths[0], c)
+    full = O.OracleModel(widths, c, seed=3, bs=30, gamma=[4, 4, 4])
+    full.train(x[:60], y[:60])
+    pl = full.predict_layers(x)
+    assert pl.shape == (3, 90)
+    assert np.array_equal(pl[-1], full.predict(x))
+    for l in (1, 2):
+        cut = O.OracleModel(widths[:l + 1], c, seed=3, bs=30, gamma=[4] * l)
+        for j in range(1, l + 1):
+            cut.set_H(j, full.H(j))
+        assert np.array_equal(cut.predict(x), pl[l - 1]), l
+
+
+def check_layer_errors_match_eval(seed=11):
+    """The local 01-loss count of layer l (O17) adds up, mini-batch by
+    mini-batch, the patterns whose layer-l early-exit prediction with that
+    mini-batch's pre-update weights differs from the label; the last layer's
+    count is the train call's error count."""
+    rng = np.random.default_rng(seed)
+    widths, c, bs = [36, 20, 16], 4, 25
+    x, y = _bias_data(rng, 100, widths[0], c)
+    m = O.OracleModel(widths, c, seed=6, bs=bs, gamma=[4, 4])
+    want = np.zeros(2, np.int64)
+    last = 0
+    for s0 in range(0, 100, bs):
+        pl = m.predict_layers(x[s0:s0 + bs])
+        want += (pl != y[s0:s0 + bs][None, :]).sum(axis=1)
+        last += m.train(x[s0:s0 + bs], y[s0:s0 + bs])
+    got = m.layer_errors(reset=True)
+    assert got == [int(v) for v in want], (got, want)
+    assert got[-1] == last
+    assert m.layer_errors() == [0, 0]
+
+
 ALL_CHECKS = [
     check_philox_kat,
     check_gamma_golden,
@@ -466,4 +530,7 @@ ALL_CHECKS = [
     check_epoch_end_pr,
     check_learnable,
     check_resume_equivalence,
+    check_binarize_median_rank,
+    check_early_exit_truncation,
+    check_layer_errors_match_eval,
 ]

@@ -46,6 +46,12 @@ MUTANTS = [
     ("update_without_marks", "if (!any) continue; /* O6 */", "(void)any;"),
     ("gamma_ties_small", "(dist == best_dist && g > best)", "(dist == best_dist && g < best)"),
     ("pr_without_sqrt", "m->p_r = m->p_r * sqrt(E);", "m->p_r = m->p_r * E;"),
+    ("binarize_upper_median", "const float med = s[(K + 1) / 2 - 1];", "const float med = s[K / 2];"),
+    ("binarize_not_strict", "a[mu * K + i] = (int8_t)(row[i] > med ? 1 : -1);",
+     "a[mu * K + i] = (int8_t)(row[i] >= med ? 1 : -1);"),
+    ("early_exit_layers_reversed", "pred[(int64_t)(l - 1) * n + start + mu] = jmax;",
+     "pred[(int64_t)(L - l) * n + start + mu] = jmax;"),
+    ("layer_errors_count_marks", "m->layer_err[l] += ell[mu]; /* O17 */", "m->layer_err[l] += mark[l][mu];"),
     ("forward_drops_sign", "zr[k] += ai * (hrow[k] > 0 ? 1 : -1);", "zr[k] += ai * hrow[k];"),
 ]
 
