@@ -126,6 +126,41 @@ int bmlp_train(bmlp_t* h, const uint64_t* x_packed, const int32_t* labels, int64
 int bmlp_predict(bmlp_t* h, const uint64_t* x_packed, int64_t n, int32_t* labels_out,
                  void* cuda_stream);
 
+/* Early-exit evaluation (Sec. 3.1: after training, the intermediate random
+ * classifiers P_l may serve early-exit strategies).  For every layer
+ * l = 1..L: labels_out[(l-1) n + mu] = argmax_j of yhat_l = a_l P_l for
+ * pattern mu (ties to the lowest class), a_l from the same forward pass as
+ * bmlp_predict; row L equals bmlp_predict's output.  x_packed: as for
+ * bmlp_predict; labels_out: L x n int32, layer-major, caller-owned, host or
+ * device.  Asynchronous on cuda_stream when both pointers are device
+ * pointers; synchronises otherwise.  Errors as bmlp_predict. */
+int bmlp_predict_layers(bmlp_t* h, const uint64_t* x_packed, int64_t n, int32_t* labels_out,
+                        void* cuda_stream);
+
+/* Local error counts (Eq. 1 for every layer, Alg. 1 l.12): errs_out[l-1] =
+ * the number of training patterns whose layer-l local 01-loss was 1 in their
+ * training forward pass (the weights of their mini-batch before its update),
+ * counted since creation or the last reset; errs_out[L-1] counts what
+ * bmlp_train's n_errors_out reports.  errs_out: host, L values.  Synchronises
+ * the device; reset != 0 sets the counters to 0 after reading them.  The
+ * counters are not part of the state that bmlp_get_state / bmlp_set_state
+ * carry. */
+int bmlp_layer_errors(bmlp_t* h, int64_t* errs_out, int32_t reset);
+
+/* MedianBinarization (Alg. 1 l.5; Sec. 3.2: the median value is the
+ * threshold) of real-valued patterns, for data that is not already +-1:
+ * bit i of pattern mu is 1 (+1) iff x[mu][i] > m_mu, where m_mu is the
+ * ceil(K/2)-th smallest of the pattern's K values (its lower median) and the
+ * comparison is made in fp32 (-0 and +0 are equal); else 0 (-1).  Pad bits
+ * are 0, so the output is bmlp_train / bmlp_predict input for K_0 = K.
+ *   x: device, n x K fp32, row-major, 4-byte aligned, finite values (a NaN
+ *      ranks by its bit pattern and compares false); caller-owned.
+ *   out: device, n x ceil(K/64) words, 8-byte aligned, caller-owned.
+ * Needs no handle (errors read with bmlp_last_error(NULL)); asynchronous on
+ * cuda_stream.  BMLP_EINVAL for n < 0, K < 1, NULL, host or misaligned
+ * pointers; BMLP_ECUDA if the launch fails. */
+int bmlp_binarize_median(const float* x, int64_t n, int32_t K, uint64_t* out, void* cuda_stream);
+
 /* One layer of forward-only evaluation (Sec. 3.1; Alg. 1 l.8-9):
  * a_out = sign(a_in W_l), sign(0) = +1, for n packed rows.  a_in: n rows of
  * ceil(K_{l-1}/64) words (pad bits 0); a_out: n rows of ceil(K_l/64) words,

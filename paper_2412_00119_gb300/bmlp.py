@@ -74,6 +74,9 @@ SIGNATURES = [
     ("bmlp_predict_noalloc", C.c_int, [_vp, _vp, C.c_int64, _vp, _vp]),
     ("bmlp_layer_forward", C.c_int, [_vp, C.c_int32, _vp, C.c_int64, _vp, _vp]),
     ("bmlp_update_stats", C.c_int, [_vp, _vp, _vp, _vp, C.c_int32]),
+    ("bmlp_predict_layers", C.c_int, [_vp, _vp, C.c_int64, _vp, _vp]),
+    ("bmlp_layer_errors", C.c_int, [_vp, _i64p, C.c_int32]),
+    ("bmlp_binarize_median", C.c_int, [_vp, C.c_int64, C.c_int32, _vp, _vp]),
 ]
 
 
@@ -176,6 +179,27 @@ def bmlp_predict_noalloc(h, x_packed, labels_out, n=None, stream=None):
     memory (device buffers only; n * ceil(max K_l / 64) <= 2^20)."""
     n = labels_out.shape[0] if n is None else n
     _check(lib().bmlp_predict_noalloc(h, _ptr(x_packed), n, _ptr(labels_out), _stream(stream)), h)
+
+
+def bmlp_predict_layers(h, x_packed, labels_out, n=None, stream=None):
+    """Early-exit predictions of every layer into labels_out (L x n, layer-major)."""
+    n = labels_out.shape[-1] if n is None else n
+    _check(lib().bmlp_predict_layers(h, _ptr(x_packed), n, _ptr(labels_out), _stream(stream)), h)
+
+
+def bmlp_layer_errors(h, reset=False):
+    """Local 01-loss counts of layers 1..L since creation or the last reset."""
+    L = C.c_int32()
+    lib().bmlp_get_info(h, C.byref(L), None, None, None, None, None)
+    out = (C.c_int64 * L.value)()
+    _check(lib().bmlp_layer_errors(h, out, 1 if reset else 0), h)
+    return [int(v) for v in out]
+
+
+def bmlp_binarize_median(x, out, stream=None):
+    """Median binarisation of n x K fp32 patterns (device) into packed bits."""
+    n, K = x.shape
+    _check(lib().bmlp_binarize_median(_ptr(x), n, K, _ptr(out), _stream(stream)), None)
 
 
 def bmlp_layer_forward(h, layer, a_in, a_out, n=None, stream=None):
@@ -302,6 +326,12 @@ class BMLP:
 
     def predict(self, x_packed, labels_out, stream=None, n=None):
         bmlp_predict(self.h, x_packed, labels_out, n, stream)
+
+    def predict_layers(self, x_packed, labels_out, stream=None, n=None):
+        bmlp_predict_layers(self.h, x_packed, labels_out, n, stream)
+
+    def layer_errors(self, reset=False):
+        return bmlp_layer_errors(self.h, reset)
 
     def state(self, layer):
         return bmlp_get_state(self.h, layer)

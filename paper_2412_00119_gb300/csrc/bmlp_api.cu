@@ -589,7 +589,13 @@ int bmlp_train(bmlp_t* h, const uint64_t* x, const int32_t* labels, int64_t n, u
   return prof_collect(h, st);
 }
 
-int bmlp_predict(bmlp_t* h, const uint64_t* x, int64_t n, int32_t* out, void* cuda_stream) {
+namespace {
+
+// Forward-only evaluation of n patterns (Sec. 3.1).  every_layer: the argmax of
+// a_l P_l of every layer l into out[(l-1) n + mu] (early exit); else of the
+// last layer only into out[mu].
+int predict_impl(bmlp_t* h, const uint64_t* x, int64_t n, int32_t* out, void* cuda_stream,
+                 bool every_layer) {
   if (!h) return BMLP_EINVAL;
   h->err.clear();
   if (n < 0) return fail(h, BMLP_EINVAL, "n < 0");
@@ -624,19 +630,22 @@ int bmlp_predict(bmlp_t* h, const uint64_t* x, int64_t n, int32_t* out, void* cu
       prof_end(h, st);
       in = h->evA[cur];
       cur ^= 1;
-    }
-    const DevLayer& DL = h->hp.layer[h->L - 1];
-    int32_t* o = odev ? out + s0 : h->stOut;
-    prof_begin(h, kProfOut, st);
-    k_predict_out<<<(unsigned)((m + 7) / 8), 256, 0, st>>>(in, m, DL.nw_out, DL.PT, h->c, DL.Kout, o);
-    prof_end(h, st);
-    CK(h, cudaGetLastError());
-    h->launches += h->L + 1;
-    if (!odev) {
-      prof_begin(h, kProfCopy, st);
-      CK(h, cudaMemcpyAsync(out + s0, h->stOut, sizeof(int32_t) * m, cudaMemcpyDeviceToHost, st));
+      if (!every_layer && l < h->L) continue;
+      // argmax of a_l P_l (lowest class on ties)
+      int32_t* dst = out + (every_layer ? (int64_t)(l - 1) * n : 0) + s0;
+      int32_t* o = odev ? dst : h->stOut;
+      prof_begin(h, kProfOut, st);
+      k_predict_out<<<(unsigned)((m + 7) / 8), 256, 0, st>>>(in, m, D.nw_out, D.PT, h->c, D.Kout, o);
       prof_end(h, st);
+      CK(h, cudaGetLastError());
+      h->launches += 1;
+      if (!odev) {
+        prof_begin(h, kProfCopy, st);
+        CK(h, cudaMemcpyAsync(dst, h->stOut, sizeof(int32_t) * m, cudaMemcpyDeviceToHost, st));
+        prof_end(h, st);
+      }
     }
+    h->launches += h->L;
   }
   if (!odev) {
     if (h->fwd_impl == BMLP_FWD_TCGEN05)
@@ -650,6 +659,44 @@ int bmlp_predict(bmlp_t* h, const uint64_t* x, int64_t n, int32_t* out, void* cu
     }
   }
   return prof_collect(h, st);
+}
+
+}  // namespace
+
+int bmlp_predict(bmlp_t* h, const uint64_t* x, int64_t n, int32_t* out, void* cuda_stream) {
+  return predict_impl(h, x, n, out, cuda_stream, false);
+}
+
+int bmlp_predict_layers(bmlp_t* h, const uint64_t* x, int64_t n, int32_t* out, void* cuda_stream) {
+  return predict_impl(h, x, n, out, cuda_stream, true);
+}
+
+int bmlp_layer_errors(bmlp_t* h, int64_t* errs_out, int32_t reset) {
+  if (!h) return BMLP_EINVAL;
+  h->err.clear();
+  if (!errs_out) return fail(h, BMLP_EINVAL, "errs_out is NULL");
+  CK(h, cudaDeviceSynchronize());
+  unsigned long long v[BMLP_MAX_LAYERS];
+  CK(h, cudaMemcpy(v, h->dCtrl->layer_err, sizeof(unsigned long long) * h->L, cudaMemcpyDeviceToHost));
+  for (int l = 0; l < h->L; ++l) errs_out[l] = (int64_t)v[l];
+  if (reset) {
+    CK(h, cudaMemset(h->dCtrl->layer_err, 0, sizeof(unsigned long long) * h->L));
+    CK(h, cudaDeviceSynchronize());
+  }
+  return BMLP_OK;
+}
+
+int bmlp_binarize_median(const float* x, int64_t n, int32_t K, uint64_t* out, void* cuda_stream) {
+  if (n < 0 || K < 1) return fail(nullptr, BMLP_EINVAL, "bmlp_binarize_median: n < 0 or K < 1");
+  if (n == 0) return BMLP_OK;
+  if (!x || !out || !is_device_ptr(x) || !is_device_ptr(out))
+    return fail(nullptr, BMLP_EINVAL, "bmlp_binarize_median: x and out must be device pointers");
+  if ((reinterpret_cast<uintptr_t>(x) & 3) || (reinterpret_cast<uintptr_t>(out) & 7))
+    return fail(nullptr, BMLP_EINVAL, "bmlp_binarize_median: misaligned x or out");
+  launch_binarize_median(x, n, K, (K + 63) / 64, out, static_cast<cudaStream_t>(cuda_stream));
+  const cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_fail(nullptr, e, "k_binarize_median");
+  return BMLP_OK;
 }
 
 int bmlp_get_state(const bmlp_t* hc, int32_t layer, int16_t* H_out, uint64_t* W_out, int8_t* P_out,

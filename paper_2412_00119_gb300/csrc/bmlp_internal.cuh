@@ -68,6 +68,7 @@ struct Ctrl {
   unsigned long long upd_streamed;   // rows streamed (at least one CP tuple)
   unsigned long long upd_bytes;      // algorithmic bytes: H read + write and W write of the
                                      // streamed rows, int16 read + write per sparse event
+  unsigned long long layer_err[BMLP_MAX_LAYERS];  // local 01-loss count of each layer
 };
 
 // Thresholds of the reinforcement sampler of one layer (Alg. 3 l.5-12): the
@@ -188,6 +189,8 @@ size_t act_tile_bytes(int K);  // bytes of an AE image for K activations
 // Tensor-core forward for evaluation: A (M x nw_in) against W -> Aout
 // (M x nw_out), 128-pattern x 256-neuron tiles; an expired bounded wait adds
 // one to *timeouts.
+void launch_binarize_median(const float* x, int64_t n, int K, int nw, uint64_t* out,
+                            cudaStream_t st);
 cudaError_t prepare_forward_eval_tc();
 void launch_forward_eval_tc(const uint64_t* A, int64_t M, int nw_in, const uint64_t* W, int N,
                             int Kin, uint64_t* Aout, int nw_out, unsigned int* timeouts,

@@ -73,6 +73,7 @@ __global__ void __launch_bounds__(kClsThreads) k_cls_select(const StepParams* __
     const int mark = loss || ((long long)tau * P->r_den < (long long)P->r_num * Ly.Kout);
     Ly.mark[mu] = (uint8_t)mark;
     if (mark) atomicOr(&ctrl->any_mark[li], 1u);
+    if (loss) atomicAdd(&ctrl->layer_err[li], 1ull);
     if (li == P->L - 1 && loss) atomicAdd(&ctrl->err, 1ull);
     s_mark = mark;
     s_y = yv;

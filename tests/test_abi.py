@@ -79,8 +79,22 @@ def test_create_without_gpu_reports_no_device():
     assert ei.value.code == B.BMLP_ENODEV
 
 
+def test_binarize_rejects_bad_arguments():
+    lib = pkg.lib()
+    assert lib.bmlp_binarize_median(None, -1, 8, None, None) == B.BMLP_EINVAL
+    assert b"n < 0" in lib.bmlp_last_error(None)
+    assert lib.bmlp_binarize_median(None, 4, 0, None, None) == B.BMLP_EINVAL
+    assert lib.bmlp_binarize_median(None, 0, 8, None, None) == B.BMLP_OK
+    x = np.zeros((4, 8), np.float32)
+    out = np.zeros((4, 1), np.uint64)
+    assert lib.bmlp_binarize_median(x.ctypes.data, 4, 8, out.ctypes.data, None) == B.BMLP_EINVAL
+    assert b"device pointers" in lib.bmlp_last_error(None)
+
+
 def test_null_handle_calls_fail_cleanly():
     lib = pkg.lib()
+    assert lib.bmlp_predict_layers(None, None, 0, None, None) == B.BMLP_EINVAL
+    assert lib.bmlp_layer_errors(None, None, 0) == B.BMLP_EINVAL
     assert lib.bmlp_train(None, None, None, 0, 0, None, None) == B.BMLP_EINVAL
     assert lib.bmlp_predict(None, None, 0, None, None) == B.BMLP_EINVAL
     assert lib.bmlp_get_state(None, 1, None, None, None, None, None) == B.BMLP_EINVAL

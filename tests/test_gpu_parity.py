@@ -149,6 +149,40 @@ def test_layer_forward_eval_8byte_aligned_input(widths, n):
     gpu.close()
 
 
+@pytest.mark.parametrize("n,K,kind", [(1, 1, "gauss"), (7, 63, "ties"), (33, 64, "ties"),
+                                       (100, 784, "pixels"), (5, 3072, "gauss"), (3, 8193, "pixels"),
+                                       (2000, 100, "ties")])
+def test_binarize_median_matches_oracle(n, K, kind):
+    """MedianBinarization (Alg. 1 l.5): every packed bit, pads 0, equals the
+    oracle's lower-median threshold with a strict comparison."""
+    x = W.real_patterns(31 + K, n, K, kind)
+    out = torch.full((n, W.words(K)), -1, dtype=torch.int64, device=DEV)
+    B.bmlp_binarize_median(torch.from_numpy(x).to(DEV), out)
+    want = W.pack(O.binarize_median(x))
+    assert np.array_equal(out.cpu().numpy().view(np.uint64), want)
+
+
+@pytest.mark.parametrize("engine", sorted(ENGINES))
+def test_early_exit_and_layer_errors(engine):
+    """Early-exit predictions of every layer (Sec. 3.1) and the local 01-loss
+    counts of every layer equal the oracle's, device and host buffers."""
+    gpu, ref = run_pair(widths=(200, 130, 96, 70), classes=10, n_train=400, n_test=0, bs=50,
+                        gamma=[13, 8, 7], fwd=ENGINES[engine])
+    assert gpu.layer_errors() == ref.layer_errors()
+    assert gpu.layer_errors(reset=True)[-1] == ref.layer_errors()[-1]
+    assert gpu.layer_errors() == [0, 0, 0]
+    cfg = W.small_config((200, 130, 96, 70), 10, 400, 300)
+    te = W.make_split(cfg, "test")
+    want = ref.predict_layers(te.pm1())
+    o = torch.full((3, 300), -7, dtype=torch.int32, device=DEV)
+    gpu.predict_layers(dev_x(te.xp), o)
+    assert np.array_equal(o.cpu().numpy(), want)
+    host = np.full((3, 300), -7, np.int32)
+    gpu.predict_layers(te.xp, host)
+    assert np.array_equal(host, want)
+    gpu.close()
+
+
 CASES = {
     "ragged_3layer": dict(widths=(200, 130, 70), classes=10, n_train=300, bs=50, gamma=[13, 7]),
     "tail_batch": dict(widths=(64, 64), classes=4, n_train=250),

@@ -129,6 +129,23 @@ def random_packed(seed: int, n: int, K: int) -> np.ndarray:
     return _iid_packed(np.random.default_rng(seed), n, K)
 
 
+def real_patterns(seed: int, n: int, K: int, kind: str = "pixels") -> np.ndarray:
+    """n x K fp32 real-valued patterns for the median-binarisation front end:
+    "pixels" = integer intensities 0..255 with about 60 % zeros (an image-like
+    mix with many ties), "gauss" = N(0, 1), "ties" = a pool of seven values
+    including -0.0 and +0.0."""
+    rng = np.random.default_rng(seed)
+    if kind == "pixels":
+        v = rng.integers(1, 256, (n, K)).astype(np.float32)
+        return np.where(rng.random((n, K)) < 0.6, np.float32(0), v).astype(np.float32)
+    if kind == "gauss":
+        return rng.standard_normal((n, K)).astype(np.float32)
+    if kind == "ties":
+        pool = np.array([-2.0, -1.0, -0.0, 0.0, 0.5, 1.0, 3.0], np.float32)
+        return pool[rng.integers(0, len(pool), (n, K))]
+    raise ValueError(kind)
+
+
 # -- teacher -------------------------------------------------------------------
 
 @dataclasses.dataclass
