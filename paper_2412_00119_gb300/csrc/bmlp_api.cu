@@ -51,7 +51,8 @@ struct bmlp {
   int64_t stCap = 0;
   unsigned long long* hostPinned = nullptr;  // [4] D2H landing zone
   // graph of one training step
-  cudaGraphExec_t stepExec = nullptr;
+  cudaGraphExec_t stepExec = nullptr;   // one mini-batch step
+  cudaGraphExec_t multiExec = nullptr;  // kGraphSteps consecutive steps
   cudaStream_t capStream = nullptr;
   cudaStream_t sideStream = nullptr;  // the event-draw branch of the step graph
   cudaEvent_t evFork = nullptr, evJoin = nullptr;
@@ -197,7 +198,14 @@ int prof_collect(bmlp_t* h, cudaStream_t st) {
 // (graph capture) their kernel runs on a side stream next to the forward
 // passes, which leave most of every SM idle, and joins before the update;
 // otherwise it runs first on `st`.
-int enqueue_step(bmlp_t* h, cudaStream_t st, bool fork) {
+// Mini-batch steps per captured training graph (a shorter run, or one that
+// has sampled steps in the way, uses the one-step graph).
+constexpr int kGraphSteps = 8;
+
+// One mini-batch step.  fork: the graph form (event draws on a branch,
+// programmatic dependent launches); chained: the step follows another step in
+// the same graph, so its first forward is a dependent of that step's update.
+int enqueue_step(bmlp_t* h, cudaStream_t st, bool fork, bool chained = false) {
   if (!fork) {
     prof_begin(h, kProfEvents, st);
     launch_r_events((unsigned)h->hp.ev_ctas_total, st, h->dP, h->hp.key0, h->hp.key1);
@@ -214,13 +222,17 @@ int enqueue_step(bmlp_t* h, cudaStream_t st, bool fork) {
     }
     prof_begin(h, kProfTrainFwd, st);
     if (h->fwd_impl == BMLP_FWD_TCGEN05)
-      launch_train_forward_tc(l > 1, h->K[l], st, h->dP, l);
+      CK(h, launch_train_forward_tc(l > 1, h->K[l], st, fork && (l > 1 || chained), h->dP, l));
     else
       k_train_forward<<<train_forward_grid(h->bs, h->K[l]), train_forward_block(), 0, st>>>(h->dP, l);
     prof_end(h, st);
   }
   prof_begin(h, kProfCls, st);
-  k_cls_select<<<dim3((unsigned)h->bs, (unsigned)h->L), kClsThreads, 0, st>>>(h->dP);
+  // inside the step graph each kernel after the first is launched as a
+  // programmatic dependent of the one before it (launch and prologue overlap
+  // the previous kernel's tail); the event-draw branch joins with a full edge
+  CK(h, launch_kernel(k_cls_select, dim3((unsigned)h->bs, (unsigned)h->L), dim3(kClsThreads), 0, st,
+                      fork && h->fwd_impl == BMLP_FWD_TCGEN05, h->dP));
   prof_end(h, st);
   if (fork && h->L == 1) {
     CK(h, cudaEventRecord(h->evFork, st));
@@ -230,15 +242,36 @@ int enqueue_step(bmlp_t* h, cudaStream_t st, bool fork) {
   }
   if (fork) CK(h, cudaStreamWaitEvent(st, h->evJoin, 0));
   prof_begin(h, kProfUpd, st);
-  launch_update(update_hb_mode(h->h_max, h->hp.hb), (unsigned)h->updCtas, h->updSmem, st, h->dP,
-                h->hp.key0, h->hp.key1);
+  CK(h, launch_update(update_hb_mode(h->h_max, h->hp.hb), (unsigned)h->updCtas, h->updSmem, st, fork,
+                      h->dP, h->hp.key0, h->hp.key1));
   prof_end(h, st);
   CK(h, cudaGetLastError());
   return BMLP_OK;
 }
 
+// Capture `steps` consecutive mini-batch steps into one executable graph.
+int capture_steps(bmlp_t* h, int steps, cudaGraphExec_t* exec) {
+  cudaGraph_t g = nullptr;
+  CK(h, cudaStreamBeginCapture(h->capStream, cudaStreamCaptureModeThreadLocal));
+  const bool prof = h->profiling;
+  h->profiling = false;
+  int rc = BMLP_OK;
+  for (int i = 0; i < steps && rc == BMLP_OK; ++i) rc = enqueue_step(h, h->capStream, true, i > 0);
+  h->profiling = prof;
+  cudaError_t e = cudaStreamEndCapture(h->capStream, &g);
+  if (rc != BMLP_OK) {
+    if (g) cudaGraphDestroy(g);
+    return rc;
+  }
+  if (e != cudaSuccess) return cuda_fail(h, e, "cudaStreamEndCapture");
+  e = cudaGraphInstantiate(exec, g, cudaGraphInstantiateFlagUseNodePriority);
+  cudaGraphDestroy(g);
+  if (e != cudaSuccess) return cuda_fail(h, e, "cudaGraphInstantiate");
+  return BMLP_OK;
+}
+
 int ensure_graph(bmlp_t* h) {
-  if (h->stepExec) return BMLP_OK;
+  if (h->stepExec && h->multiExec) return BMLP_OK;
   // the forward chain is captured at the highest stream priority and the
   // event-draw branch at the lowest, so that the block scheduler places
   // forward CTAs first and the event draws fill the remaining room
@@ -250,21 +283,9 @@ int ensure_graph(bmlp_t* h) {
     CK(h, cudaStreamCreateWithPriority(&h->sideStream, cudaStreamNonBlocking, prio_low));
   if (!h->evFork) CK(h, cudaEventCreateWithFlags(&h->evFork, cudaEventDisableTiming));
   if (!h->evJoin) CK(h, cudaEventCreateWithFlags(&h->evJoin, cudaEventDisableTiming));
-  cudaGraph_t g = nullptr;
-  CK(h, cudaStreamBeginCapture(h->capStream, cudaStreamCaptureModeThreadLocal));
-  const bool prof = h->profiling;
-  h->profiling = false;
-  int rc = enqueue_step(h, h->capStream, true);
-  h->profiling = prof;
-  cudaError_t e = cudaStreamEndCapture(h->capStream, &g);
-  if (rc != BMLP_OK) {
-    if (g) cudaGraphDestroy(g);
-    return rc;
-  }
-  if (e != cudaSuccess) return cuda_fail(h, e, "cudaStreamEndCapture");
-  e = cudaGraphInstantiate(&h->stepExec, g, cudaGraphInstantiateFlagUseNodePriority);
-  cudaGraphDestroy(g);
-  if (e != cudaSuccess) return cuda_fail(h, e, "cudaGraphInstantiate");
+  int rc;
+  if (!h->stepExec && (rc = capture_steps(h, 1, &h->stepExec)) != BMLP_OK) return rc;
+  if (!h->multiExec && (rc = capture_steps(h, kGraphSteps, &h->multiExec)) != BMLP_OK) return rc;
   return BMLP_OK;
 }
 
@@ -282,15 +303,23 @@ int run_steps(bmlp_t* h, const uint64_t* xd, const int32_t* yd, int64_t n, cudaS
     int rc = ensure_graph(h);
     if (rc != BMLP_OK) return rc;
   }
-  for (int64_t s = 0; s < steps; ++s) {
-    // sampled mini-batches are launched kernel by kernel between CUDA events
-    h->profiling = h->profEvery > 0 && ((h->t_host + s) % h->profEvery) == 0;
+  auto sampled = [&](int64_t s) {
+    return h->profEvery > 0 && ((h->t_host + s) % h->profEvery) == 0;
+  };
+  for (int64_t s = 0; s < steps;) {
+    // sampled mini-batches are launched kernel by kernel between CUDA events;
+    // the others as graphs of kGraphSteps steps, or of one step
+    h->profiling = sampled(s);
     if (h->profiling) {
       int rc = enqueue_step(h, st, false);
       if (rc != BMLP_OK) return rc;
-    } else {
-      CK(h, cudaGraphLaunch(h->stepExec, st));
+      ++s;
+      continue;
     }
+    bool multi = s + kGraphSteps <= steps;
+    for (int64_t i = 1; multi && i < kGraphSteps; ++i) multi = !sampled(s + i);
+    CK(h, cudaGraphLaunch(multi ? h->multiExec : h->stepExec, st));
+    s += multi ? kGraphSteps : 1;
   }
   h->profiling = h->profEvery > 0;
   h->launches += steps * (h->L + 3);
@@ -511,6 +540,7 @@ void bmlp_destroy(bmlp_t* h) {
   if (!h) return;
   cudaDeviceSynchronize();
   if (h->stepExec) cudaGraphExecDestroy(h->stepExec);
+  if (h->multiExec) cudaGraphExecDestroy(h->multiExec);
   if (h->capStream) cudaStreamDestroy(h->capStream);
   if (h->sideStream) cudaStreamDestroy(h->sideStream);
   if (h->evFork) cudaEventDestroy(h->evFork);

@@ -107,9 +107,10 @@ constexpr int kClsThreads = 512;
 // Counter layout of the library's random streams (purpose tag in c2):
 //   initial h_ik of layer l : (i/4, k, 1*2^16 + l, 0)   word i%4, +1 iff bit 31
 //   rho_kj of P_l           : (j/4, k, 2*2^16 + l, 0)   word j%4, +1 iff bit 31
-//   reinforcement draw U of h_ik at step t: high 16 bits = lane i%8 of
-//     (i/8, k, 3*2^16 + l, t), low 16 bits = lane i%8 of (i/8, k, 4*2^16 + l, t);
-//     lane j of (w0..w3) is the 16-bit half j%2 (low half first) of w_{j/2}.
+//   block draw U of block b (inputs 64b .. 64b+63) of neuron k at step t:
+//                             (b/4, k, 3*2^16 + l, t)   word b%4
+//   event draws V_0, V_1, .. of that block: words 0..3 of (b, k, (4+r)*2^16 + l, t),
+//                             r = 0, 1, ..
 // ---------------------------------------------------------------------------
 __device__ __forceinline__ uint4 philox4x32_10(uint4 ctr, uint32_t k0, uint32_t k1) {
 #pragma unroll
@@ -122,9 +123,33 @@ __device__ __forceinline__ uint4 philox4x32_10(uint4 ctr, uint32_t k0, uint32_t 
   return ctr;
 }
 
-__device__ __forceinline__ uint32_t lane16(const uint4& w, int j) {
-  const uint32_t word = (j < 2) ? w.x : (j < 4) ? w.y : (j < 6) ? w.z : w.w;
-  return (j & 1) ? (word >> 16) : (word & 0xFFFFu);
+// Programmatic dependent launch: a kernel launched with the
+// programmatic-stream-serialization attribute may start while the kernel
+// before it in the stream is still running.  pdl_wait() returns once that
+// kernel has completed and its memory is visible (at once without the
+// attribute); pdl_trigger() lets the next kernel start launching.  Every
+// kernel that triggers does so only after its own wait, so when a kernel
+// starts, every kernel two or more launches before it has completed.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+// Launch with or without the programmatic-stream-serialization attribute.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_kernel(void (*k)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                          bool pdl, Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, k, args...);
 }
 
 __device__ __forceinline__ int clip_h(int h, int h_max) {
@@ -144,8 +169,9 @@ __global__ void k_cls_select(const StepParams* P);
 // boundaries of the lattice index).
 // hb_mode: 8 when h_max = 255 (compile-time lattice exponent), -1 for another
 // h_max + 1 that is a power of two, 0 otherwise (update_hb_mode).
-void launch_update(int hb_mode, unsigned grid, size_t smem, cudaStream_t st, const StepParams* P,
-                   uint32_t key0, uint32_t key1);
+// pdl: launched with the programmatic-stream-serialization attribute.
+cudaError_t launch_update(int hb_mode, unsigned grid, size_t smem, cudaStream_t st, bool pdl,
+                          const StepParams* P, uint32_t key0, uint32_t key1);
 inline int update_hb_mode(int h_max, int hb) {
   return ((h_max + 1) & h_max) != 0 ? 0 : (hb == 8 ? 8 : -1);
 }
@@ -184,13 +210,16 @@ __global__ void k_repack_w(const int16_t* H, uint64_t* W, int Kin, int Kout, int
 // needs bs <= 128.  tiles: take the A operand from layer l-1's AE image.
 size_t train_forward_tc_smem();
 cudaError_t prepare_train_forward_tc();
-void launch_train_forward_tc(bool tiles, int Kout, cudaStream_t st, const StepParams* P, int l);
+// pdl: launched with the programmatic-stream-serialization attribute.
+cudaError_t launch_train_forward_tc(bool tiles, int Kout, cudaStream_t st, bool pdl,
+                                   const StepParams* P, int l);
 size_t act_tile_bytes(int K);  // bytes of an AE image for K activations
+// Median binarisation of n x K fp32 patterns into n x nw packed words.
+void launch_binarize_median(const float* x, int64_t n, int K, int nw, uint64_t* out,
+                            cudaStream_t st);
 // Tensor-core forward for evaluation: A (M x nw_in) against W -> Aout
 // (M x nw_out), 128-pattern x 256-neuron tiles; an expired bounded wait adds
 // one to *timeouts.
-void launch_binarize_median(const float* x, int64_t n, int K, int nw, uint64_t* out,
-                            cudaStream_t st);
 cudaError_t prepare_forward_eval_tc();
 void launch_forward_eval_tc(const uint64_t* A, int64_t M, int nw_in, const uint64_t* W, int N,
                             int Kin, uint64_t* Aout, int nw_out, unsigned int* timeouts,

@@ -116,12 +116,12 @@ cudaError_t prepare_train_forward_tc() {
                               (int)kSmemBytes);
 }
 
-void launch_train_forward_tc(bool tiles, int Kout, cudaStream_t st, const StepParams* P, int l) {
+cudaError_t launch_train_forward_tc(bool tiles, int Kout, cudaStream_t st, bool pdl,
+                                   const StepParams* P, int l) {
   const dim3 grid((unsigned)(((Kout + TN - 1) / TN) * kSplit));
   if (tiles)
-    k_train_forward_tc<true><<<grid, THREADS, kSmemBytes, st>>>(P, l);
-  else
-    k_train_forward_tc<false><<<grid, THREADS, kSmemBytes, st>>>(P, l);
+    return launch_kernel(k_train_forward_tc<true>, grid, dim3(THREADS), kSmemBytes, st, pdl, P, l);
+  return launch_kernel(k_train_forward_tc<false>, grid, dim3(THREADS), kSmemBytes, st, pdl, P, l);
 }
 
 size_t act_tile_bytes(int K) { return (size_t)((K + KB - 1) / KB) * A_BYTES; }
@@ -136,10 +136,16 @@ __global__ void __cluster_dims__(kSplit, 1, 1) __launch_bounds__(THREADS, 1)
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   TcShared* sh = reinterpret_cast<TcShared*>(base + kStages * STAGE_BYTES);
   const DevLayer& Ly = P->layer[l - 1];
-  const int64_t start = (int64_t)P->ctrl->s * P->bs;
-  const int64_t rem = P->n - start;
-  const int M = (int)(rem < P->bs ? rem : P->bs);
-  const uint64_t* A = (l == 1) ? P->x + start * P->nw0 : P->layer[l - 2].A;
+  // the mini-batch index is advanced by the previous step's update kernel; a
+  // layer >= 2 launch reads it after the wait below, layer 1 (which zeroes
+  // the pattern rows >= M in its prologue) before anything else
+  int64_t start = 0;
+  int M = 0;
+  if (!kTiles) {
+    pdl_wait();
+    start = (int64_t)P->ctrl->s * P->bs;
+    M = (int)min((int64_t)P->bs, P->n - start);
+  }
   const uint32_t rank = cluster_rank();
   const int n0 = (int)(blockIdx.x / kSplit) * TN;
   const int N = Ly.Kout, Kin = Ly.Kin, nw = Ly.nw_in;
@@ -183,6 +189,16 @@ __global__ void __cluster_dims__(kSplit, 1, 1) __launch_bounds__(THREADS, 1)
   __syncthreads();
   asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
   const uint32_t tmem = sh->tmem_base;
+  if (kTiles) {
+    // everything above depends on no earlier kernel; the activations, the
+    // mini-batch index and this layer's outputs (read by the previous step's
+    // update) do
+    pdl_wait();
+    start = (int64_t)P->ctrl->s * P->bs;
+    M = (int)min((int64_t)P->bs, P->n - start);
+  }
+  pdl_trigger();
+  const uint64_t* A = (l == 1) ? P->x + start * P->nw0 : P->layer[l - 2].A;
 
   if (threadIdx.x < kProducers) {
     // ---------------- producers ----------------

@@ -39,6 +39,8 @@ __global__ void __launch_bounds__(kClsThreads) k_cls_select(const StepParams* __
   const int mu = blockIdx.x;
   const DevLayer& Ly = P->layer[li];
   Ctrl* ctrl = P->ctrl;
+  pdl_wait();
+  pdl_trigger();
   const int64_t start = batch_start(P);
   const int64_t bsz = batch_size(P, start);
   if (mu >= bsz) return;
@@ -384,11 +386,7 @@ __global__ void __launch_bounds__(kUpdThreads, 4) k_update(const StepParams* __r
   __shared__ uint2 s_fire[16];
   __shared__ unsigned long long s_stats[3];
   Ctrl* ctrl = P->ctrl;
-  const unsigned long long t = ctrl->t;
-  const uint32_t s = ctrl->s;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nwarps = blockDim.x >> 5;
-  const int64_t start = (int64_t)s * P->bs;
-  const int bsz = (int)batch_size(P, start);
   // dynamic shared memory, per warp: s_list [bs] int32 | (8-byte aligned)
   // s_ev [nblk_max] uint64
   const size_t wbytes = update_warp_smem(P->bs, P->nblk_max);
@@ -417,6 +415,13 @@ __global__ void __launch_bounds__(kUpdThreads, 4) k_update(const StepParams* __r
       s_fire[n] = make_uint2((uint32_t)((n & 1) | ((n >> 1) & 1) << 16),
                              (uint32_t)(((n >> 2) & 1) | ((n >> 3) & 1) << 16));
   }
+  // the tables above depend on no earlier kernel; everything below does
+  pdl_wait();
+  pdl_trigger();
+  const unsigned long long t = ctrl->t;
+  const uint32_t s = ctrl->s;
+  const int64_t start = (int64_t)s * P->bs;
+  const int bsz = (int)batch_size(P, start);
   __syncthreads();
 
   const int c = P->c;
@@ -733,14 +738,13 @@ void launch_r_events(unsigned grid, cudaStream_t st, const StepParams* P, uint32
   k_r_events<<<grid, kEvThreads, 0, st>>>(P, key0, key1);
 }
 
-void launch_update(int hb_mode, unsigned grid, size_t smem, cudaStream_t st, const StepParams* P,
-                   uint32_t key0, uint32_t key1) {
+cudaError_t launch_update(int hb_mode, unsigned grid, size_t smem, cudaStream_t st, bool pdl,
+                          const StepParams* P, uint32_t key0, uint32_t key1) {
   if (hb_mode == 8)
-    k_update<8><<<grid, kUpdThreads, smem, st>>>(P, key0, key1);
-  else if (hb_mode != 0)
-    k_update<-1><<<grid, kUpdThreads, smem, st>>>(P, key0, key1);
-  else
-    k_update<0><<<grid, kUpdThreads, smem, st>>>(P, key0, key1);
+    return launch_kernel(k_update<8>, dim3(grid), dim3(kUpdThreads), smem, st, pdl, P, key0, key1);
+  if (hb_mode != 0)
+    return launch_kernel(k_update<-1>, dim3(grid), dim3(kUpdThreads), smem, st, pdl, P, key0, key1);
+  return launch_kernel(k_update<0>, dim3(grid), dim3(kUpdThreads), smem, st, pdl, P, key0, key1);
 }
 
 cudaError_t update_kernel_occupancy(int hb_mode, size_t smem, int* per_sm) {
