@@ -13,6 +13,10 @@ these seeded generators stand in for their shapes:
   C5  8192 -> 8192 x4 -> 10        1,000,000 streamed samples, 1 pass;
                                    plus a 65,536-sample forward-only sweep
 
+Random Prototypes (Sec. 4.1.1, ``random_prototypes``): K_0 = 1000 bits,
+10 classes, each sample a class prototype with every entry flipped with
+probability 0.44, all samples distinct; 10,000 training and 2,000 test samples.
+
 Input distributions:
   "bias"  : bit j of a sample is +1 with probability p_j, p_j ~ U[0.3, 0.7]
             drawn once per feature (C1, C2, the 784-pixel FashionMNIST shape);
@@ -235,6 +239,34 @@ def make_split(cfg: Config, split: str, n: int | None = None) -> Split:
     t = make_teacher(cfg)
     y = teacher_labels_pm1(t, unpack(xp, cfg.widths[0]))
     return Split(xp, y, cfg.widths[0])
+
+
+def random_prototypes(seed: int, n_train: int = 10000, n_test: int = 2000, K0: int = 1000,
+                      classes: int = 10, p: float = 0.44):
+    """The Random Prototypes set of Sec. 4.1.1: one uniformly random +-1
+    prototype per class; a sample of class j is prototype j with each entry
+    flipped independently with probability p; a sample equal to an earlier one
+    (train or test) is discarded and redrawn, so all n_train + n_test samples
+    are distinct.  Sample i (train first, then test) has class i mod classes,
+    so every mini-batch in dataset order mixes the classes.  Returns
+    (train Split, test Split) with labels = the classes."""
+    rng = np.random.Generator(np.random.PCG64(np.random.SeedSequence([seed, 77])))
+    proto = np.where(rng.random((classes, K0)) < 0.5, 1, -1).astype(np.int8)
+    n = n_train + n_test
+    x = np.empty((n, K0), np.int8)
+    y = (np.arange(n) % classes).astype(np.int32)
+    seen = set()
+    for i in range(n):
+        while True:
+            flip = rng.random(K0) < p
+            v = np.where(flip, -proto[y[i]], proto[y[i]]).astype(np.int8)
+            key = v.tobytes()
+            if key not in seen:
+                seen.add(key)
+                x[i] = v
+                break
+    xp = pack(x)
+    return Split(xp[:n_train], y[:n_train], K0), Split(xp[n_train:], y[n_train:], K0)
 
 
 def small_config(widths, classes, n_train, n_test=0, gen="bias", teacher_hidden=32, number=99):
