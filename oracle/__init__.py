@@ -125,7 +125,11 @@ def _declare(L):
                                 C.c_int32, _i32p, _u8p, _i32p, _u8p]
     L.or_local_loss.restype = None
     L.or_select.argtypes = [_i32p, C.c_int32, C.c_int32, _i8p, C.c_int32, _i32p, _u8p,
-                            C.c_int32, _i32p]
+                            C.c_int32, _i32p, _i32p]
+    L.or_group_members.argtypes = [C.c_uint64, C.c_int32, C.c_int32, C.c_int32, C.c_uint32, _i32p]
+    L.or_group_members.restype = C.c_int
+    L.or_set_group_mode.argtypes = [C.c_void_p, C.c_int32]
+    L.or_set_group_mode.restype = C.c_int
     L.or_select.restype = None
     L.or_perceptron_update.argtypes = [_i32p, C.c_int32, C.c_int32, _i8p, _i32p, _i8p,
                                        C.c_int32, _i32p, C.c_int32, C.c_int32, C.c_int32,
@@ -261,8 +265,9 @@ def local_loss(yhat, y, K, r_num=1, r_den=4):
     return pred, ell, tau, mark
 
 
-def select(z, P, y, mark, gamma):
-    """Alg. 2 l.4-10.  Returns sel: b x G (selected neuron per group, -1 = none)."""
+def select(z, P, y, mark, gamma, member=None):
+    """Alg. 2 l.4-10.  Returns sel: b x G (selected neuron per group, -1 = none).
+    member (O19): group g = member[g*gamma:(g+1)*gamma]; None = contiguous."""
     z = _c(z, np.int32)
     P = _c(P, np.int8)
     y = _c(y, np.int32)
@@ -271,9 +276,19 @@ def select(z, P, y, mark, gamma):
     c = P.shape[1]
     G = K // gamma
     sel = np.zeros((b, G), np.int32)
+    mem = None if member is None else _c(member, np.int32)
     lib().or_select(_p(z, _i32p), b, K, _p(P, _i8p), c, _p(y, _i32p), _p(mark, _u8p), gamma,
-                    _p(sel, _i32p))
+                    None if mem is None else _p(mem, _i32p), _p(sel, _i32p))
     return sel
+
+
+def group_members(seed, l, K, mode, t=0):
+    """Group order of layer l (O19): member[j] = neuron at position j."""
+    out = np.zeros(K, np.int32)
+    rc = lib().or_group_members(seed & (2**64 - 1), l, K, mode, t & 0xFFFFFFFF, _p(out, _i32p))
+    if rc != 0:
+        raise ValueError("or_group_members failed: %d" % rc)
+    return out
 
 
 def perceptron_update(H, a_prev, y, P, sel, h_max, q, seed, l, t):
@@ -370,6 +385,12 @@ class OracleModel:
         out = np.zeros(self.L, np.int64)
         lib().or_layer_errors(self._h, _p(out, _i64p), 1 if reset else 0)
         return [int(v) for v in out]
+
+    def set_group_mode(self, mode):
+        """Group membership of every layer (O19): 0 contiguous, 1 fixed random,
+        2 redrawn at every mini-batch step."""
+        if lib().or_set_group_mode(self._h, mode) != 0:
+            raise ValueError("or_set_group_mode failed")
 
     def gamma(self, l):
         return lib().or_gamma(self._h, l)

@@ -73,6 +73,14 @@
  *       ceil(K/2)-th smallest; a_i = +1 iff x_i > m (strict, compared in
  *       fp32), else -1.  With distinct values exactly floor(K/2) inputs are
  *       +1; a constant pattern is all -1.
+ *   O19 Group membership (Sec. 4.3: by permutation symmetry the groups may
+ *       be a random partition fixed once, or redrawn at every step).  Mode 0:
+ *       contiguous groups (O7).  Modes 1 and 2: order the neurons k of layer l
+ *       by the key u_k = word k%4 of Philox (k/4, 0, 32*2^16 + l, t'), ties to
+ *       the smaller k; group g is the neurons at positions g*gamma ..
+ *       (g+1)*gamma - 1 of that order; t' = 0 (mode 1, fixed) or the step t
+ *       (mode 2, redrawn every mini-batch).  Inside a group the easiest
+ *       neuron is chosen as in O7, ties to the lowest neuron index k.
  *   O17 Early exit (Sec. 3.1: the intermediate P_l may serve early-exit
  *       strategies): the prediction of layer l is argmax_j of
  *       yhat_l = a_l P_l, ties to the lowest class (O2); the local error
@@ -88,6 +96,8 @@
  *                               (b/4, k, 3*2^16 + l, t); word b%4
  *   event draws V_0, V_1, ... of that block, in this order:
  *                               words 0..3 of (b, k, (4 + r)*2^16 + l, t), r = 0, 1, ...
+ *                               (at most 16 calls per block: r <= 15)
+ *   group-order key u_k of neuron k (O19): (k/4, 0, 32*2^16 + l, t'); word k%4
  *   Layers are numbered l = 1..L as in the paper.
  */
 #include <math.h>
@@ -249,6 +259,42 @@ static int32_t clip(int32_t h, int32_t h_max) {
 
 static int32_t sign_of(int32_t v) { return v >= 0 ? +1 : -1; } /* O1 */
 
+/* Group membership of layer l (O19): member[j] = the neuron at position j of
+ * the group order (group g = member[g*gamma .. (g+1)*gamma - 1]). */
+typedef struct {
+  uint32_t u;
+  int32_t k;
+} or_keyed;
+
+static int or_cmp_keyed(const void* pa, const void* pb) {
+  const or_keyed* a = (const or_keyed*)pa;
+  const or_keyed* b = (const or_keyed*)pb;
+  if (a->u != b->u) return a->u < b->u ? -1 : 1;
+  return (a->k > b->k) - (a->k < b->k);
+}
+
+int or_group_members(uint64_t seed, int32_t l, int32_t K, int32_t mode, uint32_t t,
+                     int32_t* member) {
+  if (K < 1 || !member || mode < 0 || mode > 2) return OR_EINVAL;
+  if (mode == 0) {
+    for (int32_t k = 0; k < K; k++) member[k] = k;
+    return OR_OK;
+  }
+  or_keyed* v = (or_keyed*)malloc(sizeof(or_keyed) * (size_t)K);
+  if (!v) return OR_ENOMEM;
+  const uint32_t tt = (mode == 2) ? t : 0u;
+  for (int32_t k = 0; k < K; k++) {
+    uint32_t w[4];
+    philox_at(seed, (uint32_t)k / 4u, 0u, (32u << 16) + (uint32_t)l, tt, w);
+    v[k].u = w[k % 4];
+    v[k].k = k;
+  }
+  qsort(v, (size_t)K, sizeof(or_keyed), or_cmp_keyed);
+  for (int32_t j = 0; j < K; j++) member[j] = v[j].k;
+  free(v);
+  return OR_OK;
+}
+
 /* ------------------------------------------------------------------------ */
 /* Network level, Algorithm 1                                                 */
 /* ------------------------------------------------------------------------ */
@@ -310,11 +356,14 @@ void or_local_loss(const int32_t* yhat, int32_t b, int32_t c, const int32_t* y, 
 /* Layer level, Algorithm 2                                                   */
 /* ------------------------------------------------------------------------ */
 
-/* For every mu in M_l (mark[mu] != 0) and every group g of gamma contiguous
- * neurons: delta_k = z^mu_k rho_{k, y^mu}; k* = argmax_{k in g} {delta_k : delta_k < 0}.
- * sel[mu * G + g] = k*, or -1 when mu is not marked or no delta in g is negative. */
+/* For every mu in M_l (mark[mu] != 0) and every group g of gamma neurons
+ * (member == NULL: contiguous, neuron g*gamma + j; else neuron member[g*gamma + j],
+ * O19): delta_k = z^mu_k rho_{k, y^mu}; k* = argmax_{k in g} {delta_k : delta_k < 0},
+ * ties to the lowest k.  sel[mu * G + g] = k*, or -1 when mu is not marked or
+ * no delta in g is negative. */
 void or_select(const int32_t* z, int32_t b, int32_t K, const int8_t* P, int32_t c,
-               const int32_t* y, const uint8_t* mark, int32_t gamma, int32_t* sel) {
+               const int32_t* y, const uint8_t* mark, int32_t gamma, const int32_t* member,
+               int32_t* sel) {
   const int32_t G = K / gamma;
   int32_t* delta = (int32_t*)malloc(sizeof(int32_t) * (size_t)(K > 0 ? K : 1));
   for (int32_t mu = 0; mu < b; mu++) {
@@ -324,8 +373,12 @@ void or_select(const int32_t* z, int32_t b, int32_t K, const int8_t* P, int32_t 
       delta[k] = z[(int64_t)mu * K + k] * P[(int64_t)k * c + y[mu]];
     for (int32_t g = 0; g < G; g++) {
       int32_t best = -1;
-      for (int32_t k = g * gamma; k < (g + 1) * gamma; k++)
-        if (delta[k] < 0 && (best < 0 || delta[k] > delta[best])) best = k;
+      for (int32_t j = g * gamma; j < (g + 1) * gamma; j++) {
+        const int32_t k = member ? member[j] : j;
+        if (delta[k] < 0 &&
+            (best < 0 || delta[k] > delta[best] || (delta[k] == delta[best] && k < best)))
+          best = k;
+      }
       sel[(int64_t)mu * G + g] = best;
     }
   }
@@ -386,6 +439,7 @@ typedef struct {
   int64_t t;        /* mini-batches processed since creation */
   int64_t epoch_err, epoch_n;
   int64_t* layer_err; /* layer_err[l]: local 01-loss count of layer l (O17) */
+  int32_t group_mode; /* O19: 0 contiguous, 1 fixed random, 2 redrawn every step */
   int32_t** H;      /* H[l]: K[l-1] x K[l] */
   int8_t** P;       /* P[l]: K[l] x c */
 } or_model;
@@ -476,6 +530,7 @@ int or_train(or_model* m, const int8_t* x, const int32_t* y, int64_t n, int32_t 
   int32_t* yhat = (int32_t*)malloc(sizeof(int32_t) * (size_t)m->bs * (size_t)c);
   uint8_t* ell = (uint8_t*)malloc((size_t)m->bs);
   int32_t* sel = NULL;
+  int32_t* member = NULL;
   int64_t n_err = 0;
   int rc = OR_OK;
   if (!a || !z || !mark || !yhat || !ell) rc = OR_ENOMEM;
@@ -490,7 +545,8 @@ int or_train(or_model* m, const int8_t* x, const int32_t* y, int64_t n, int32_t 
     if (m->K[l] > Kmax) Kmax = m->K[l];
   if (rc == OR_OK) {
     sel = (int32_t*)malloc(sizeof(int32_t) * (size_t)m->bs * (size_t)Kmax);
-    if (!sel) rc = OR_ENOMEM;
+    member = (int32_t*)malloc(sizeof(int32_t) * (size_t)Kmax);
+    if (!sel || !member) rc = OR_ENOMEM;
   }
   for (int64_t start = 0; rc == OR_OK && start < n; start += m->bs) {
     const int32_t b = (int32_t)((n - start) < m->bs ? (n - start) : m->bs); /* O13 */
@@ -511,7 +567,10 @@ int or_train(or_model* m, const int8_t* x, const int32_t* y, int64_t n, int32_t 
       for (int32_t mu = 0; mu < b; mu++) any |= mark[l][mu];
       if (!any) continue; /* O6 */
       const int32_t G = m->K[l] / m->gamma[l];
-      or_select(z[l], b, m->K[l], m->P[l], c, yb, mark[l], m->gamma[l], sel);
+      if (m->group_mode != 0)
+        or_group_members(m->seed, l, m->K[l], m->group_mode, (uint32_t)m->t, member);
+      or_select(z[l], b, m->K[l], m->P[l], c, yb, mark[l], m->gamma[l],
+                m->group_mode != 0 ? member : NULL, sel);
       or_perceptron_update(m->H[l], m->K[l - 1], m->K[l], a[l - 1], yb, m->P[l], c, sel, b, G,
                            m->h_max, or_reinforce_prob(m->p_r, m->K[l]), m->seed, l,
                            (uint32_t)m->t);
@@ -540,6 +599,7 @@ int or_train(or_model* m, const int8_t* x, const int32_t* y, int64_t n, int32_t 
   free(yhat);
   free(ell);
   free(sel);
+  free(member);
   return rc;
 }
 
@@ -678,6 +738,13 @@ int or_get_layer(const or_model* m, int32_t l, int32_t* H, int8_t* P) {
 int or_set_layer(or_model* m, int32_t l, const int32_t* H) {
   if (!m || l < 1 || l > m->L || !H) return OR_EINVAL;
   memcpy(m->H[l], H, sizeof(int32_t) * (size_t)m->K[l - 1] * (size_t)m->K[l]);
+  return OR_OK;
+}
+
+/* Group membership mode of every layer (O19). */
+int or_set_group_mode(or_model* m, int32_t mode) {
+  if (!m || mode < 0 || mode > 2) return OR_EINVAL;
+  m->group_mode = mode;
   return OR_OK;
 }
 

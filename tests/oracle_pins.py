@@ -510,6 +510,87 @@ def check_layer_errors_match_eval(seed=11):
     assert m.layer_errors() == [0, 0]
 
 
+# -- group membership (O19) -------------------------------------------------------
+
+def check_group_members(seed=12):
+    """Modes 1 and 2 order the neurons by the Philox key of O19 (recomputed here
+    from the KAT-pinned Philox with numpy's stable lexsort); mode 0 is the
+    identity; mode 1 does not depend on the step, mode 2 does, and equals
+    mode 1 at t = 0.  Over many layers the partition is uniform: neurons 0 and
+    1 share a group with probability (gamma-1)/(K-1), and neuron 0's position
+    is uniform (chi-square)."""
+    for K in (1, 5, 24, 130):
+        assert np.array_equal(O.group_members(seed, 1, K, 0), np.arange(K))
+        for l in (1, 3):
+            for t in (0, 7):
+                u = np.array([O.philox4x32_10([k // 4, 0, (32 << 16) + l, t],
+                                              [seed & 0xFFFFFFFF, seed >> 32])[k % 4]
+                              for k in range(K)], np.uint64)
+                want = np.lexsort((np.arange(K), u))
+                assert np.array_equal(O.group_members(seed, l, K, 2, t), want), (K, l, t)
+                assert np.array_equal(O.group_members(seed, l, K, 1, t),
+                                      O.group_members(seed, l, K, 2, 0))
+    assert not np.array_equal(O.group_members(seed, 1, 130, 2, 1), O.group_members(seed, 1, 130, 2, 2))
+    K, gamma, trials = 24, 6, 3000
+    same, pos0 = 0, np.zeros(K, np.int64)
+    for s in range(trials):
+        m = O.group_members(1000 + s, 1 + s % 7, K, 1)
+        where = np.argsort(m)
+        same += int(where[0] // gamma == where[1] // gamma)
+        pos0[where[0]] += 1
+    p = (gamma - 1) / (K - 1)
+    assert abs(same - p * trials) < 5 * np.sqrt(trials * p * (1 - p)), same
+    chi2 = ((pos0 - trials / K) ** 2 / (trials / K)).sum()
+    assert chi2 < 60, chi2   # 23 degrees of freedom: P(chi2 > 60) < 1e-4
+
+
+def check_select_with_members(seed=13):
+    """Alg. 2 over an arbitrary partition: the selected neuron lies in its
+    group, has delta < 0, and no member of the group has a larger negative
+    delta or the same delta with a smaller index; a group without a negative
+    delta gives -1; the identity order reproduces contiguous groups."""
+    rng = np.random.default_rng(seed)
+    b, K, c, gamma = 30, 24, 4, 6
+    for _ in range(20):
+        z = rng.integers(-3, 4, size=(b, K)).astype(np.int32)    # many ties
+        P = np.where(rng.random((K, c)) < 0.5, 1, -1).astype(np.int8)
+        y = rng.integers(0, c, size=b).astype(np.int32)
+        mark = (rng.random(b) < 0.8).astype(np.uint8)
+        member = rng.permutation(K).astype(np.int32)
+        sel = O.select(z, P, y, mark, gamma, member)
+        assert np.array_equal(O.select(z, P, y, mark, gamma, np.arange(K)),
+                              O.select(z, P, y, mark, gamma))
+        delta = z * P[:, y].T
+        for mu in range(b):
+            for g in range(K // gamma):
+                grp = member[g * gamma:(g + 1) * gamma]
+                neg = [k for k in grp if delta[mu, k] < 0]
+                if not mark[mu] or not neg:
+                    assert sel[mu, g] == -1
+                    continue
+                best = max(delta[mu, k] for k in neg)
+                assert sel[mu, g] == min(k for k in neg if delta[mu, k] == best), (mu, g)
+
+
+def check_group_mode_single_group(seed=14):
+    """With gamma = K_l the only group is the whole layer whatever the order,
+    so training in modes 1 and 2 equals mode 0 exactly."""
+    rng = np.random.default_rng(seed)
+    x, y = _bias_data(rng, 120, 30, 3)
+    ref = O.OracleModel([30, 12, 8], 3, seed=2, bs=20, gamma=[12, 8])
+    ref.train(x, y)
+    for mode in (1, 2):
+        m = O.OracleModel([30, 12, 8], 3, seed=2, bs=20, gamma=[12, 8])
+        m.set_group_mode(mode)
+        m.train(x, y)
+        for l in (1, 2):
+            assert np.array_equal(m.H(l), ref.H(l)), (mode, l)
+    a = O.OracleModel([30, 12, 8], 3, seed=2, bs=20, gamma=[4, 4])
+    a.set_group_mode(2)
+    a.train(x, y)
+    assert not np.array_equal(a.H(1), ref.H(1))
+
+
 ALL_CHECKS = [
     check_philox_kat,
     check_gamma_golden,
@@ -533,4 +614,7 @@ ALL_CHECKS = [
     check_binarize_median_rank,
     check_early_exit_truncation,
     check_layer_errors_match_eval,
+    check_group_members,
+    check_select_with_members,
+    check_group_mode_single_group,
 ]

@@ -52,6 +52,9 @@ MUTANTS = [
     ("early_exit_layers_reversed", "pred[(int64_t)(l - 1) * n + start + mu] = jmax;",
      "pred[(int64_t)(L - l) * n + start + mu] = jmax;"),
     ("layer_errors_count_marks", "m->layer_err[l] += ell[mu]; /* O17 */", "m->layer_err[l] += mark[l][mu];"),
+    ("group_ties_by_position", "(delta[k] == delta[best] && k < best)", "(0)"),
+    ("group_key_word", "v[k].u = w[k % 4];", "v[k].u = w[0];"),
+    ("group_mode2_fixed", "const uint32_t tt = (mode == 2) ? t : 0u;", "const uint32_t tt = 0u;"),
     ("forward_drops_sign", "zr[k] += ai * (hrow[k] > 0 ? 1 : -1);", "zr[k] += ai * hrow[k];"),
 ]
 
