@@ -95,7 +95,22 @@ typedef struct bmlp_hparams {
   double p_r0;           /* initial reinforcement probability; < 0 -> 0.5 */
   const int32_t* gamma;  /* L group sizes, each dividing K_l; NULL -> Sec. 4.3 rule */
   int32_t fwd_impl;      /* BMLP_FWD_*; 0 -> auto */
+  int32_t group_mode;    /* BMLP_GROUPS_*: group membership of Alg. 2 (Sec. 4.3); 0 -> contiguous */
 } bmlp_hparams;
+
+/* Group membership (Sec. 4.3: by the permutation symmetry of a hidden layer
+ * its groups may be any fixed random partition, or one redrawn at every
+ * step).  CONTIGUOUS: group g = neurons g*gamma .. (g+1)*gamma - 1.  FIXED /
+ * RESHUFFLED: order the neurons k of layer l by the key u_k = word k%4 of
+ * Philox4x32-10 at counter (k/4, 0, 32*2^16 + l, t') with the model's key,
+ * ties to the smaller k; group g = the neurons at positions g*gamma ..
+ * (g+1)*gamma - 1 of that order, with t' = 0 (FIXED) or t' = the step counter
+ * (RESHUFFLED, a new partition every mini-batch).  Within a group the easiest
+ * neuron is chosen with ties to the lowest neuron index.  FIXED and
+ * RESHUFFLED need every K_l <= 16384. */
+#define BMLP_GROUPS_CONTIGUOUS 0
+#define BMLP_GROUPS_FIXED 1
+#define BMLP_GROUPS_RESHUFFLED 2
 
 /* Create a model and initialise H_l, P_l uniformly on {+-1} from `seed`
  * (Alg. 1 l.2).  widths: K_0..K_L (n_widths = L + 1, 2..BMLP_MAX_LAYERS + 1,

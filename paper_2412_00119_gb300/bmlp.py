@@ -29,6 +29,7 @@ BMLP_ESTATE = -5
 BMLP_ENODEV = -6
 BMLP_EPOCH_END = 1
 BMLP_FWD_AUTO, BMLP_FWD_POPC, BMLP_FWD_TCGEN05 = 0, 1, 2
+BMLP_GROUPS_CONTIGUOUS, BMLP_GROUPS_FIXED, BMLP_GROUPS_RESHUFFLED = 0, 1, 2
 PROFILE_KINDS = ("train_forward", "cls_select", "update", "eval_forward", "eval_out", "copy",
                  "r_events")
 
@@ -43,7 +44,8 @@ class BmlpError(RuntimeError):
 
 class bmlp_hparams(C.Structure):
     _fields_ = [("bs", C.c_int32), ("r_num", C.c_int32), ("r_den", C.c_int32),
-                ("p_r0", C.c_double), ("gamma", C.POINTER(C.c_int32)), ("fwd_impl", C.c_int32)]
+                ("p_r0", C.c_double), ("gamma", C.POINTER(C.c_int32)), ("fwd_impl", C.c_int32),
+                ("group_mode", C.c_int32)]
 
 
 _lib = None
@@ -139,7 +141,7 @@ def _stream(stream):
 # -- the C-ABI, one Python function per entry point ------------------------------
 
 def bmlp_create(widths, classes, h_max=255, seed=0, bs=100, r=(1, 4), p_r0=0.5, gamma=None,
-                fwd_impl=BMLP_FWD_AUTO):
+                fwd_impl=BMLP_FWD_AUTO, group_mode=BMLP_GROUPS_CONTIGUOUS):
     w = (C.c_int32 * len(widths))(*[int(v) for v in widths])
     hp = bmlp_hparams()
     hp.bs = bs
@@ -150,6 +152,7 @@ def bmlp_create(widths, classes, h_max=255, seed=0, bs=100, r=(1, 4), p_r0=0.5, 
         g = (C.c_int32 * len(gamma))(*[int(v) for v in gamma])
         hp.gamma = C.cast(g, _i32p)
     hp.fwd_impl = fwd_impl
+    hp.group_mode = group_mode
     h = _vp()
     rc = lib().bmlp_create(w, len(widths), classes, h_max, seed & (2 ** 64 - 1), C.byref(hp), C.byref(h))
     _check(rc, None)
@@ -305,8 +308,9 @@ class BMLP:
     """Owning wrapper of a bmlp_t handle."""
 
     def __init__(self, widths, classes, h_max=255, seed=0, bs=100, r=(1, 4), p_r0=0.5,
-                 gamma=None, fwd_impl=BMLP_FWD_AUTO):
-        self.h = bmlp_create(widths, classes, h_max, seed, bs, r, p_r0, gamma, fwd_impl)
+                 gamma=None, fwd_impl=BMLP_FWD_AUTO, group_mode=BMLP_GROUPS_CONTIGUOUS):
+        self.h = bmlp_create(widths, classes, h_max, seed, bs, r, p_r0, gamma, fwd_impl,
+                             group_mode)
         self.info = bmlp_get_info(self.h)
 
     def close(self):

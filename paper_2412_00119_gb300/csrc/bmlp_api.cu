@@ -31,6 +31,7 @@ enum ProfKind { kProfTrainFwd = 0, kProfCls = 1, kProfUpd = 2, kProfEvalFwd = 3,
 struct bmlp {
   int device = 0;
   int L = 0, c = 0, h_max = 0, bs = 0, r_num = 0, r_den = 1, fwd_impl = BMLP_FWD_POPC;
+  int group_mode = BMLP_GROUPS_CONTIGUOUS, max_K = 0;  // group membership (Sec. 4.3), widest layer
   uint64_t seed = 0;
   std::vector<int> K, gamma;
   double p_r = 0.5;
@@ -227,6 +228,10 @@ int enqueue_step(bmlp_t* h, cudaStream_t st, bool fork, bool chained = false) {
       k_train_forward<<<train_forward_grid(h->bs, h->K[l]), train_forward_block(), 0, st>>>(h->dP, l);
     prof_end(h, st);
   }
+  if (h->group_mode == BMLP_GROUPS_RESHUFFLED) {
+    // this step's partition (keyed by the step counter) before the selection
+    CK(h, launch_group_order(h->L, h->max_K, true, st, h->dP));
+  }
   prof_begin(h, kProfCls, st);
   // inside the step graph each kernel after the first is launched as a
   // programmatic dependent of the one before it (launch and prologue overlap
@@ -322,7 +327,7 @@ int run_steps(bmlp_t* h, const uint64_t* xd, const int32_t* yd, int64_t n, cudaS
     s += multi ? kGraphSteps : 1;
   }
   h->profiling = h->profEvery > 0;
-  h->launches += steps * (h->L + 3);
+  h->launches += steps * (h->L + 3 + (h->group_mode == BMLP_GROUPS_RESHUFFLED ? 1 : 0));
   h->t_host += steps;
   return BMLP_OK;
 }
@@ -416,6 +421,13 @@ int bmlp_create(const int32_t* widths, int32_t n_widths, int32_t classes, int16_
   if (fwd == BMLP_FWD_TCGEN05 && bs > 128)
     return fail(nullptr, BMLP_EINVAL, "fwd_impl TCGEN05 needs bs <= 128");
   const int L = n_widths - 1;
+  const int group_mode = hp.group_mode;
+  if (group_mode < BMLP_GROUPS_CONTIGUOUS || group_mode > BMLP_GROUPS_RESHUFFLED)
+    return fail(nullptr, BMLP_EINVAL, "group_mode must be 0, 1 or 2");
+  int max_K = 0;
+  for (int l = 1; l <= L; ++l) max_K = std::max(max_K, (int)widths[l]);
+  if (group_mode != BMLP_GROUPS_CONTIGUOUS && max_K > 16384)
+    return fail(nullptr, BMLP_EINVAL, "random group membership needs every K_l <= 16384");
   std::vector<int> gam(L + 1, 0);
   for (int l = 1; l <= L; ++l) {
     const int g = hp.gamma ? hp.gamma[l - 1] : bmlp_gamma_rule(widths[l]);
@@ -441,6 +453,7 @@ int bmlp_create(const int32_t* widths, int32_t n_widths, int32_t classes, int16_
   }
   h->L = L; h->c = classes; h->h_max = h_max; h->bs = bs; h->r_num = r_num; h->r_den = r_den;
   h->fwd_impl = fwd; h->seed = seed; h->p_r = p_r0;
+  h->group_mode = group_mode; h->max_K = max_K;
   h->K.assign(widths, widths + n_widths);
   h->gamma = gam;
 
@@ -475,6 +488,10 @@ int bmlp_create(const int32_t* widths, int32_t n_widths, int32_t classes, int16_
         (rc = dalloc(h, &D.mark, (size_t)bs)) ||
         (rc = dalloc(h, &D.sel, (size_t)bs * D.G)) ||
         (rc = dalloc(h, &D.EV, (size_t)D.Kout * D.nblk)))
+      return bail(rc);
+    D.member = D.group_of = nullptr;
+    if (group_mode != BMLP_GROUPS_CONTIGUOUS &&
+        ((rc = dalloc(h, &D.member, (size_t)D.Kout)) || (rc = dalloc(h, &D.group_of, (size_t)D.Kout))))
       return bail(rc);
     D.AE = nullptr;
     if (fwd == BMLP_FWD_TCGEN05 && l < L) {
@@ -530,6 +547,11 @@ int bmlp_create(const int32_t* widths, int32_t n_widths, int32_t classes, int16_
   if ((e = cudaMemcpy(h->dP, &P, sizeof(P), cudaMemcpyHostToDevice)) != cudaSuccess)
     return bail(cuda_fail(h, e, "param upload"));
   if ((rc = upload_thresholds(h, 0)) != BMLP_OK) return bail(rc);
+  // the partition of step 0 (the fixed one, or the first redrawn one)
+  if (group_mode != BMLP_GROUPS_CONTIGUOUS &&
+      ((e = prepare_group_order(max_K)) != cudaSuccess ||
+       (e = launch_group_order(L, max_K, false, 0, h->dP)) != cudaSuccess))
+    return bail(cuda_fail(h, e, "group order"));
   if ((e = cudaDeviceSynchronize()) != cudaSuccess) return bail(cuda_fail(h, e, "init"));
   h->launches += 4 * L;
   *out = h;

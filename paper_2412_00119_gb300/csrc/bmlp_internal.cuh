@@ -43,6 +43,8 @@ struct DevLayer {
   uint8_t* mark;
   int16_t* sel;
   uint8_t* AE;
+  int16_t* member;    // [K_out] group order (neuron at position j), or null: contiguous groups
+  int16_t* group_of;  // [K_out] group of neuron k (with member)
   int32_t Kin, Kout, nw_in, nw_out, ldh, gamma, G;
   int32_t ev_cta_base;   // first CTA of this layer in the event-draw grid
   int32_t row_base;      // first row of this layer in the update's row numbering
@@ -175,6 +177,10 @@ cudaError_t launch_update(int hb_mode, unsigned grid, size_t smem, cudaStream_t 
 inline int update_hb_mode(int h_max, int hb) {
   return ((h_max + 1) & h_max) != 0 ? 0 : (hb == 8 ? 8 : -1);
 }
+// Group order of every layer with a random partition (DevLayer::member /
+// group_of); redraw: keyed by the current step (else by step 0).
+cudaError_t prepare_group_order(int max_K);  // shared-memory attribute, once
+cudaError_t launch_group_order(int L, int max_K, bool redraw, cudaStream_t st, const StepParams* P);
 // Reinforcement events of every neuron row of every layer for the current
 // step into DevLayer::EV (Alg. 3 l.5-12); grid = P->ev_ctas_total CTAs.
 void launch_r_events(unsigned grid, cudaStream_t st, const StepParams* P, uint32_t key0,

@@ -91,7 +91,7 @@ __global__ void __launch_bounds__(kClsThreads) k_cls_select(const StepParams* __
   const int16_t* z = Ly.Z + (int64_t)mu * Ly.Kout;
   const int gamma = Ly.gamma;
   const int per = gamma >> 3;  // 8-neuron chunks per group
-  if ((gamma & 7) == 0 && per <= 32 && (per & (per - 1)) == 0) {
+  if (Ly.member == nullptr && (gamma & 7) == 0 && per <= 32 && (per & (per - 1)) == 0) {
     // one thread per 8 neurons: 16-byte z loads, 8 bytes of rho^T, then the
     // group's per lanes (consecutive, aligned) reduce with shuffles
     const int8_t* rt = Ly.rhoT + (int64_t)y * Ly.Kout;
@@ -128,12 +128,15 @@ __global__ void __launch_bounds__(kClsThreads) k_cls_select(const StepParams* __
     }
     return;
   }
+  // warp per group; the group's neurons are contiguous or listed by the group
+  // order (random partition), so ties compare neuron indices explicitly
+  const int16_t* member = Ly.member;
   for (int g = warp; g < Ly.G; g += nwarps) {
     int bestd = INT_MIN, bestk = INT_MAX;
     for (int kk = lane; kk < gamma; kk += 32) {
-      const int k = g * gamma + kk;
+      const int k = member ? (int)member[g * gamma + kk] : g * gamma + kk;
       const int d = (int)z[k] * (int)Ly.rho[(int64_t)k * c + y];
-      if (d < 0 && d > bestd) {  // ascending k per lane: strict '>' keeps the lowest
+      if (d < 0 && (d > bestd || (d == bestd && k < bestk))) {
         bestd = d;
         bestk = k;
       }
@@ -454,7 +457,7 @@ __global__ void __launch_bounds__(kUpdThreads, 4) k_update(const StepParams* __r
       const DevLayer& Ly = P->layer[li];
       const int k = gr - Ly.row_base;
       const int gamma = Ly.gamma;
-      const int g = k / gamma;
+      const int g = Ly.group_of ? (int)Ly.group_of[k] : k / gamma;
       const int Kin = Ly.Kin;
       const int nch = (Kin + 7) >> 3;             // chunks holding at least one input
       const int full = Kin >> 3;                  // chunks of 8 real inputs
@@ -731,6 +734,74 @@ __global__ void __launch_bounds__(kEvThreads) k_r_events(const StepParams* __res
     }
     __syncwarp();
   }
+}
+
+// ---------------------------------------------------------------------------
+// Group order of a layer with a random partition (Sec. 4.3): CTA l sorts the
+// 64-bit keys (u_k << 32 | k), u_k = word k%4 of Philox (k/4, 0, 32*2^16 + l,
+// t'), ascending with a bitonic network in shared memory (keys are distinct,
+// so ties in u_k go to the smaller k), then member[j] = the k of the j-th key
+// and group_of[k] = j / gamma.  t' = the step counter when redrawn every
+// step, else 0.
+// ---------------------------------------------------------------------------
+constexpr int kGroupThreads = 1024;
+
+__global__ void __launch_bounds__(kGroupThreads) k_group_order(const StepParams* __restrict__ P,
+                                                               int redraw) {
+  extern __shared__ unsigned long long keys[];
+  const DevLayer& Ly = P->layer[blockIdx.x];
+  if (Ly.member == nullptr) return;
+  const int K = Ly.Kout;
+  int n = 1;
+  while (n < K) n <<= 1;
+  const uint32_t t = redraw ? (uint32_t)P->ctrl->t : 0u;
+  const uint32_t c2 = (32u << 16) + (uint32_t)(blockIdx.x + 1);
+  for (int k = threadIdx.x; k < n; k += kGroupThreads) {
+    unsigned long long v = ~0ull;
+    if (k < K) {
+      const uint4 w = philox4x32_10(make_uint4((uint32_t)k >> 2, 0u, c2, t), P->key0, P->key1);
+      const uint32_t u = (k & 3) == 0 ? w.x : (k & 3) == 1 ? w.y : (k & 3) == 2 ? w.z : w.w;
+      v = ((unsigned long long)u << 32) | (uint32_t)k;
+    }
+    keys[k] = v;
+  }
+  __syncthreads();
+  for (int size = 2; size <= n; size <<= 1) {
+    for (int stride = size >> 1; stride > 0; stride >>= 1) {
+      for (int i = threadIdx.x; i < (n >> 1); i += kGroupThreads) {
+        const int lo = 2 * i - (i & (stride - 1));
+        const int hi = lo + stride;
+        const bool up = (lo & size) == 0;
+        const unsigned long long a = keys[lo], b = keys[hi];
+        if ((a > b) == up) {
+          keys[lo] = b;
+          keys[hi] = a;
+        }
+      }
+      __syncthreads();
+    }
+  }
+  for (int j = threadIdx.x; j < K; j += kGroupThreads) {
+    const int k = (int)(uint32_t)keys[j];
+    Ly.member[j] = (int16_t)k;
+    Ly.group_of[k] = (int16_t)(j / Ly.gamma);
+  }
+}
+
+static size_t group_order_smem(int max_K) {
+  int n = 1;
+  while (n < max_K) n <<= 1;
+  return sizeof(unsigned long long) * (size_t)n;
+}
+
+cudaError_t prepare_group_order(int max_K) {
+  return cudaFuncSetAttribute(k_group_order, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              (int)group_order_smem(max_K));
+}
+
+cudaError_t launch_group_order(int L, int max_K, bool redraw, cudaStream_t st, const StepParams* P) {
+  k_group_order<<<(unsigned)L, kGroupThreads, group_order_smem(max_K), st>>>(P, redraw ? 1 : 0);
+  return cudaGetLastError();
 }
 
 void launch_r_events(unsigned grid, cudaStream_t st, const StepParams* P, uint32_t key0,

@@ -62,6 +62,8 @@ def test_sampler_tables_match_oracle(oracle_mod):
     (dict(widths=[10, 8], classes=2, gamma=[3]), "gamma"),
     (dict(widths=[10, 8], classes=2, r=(-1, 4)), "r must"),
     (dict(widths=[10, 8], classes=2, fwd_impl=7), "fwd_impl"),
+    (dict(widths=[10, 8], classes=2, group_mode=3), "group_mode"),
+    (dict(widths=[10, 20000], classes=2, gamma=[100], group_mode=1), "16384"),
 ])
 def test_create_rejects_bad_arguments(kw, msg):
     with pytest.raises(B.BmlpError) as ei:

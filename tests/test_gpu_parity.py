@@ -53,16 +53,17 @@ def assert_same_state(gpu, ref, where=""):
 
 def run_pair(widths, classes, n_train, n_test=64, epochs=2, seed=5, bs=100, gamma=None, h_max=255,
              r=(1, 4), p_r0=0.5, gen="bias", host=False, profiling=False, teacher_hidden=16,
-             data_number=99, fwd=B.BMLP_FWD_AUTO):
+             data_number=99, fwd=B.BMLP_FWD_AUTO, group_mode=0):
     cfg = W.small_config(widths, classes, n_train, n_test, gen=gen, teacher_hidden=teacher_hidden,
                          number=data_number)
     tr = W.make_split(cfg, "train")
     gpu = B.BMLP(widths, classes, h_max=h_max, seed=seed, bs=bs, r=r, p_r0=p_r0, gamma=gamma,
-                 fwd_impl=fwd)
+                 fwd_impl=fwd, group_mode=group_mode)
     assert gpu.info["fwd_impl"] == (fwd if fwd else
                                     (B.BMLP_FWD_TCGEN05 if bs <= 128 else B.BMLP_FWD_POPC))
     ref = O.OracleModel(list(widths), classes, h_max=h_max, seed=seed, bs=bs, r=r, p_r0=p_r0,
                         gamma=gamma)
+    ref.set_group_mode(group_mode)
     if profiling:
         B.bmlp_set_profiling(gpu.h, True)
     assert_same_state(gpu, ref, "after init")
@@ -201,6 +202,14 @@ CASES = {
     "field_inputs": dict(widths=(3072, 128), classes=10, n_train=200, gen="field", teacher_hidden=32),
     "h_max_5_clipping": dict(widths=(96, 64, 64), classes=4, n_train=500, h_max=5, p_r0=1.0),
     "q_above_half": dict(widths=(40, 8), classes=3, n_train=120, bs=20, p_r0=2.0, gamma=[4]),
+    "groups_fixed": dict(widths=(200, 130, 70), classes=10, n_train=300, bs=50, gamma=[13, 7],
+                         group_mode=1),
+    "groups_reshuffled": dict(widths=(200, 130, 70), classes=10, n_train=300, bs=50, gamma=[13, 7],
+                              group_mode=2),
+    "groups_fixed_gamma64": dict(widths=(300, 256, 256), classes=10, n_train=300, gamma=[64, 64],
+                                 group_mode=1),
+    "groups_reshuffled_wide": dict(widths=(256, 1024), classes=10, n_train=400, gamma=[64],
+                                   group_mode=2),
 }
 
 

@@ -102,3 +102,35 @@ def test_table_c1_reproduction():
         print("%5d  %6.2f +- %.2f      %6.2f +- %.2f" % r)
     for width, mean, _, mean_p, std_p in rows:
         assert abs(mean - mean_p) <= 3 * std_p + 1.0, (width, mean, mean_p)
+
+
+@pytest.mark.gpu
+def test_group_membership_does_not_matter():
+    """Sec. 4.3: a fixed random partition, or one redrawn at every step, trains
+    as well as contiguous groups.  1000 -> 255 -> 255 -> 10 (gamma 85, three
+    groups per layer), 20 epochs, 10 model seeds: the three mean test
+    accuracies lie within 1.5 points of each other."""
+    import torch
+
+    from paper_2412_00119_gb300 import bmlp as B
+
+    if not torch.cuda.is_available():
+        pytest.skip("needs a GPU")
+    tr, te = W.random_prototypes(2024)
+    x = torch.from_numpy(tr.xp.view(np.int64)).cuda()
+    y = torch.from_numpy(tr.y).cuda()
+    xt = torch.from_numpy(te.xp.view(np.int64)).cuda()
+    out = torch.empty(len(te.y), dtype=torch.int32, device="cuda")
+    means = []
+    for mode in (B.BMLP_GROUPS_CONTIGUOUS, B.BMLP_GROUPS_FIXED, B.BMLP_GROUPS_RESHUFFLED):
+        acc = []
+        for seed in range(10):
+            m = B.BMLP([1000, 255, 255], 10, seed=seed, bs=100, group_mode=mode)
+            for _ in range(20):
+                m.train(x, y, epoch_end=True)
+            m.predict(xt, out)
+            acc.append(100.0 * float((out.cpu().numpy() == te.y).mean()))
+            m.close()
+        means.append(float(np.mean(acc)))
+    print("\ncontiguous / fixed random / reshuffled: %.2f / %.2f / %.2f" % tuple(means))
+    assert max(means) - min(means) <= 1.5, means
