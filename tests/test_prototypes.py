@@ -134,3 +134,35 @@ def test_group_membership_does_not_matter():
         means.append(float(np.mean(acc)))
     print("\ncontiguous / fixed random / reshuffled: %.2f / %.2f / %.2f" % tuple(means))
     assert max(means) - min(means) <= 1.5, means
+
+
+@pytest.mark.gpu
+def test_hidden_bits_sweep():
+    """App. A.5: fewer bits for the hidden weights (h_max = 2^b - 1) bring
+    catastrophic forgetting; with one bit only the visible weights remain.
+    1000 -> 135 -> 135 -> 10, 50 epochs, 3 model seeds: accuracy rises with b,
+    one bit stays near chance (< 20 %) and eight bits reach > 85 %."""
+    import torch
+
+    from paper_2412_00119_gb300 import bmlp as B
+
+    if not torch.cuda.is_available():
+        pytest.skip("needs a GPU")
+    tr, te = W.random_prototypes(2024)
+    x = torch.from_numpy(tr.xp.view(np.int64)).cuda()
+    y = torch.from_numpy(tr.y).cuda()
+    xt = torch.from_numpy(te.xp.view(np.int64)).cuda()
+    out = torch.empty(len(te.y), dtype=torch.int32, device="cuda")
+    means = []
+    for bits in (1, 4, 8):
+        acc = []
+        for seed in range(3):
+            m = B.BMLP([1000, 135, 135], 10, h_max=2 ** bits - 1, seed=seed, bs=100)
+            for _ in range(50):
+                m.train(x, y, epoch_end=True)
+            m.predict(xt, out)
+            acc.append(100.0 * float((out.cpu().numpy() == te.y).mean()))
+            m.close()
+        means.append(float(np.mean(acc)))
+    print("\nbits 1 / 4 / 8: %.2f / %.2f / %.2f" % tuple(means))
+    assert means[0] < 20.0 < means[1] < means[2] and means[2] > 85.0, means
