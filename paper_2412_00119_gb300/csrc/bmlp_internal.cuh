@@ -224,8 +224,8 @@ size_t act_tile_bytes(int K);  // bytes of an AE image for K activations
 void launch_binarize_median(const float* x, int64_t n, int K, int nw, uint64_t* out,
                             cudaStream_t st);
 // Tensor-core forward for evaluation: A (M x nw_in) against W -> Aout
-// (M x nw_out), 128-pattern x 256-neuron tiles; an expired bounded wait adds
-// one to *timeouts.
+// (M x nw_out), 256-pattern x 256-neuron tiles per CTA pair; an expired
+// bounded wait adds one to *timeouts.
 cudaError_t prepare_forward_eval_tc();
 void launch_forward_eval_tc(const uint64_t* A, int64_t M, int nw_in, const uint64_t* W, int N,
                             int Kin, uint64_t* Aout, int nw_out, unsigned int* timeouts,

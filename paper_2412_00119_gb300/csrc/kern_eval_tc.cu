@@ -2,21 +2,32 @@
 // (Sec. 3.1; Alg. 1 l.8-9 without the training side outputs).
 //
 // Same exact e4m3 formulation as the training forward (+-1 -> 0x38 / 0xB8,
-// pads 0, fp32 sums exact), tiled for large batches: a CTA computes 128
-// patterns x 256 neurons over the whole K range.
-//   - 12 producer warps, one thread per stage row (128 activation rows, then
-//     256 weight rows): per 128-element k-block the thread loads the row's
-//     two bit words (one 16-byte load when the rows are 16-byte aligned),
-//     kPrefetch blocks ahead, and expands them into the row's eight 16-byte
-//     chunks of the 128B-swizzled K-major stage (48 KB, 4-stage ring);
-//   - 1 MMA warp issues tcgen05.mma.kind::f8f6f4 M128 N256 K32 (four per stage)
-//     into a 128 x 256 fp32 accumulator in TMEM (256 columns) and commits to
-//     the stage's "empty" mbarrier;
-//   - the epilogue: the producer warps read TMEM (warp w: lanes 32 (w % 4) ..,
-//     column blocks w / 4, w / 4 + 3, ..) and write the sign bits of each
-//     pattern as 32-bit pieces of its packed row (pad bits 0).
-// Every mbarrier wait is bounded; the first expiry stops every other wait and
-// the kernel counts it in *timeouts, releases TMEM and returns.
+// pads 0, fp32 sums exact), tiled for large batches.
+//
+// Tile.  A cluster of two CTAs computes 256 patterns x 256 neurons with
+// tcgen05.mma.cta_group::2 (M = 256, N = 256, K = 32): CTA r of the pair
+// stages activation rows m0 + 128 r .. + 127 and weight rows n0 + 128 r ..
+// + 127; the even CTA issues the MMAs, which read the A and B halves of both
+// CTAs at the same shared-memory offsets, and CTA r's TMEM receives D rows
+// 128 r .. + 127 for all 256 neurons (256 columns).  Per MAC each CTA expands
+// and the MMAs read a third less than with a one-CTA 128 x 256 tile.
+//   - producer warps: kRowSplit threads per stage row (128 activation rows,
+//     then 128 weight rows); per 128-element k-block a thread loads its
+//     16 / kRowSplit bytes of bits (kStages blocks ahead, in registers) and
+//     expands them into its chunks of the 6-stage ring of 32 KB stages;
+//     every producer warp arrives on its own CTA's "full" barrier;
+//   - in the odd CTA one relay thread waits on that barrier and forwards one
+//     arrival (cluster release) to the even CTA's, so no thread with bit
+//     loads in flight executes a cluster-scope release;
+//   - the even CTA's MMA thread waits on "full" (cluster acquire), issues four
+//     MMAs and commits to the "empty" barrier of both CTAs (multicast);
+//   - the epilogue: producer warps 0..7 read TMEM (warp w: lanes 32 (w % 4) ..,
+//     column blocks w / 4, w / 4 + 2, ..) and write the sign bits of their
+//     patterns as 32-bit pieces of the packed rows (pad bits 0);
+//   - both CTAs pass a cluster barrier after initialisation (no remote arrive
+//     or commit reaches an uninitialised barrier) and before releasing TMEM.
+// Every mbarrier wait is bounded; the first expiry stops every other wait of
+// the CTA and the kernel counts it in *timeouts, releases TMEM and returns.
 #include "tc_common.cuh"
 
 namespace bk {
@@ -24,19 +35,19 @@ namespace {
 
 using namespace tc;
 
-constexpr int TM = 128;
-constexpr int TN = 256;
-constexpr int kStages = 4;
-constexpr int kPrefetch = 4;  // == kStages: the stage of k-block kb0 + d is d
-constexpr int kProducers = TM + TN;  // one stage row per producer thread
+constexpr int TM = 128;                  // pattern rows per CTA (MMA M = 256 per pair)
+constexpr int TN = 256;                  // neurons per pair (MMA N)
+constexpr int TB = 128;                  // weight rows per CTA
+constexpr int kStages = 6;
+constexpr int kRowSplit = 1;             // producer threads per stage row
+constexpr int kProducers = (TM + TB) * kRowSplit;
 constexpr int kProdWarps = kProducers / 32;
 constexpr int THREADS = kProducers + 32;
-constexpr int A_BYTES = TM * KB;   // 16 KB
-constexpr int B_BYTES = TN * KB;   // 32 KB
+constexpr int A_BYTES = TM * KB;         // 16 KB
+constexpr int B_BYTES = TB * KB;         // 16 KB
 constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-constexpr int TMEM_COLS = 256;
-constexpr uint32_t kIdesc = idesc_f8(TM, TN);
-static_assert(kPrefetch == kStages, "stage index is the unrolled prefetch slot");
+constexpr int TMEM_COLS = TN;
+constexpr uint32_t kIdesc = idesc_f8(2 * TM, TN);
 
 struct __align__(8) EvShared {
   unsigned long long full[kStages];
@@ -59,54 +70,98 @@ __device__ __forceinline__ uint32_t e4m3_quad(uint32_t x) {
   return ((x & (0xFu << P)) * kMul & 0x80808080u) ^ 0xB8B8B8B8u;
 }
 
-// The row's 128 K-elements of one k-block (four 32-bit words, element e =
-// bit e % 32 of word e / 32) -> its eight chunks; chunk c (elements 16 c ..
-// 16 c + 15) goes to physical chunk c ^ swz.  Elements at index >= valid are
-// written 0 (valid < 128 only in the last k-block of a ragged K).
-__device__ __forceinline__ void expand_row(uint8_t* row, int swz, uint4 w, int valid) {
-  const uint32_t x[4] = {w.x, w.y, w.z, w.w};
-#pragma unroll
-  for (int c = 0; c < 8; ++c) {
-    const uint32_t h = x[c >> 1] >> (16 * (c & 1));
-    uint4 v = make_uint4(e4m3_quad<0>(h), e4m3_quad<4>(h), e4m3_quad<0>(h >> 8),
-                         e4m3_quad<4>(h >> 8));
-    if (valid < KB) {
-      const int n = valid - 16 * c;
-      v.x &= keep_mask(n);
-      v.y &= keep_mask(n - 4);
-      v.z &= keep_mask(n - 8);
-      v.w &= keep_mask(n - 12);
+// 16 K-elements (bits 0..15 of h) -> one 16-byte chunk.
+__device__ __forceinline__ uint4 chunk16(uint32_t h) {
+  return make_uint4(e4m3_quad<0>(h), e4m3_quad<4>(h), e4m3_quad<0>(h >> 8), e4m3_quad<4>(h >> 8));
+}
+
+// The same with the elements at index >= valid set to 0 (ragged K only).
+__device__ __forceinline__ uint4 chunk16_masked(uint32_t h, int valid) {
+  uint4 v = chunk16(h);
+  v.x &= keep_mask(valid);
+  v.y &= keep_mask(valid - 4);
+  v.z &= keep_mask(valid - 8);
+  v.w &= keep_mask(valid - 12);
+  return v;
+}
+
+// -------- the pair kernel -----------------------------------------------------
+__device__ __forceinline__ uint32_t pair_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+
+__device__ __forceinline__ void pair_sync() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;"
+               ::: "memory");
+}
+
+// Bounded wait with cluster-scope acquire (the barrier collects an arrival
+// from the peer CTA).
+__device__ __forceinline__ bool mbar_wait_cluster(unsigned long long* bar, uint32_t parity,
+                                                  volatile int* failed) {
+  const uint32_t a = smem_u32(bar);
+  const unsigned long long t0 = clock64();
+  while (true) {
+    uint32_t ok;
+    asm volatile(
+        "{\n .reg .pred p;\n mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n"
+        " selp.u32 %0, 1, 0, p;\n}"
+        : "=r"(ok) : "r"(a), "r"(parity) : "memory");
+    if (ok) return true;
+    if (*failed) return false;
+    if (clock64() - t0 > kWaitCycles) {
+      *failed = 1;
+      return false;
     }
-    *reinterpret_cast<uint4*>(row + 16 * (c ^ swz)) = v;
   }
 }
 
-// Bits of k-block kb of a row (words 2 kb, 2 kb + 1; 0 past the nw words).
-template <bool kVec>
-__device__ __forceinline__ uint4 load_block(const uint64_t* src, int kb, int nkb, int nw) {
-  if (src == nullptr || kb >= nkb) return make_uint4(0, 0, 0, 0);
-  if (kVec) return __ldg(reinterpret_cast<const uint4*>(src) + kb);
-  const uint64_t lo = __ldg(src + 2 * kb);
-  const uint64_t hi = 2 * kb + 1 < nw ? __ldg(src + 2 * kb + 1) : 0ull;
-  return make_uint4((uint32_t)lo, (uint32_t)(lo >> 32), (uint32_t)hi, (uint32_t)(hi >> 32));
+// Arrive on the barrier at the same offset in CTA 0 of the cluster.
+__device__ __forceinline__ void mbar_arrive_rank0(unsigned long long* bar) {
+  uint32_t remote;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, 0;" : "=r"(remote) : "r"(smem_u32(bar)));
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(remote) : "memory");
 }
 
-// kVec: nw even and both operands 16-byte aligned (every row then is)
+__device__ __forceinline__ void mma_f8_pair(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc,
+                                            uint32_t accumulate) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::2.kind::f8f6f4 [%0], %1, %2, %3, p;\n}"
+      ::"r"(tmem_d), "l"(adesc), "l"(bdesc), "r"(kIdesc), "r"(accumulate));
+}
+
+// Arrive once on the barrier at this offset in both CTAs of the pair when the
+// MMAs issued so far complete.
+__device__ __forceinline__ void mma_commit_pair(unsigned long long* bar) {
+  const uint16_t mask = 0x3;
+  asm volatile(
+      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;"
+      ::"r"(smem_u32(bar)), "h"(mask) : "memory");
+}
+
+// kVec: nw even and both operands 16-byte aligned (every row then is); with
+// one thread per row its two words of a k-block are then one 16-byte load
 template <bool kVec>
-__global__ void __launch_bounds__(THREADS, 1)
-    k_forward_eval_tc(const uint64_t* __restrict__ A, int64_t M, int nw, const uint64_t* __restrict__ W,
-                      int N, int Kin, uint64_t* __restrict__ Aout, int nw_out,
-                      unsigned int* __restrict__ timeouts) {
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
+    k_forward_eval_tc(const uint64_t* __restrict__ A, int64_t M, int nw,
+                      const uint64_t* __restrict__ W, int N, int Kin, uint64_t* __restrict__ Aout,
+                      int nw_out, unsigned int* __restrict__ timeouts) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* base = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   EvShared* sh = reinterpret_cast<EvShared*>(base + kStages * STAGE_BYTES);
-  const int64_t m0 = (int64_t)blockIdx.y * TM;
-  const int MR = (int)min((int64_t)TM, M - m0);   // pattern rows of this CTA
-  const int n0 = blockIdx.x * TN;
-  const int NB = min(TN, N - n0);                 // neuron rows of this CTA
+  const uint32_t rank = pair_rank();
+  // neuron tiles vary fastest: the pairs in flight share a tile of patterns,
+  // and the layer's packed W (8 MB at 8192 x 8192) stays in L2
+  const int64_t m0 = (int64_t)blockIdx.y * (2 * TM) + (int64_t)rank * TM;  // this CTA's patterns
+  const int MR = (int)max((int64_t)0, min((int64_t)TM, M - m0));
+  const int n0 = (int)(blockIdx.x >> 1) * TN;                               // the pair's neurons
+  const int nb0 = n0 + (int)rank * TB;                                      // this CTA's weight rows
+  const int NB = max(0, min(TB, N - nb0));
   const int nkb = (Kin + KB - 1) / KB;
-  const int tail = Kin - KB * (nkb - 1);          // valid elements of the last k-block
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   volatile int* failed = &sh->failed;
 
@@ -115,12 +170,13 @@ __global__ void __launch_bounds__(THREADS, 1)
     for (int i = MR * (KB / 16) + threadIdx.x; i < TM * (KB / 16); i += THREADS)
       a4[i] = make_uint4(0, 0, 0, 0);
     uint4* b4 = reinterpret_cast<uint4*>(base + s * STAGE_BYTES + A_BYTES);
-    for (int i = NB * (KB / 16) + threadIdx.x; i < TN * (KB / 16); i += THREADS)
+    for (int i = NB * (KB / 16) + threadIdx.x; i < TB * (KB / 16); i += THREADS)
       b4[i] = make_uint4(0, 0, 0, 0);
   }
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
-      mbar_init(&sh->full[s], kProdWarps);  // one arrival per producer warp
+      // the producer warps and, on the even CTA, the odd CTA's relayed arrival
+      mbar_init(&sh->full[s], kProdWarps + (rank == 0 ? 1 : 0));
       mbar_init(&sh->empty[s], 1);
     }
     mbar_init(&sh->done, 1);
@@ -128,68 +184,110 @@ __global__ void __launch_bounds__(THREADS, 1)
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   if (warp == 0) {
-    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;"
+    asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;"
                  ::"r"(smem_u32(&sh->tmem_base)), "r"(TMEM_COLS) : "memory");
-    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
   }
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
   asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-  __syncthreads();
+  pair_sync();
   asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
   const uint32_t tmem = sh->tmem_base;
 
   if (threadIdx.x < kProducers) {
-    // this thread's stage row: activation row p (p < TM) or weight row p - TM
-    const int p = threadIdx.x;
+    // stage row p (activation row p < TM, else weight row p - TM), part `part`
+    // of its 128 K-elements per k-block: chunks kCh part .. kCh part + kCh - 1
+    constexpr int kCh = 8 / kRowSplit;          // 16-byte chunks per thread and stage
+    constexpr int kWords = 2 / kRowSplit > 0 ? 2 / kRowSplit : 1;
+    const int p = threadIdx.x / kRowSplit, part = threadIdx.x % kRowSplit;
     const bool isA = p < TM;
     const int r = isA ? p : p - TM;
     const uint64_t* src = nullptr;
     if (isA && r < MR) src = A + (m0 + r) * nw;
-    if (!isA && r < NB) src = W + (int64_t)(n0 + r) * nw;
+    if (!isA && r < NB) src = W + (int64_t)(nb0 + r) * nw;
     const uint32_t row_off = (isA ? 0u : (uint32_t)A_BYTES) + (uint32_t)(r * KB);
     const int swz = r & 7;
-
-    uint4 pre[kPrefetch];
+    // bits of k-block kb for this thread: words 2 kb + kWords part .. (0 past nw)
+    auto load = [&](int kb) -> uint4 {
+      uint4 v = make_uint4(0, 0, 0, 0);
+      if (src == nullptr || kb >= nkb) return v;
+      if (kVec && kWords == 2) return __ldg(reinterpret_cast<const uint4*>(src) + kb);
+      const int w0 = 2 * kb + kWords * part;
+      const uint64_t lo = w0 < nw ? __ldg(src + w0) : 0ull;
+      v.x = (uint32_t)lo;
+      v.y = (uint32_t)(lo >> 32);
+      if (kWords == 2) {
+        const uint64_t hi = w0 + 1 < nw ? __ldg(src + w0 + 1) : 0ull;
+        v.z = (uint32_t)hi;
+        v.w = (uint32_t)(hi >> 32);
+      }
+      return v;
+    };
+    uint4 pre[kStages];
 #pragma unroll
-    for (int d = 0; d < kPrefetch; ++d) pre[d] = load_block<kVec>(src, d, nkb, nw);
+    for (int d = 0; d < kStages; ++d) pre[d] = load(d);
 
-    for (int kb0 = 0; kb0 < nkb; kb0 += kPrefetch) {
+    for (int kb0 = 0; kb0 < nkb; kb0 += kStages) {
 #pragma unroll
-      for (int d = 0; d < kPrefetch; ++d) {
+      for (int d = 0; d < kStages; ++d) {  // the stage of k-block kb0 + d is d
         const int kb = kb0 + d;
         if (kb >= nkb) break;
         if (kb0 > 0 &&
             !__all_sync(kFull, mbar_wait(&sh->empty[d], (uint32_t)((kb0 / kStages - 1) & 1), failed)))
           break;
-        if (src != nullptr)
-          expand_row(base + d * STAGE_BYTES + row_off, swz, pre[d], kb == nkb - 1 ? tail : KB);
-        pre[d] = load_block<kVec>(src, kb + kPrefetch, nkb, nw);
+        if (src != nullptr) {
+          uint8_t* row = base + d * STAGE_BYTES + row_off;
+          const uint32_t x[4] = {pre[d].x, pre[d].y, pre[d].z, pre[d].w};
+          const int valid = Kin - KB * kb - 16 * kCh * part;
+          if (valid >= 16 * kCh) {
+#pragma unroll
+            for (int q = 0; q < kCh; ++q) {
+              const int c = kCh * part + q;
+              *reinterpret_cast<uint4*>(row + 16 * (c ^ swz)) = chunk16(x[q >> 1] >> (16 * (q & 1)));
+            }
+          } else {
+#pragma unroll
+            for (int q = 0; q < kCh; ++q) {
+              const int c = kCh * part + q;
+              *reinterpret_cast<uint4*>(row + 16 * (c ^ swz)) =
+                  chunk16_masked(x[q >> 1] >> (16 * (q & 1)), valid - 16 * q);
+            }
+          }
+        }
+        pre[d] = load(kb + kStages);
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
         __syncwarp();
         if (lane == 0) mbar_arrive(&sh->full[d]);
       }
       if (__any_sync(kFull, *failed != 0)) break;
     }
-  } else if (threadIdx.x == kProducers) {
-    // MMA issuer: lane 0 of the last warp
+  } else if (threadIdx.x == kProducers && rank == 0) {
+    // MMA issuer of the pair: lane 0 of the even CTA's last warp
     for (int kb = 0; kb < nkb; ++kb) {
       const int s = kb % kStages;
-      if (!mbar_wait(&sh->full[s], (uint32_t)((kb / kStages) & 1), failed)) break;
+      if (!mbar_wait_cluster(&sh->full[s], (uint32_t)((kb / kStages) & 1), failed)) break;
       asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
       const uint8_t* sa = base + s * STAGE_BYTES;
       const uint64_t ad = smem_desc(smem_u32(sa));
       const uint64_t bd = smem_desc(smem_u32(sa + A_BYTES));
 #pragma unroll
       for (int j = 0; j < KB / 32; ++j)
-        mma_f8<kIdesc>(tmem, ad + 2 * j, bd + 2 * j, (kb > 0 || j > 0) ? 1u : 0u);
-      mma_commit(&sh->empty[s]);
+        mma_f8_pair(tmem, ad + 2 * j, bd + 2 * j, (kb > 0 || j > 0) ? 1u : 0u);
+      mma_commit_pair(&sh->empty[s]);
     }
-    if (!*failed) mma_commit(&sh->done);
+    if (!*failed) mma_commit_pair(&sh->done);
+  } else if (threadIdx.x == kProducers) {
+    // relay of the odd CTA: its stage is full -> one arrival on the even CTA's
+    for (int kb = 0; kb < nkb; ++kb) {
+      const int s = kb % kStages;
+      if (!mbar_wait(&sh->full[s], (uint32_t)((kb / kStages) & 1), failed)) break;
+      mbar_arrive_rank0(&sh->full[s]);
+    }
   }
 
-  // epilogue: tcgen05.ld is warp-collective, so the decision is per warp
+  // epilogue: this CTA's 128 rows of D, all 256 neurons
   bool go = false;
-  if (threadIdx.x < kProducers) {
+  if (warp < 8) {
     go = !*failed && mbar_wait(&sh->done, 0, failed);
     go = __all_sync(0xffffffffu, go);
   }
@@ -197,7 +295,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
     const int sub = warp & 3;
     const int m = 32 * sub + lane;
-    for (int cb = warp >> 2; cb < TN / 32; cb += kProdWarps / 4) {
+    for (int cb = warp >> 2; cb < TN / 32; cb += 2) {
       const int col0 = 32 * cb;
       uint32_t v[32];
       asm volatile(
@@ -223,10 +321,11 @@ __global__ void __launch_bounds__(THREADS, 1)
     }
   }
   asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-  __syncthreads();
+  pair_sync();   // no CTA releases TMEM or leaves while its peer may still use the pair
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
   if (threadIdx.x == 0 && *failed) atomicAdd(timeouts, 1u);
   if (warp == 0)
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(TMEM_COLS) : "memory");
+    asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(TMEM_COLS) : "memory");
 }
 
 }  // namespace
@@ -242,15 +341,15 @@ cudaError_t prepare_forward_eval_tc() {
 void launch_forward_eval_tc(const uint64_t* A, int64_t M, int nw_in, const uint64_t* W, int N,
                             int Kin, uint64_t* Aout, int nw_out, unsigned int* timeouts,
                             cudaStream_t st) {
-  const dim3 grid((unsigned)((N + TN - 1) / TN), (unsigned)((M + TM - 1) / TM));
+  const dim3 grid((unsigned)(2 * ((N + TN - 1) / TN)), (unsigned)((M + 2 * TM - 1) / (2 * TM)));
   const bool vec = (nw_in % 2 == 0) && (reinterpret_cast<uintptr_t>(A) % 16 == 0) &&
                    (reinterpret_cast<uintptr_t>(W) % 16 == 0);
   if (vec)
-    k_forward_eval_tc<true><<<grid, THREADS, kSmemBytes, st>>>(A, M, nw_in, W, N, Kin, Aout,
-                                                                nw_out, timeouts);
+    k_forward_eval_tc<true><<<grid, THREADS, kSmemBytes, st>>>(A, M, nw_in, W, N, Kin, Aout, nw_out,
+                                                                timeouts);
   else
-    k_forward_eval_tc<false><<<grid, THREADS, kSmemBytes, st>>>(A, M, nw_in, W, N, Kin, Aout,
-                                                                 nw_out, timeouts);
+    k_forward_eval_tc<false><<<grid, THREADS, kSmemBytes, st>>>(A, M, nw_in, W, N, Kin, Aout, nw_out,
+                                                                 timeouts);
 }
 
 }  // namespace bk
