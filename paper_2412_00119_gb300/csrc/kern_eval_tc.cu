@@ -36,18 +36,19 @@ namespace {
 using namespace tc;
 
 constexpr int TM = 128;                  // pattern rows per CTA (MMA M = 256 per pair)
-constexpr int TN = 256;                  // neurons per pair (MMA N)
-constexpr int TB = 128;                  // weight rows per CTA
-constexpr int kStages = 6;
+constexpr int kHalves = 2;               // N = 256 MMAs per k-step (TMEM column ranges)
+constexpr int TN = 256 * kHalves;        // neurons per pair
+constexpr int TB = 128 * kHalves;        // weight rows per CTA
+constexpr int kStages = 4;
 constexpr int kRowSplit = 1;             // producer threads per stage row
 constexpr int kProducers = (TM + TB) * kRowSplit;
 constexpr int kProdWarps = kProducers / 32;
 constexpr int THREADS = kProducers + 32;
 constexpr int A_BYTES = TM * KB;         // 16 KB
-constexpr int B_BYTES = TB * KB;         // 16 KB
+constexpr int B_BYTES = TB * KB;         // 16 KB per N half
 constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
 constexpr int TMEM_COLS = TN;
-constexpr uint32_t kIdesc = idesc_f8(2 * TM, TN);
+constexpr uint32_t kIdesc = idesc_f8(2 * TM, 256);
 
 struct __align__(8) EvShared {
   unsigned long long full[kStages];
@@ -159,8 +160,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
   const int64_t m0 = (int64_t)blockIdx.y * (2 * TM) + (int64_t)rank * TM;  // this CTA's patterns
   const int MR = (int)max((int64_t)0, min((int64_t)TM, M - m0));
   const int n0 = (int)(blockIdx.x >> 1) * TN;                               // the pair's neurons
-  const int nb0 = n0 + (int)rank * TB;                                      // this CTA's weight rows
-  const int NB = max(0, min(TB, N - nb0));
+  // weight row q of this CTA (block q / 128 of the B stage) is neuron
+  // n0 + 256 (q / 128) + 128 rank + q % 128: half h of the pair's MMAs covers
+  // neurons n0 + 256 h .. + 255, 128 from each CTA
+  auto neuron_of = [&](int q) { return n0 + 256 * (q >> 7) + 128 * (int)rank + (q & 127); };
   const int nkb = (Kin + KB - 1) / KB;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   volatile int* failed = &sh->failed;
@@ -170,8 +173,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
     for (int i = MR * (KB / 16) + threadIdx.x; i < TM * (KB / 16); i += THREADS)
       a4[i] = make_uint4(0, 0, 0, 0);
     uint4* b4 = reinterpret_cast<uint4*>(base + s * STAGE_BYTES + A_BYTES);
-    for (int i = NB * (KB / 16) + threadIdx.x; i < TB * (KB / 16); i += THREADS)
-      b4[i] = make_uint4(0, 0, 0, 0);
+    for (int i = threadIdx.x; i < TB * (KB / 16); i += THREADS)
+      if (neuron_of(i / (KB / 16)) >= N) b4[i] = make_uint4(0, 0, 0, 0);
   }
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
@@ -204,7 +207,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
     const int r = isA ? p : p - TM;
     const uint64_t* src = nullptr;
     if (isA && r < MR) src = A + (m0 + r) * nw;
-    if (!isA && r < NB) src = W + (int64_t)(nb0 + r) * nw;
+    if (!isA && neuron_of(r) < N) src = W + (int64_t)neuron_of(r) * nw;
     const uint32_t row_off = (isA ? 0u : (uint32_t)A_BYTES) + (uint32_t)(r * KB);
     const int swz = r & 7;
     // bits of k-block kb for this thread: words 2 kb + kWords part .. (0 past nw)
@@ -269,10 +272,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
       asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
       const uint8_t* sa = base + s * STAGE_BYTES;
       const uint64_t ad = smem_desc(smem_u32(sa));
-      const uint64_t bd = smem_desc(smem_u32(sa + A_BYTES));
 #pragma unroll
       for (int j = 0; j < KB / 32; ++j)
-        mma_f8_pair(tmem, ad + 2 * j, bd + 2 * j, (kb > 0 || j > 0) ? 1u : 0u);
+#pragma unroll
+        for (int h = 0; h < kHalves; ++h)
+          mma_f8_pair(tmem + 256u * (uint32_t)h, ad + 2 * j,
+                      smem_desc(smem_u32(sa + A_BYTES + h * (B_BYTES / kHalves))) + 2 * j,
+                      (kb > 0 || j > 0) ? 1u : 0u);
       mma_commit_pair(&sh->empty[s]);
     }
     if (!*failed) mma_commit_pair(&sh->done);
@@ -285,7 +291,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
     }
   }
 
-  // epilogue: this CTA's 128 rows of D, all 256 neurons
+  // epilogue: this CTA's 128 rows of D, all TN neurons (TMEM column c = neuron n0 + c)
   bool go = false;
   if (warp < 8) {
     go = !*failed && mbar_wait(&sh->done, 0, failed);
