@@ -235,6 +235,17 @@ int bmlp_reinforce_tables(double p_r, int32_t K, int32_t n, uint64_t* any_out,
 int bmlp_debug_last_step(const bmlp_t* h, int32_t layer, int16_t* Z, uint64_t* A,
                          uint8_t* mark, int16_t* sel);
 
+/* Failure-path probe of the bounded device waits (no counterpart in the
+ * paper): one CTA initialises an mbarrier and waits on its first phase with
+ * the same bounded wait the tensor-core kernels use, limited to `seconds`
+ * (0 < seconds <= 10) of SM clock.  arrive != 0: one arrival completes the
+ * phase first, so the wait succeeds.  arrive == 0: nothing arrives, the wait
+ * gives up when the limit expires, the kernel counts it as a timeout and
+ * returns (no trap, no fault; the context stays usable).  Synchronises, then
+ * returns BMLP_ETIMEOUT if any timeout is pending (and clears it), else
+ * BMLP_OK. */
+int bmlp_debug_wait_probe(bmlp_t* h, int32_t arrive, double seconds);
+
 /* Per-kernel timing.  every = 0: off.  every = S > 0: every S-th training
  * mini-batch (counted by the step counter t) and every evaluation launch is
  * enqueued kernel by kernel between two CUDA events on the caller's stream; the

@@ -79,6 +79,7 @@ SIGNATURES = [
     ("bmlp_predict_layers", C.c_int, [_vp, _vp, C.c_int64, _vp, _vp]),
     ("bmlp_layer_errors", C.c_int, [_vp, _i64p, C.c_int32]),
     ("bmlp_binarize_median", C.c_int, [_vp, C.c_int64, C.c_int32, _vp, _vp]),
+    ("bmlp_debug_wait_probe", C.c_int, [_vp, C.c_int32, C.c_double]),
 ]
 
 
@@ -203,6 +204,11 @@ def bmlp_binarize_median(x, out, stream=None):
     """Median binarisation of n x K fp32 patterns (device) into packed bits."""
     n, K = x.shape
     _check(lib().bmlp_binarize_median(_ptr(x), n, K, _ptr(out), _stream(stream)), None)
+
+
+def bmlp_debug_wait_probe(h, arrive, seconds=0.05):
+    """Run the bounded-wait probe; raises BmlpError(BMLP_ETIMEOUT) if it expired."""
+    _check(lib().bmlp_debug_wait_probe(h, 1 if arrive else 0, float(seconds)), h)
 
 
 def bmlp_layer_forward(h, layer, a_in, a_out, n=None, stream=None):

@@ -862,6 +862,25 @@ int bmlp_layer_forward(bmlp_t* h, int32_t layer, const uint64_t* a_in, int64_t n
   return prof_collect(h, st);
 }
 
+int bmlp_debug_wait_probe(bmlp_t* h, int32_t arrive, double seconds) {
+  if (!h) return BMLP_EINVAL;
+  h->err.clear();
+  if (!(seconds > 0.0) || seconds > 10.0) return fail(h, BMLP_EINVAL, "seconds must be in (0, 10]");
+  int khz = 0;
+  CK(h, cudaDeviceGetAttribute(&khz, cudaDevAttrClockRate, h->device));
+  const unsigned long long limit = (unsigned long long)(seconds * 1e3 * (double)khz);
+  launch_wait_probe(&h->dCtrl->timeouts, arrive ? 1 : 0, limit, 0);
+  CK(h, cudaGetLastError());
+  CK(h, cudaDeviceSynchronize());
+  uint32_t t = 0;
+  CK(h, cudaMemcpy(&t, &h->dCtrl->timeouts, sizeof(t), cudaMemcpyDeviceToHost));
+  if (t != 0) {
+    CK(h, cudaMemset(&h->dCtrl->timeouts, 0, sizeof(uint32_t)));
+    return fail(h, BMLP_ETIMEOUT, "a bounded device-side wait expired");
+  }
+  return BMLP_OK;
+}
+
 int bmlp_debug_last_step(const bmlp_t* hc, int32_t layer, int16_t* Z, uint64_t* A, uint8_t* mark,
                          int16_t* sel) {
   bmlp_t* h = const_cast<bmlp_t*>(hc);

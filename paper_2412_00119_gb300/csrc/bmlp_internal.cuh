@@ -227,6 +227,10 @@ void launch_binarize_median(const float* x, int64_t n, int K, int nw, uint64_t* 
 // (M x nw_out), 256-pattern x 256-neuron tiles per CTA pair; an expired
 // bounded wait adds one to *timeouts.
 cudaError_t prepare_forward_eval_tc();
+// One CTA waiting (bounded by limit_cycles) on an mbarrier that completes only
+// with arrive != 0; an expired wait adds one to *timeouts.
+void launch_wait_probe(unsigned int* timeouts, int arrive, unsigned long long limit_cycles,
+                       cudaStream_t st);
 void launch_forward_eval_tc(const uint64_t* A, int64_t M, int nw_in, const uint64_t* W, int N,
                             int Kin, uint64_t* Aout, int nw_out, unsigned int* timeouts,
                             cudaStream_t st);

@@ -334,7 +334,27 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
     asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(TMEM_COLS) : "memory");
 }
 
+// Failure-path probe: the bounded mbarrier wait of the kernels above on a
+// barrier whose phase completes only if `arrive` (one arrival before the wait).
+__global__ void k_wait_probe(unsigned int* __restrict__ timeouts, int arrive,
+                             unsigned long long limit) {
+  __shared__ unsigned long long bar;
+  __shared__ int failed;
+  if (threadIdx.x == 0) {
+    mbar_init(&bar, 1);
+    failed = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    if (arrive) mbar_arrive(&bar);
+    if (!mbar_wait(&bar, 0, &failed, limit)) atomicAdd(timeouts, 1u);
+  }
+}
+
 }  // namespace
+
+void launch_wait_probe(unsigned int* timeouts, int arrive, unsigned long long limit_cycles,
+                       cudaStream_t st) {
+  k_wait_probe<<<1, 32, 0, st>>>(timeouts, arrive, limit_cycles);
+}
 
 cudaError_t prepare_forward_eval_tc() {
   cudaError_t e = cudaFuncSetAttribute(k_forward_eval_tc<true>,

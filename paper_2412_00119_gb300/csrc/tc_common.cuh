@@ -26,10 +26,11 @@ __device__ __forceinline__ void mbar_arrive(unsigned long long* bar) {
                ::"r"(smem_u32(bar)) : "memory");
 }
 
-// Bounded wait for the phase with the given parity; false on expiry or when
-// another thread already recorded a failure.
+// Bounded wait for the phase with the given parity; false on expiry (after
+// `limit` SM clock cycles) or when another thread already recorded a failure.
 __device__ __forceinline__ bool mbar_wait(unsigned long long* bar, uint32_t parity,
-                                          volatile int* failed) {
+                                          volatile int* failed,
+                                          unsigned long long limit = kWaitCycles) {
   const uint32_t a = smem_u32(bar);
   const unsigned long long t0 = clock64();
   while (true) {
@@ -40,7 +41,7 @@ __device__ __forceinline__ bool mbar_wait(unsigned long long* bar, uint32_t pari
         : "=r"(ok) : "r"(a), "r"(parity) : "memory");
     if (ok) return true;
     if (*failed) return false;
-    if (clock64() - t0 > kWaitCycles) {
+    if (clock64() - t0 > limit) {
       *failed = 1;
       return false;
     }

@@ -97,6 +97,7 @@ def test_null_handle_calls_fail_cleanly():
     lib = pkg.lib()
     assert lib.bmlp_predict_layers(None, None, 0, None, None) == B.BMLP_EINVAL
     assert lib.bmlp_layer_errors(None, None, 0) == B.BMLP_EINVAL
+    assert lib.bmlp_debug_wait_probe(None, 0, 0.05) == B.BMLP_EINVAL
     assert lib.bmlp_train(None, None, None, 0, 0, None, None) == B.BMLP_EINVAL
     assert lib.bmlp_predict(None, None, 0, None, None) == B.BMLP_EINVAL
     assert lib.bmlp_get_state(None, 1, None, None, None, None, None) == B.BMLP_EINVAL

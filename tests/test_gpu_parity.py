@@ -395,3 +395,18 @@ def test_update_stats_count_rows_and_bytes():
     assert nbytes >= streamed * min(row_bytes) and (nbytes - streamed * min(row_bytes)) % 4 == 0
     assert B.bmlp_update_stats(gpu.h) == (0, 0, 0)
     gpu.close()
+
+
+def test_bounded_wait_expiry_is_reported_and_recoverable():
+    """Failure handling without a fault: a bounded mbarrier wait on a phase that
+    nothing completes gives up after 50 ms and is reported as BMLP_ETIMEOUT;
+    the same wait with its arrival succeeds; training and evaluation on the
+    same context afterwards still match the oracle."""
+    gpu = B.BMLP((64, 64), 4, seed=3, bs=32, fwd_impl=B.BMLP_FWD_TCGEN05)
+    with pytest.raises(B.BmlpError) as ei:
+        B.bmlp_debug_wait_probe(gpu.h, arrive=False, seconds=0.05)
+    assert ei.value.code == B.BMLP_ETIMEOUT
+    B.bmlp_debug_wait_probe(gpu.h, arrive=True, seconds=0.05)
+    gpu.close()
+    g2, _ = run_pair(widths=(130, 96), classes=5, n_train=200, bs=50, fwd=B.BMLP_FWD_TCGEN05)
+    g2.close()
