@@ -892,7 +892,13 @@ int bmlp_debug_last_step(const bmlp_t* hc, int32_t layer, int16_t* Z, uint64_t* 
   if (Z) CK(h, cudaMemcpy(Z, D.Z, sizeof(int16_t) * h->bs * D.Kout, cudaMemcpyDeviceToHost));
   if (A) CK(h, cudaMemcpy(A, D.A, sizeof(uint64_t) * h->bs * D.nw_out, cudaMemcpyDeviceToHost));
   if (mark) CK(h, cudaMemcpy(mark, D.mark, (size_t)h->bs, cudaMemcpyDeviceToHost));
-  if (sel) CK(h, cudaMemcpy(sel, D.sel, sizeof(int16_t) * h->bs * D.G, cudaMemcpyDeviceToHost));
+  if (sel) {
+    // device layout [G][bs] -> the documented [bs][G]
+    std::vector<int16_t> t((size_t)h->bs * D.G);
+    CK(h, cudaMemcpy(t.data(), D.sel, sizeof(int16_t) * t.size(), cudaMemcpyDeviceToHost));
+    for (int g = 0; g < D.G; ++g)
+      for (int m = 0; m < h->bs; ++m) sel[(size_t)m * D.G + g] = t[(size_t)g * h->bs + m];
+  }
   return BMLP_OK;
 }
 

@@ -41,7 +41,7 @@ struct DevLayer {
   int16_t* Z;
   uint64_t* A;
   uint8_t* mark;
-  int16_t* sel;
+  int16_t* sel;       // [G][bs] selected neuron per group and pattern, or -1 (group-major)
   uint8_t* AE;
   int16_t* member;    // [K_out] group order (neuron at position j), or null: contiguous groups
   int16_t* group_of;  // [K_out] group of neuron k (with member)

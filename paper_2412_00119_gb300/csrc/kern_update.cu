@@ -82,9 +82,12 @@ __global__ void __launch_bounds__(kClsThreads) k_cls_select(const StepParams* __
   }
   __syncthreads();
 
-  int16_t* sel = Ly.sel + (int64_t)mu * Ly.G;
+  // selections are stored group-major (sel[g][mu]): the update kernel reads a
+  // group's bs selections as one contiguous run
+  int16_t* sel = Ly.sel + mu;
+  const int64_t sstride = P->bs;
   if (!s_mark) {
-    for (int g = threadIdx.x; g < Ly.G; g += blockDim.x) sel[g] = -1;
+    for (int g = threadIdx.x; g < Ly.G; g += blockDim.x) sel[g * sstride] = -1;
     return;
   }
   const int y = s_y;
@@ -124,7 +127,7 @@ __global__ void __launch_bounds__(kClsThreads) k_cls_select(const StepParams* __
         }
       }
       if (ci < nchunk && (ci & (per - 1)) == 0)
-        sel[ci / per] = (bestd == INT_MIN) ? (int16_t)-1 : (int16_t)bestk;
+        sel[(ci / per) * sstride] = (bestd == INT_MIN) ? (int16_t)-1 : (int16_t)bestk;
     }
     return;
   }
@@ -150,7 +153,7 @@ __global__ void __launch_bounds__(kClsThreads) k_cls_select(const StepParams* __
         bestk = ok;
       }
     }
-    if (lane == 0) sel[g] = (bestd == INT_MIN) ? (int16_t)-1 : (int16_t)bestk;
+    if (lane == 0) sel[g * sstride] = (bestd == INT_MIN) ? (int16_t)-1 : (int16_t)bestk;
   }
 }
 
@@ -475,7 +478,7 @@ __global__ void __launch_bounds__(kUpdThreads, 4) k_update(const StepParams* __r
       int n_t = 0;
       for (int mb = 0; mb < bsz; mb += 32) {
         const int m = mb + lane;
-        const bool hit = (m < bsz) && (Ly.sel[(int64_t)m * Ly.G + g] == k);
+        const bool hit = (m < bsz) && (Ly.sel[(int64_t)g * P->bs + m] == k);
         const unsigned bal = __ballot_sync(kFull, hit);
         if (hit) {
           int yv = P->y[start + m];
