@@ -52,8 +52,8 @@ EVAL_BATCH = 65_536
 # of this bench (dram__bytes_read.sum + dram__bytes_write.sum, one pass; see
 # profiles/k_update_c5.md), valid while the kernel source hashes to
 # UPDATE_TRAFFIC_SRC_SHA; otherwise reported as null.
-UPDATE_TRAFFIC_BYTES = 463_731_456 + 384_116_992  # dram read + write of one timed-region launch (ncu)
-UPDATE_TRAFFIC_SRC_SHA = "2ef29d2006466a1b"
+UPDATE_TRAFFIC_BYTES = 463_731_712 + 383_939_840  # dram read + write of one timed-region launch (ncu)
+UPDATE_TRAFFIC_SRC_SHA = "8d7fd0f8e4d76002"
 
 
 def bitpairs_per_sample(widths, classes):
