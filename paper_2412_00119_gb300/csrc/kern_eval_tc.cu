@@ -4,23 +4,27 @@
 // Same exact e4m3 formulation as the training forward (+-1 -> 0x38 / 0xB8,
 // pads 0, fp32 sums exact), tiled for large batches.
 //
-// Tile.  A cluster of two CTAs computes 256 patterns x 256 neurons with
-// tcgen05.mma.cta_group::2 (M = 256, N = 256, K = 32): CTA r of the pair
-// stages activation rows m0 + 128 r .. + 127 and weight rows n0 + 128 r ..
-// + 127; the even CTA issues the MMAs, which read the A and B halves of both
-// CTAs at the same shared-memory offsets, and CTA r's TMEM receives D rows
-// 128 r .. + 127 for all 256 neurons (256 columns).  Per MAC each CTA expands
-// and the MMAs read a third less than with a one-CTA 128 x 256 tile.
+// Tile.  A cluster of two CTAs computes 256 patterns x 512 neurons with
+// tcgen05.mma.cta_group::2 (M = 256, N = 256, K = 32), two MMAs per 32-element
+// k-step, one per N half (neurons n0 .. n0 + 255 and n0 + 256 .. n0 + 511):
+// CTA r of the pair stages activation rows m0 + 128 r .. + 127 and, for half
+// h, weight rows n0 + 256 h + 128 r .. + 127; the even CTA issues the MMAs,
+// which read the A and B halves of both CTAs at the same shared-memory
+// offsets, and CTA r's TMEM receives D rows 128 r .. + 127 for all 512
+// neurons (all 512 columns; column c is neuron n0 + c).  Each CTA stages 384
+// rows per 128 x 512 outputs, against 384 per 128 x 256 with one CTA: the
+// expansion, not the tensor core, sets the pace.
 //   - producer warps: kRowSplit threads per stage row (128 activation rows,
-//     then 128 weight rows); per 128-element k-block a thread loads its
+//     then 256 weight rows); per 128-element k-block a thread loads its
 //     16 / kRowSplit bytes of bits (kStages blocks ahead, in registers) and
-//     expands them into its chunks of the 6-stage ring of 32 KB stages;
+//     expands them into its chunks of the 4-stage ring of 48 KB stages;
 //     every producer warp arrives on its own CTA's "full" barrier;
 //   - in the odd CTA one relay thread waits on that barrier and forwards one
 //     arrival (cluster release) to the even CTA's, so no thread with bit
 //     loads in flight executes a cluster-scope release;
-//   - the even CTA's MMA thread waits on "full" (cluster acquire), issues four
-//     MMAs and commits to the "empty" barrier of both CTAs (multicast);
+//   - the even CTA's MMA thread waits on "full" (cluster acquire), issues the
+//     eight MMAs of the stage and commits to the "empty" barrier of both CTAs
+//     (multicast);
 //   - the epilogue: producer warps 0..7 read TMEM (warp w: lanes 32 (w % 4) ..,
 //     column blocks w / 4, w / 4 + 2, ..) and write the sign bits of their
 //     patterns as 32-bit pieces of the packed rows (pad bits 0);
@@ -45,7 +49,7 @@ constexpr int kProducers = (TM + TB) * kRowSplit;
 constexpr int kProdWarps = kProducers / 32;
 constexpr int THREADS = kProducers + 32;
 constexpr int A_BYTES = TM * KB;         // 16 KB
-constexpr int B_BYTES = TB * KB;         // 16 KB per N half
+constexpr int B_BYTES = TB * KB;         // 32 KB: 16 KB per N half
 constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
 constexpr int TMEM_COLS = TN;
 constexpr uint32_t kIdesc = idesc_f8(2 * TM, 256);
