@@ -53,7 +53,11 @@ constexpr int TN = 256;           // MMA N: neurons per tile
 constexpr int kSplit = 4;         // CTAs per cluster, each a quarter of K
 constexpr int kStages = 4;
 constexpr int kPrefetch = 4;      // stages of bit-words held in registers ahead
-constexpr int kProducers = 512;   // 16 warps
+constexpr int kProducers = 512;   // 16 warps: the epilogue's partial and reduction
+// producer warps of the mainloop: one thread per stage row -- 256 weight rows,
+// plus 128 input rows on layer 1
+template <bool kTiles>
+constexpr int kRowWarps = kTiles ? 8 : 12;
 constexpr int THREADS = kProducers + 32;
 constexpr int A_BYTES = TM * KB;  // 16 KB
 constexpr int B_BYTES = TN * KB;  // 32 KB
@@ -170,9 +174,9 @@ __global__ void __cluster_dims__(kSplit, 1, 1) __launch_bounds__(THREADS, 1)
   }
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
-      // one arrival per producer warp, plus (kTiles) the tile copy's
+      // one arrival per row-producer warp, plus (kTiles) the tile copy's
       // expect_tx arrival
-      mbar_init(&sh->full[s], kProducers / 32 + (kTiles ? 1 : 0));
+      mbar_init(&sh->full[s], kRowWarps<kTiles> + (kTiles ? 1 : 0));
       mbar_init(&sh->empty[s], 1);
     }
     mbar_init(&sh->done, 1);
@@ -200,31 +204,31 @@ __global__ void __cluster_dims__(kSplit, 1, 1) __launch_bounds__(THREADS, 1)
   pdl_trigger();
   const uint64_t* A = (l == 1) ? P->x + start * P->nw0 : P->layer[l - 2].A;
 
-  if (threadIdx.x < kProducers) {
-    // ---------------- producers ----------------
-    // items: W rows [0, NB) x 2 halves (item i: row i / 2, half i % 2), then
-    // (layer 1 only) input rows [0, M) x 2 halves; item i -> thread i % 512
-    constexpr int kItems = kTiles ? 1 : 2;
-    const int nB = 2 * NB, nItems = nB + (kTiles ? 0 : 2 * M);
-    Item it[kItems];
+  if (threadIdx.x < 32 * kRowWarps<kTiles>) {
+    // ---------------- producers: one thread per stage row ----------------
+    // threads 0 .. 255: weight rows (neurons n0 ..); layer 1 also threads
+    // 256 .. 383: input rows (patterns 0 .. M - 1); per k-block the thread
+    // loads the row's two bit words (one 16-byte load when the rows are
+    // 16-byte aligned) and expands them into the row's eight 16-byte chunks
+    const int p = threadIdx.x;
+    const bool isW = p < TN;
+    const int r = isW ? p : p - TN;
+    const uint64_t* src = nullptr;
+    if (isW && r < NB) src = Ly.W + (int64_t)(n0 + r) * nw;
+    if (!isW && !kTiles && r < M) src = A + (int64_t)r * nw;
+    const bool vec = (nw % 2 == 0) && src != nullptr && (reinterpret_cast<uintptr_t>(src) % 16 == 0);
+    const uint32_t row_off = (isW ? (uint32_t)A_BYTES : 0u) + (uint32_t)(r * KB);
+    const int swz = r & 7;
+    auto load = [&](int kb) -> uint4 {
+      if (src == nullptr || kb >= kb0 + nk) return make_uint4(0, 0, 0, 0);
+      if (vec) return __ldg(reinterpret_cast<const uint4*>(src) + kb);
+      const uint64_t lo = __ldg(src + 2 * kb);
+      const uint64_t hi = 2 * kb + 1 < nw ? __ldg(src + 2 * kb + 1) : 0ull;
+      return make_uint4((uint32_t)lo, (uint32_t)(lo >> 32), (uint32_t)hi, (uint32_t)(hi >> 32));
+    };
+    uint4 pre[kPrefetch];
 #pragma unroll
-    for (int j = 0; j < kItems; ++j) {
-      const int i = threadIdx.x + j * kProducers;
-      if (i < nB) {
-        it[j] = Item{Ly.W + (int64_t)(n0 + (i >> 1)) * nw, (uint32_t)(A_BYTES + (i >> 1) * KB), i >> 1,
-                     i & 1};
-      } else if (i < nItems) {
-        const int a = i - nB;
-        it[j] = Item{A + (int64_t)(a >> 1) * nw, (uint32_t)((a >> 1) * KB), a >> 1, a & 1};
-      } else {
-        it[j] = Item{nullptr, 0u, 0, 0};
-      }
-    }
-    uint64_t pre[kPrefetch][kItems];
-#pragma unroll
-    for (int d = 0; d < kPrefetch; ++d)
-#pragma unroll
-      for (int j = 0; j < kItems; ++j) pre[d][j] = load_word(it[j], kb0 + d, nw);
+    for (int d = 0; d < kPrefetch; ++d) pre[d] = load(kb0 + d);
 
     for (int k0 = 0; k0 < nk; k0 += kPrefetch) {
 #pragma unroll
@@ -242,11 +246,22 @@ __global__ void __cluster_dims__(kSplit, 1, 1) __launch_bounds__(THREADS, 1)
           mbar_arrive_tx(&sh->full[s], A_BYTES);
           bulk_g2s(stage, P->layer[l - 2].AE + (size_t)kb * A_BYTES, A_BYTES, &sh->full[s]);
         }
+        if (src != nullptr) {
+          uint8_t* row = stage + row_off;
+          const uint32_t x[4] = {pre[d].x, pre[d].y, pre[d].z, pre[d].w};
+          const int valid = Kin - KB * kb;
+          if (valid >= KB) {
 #pragma unroll
-        for (int j = 0; j < kItems; ++j) {
-          if (it[j].src != nullptr) store_word(stage, it[j], pre[d][j], kb, Kin);
-          pre[d][j] = load_word(it[j], kb + kPrefetch, nw);
+            for (int c = 0; c < 8; ++c)
+              *reinterpret_cast<uint4*>(row + 16 * (c ^ swz)) = chunk16(x[c >> 1] >> (16 * (c & 1)));
+          } else {
+#pragma unroll
+            for (int c = 0; c < 8; ++c)
+              *reinterpret_cast<uint4*>(row + 16 * (c ^ swz)) =
+                  chunk16_masked(x[c >> 1] >> (16 * (c & 1)), valid - 16 * c);
+          }
         }
+        pre[d] = load(kb + kPrefetch);
         // every writer orders its stores for the async proxy; one arrival per warp
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
         __syncwarp();

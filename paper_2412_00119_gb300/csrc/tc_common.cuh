@@ -131,6 +131,32 @@ __device__ __forceinline__ uint32_t keep_mask(int n_ok) {
   return n_ok >= 4 ? 0xFFFFFFFFu : (n_ok <= 0 ? 0u : ((1u << (8 * n_ok)) - 1u));
 }
 
+// Four K-elements, bits P .. P + 3 of x (P = 0 or 4), as four e4m3 bytes
+// (bit 1 -> 0x38 = +1, bit 0 -> 0xB8 = -1): the product places bit P + j at
+// bit 8 j + 7; its four shifted copies of the masked nibble do not overlap,
+// so it carries nothing.
+template <int P>
+__device__ __forceinline__ uint32_t e4m3_quad(uint32_t x) {
+  static_assert(P == 0 || P == 4, "nibble position");
+  constexpr uint32_t kMul = P == 0 ? 0x10204080u : 0x01020408u;
+  return ((x & (0xFu << P)) * kMul & 0x80808080u) ^ 0xB8B8B8B8u;
+}
+
+// 16 K-elements (bits 0..15 of h) -> one 16-byte chunk.
+__device__ __forceinline__ uint4 chunk16(uint32_t h) {
+  return make_uint4(e4m3_quad<0>(h), e4m3_quad<4>(h), e4m3_quad<0>(h >> 8), e4m3_quad<4>(h >> 8));
+}
+
+// The same with the elements at index >= valid set to 0 (ragged K only).
+__device__ __forceinline__ uint4 chunk16_masked(uint32_t h, int valid) {
+  uint4 v = chunk16(h);
+  v.x &= keep_mask(valid);
+  v.y &= keep_mask(valid - 4);
+  v.z &= keep_mask(valid - 8);
+  v.w &= keep_mask(valid - 12);
+  return v;
+}
+
 // Expand the item's bits into its stage chunk; elements at K >= Kin are 0.
 __device__ __forceinline__ void store_chunk(uint8_t* stage, const Chunk& ch, uint32_t bits, int kb,
                                             int Kin) {
