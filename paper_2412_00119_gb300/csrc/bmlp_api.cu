@@ -1,11 +1,14 @@
 // bmlp_api.cu -- host side of the C-ABI declared in include/bmlp.h.
 //
-// One training mini-batch is L forward launches, one local-classifier +
-// selection launch and one update launch.  All of them read the batch index s
-// and the step counter t from a device-resident control block that the update
-// kernel advances, so a single captured CUDA graph replays step after step with
-// no host work between steps.  Batch pointers live in a device-resident
-// parameter block that a stream-ordered copy refreshes at the start of a call.
+// One training mini-batch is one event-draw launch, L forward launches, one
+// local-classifier + selection launch and one update launch.  All of them read
+// the batch index s and the step counter t from a device-resident control block
+// that the update kernel advances, so captured CUDA graphs (of eight steps, or
+// one) replay step after step with no host work between steps.  Batch pointers
+// live in a device-resident parameter block that a stream-ordered copy
+// refreshes at the start of a call.  Each entry point that launches work opens
+// an NVTX range named after it (header-only NVTX v3: a no-op unless a tracing
+// tool is attached).
 #include <algorithm>
 #include <cmath>
 #include <cstddef>
@@ -15,6 +18,8 @@
 #include <string>
 #include <vector>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "bmlp_internal.cuh"
 
 using namespace bk;
@@ -22,6 +27,14 @@ using namespace bk;
 namespace {
 
 thread_local std::string g_create_error;
+
+// NVTX range for the lifetime of an entry point call.
+struct TraceRange {
+  explicit TraceRange(const char* name) { nvtxRangePushA(name); }
+  ~TraceRange() { nvtxRangePop(); }
+  TraceRange(const TraceRange&) = delete;
+  TraceRange& operator=(const TraceRange&) = delete;
+};
 
 enum ProfKind { kProfTrainFwd = 0, kProfCls = 1, kProfUpd = 2, kProfEvalFwd = 3, kProfOut = 4,
                 kProfCopy = 5, kProfEvents = 6, kProfKinds = 7 };
@@ -392,6 +405,7 @@ const char* bmlp_last_error(const bmlp_t* h) {
 
 int bmlp_create(const int32_t* widths, int32_t n_widths, int32_t classes, int16_t h_max,
                 uint64_t seed, const bmlp_hparams* hpin, bmlp_t** out) {
+  TraceRange trace("bmlp_create");
   g_create_error.clear();
   if (!out) return fail(nullptr, BMLP_EINVAL, "out is NULL");
   *out = nullptr;
@@ -575,6 +589,7 @@ void bmlp_destroy(bmlp_t* h) {
 
 int bmlp_train(bmlp_t* h, const uint64_t* x, const int32_t* labels, int64_t n, uint32_t flags,
                void* cuda_stream, int64_t* n_errors_out) {
+  TraceRange trace("bmlp_train");
   if (!h) return BMLP_EINVAL;
   h->err.clear();
   if (n < 0) return fail(h, BMLP_EINVAL, "n < 0");
@@ -716,10 +731,12 @@ int predict_impl(bmlp_t* h, const uint64_t* x, int64_t n, int32_t* out, void* cu
 }  // namespace
 
 int bmlp_predict(bmlp_t* h, const uint64_t* x, int64_t n, int32_t* out, void* cuda_stream) {
+  TraceRange trace("bmlp_predict");
   return predict_impl(h, x, n, out, cuda_stream, false);
 }
 
 int bmlp_predict_layers(bmlp_t* h, const uint64_t* x, int64_t n, int32_t* out, void* cuda_stream) {
+  TraceRange trace("bmlp_predict_layers");
   return predict_impl(h, x, n, out, cuda_stream, true);
 }
 
@@ -739,6 +756,7 @@ int bmlp_layer_errors(bmlp_t* h, int64_t* errs_out, int32_t reset) {
 }
 
 int bmlp_binarize_median(const float* x, int64_t n, int32_t K, uint64_t* out, void* cuda_stream) {
+  TraceRange trace("bmlp_binarize_median");
   if (n < 0 || K < 1) return fail(nullptr, BMLP_EINVAL, "bmlp_binarize_median: n < 0 or K < 1");
   if (n == 0) return BMLP_OK;
   if (!x || !out || !is_device_ptr(x) || !is_device_ptr(out))
@@ -835,6 +853,7 @@ int bmlp_get_info(const bmlp_t* h, int32_t* n_layers, int32_t* widths_out, int32
 
 int bmlp_layer_forward(bmlp_t* h, int32_t layer, const uint64_t* a_in, int64_t n, uint64_t* a_out,
                        void* cuda_stream) {
+  TraceRange trace("bmlp_layer_forward");
   if (!h) return BMLP_EINVAL;
   h->err.clear();
   if (layer < 1 || layer > h->L) return fail(h, BMLP_EINVAL, "layer must be in 1..%d", h->L);
