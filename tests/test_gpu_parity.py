@@ -368,6 +368,14 @@ def test_c1_784_256_full_epoch_popc_engine():
     _full_width("C1", n_test=500, fwd=B.BMLP_FWD_POPC)
 
 
+def test_c5_8192x5_20_step_prefix():
+    """The 8192 -> 8192 x4 -> 10 network in the bench's launch configuration
+    (tensor-core forward, eight-step graphs): H, W, P, p_r and the step
+    counter after 20 mini-batches equal the oracle's (a difference at any
+    step would persist), and so does the error count."""
+    _full_width("C5", steps=20, n_test=0)
+
+
 def test_c5_8192x5_prefix_popc_engine():
     _full_width("C5", steps=1, n_test=0, fwd=B.BMLP_FWD_POPC)
 
