@@ -54,6 +54,12 @@ EVAL_BATCH = 65_536
 # UPDATE_TRAFFIC_SRC_SHA; otherwise reported as null.
 UPDATE_TRAFFIC_BYTES = 463_731_712 + 383_939_840  # dram read + write of one timed-region launch (ncu)
 UPDATE_TRAFFIC_SRC_SHA = "8d7fd0f8e4d76002"
+# The same for one 8192 -> 8192 k_forward_eval_tc launch at 65,536 patterns
+# (profiles/k_forward_eval_tc_c5eval.md), keyed to the kernel and its shared
+# tcgen05 header.  Part of the 67 MB output is still in the write-back L2 when
+# the launch ends, so the write figure is below the output's size.
+EVAL_TRAFFIC_BYTES = 75_599_360 + 32_936_448
+EVAL_TRAFFIC_SRC_SHA = "f8b34ceea49eb88e"
 
 
 def bitpairs_per_sample(widths, classes):
@@ -396,9 +402,13 @@ def run_ours(args):
     efwd_bp = EVAL_BATCH * cfg.widths[1] * cfg.widths[0]
     if tc:
         fp8 = FP8_PER_BF16 * bf16_tf
+        etraffic = None
+        if (EVAL_TRAFFIC_BYTES is not None and cfg.widths[0] == cfg.widths[1] == 8192
+                and EVAL_TRAFFIC_SRC_SHA == src_sha("kern_eval_tc.cu", "tc_common.cuh")):
+            etraffic = EVAL_TRAFFIC_BYTES
         eroof = {"bound": "tensor", "kernel": "k_forward_eval_tc",
                  "achieved": 2 * efwd_bp / efwd_s / 1e12, "peak": fp8, "unit": "TFLOP/s",
-                 "frac": 2 * efwd_bp / efwd_s / 1e12 / fp8, "traffic": None,
+                 "frac": 2 * efwd_bp / efwd_s / 1e12 / fp8, "traffic": etraffic,
                  "peak_source": peak_src + " bf16 burst x 2 (e4m3 / bf16 nominal)"}
     else:
         eroof = {"bound": "alu", "kernel": "k_forward_eval",
