@@ -176,6 +176,33 @@ int bmlp_layer_errors(bmlp_t* h, int64_t* errs_out, int32_t reset);
  * pointers; BMLP_ECUDA if the launch fails. */
 int bmlp_binarize_median(const float* x, int64_t n, int32_t K, uint64_t* out, void* cuda_stream);
 
+/* Weights of a fixed random expansion layer (Sec. 3.2, footnote to the
+ * binarisation step: a fixed random input layer with weights in {+-1} and
+ * sign activation lets the BMLP take non-binary inputs directly):
+ * e_k,i = +1 iff bit 31 of word i%4 of Philox4x32-10 at counter
+ * (i/4, k, 33*2^16, 0) with key (seed mod 2^32, seed div 2^32), else -1.
+ *   E_out: device, K x ceil(D/64) words (bit i % 64 of word i / 64 of row k
+ *          = 1 <-> e_k,i = +1; pad bits 0), 8-byte aligned, caller-owned.
+ * No handle (errors: bmlp_last_error(NULL)); asynchronous on cuda_stream.
+ * BMLP_EINVAL for K < 1, D < 1, D > 2^23, NULL, host or misaligned E_out. */
+int bmlp_expand_weights(uint64_t seed, int32_t K, int32_t D, uint64_t* E_out, void* cuda_stream);
+
+/* The expansion layer itself, for unsigned 8-bit inputs (pixel
+ * intensities): bit k of pattern mu is 1 (+1) iff
+ * sum_i x[mu][i] e_k,i >= 0 (sign(0) = +1, as for every activation), the
+ * sum taken exactly in integers; else 0 (-1).  Pad bits are 0, so the output
+ * is bmlp_train / bmlp_predict input for K_0 = K.
+ *   x: device, n x D uint8, row-major (row mu at x + mu D), caller-owned;
+ *      any alignment.
+ *   E: device, K x ceil(D/64) words as written by bmlp_expand_weights (any
+ *      +-1 matrix in that layout; pad bits ignored), 8-byte aligned.
+ *   out: device, n x ceil(K/64) words, 8-byte aligned, caller-owned.
+ * No handle (errors: bmlp_last_error(NULL)); asynchronous on cuda_stream.
+ * BMLP_EINVAL for n < 0, K < 1, D < 1, D > 2^23 (the int32 sum bound),
+ * NULL, host or misaligned pointers; BMLP_ECUDA if the launch fails. */
+int bmlp_expand_sign(const uint8_t* x, int64_t n, int32_t D, const uint64_t* E, int32_t K,
+                     uint64_t* out, void* cuda_stream);
+
 /* One layer of forward-only evaluation (Sec. 3.1; Alg. 1 l.8-9):
  * a_out = sign(a_in W_l), sign(0) = +1, for n packed rows.  a_in: n rows of
  * ceil(K_{l-1}/64) words (pad bits 0); a_out: n rows of ceil(K_l/64) words,

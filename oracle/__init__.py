@@ -150,6 +150,12 @@ def _declare(L):
     L.or_layer_errors.restype = C.c_int
     L.or_binarize_median.argtypes = [C.POINTER(C.c_float), C.c_int64, C.c_int32, _i8p]
     L.or_binarize_median.restype = C.c_int
+    L.or_expand_weight.argtypes = [C.c_uint64, C.c_int32, C.c_int32]
+    L.or_expand_weight.restype = C.c_int32
+    L.or_expand_weights.argtypes = [C.c_uint64, C.c_int32, C.c_int32, _i8p]
+    L.or_expand_weights.restype = C.c_int
+    L.or_expand_sign.argtypes = [_u8p, C.c_int64, C.c_int32, _i8p, C.c_int32, _i8p]
+    L.or_expand_sign.restype = C.c_int
     L.or_num_layers.argtypes = [C.c_void_p]
     L.or_num_layers.restype = C.c_int32
     L.or_width.argtypes = [C.c_void_p, C.c_int32]
@@ -315,6 +321,35 @@ def binarize_median(x):
     rc = lib().or_binarize_median(x.ctypes.data_as(C.POINTER(C.c_float)), n, K, _p(a, _i8p))
     if rc != 0:
         raise ValueError("or_binarize_median failed: %d" % rc)
+    return a
+
+
+def expand_weight(seed, k, i):
+    """Expansion weight e_{k,i} in {+-1} (O20)."""
+    return int(lib().or_expand_weight(seed, k, i))
+
+
+def expand_weights(seed, K, D):
+    """The K x D +-1 int8 expansion matrix of O20."""
+    e = np.zeros((K, D), np.int8)
+    rc = lib().or_expand_weights(seed, K, D, _p(e, _i8p))
+    if rc != 0:
+        raise ValueError("or_expand_weights failed: %d" % rc)
+    return e
+
+
+def expand_sign(x, e):
+    """Expansion layer (O20): n x D uint8, K x D +-1 -> n x K +-1 int8."""
+    x = _c(x, np.uint8)
+    e = _c(e, np.int8)
+    n, D = x.shape
+    K, De = e.shape
+    if De != D:
+        raise ValueError("x has %d inputs, e has %d" % (D, De))
+    a = np.zeros((n, K), np.int8)
+    rc = lib().or_expand_sign(_p(x, _u8p), n, D, _p(e, _i8p), K, _p(a, _i8p))
+    if rc != 0:
+        raise ValueError("or_expand_sign failed: %d" % rc)
     return a
 
 

@@ -86,6 +86,14 @@
  *       yhat_l = a_l P_l, ties to the lowest class (O2); the local error
  *       count of layer l is the number of training patterns whose 01-loss
  *       l_l of Eq. 1 was 1 in their training forward pass.
+ *   O20 Expansion layer for integer-valued inputs (Sec. 3.2, footnote to the
+ *       binarisation step: a fixed random input layer with weights in {+-1}
+ *       and sign activation lets the BMLP take non-binary inputs directly).
+ *       Inputs are unsigned 8-bit integers (pixel intensities); expansion
+ *       weight e_{k,i} (k < K expansion neurons, i < D inputs) is uniform on
+ *       {+-1}, drawn like the initial weights from its own Philox stream
+ *       (below); a_k = +1 iff sum_i x_i e_{k,i} >= 0 (O1), the sum taken
+ *       exactly in integers.
  *
  * Philox stream layout (counter-based; Salmon, Moraes, Dror, Shaw, "Parallel
  * random numbers: as easy as 1, 2, 3", SC'11).  key = (seed mod 2^32,
@@ -98,6 +106,8 @@
  *                               words 0..3 of (b, k, (4 + r)*2^16 + l, t), r = 0, 1, ...
  *                               (at most 16 calls per block: r <= 15)
  *   group-order key u_k of neuron k (O19): (k/4, 0, 32*2^16 + l, t'); word k%4
+ *   expansion weight e_{k,i} (O20)         : (i/4, k, 33*2^16, 0); word i%4;
+ *                               e = +1 iff bit 31 set
  *   Layers are numbered l = 1..L as in the paper.
  */
 #include <math.h>
@@ -716,6 +726,37 @@ int or_binarize_median(const float* x, int64_t n, int32_t K, int8_t* a) {
     free(s);
   }
   return rc;
+}
+
+/* Fixed random expansion weight e_{k,i} (O20): uniform on {+-1}. */
+int32_t or_expand_weight(uint64_t seed, int32_t k, int32_t i) {
+  uint32_t w[4];
+  philox_at(seed, (uint32_t)(i / 4), (uint32_t)k, 33u << 16, 0u, w);
+  return (w[i % 4] >> 31) ? +1 : -1;
+}
+
+/* The K x D expansion matrix, e[k*D + i] = e_{k,i}. */
+int or_expand_weights(uint64_t seed, int32_t K, int32_t D, int8_t* e) {
+  if (K < 1 || D < 1 || !e) return OR_EINVAL;
+#pragma omp parallel for schedule(static)
+  for (int32_t k = 0; k < K; k++)
+    for (int32_t i = 0; i < D; i++) e[(int64_t)k * D + i] = (int8_t)or_expand_weight(seed, k, i);
+  return OR_OK;
+}
+
+/* Expansion layer (O20): x is n x D uint8, e is K x D +-1, a is n x K +-1;
+ * a[mu][k] = sign(sum_i x[mu][i] e[k][i]) with sign(0) = +1 (O1). */
+int or_expand_sign(const uint8_t* x, int64_t n, int32_t D, const int8_t* e, int32_t K, int8_t* a) {
+  if (n < 0 || D < 1 || K < 1 || (n > 0 && (!x || !e || !a))) return OR_EINVAL;
+#pragma omp parallel for schedule(static)
+  for (int64_t mu = 0; mu < n; mu++) {
+    for (int32_t k = 0; k < K; k++) {
+      int64_t z = 0;
+      for (int32_t i = 0; i < D; i++) z += (int64_t)x[mu * D + i] * (int64_t)e[(int64_t)k * D + i];
+      a[mu * K + k] = (int8_t)(z >= 0 ? 1 : -1);
+    }
+  }
+  return OR_OK;
 }
 
 /* ------------------------------------------------------------------------ */

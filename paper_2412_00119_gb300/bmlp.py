@@ -79,6 +79,8 @@ SIGNATURES = [
     ("bmlp_predict_layers", C.c_int, [_vp, _vp, C.c_int64, _vp, _vp]),
     ("bmlp_layer_errors", C.c_int, [_vp, _i64p, C.c_int32]),
     ("bmlp_binarize_median", C.c_int, [_vp, C.c_int64, C.c_int32, _vp, _vp]),
+    ("bmlp_expand_weights", C.c_int, [C.c_uint64, C.c_int32, C.c_int32, _vp, _vp]),
+    ("bmlp_expand_sign", C.c_int, [_vp, C.c_int64, C.c_int32, _vp, C.c_int32, _vp, _vp]),
     ("bmlp_debug_wait_probe", C.c_int, [_vp, C.c_int32, C.c_double]),
 ]
 
@@ -204,6 +206,17 @@ def bmlp_binarize_median(x, out, stream=None):
     """Median binarisation of n x K fp32 patterns (device) into packed bits."""
     n, K = x.shape
     _check(lib().bmlp_binarize_median(_ptr(x), n, K, _ptr(out), _stream(stream)), None)
+
+
+def bmlp_expand_weights(seed, K, D, E_out, stream=None):
+    """The packed K x D +-1 expansion matrix (device, K x ceil(D/64) int64)."""
+    _check(lib().bmlp_expand_weights(seed, K, D, _ptr(E_out), _stream(stream)), None)
+
+
+def bmlp_expand_sign(x, E, K, out, stream=None):
+    """Expansion layer: n x D uint8 patterns (device) -> packed sign(x E^T)."""
+    n, D = x.shape
+    _check(lib().bmlp_expand_sign(_ptr(x), n, D, _ptr(E), K, _ptr(out), _stream(stream)), None)
 
 
 def bmlp_debug_wait_probe(h, arrive, seconds=0.05):

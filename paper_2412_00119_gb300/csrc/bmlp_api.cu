@@ -769,6 +769,36 @@ int bmlp_binarize_median(const float* x, int64_t n, int32_t K, uint64_t* out, vo
   return BMLP_OK;
 }
 
+int bmlp_expand_weights(uint64_t seed, int32_t K, int32_t D, uint64_t* E_out, void* cuda_stream) {
+  TraceRange trace("bmlp_expand_weights");
+  if (K < 1 || D < 1 || D > (1 << 23))
+    return fail(nullptr, BMLP_EINVAL, "bmlp_expand_weights: K < 1, D < 1 or D > 2^23");
+  if (!E_out || !is_device_ptr(E_out))
+    return fail(nullptr, BMLP_EINVAL, "bmlp_expand_weights: E_out must be a device pointer");
+  if (reinterpret_cast<uintptr_t>(E_out) & 7)
+    return fail(nullptr, BMLP_EINVAL, "bmlp_expand_weights: misaligned E_out");
+  launch_expand_weights(seed, K, D, E_out, static_cast<cudaStream_t>(cuda_stream));
+  const cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_fail(nullptr, e, "k_expand_weights");
+  return BMLP_OK;
+}
+
+int bmlp_expand_sign(const uint8_t* x, int64_t n, int32_t D, const uint64_t* E, int32_t K,
+                     uint64_t* out, void* cuda_stream) {
+  TraceRange trace("bmlp_expand_sign");
+  if (n < 0 || K < 1 || D < 1 || D > (1 << 23))
+    return fail(nullptr, BMLP_EINVAL, "bmlp_expand_sign: n < 0, K < 1, D < 1 or D > 2^23");
+  if (n == 0) return BMLP_OK;
+  if (!x || !E || !out || !is_device_ptr(x) || !is_device_ptr(E) || !is_device_ptr(out))
+    return fail(nullptr, BMLP_EINVAL, "bmlp_expand_sign: x, E and out must be device pointers");
+  if ((reinterpret_cast<uintptr_t>(E) & 7) || (reinterpret_cast<uintptr_t>(out) & 7))
+    return fail(nullptr, BMLP_EINVAL, "bmlp_expand_sign: misaligned E or out");
+  launch_expand_sign(x, n, D, E, K, out, static_cast<cudaStream_t>(cuda_stream));
+  const cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_fail(nullptr, e, "k_expand_sign");
+  return BMLP_OK;
+}
+
 int bmlp_get_state(const bmlp_t* hc, int32_t layer, int16_t* H_out, uint64_t* W_out, int8_t* P_out,
                    double* p_r_out, int64_t* step_out) {
   bmlp_t* h = const_cast<bmlp_t*>(hc);

@@ -113,6 +113,8 @@ constexpr int kClsThreads = 512;
 //                             (b/4, k, 3*2^16 + l, t)   word b%4
 //   event draws V_0, V_1, .. of that block: words 0..3 of (b, k, (4+r)*2^16 + l, t),
 //                             r = 0, 1, ..
+//   group-order key u_k of neuron k: (k/4, 0, 32*2^16 + l, t')   word k%4
+//   expansion weight e_ki   : (i/4, k, 33*2^16, 0)      word i%4, +1 iff bit 31
 // ---------------------------------------------------------------------------
 __device__ __forceinline__ uint4 philox4x32_10(uint4 ctr, uint32_t k0, uint32_t k1) {
 #pragma unroll
@@ -223,6 +225,11 @@ size_t act_tile_bytes(int K);  // bytes of an AE image for K activations
 // Median binarisation of n x K fp32 patterns into n x nw packed words.
 void launch_binarize_median(const float* x, int64_t n, int K, int nw, uint64_t* out,
                             cudaStream_t st);
+// Expansion layer for uint8 inputs: E (K x ceil(D/64) words) from the
+// expansion-weight stream, and out = packed sign(x E^T) (n x ceil(K/64)).
+void launch_expand_weights(uint64_t seed, int K, int D, uint64_t* E, cudaStream_t st);
+void launch_expand_sign(const uint8_t* x, int64_t n, int D, const uint64_t* E, int K,
+                        uint64_t* out, cudaStream_t st);
 // Tensor-core forward for evaluation: A (M x nw_in) against W -> Aout
 // (M x nw_out), 256-pattern x 256-neuron tiles per CTA pair; an expired
 // bounded wait adds one to *timeouts.

@@ -18,7 +18,10 @@ Sources of the expected values:
     reinforcement moves away from 0) and the learnability of a separable task;
   * the rank form of the lower median (brute force), the truncated network
     for early-exit predictions, and the evaluation path for the local error
-    counts.
+    counts;
+  * for the expansion front end: the Philox stream recomputed from the
+    KAT-pinned primitive, and special cases (zero pattern, one or two lit
+    inputs, 0/1 patterns as counts).
 """
 from __future__ import annotations
 
@@ -39,6 +42,70 @@ def check_philox_kat():
         v = [int(t, 16) for t in line.split()]
         out = O.philox4x32_10(v[0:4], v[4:6])
         assert [int(o) for o in out] == v[6:10], (line, [hex(int(o)) for o in out])
+
+
+# -- expansion front end (O20) ----------------------------------------------------
+
+def check_expand_weights_stream(seed=0x1234_5678_9ABC):
+    """Expansion weights (O20): e_{k,i} = +1 iff bit 31 of word i%4 of the
+    KAT-pinned Philox at counter (i/4, k, 33*2^16, 0), recomputed here from
+    the primitive over a ragged D; balanced (P(+1) = 1/2 within 5 sigma over
+    200,000 weights); a stream of its own, not that of the initial weights."""
+    K, D = 7, 13
+    e = O.expand_weights(seed, K, D)
+    key = [seed & 0xFFFFFFFF, seed >> 32]
+    for k in range(K):
+        for i in range(D):
+            w = O.philox4x32_10([i // 4, k, 33 << 16, 0], key)
+            assert e[k, i] == (1 if (int(w[i % 4]) >> 31) else -1), (k, i)
+            assert O.expand_weight(seed, k, i) == e[k, i], (k, i)
+    h1 = np.array([[O.init_h(seed, 1, k, i) for i in range(D)] for k in range(K)])
+    assert not np.array_equal(e, h1)
+    big = O.expand_weights(seed, 200, 1000)
+    assert set(np.unique(big)) == {-1, 1}
+    assert abs((big == 1).mean() - 0.5) < 5 * math.sqrt(0.25 / big.size)
+
+
+def check_expand_sign(seed=11):
+    """Expansion layer (O20), a_k = +1 iff sum_i x_i e_{k,i} >= 0, against
+    what fixes it without the sum as written: a zero pattern gives all +1
+    (sign(0) = +1); a pattern with one lit input i gives a_k = e_{k,i}; two
+    lit inputs u > v on weights +1 / -1 give +1 and on -1 / +1 give -1 (for
+    u >= 128 too: the inputs are unsigned); on 0/1 patterns a_k = +1 iff at
+    least half of the lit inputs carry weight +1 (a count); and, as a cross-
+    check, the exact int64 matrix product for pixel-like inputs with K != D."""
+    rng = np.random.default_rng(seed)
+    K, D = 9, 23
+    e = O.expand_weights(seed, K, D)
+    assert np.all(O.expand_sign(np.zeros((2, D), np.uint8), e) == 1)
+    for i in range(D):
+        for v in (1, 7, 128, 255):
+            x = np.zeros((1, D), np.uint8)
+            x[0, i] = v
+            assert np.array_equal(O.expand_sign(x, e)[0], e[:, i]), (i, v)
+    for k in range(K):
+        pos = np.flatnonzero(e[k] == 1)
+        neg = np.flatnonzero(e[k] == -1)
+        if len(pos) == 0 or len(neg) == 0:
+            continue
+        for u, v in ((255, 254), (200, 100), (128, 1), (2, 1)):
+            x = np.zeros((2, D), np.uint8)
+            x[0, pos[0]], x[0, neg[0]] = u, v
+            x[1, pos[0]], x[1, neg[0]] = v, u
+            a = O.expand_sign(x, e)
+            assert a[0, k] == 1 and a[1, k] == -1, (k, u, v)
+    xb = (rng.random((300, D)) < 0.4).astype(np.uint8)
+    a = O.expand_sign(xb, e)
+    for mu in range(len(xb)):
+        lit = xb[mu] == 1
+        for k in range(K):
+            plus = int((e[k][lit] == 1).sum())
+            assert a[mu, k] == (1 if 2 * plus >= int(lit.sum()) else -1), (mu, k)
+    Kp, Dp = 37, 61
+    ep = O.expand_weights(seed + 1, Kp, Dp)
+    xp = np.where(rng.random((50, Dp)) < 0.5, 0, rng.integers(1, 256, (50, Dp))).astype(np.uint8)
+    want = np.where(xp.astype(np.int64) @ ep.astype(np.int64).T >= 0, 1, -1)
+    assert np.array_equal(O.expand_sign(xp, ep), want)
 
 
 # -- group size ----------------------------------------------------------------
@@ -593,6 +660,8 @@ def check_group_mode_single_group(seed=14):
 
 ALL_CHECKS = [
     check_philox_kat,
+    check_expand_weights_stream,
+    check_expand_sign,
     check_gamma_golden,
     check_dot_bruteforce,
     check_sign_zero,

@@ -93,6 +93,26 @@ def test_binarize_rejects_bad_arguments():
     assert b"device pointers" in lib.bmlp_last_error(None)
 
 
+def test_expansion_rejects_bad_arguments():
+    lib = pkg.lib()
+    assert lib.bmlp_expand_weights(1, 0, 8, None, None) == B.BMLP_EINVAL
+    assert lib.bmlp_expand_weights(1, 8, 0, None, None) == B.BMLP_EINVAL
+    assert lib.bmlp_expand_weights(1, 8, (1 << 23) + 1, None, None) == B.BMLP_EINVAL
+    assert b"2^23" in lib.bmlp_last_error(None)
+    E = np.zeros((8, 1), np.uint64)
+    assert lib.bmlp_expand_weights(1, 8, 8, E.ctypes.data, None) == B.BMLP_EINVAL
+    assert b"device pointer" in lib.bmlp_last_error(None)
+    assert lib.bmlp_expand_sign(None, -1, 8, None, 8, None, None) == B.BMLP_EINVAL
+    assert lib.bmlp_expand_sign(None, 4, 8, None, 0, None, None) == B.BMLP_EINVAL
+    assert lib.bmlp_expand_sign(None, 4, 0, None, 8, None, None) == B.BMLP_EINVAL
+    assert lib.bmlp_expand_sign(None, 0, 8, None, 8, None, None) == B.BMLP_OK
+    x = np.zeros((4, 8), np.uint8)
+    out = np.zeros((4, 1), np.uint64)
+    assert lib.bmlp_expand_sign(x.ctypes.data, 4, 8, E.ctypes.data, 8, out.ctypes.data,
+                                None) == B.BMLP_EINVAL
+    assert b"device pointers" in lib.bmlp_last_error(None)
+
+
 def test_null_handle_calls_fail_cleanly():
     lib = pkg.lib()
     assert lib.bmlp_predict_layers(None, None, 0, None, None) == B.BMLP_EINVAL

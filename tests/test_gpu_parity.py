@@ -163,6 +163,74 @@ def test_binarize_median_matches_oracle(n, K, kind):
     assert np.array_equal(out.cpu().numpy().view(np.uint64), want)
 
 
+def _packed_e(e):
+    """Packed rows of a +-1 matrix (bit = +1), from the oracle's weights."""
+    return W.pack(e)
+
+
+@pytest.mark.parametrize("K,D", [(1, 1), (70, 63), (130, 784), (1024, 3072), (5, 65), (3, 129)])
+def test_expand_weights_match_oracle(K, D):
+    """Expansion weights (Sec. 3.2 footnote): every packed bit, pads 0, equals
+    the oracle's draw from the same Philox stream."""
+    seed = 0x5EED_0000_0000 + 17 * K + D
+    E = torch.full((K, W.words(D)), -1, dtype=torch.int64, device=DEV)
+    B.bmlp_expand_weights(seed, K, D, E)
+    assert np.array_equal(E.cpu().numpy().view(np.uint64), _packed_e(O.expand_weights(seed, K, D)))
+
+
+EXPAND_CASES = [(1, 1, 1, "pixels", 0), (130, 70, 130, "sparse", 0), (300, 784, 1024, "pixels", 0),
+                (129, 3072, 257, "full", 0), (50, 64, 2048, "saturated", 0), (257, 8, 64, "sparse", 0),
+                (260, 784, 200, "pixels", 1), (260, 784, 200, "pixels", 4), (77, 1000, 1000, "full", 3)]
+
+
+@pytest.mark.parametrize("n,D,K,kind,offset", EXPAND_CASES)
+def test_expand_sign_matches_oracle(n, D, K, kind, offset):
+    """Expansion layer on uint8 inputs: every packed bit, pads 0, equals the
+    oracle's exact sign(x e^T), sign(0) = +1; ragged tiles in both patterns
+    and neurons, exact ties, and inputs starting at odd byte offsets."""
+    x = W.pixel_bytes(41 + D + K, n, D, kind)
+    e = O.expand_weights(9 + K, K, D)
+    flat = torch.zeros(n * D + offset, dtype=torch.uint8, device=DEV)
+    flat[offset:] = torch.from_numpy(x.reshape(-1)).to(DEV)
+    xd = flat[offset:].view(n, D)
+    E = torch.from_numpy(_packed_e(e).view(np.int64)).to(DEV)
+    out = torch.full((n, W.words(K)), -1, dtype=torch.int64, device=DEV)
+    B.bmlp_expand_sign(xd, E, K, out)
+    want = W.pack(O.expand_sign(x, e))
+    assert np.array_equal(out.cpu().numpy().view(np.uint64), want)
+
+
+def test_expand_sign_fashion_shape_sampled():
+    """60,000 uint8 patterns of 784 inputs through a 1,024-wide expansion
+    (image-shaped data; 469 pattern tiles, the last one ragged): 300 sampled
+    rows, the first and last tiles among them, equal the oracle's."""
+    n, D, K = 60_000, 784, 1024
+    x = W.pixel_bytes(5, n, D, "pixels")
+    e = O.expand_weights(21, K, D)
+    E = torch.from_numpy(_packed_e(e).view(np.int64)).to(DEV)
+    out = torch.empty((n, W.words(K)), dtype=torch.int64, device=DEV)
+    B.bmlp_expand_sign(torch.from_numpy(x).to(DEV), E, K, out)
+    rng = np.random.default_rng(3)
+    rows = np.unique(np.concatenate([np.arange(128), np.arange(n - 200, n), rng.integers(0, n, 100)]))
+    got = out.cpu().numpy().view(np.uint64)[rows]
+    assert np.array_equal(got, W.pack(O.expand_sign(x[rows], e)))
+
+
+def test_expand_sign_beyond_one_grid():
+    """More patterns than one launch's 65,535 pattern tiles: the rows around
+    the split and at both ends equal the oracle's."""
+    per = 65_535 * 128
+    n, D, K = per + 300, 5, 3
+    x = W.pixel_bytes(6, n, D, "full")
+    e = O.expand_weights(22, K, D)
+    E = torch.from_numpy(_packed_e(e).view(np.int64)).to(DEV)
+    out = torch.full((n, 1), -1, dtype=torch.int64, device=DEV)
+    B.bmlp_expand_sign(torch.from_numpy(x).to(DEV), E, K, out)
+    rows = np.concatenate([np.arange(0, 200), np.arange(per - 200, per + 300)])
+    got = out.cpu().numpy().view(np.uint64)[rows]
+    assert np.array_equal(got, W.pack(O.expand_sign(x[rows], e)))
+
+
 @pytest.mark.parametrize("engine", sorted(ENGINES))
 def test_early_exit_and_layer_errors(engine):
     """Early-exit predictions of every layer (Sec. 3.1) and the local 01-loss

@@ -56,6 +56,11 @@ MUTANTS = [
     ("group_key_word", "v[k].u = w[k % 4];", "v[k].u = w[0];"),
     ("group_mode2_fixed", "const uint32_t tt = (mode == 2) ? t : 0u;", "const uint32_t tt = 0u;"),
     ("forward_drops_sign", "zr[k] += ai * (hrow[k] > 0 ? 1 : -1);", "zr[k] += ai * hrow[k];"),
+    ("expand_sign_zero_negative", "a[mu * K + k] = (int8_t)(z >= 0 ? 1 : -1);",
+     "a[mu * K + k] = (int8_t)(z > 0 ? 1 : -1);"),
+    ("expand_weights_transposed", "(int64_t)e[(int64_t)k * D + i];", "(int64_t)e[(int64_t)i * K + k];"),
+    ("expand_input_signed", "z += (int64_t)x[mu * D + i]", "z += (int64_t)(int8_t)x[mu * D + i]"),
+    ("expand_stream_tag", "(uint32_t)k, 33u << 16, 0u, w);", "(uint32_t)k, 32u << 16, 0u, w);"),
 ]
 
 

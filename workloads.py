@@ -150,6 +150,25 @@ def real_patterns(seed: int, n: int, K: int, kind: str = "pixels") -> np.ndarray
     raise ValueError(kind)
 
 
+def pixel_bytes(seed: int, n: int, D: int, kind: str = "pixels") -> np.ndarray:
+    """n x D uint8 patterns for the expansion front end: "pixels" = intensities
+    1..255 with about 60 % zeros (image-like), "full" = uniform 0..255,
+    "sparse" = 0/1 with 5 % ones (many exact ties z = 0 of the expansion
+    sums), "saturated" = every input 255 (z = 255 times the weight row's
+    sum: a tie wherever a row of an even width sums to 0)."""
+    rng = np.random.default_rng(seed)
+    if kind == "pixels":
+        v = rng.integers(1, 256, (n, D))
+        return np.where(rng.random((n, D)) < 0.6, 0, v).astype(np.uint8)
+    if kind == "full":
+        return rng.integers(0, 256, (n, D)).astype(np.uint8)
+    if kind == "sparse":
+        return (rng.random((n, D)) < 0.05).astype(np.uint8)
+    if kind == "saturated":
+        return np.full((n, D), 255, np.uint8)
+    raise ValueError(kind)
+
+
 # -- teacher -------------------------------------------------------------------
 
 @dataclasses.dataclass
