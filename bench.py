@@ -481,6 +481,38 @@ def run_ncu_case(args):
     return 0
 
 
+def run_frontend_case(args):
+    """The expansion front end alone (for timing and profiler captures): N x 1000
+    uint8 patterns of D inputs through a fixed random K-wide expansion layer,
+    the weight stream drawn once, the layer run twice (the second launch is
+    the one to time or capture)."""
+    import torch
+
+    from paper_2412_00119_gb300 import bmlp as B
+
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    D, K = (int(v) for v in args.frontend_shape.split(","))
+    n = 1000 * args.frontend_case
+    x = torch.from_numpy(W.pixel_bytes(1, n, D, "pixels")).to(dev)
+    E = torch.empty((K, W.words(D)), dtype=torch.int64, device=dev)
+    out = torch.empty((n, W.words(K)), dtype=torch.int64, device=dev)
+    st = torch.cuda.current_stream(dev)
+    B.bmlp_expand_weights(7, K, D, E, stream=st)
+    B.bmlp_expand_sign(x, E, K, out, stream=st)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    e0.record(st)
+    B.bmlp_expand_sign(x, E, K, out, stream=st)
+    e1.record(st)
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1)
+    print(json.dumps({"frontend_case": {"n": n, "D": D, "K": K, "expand_ms": ms,
+                                        "patterns_per_s": n / ms * 1e3,
+                                        "multiply_adds_per_s": n * D * K / ms * 1e3}}))
+    return 0
+
+
 def main(argv=None):
     ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
     ap.add_argument("--gpus", type=int, default=1)
@@ -490,9 +522,15 @@ def main(argv=None):
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--ncu-case", type=int, default=0, metavar="N",
                     help="run only a small N-mini-batch case (for profiler captures)")
+    ap.add_argument("--frontend-case", type=int, default=0, metavar="N",
+                    help="run only the expansion front end on N x 1000 uint8 patterns")
+    ap.add_argument("--frontend-shape", default="784,1024", metavar="D,K",
+                    help="inputs and width of the expansion layer for --frontend-case")
     args = ap.parse_args(argv)
     if args.ncu_case:
         return run_ncu_case(args)
+    if args.frontend_case:
+        return run_frontend_case(args)
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
     if args.impl == "reference":
