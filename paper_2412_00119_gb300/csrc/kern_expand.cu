@@ -14,7 +14,8 @@
 // k_expand_sign: a 128-pattern x 128-neuron tile per CTA of 256 threads, the
 // inputs in chunks of 64 (one word of E per neuron): the chunk's bytes of x
 // and the chunk's E bits, expanded to +-1 bytes, are staged in shared memory
-// (rows padded to 17 words: conflict-free reads), then thread (tx, ty) runs
+// (rows padded to 17 words: conflict-free reads; the next chunk's raw words
+// are already in flight in registers), then thread (tx, ty) runs
 // dp4a.u32.s32 for patterns ty + 16 i and neurons tx + 16 j, i, j < 8 (64
 // int32 sums).  Each warp ballots the signs of 2 patterns x 16 neurons and
 // writes 16-bit pieces of the packed rows.  Neuron tiles vary fastest in the
@@ -43,7 +44,7 @@ __device__ __forceinline__ int dp4a_us(uint32_t a, uint32_t b, int c) {
   return d;
 }
 
-__global__ void __launch_bounds__(kXThreads)
+__global__ void __launch_bounds__(kXThreads, 2)
     k_expand_sign(const uint8_t* __restrict__ x, int64_t n, int D, bool vec,
                   const uint64_t* __restrict__ E, int K, int nwD, uint64_t* __restrict__ out,
                   int nwK) {
@@ -58,42 +59,59 @@ __global__ void __launch_bounds__(kXThreads)
 #pragma unroll
     for (int j = 0; j < 8; ++j) acc[i][j] = 0;
 
-#pragma unroll 1
-  for (int kc = 0; kc < nwD; ++kc) {
+  // thread t stages words q = t + 256 v (v < 8) of the x tile -- staged row
+  // q / 16, word q % 16 = inputs 4 (q % 16) .. + 3 of the chunk, byte b = input
+  // 4 (q % 16) + b, 0 past D and past n -- and half t & 1 of the E word of
+  // neuron n0 + t / 2.  The raw words of chunk kc + 1 are loaded into
+  // registers before chunk kc is computed, so the loads overlap the dp4a work.
+  uint32_t xr[8], er;
+  auto load_chunk = [&](int kc) {
     const int i0 = 64 * kc;
-    // x: word c4 of staged row r = inputs i0 + 4 c4 .. + 3 of pattern m0 + r
-    // (byte b = input i0 + 4 c4 + b), 0 past D and past n
-    for (int q = threadIdx.x; q < kXM * 16; q += kXThreads) {
+#pragma unroll
+    for (int v = 0; v < 8; ++v) {
+      const int q = threadIdx.x + kXThreads * v;
       const int r = q >> 4, c4 = q & 15;
       const int64_t m = m0 + r;
       const int i = i0 + 4 * c4;
-      uint32_t v = 0;
+      uint32_t w = 0;
       if (m < n) {
         const uint8_t* row = x + m * (int64_t)D;
         if (vec && i + 4 <= D) {
-          v = __ldg(reinterpret_cast<const uint32_t*>(row + i));
+          w = __ldg(reinterpret_cast<const uint32_t*>(row + i));
         } else {
 #pragma unroll
           for (int b = 0; b < 4; ++b)
-            if (i + b < D) v |= (uint32_t)__ldg(row + i + b) << (8 * b);
+            if (i + b < D) w |= (uint32_t)__ldg(row + i + b) << (8 * b);
         }
       }
-      xs[r][c4] = v;
+      xr[v] = w;
     }
-    // E: thread t expands half t & 1 of word kc of neuron n0 + t / 2 into
-    // eight words of +-1 bytes (0x01 / 0xFF); neurons past K stage zeros
+    const int k = n0 + (threadIdx.x >> 1);
+    er = k < K ? (uint32_t)(E[(int64_t)k * nwD + kc] >> (32 * (threadIdx.x & 1))) : 0u;
+  };
+  load_chunk(0);
+
+#pragma unroll 1
+  for (int kc = 0; kc < nwD; ++kc) {
+#pragma unroll
+    for (int v = 0; v < 8; ++v) {
+      const int q = threadIdx.x + kXThreads * v;
+      xs[q >> 4][q & 15] = xr[v];
+    }
     {
+      // E half -> eight words of +-1 bytes (0x01 / 0xFF); neurons past K
+      // stage zeros
       const int r = threadIdx.x >> 1, h = threadIdx.x & 1;
-      const int k = n0 + r;
-      const uint32_t bits = k < K ? (uint32_t)(E[(int64_t)k * nwD + kc] >> (32 * h)) : 0u;
+      const bool live = n0 + r < K;
 #pragma unroll
       for (int q = 0; q < 8; ++q) {
         // nibble -> one bit per byte (the shifted copies do not overlap)
-        const uint32_t p = (((bits >> (4 * q)) & 0xFu) * 0x00204081u) & 0x01010101u;
-        es[r][8 * h + q] = k < K ? ~(p * 0xFEu) : 0u;
+        const uint32_t p = (((er >> (4 * q)) & 0xFu) * 0x00204081u) & 0x01010101u;
+        es[r][8 * h + q] = live ? ~(p * 0xFEu) : 0u;
       }
     }
     __syncthreads();
+    if (kc + 1 < nwD) load_chunk(kc + 1);
 #pragma unroll 4
     for (int c4 = 0; c4 < 16; ++c4) {
       uint32_t a[8], b[8];
