@@ -47,6 +47,9 @@ CONFIG_KEY = "C5"
 SAMPLES_PER_STEP = 100_000
 STEPS_PER_EPOCH = 10
 EVAL_BATCH = 65_536
+# sampled mini-batches for the per-kernel figures: one in 50, i.e. 20 per
+# step of 1,000 mini-batches
+PROFILE_EVERY = 50
 
 # HBM traffic of one k_update launch of the timed region, from an ncu capture
 # of this bench (dram__bytes_read.sum + dram__bytes_write.sum, one pass; see
@@ -292,8 +295,10 @@ def run_ours(args):
         train_step(i, xd, yd)
     torch.cuda.synchronize()
 
-    # timed region: every 10th mini-batch is launched with per-kernel events
-    B.bmlp_set_profiling(h, 10)
+    # timed region: every PROFILE_EVERY-th mini-batch is launched kernel by
+    # kernel between CUDA events (the per-kernel figures below); the others
+    # run as captured graphs
+    B.bmlp_set_profiling(h, PROFILE_EVERY)
     B.bmlp_reset_profile(h)
     B.bmlp_update_stats(h, reset=True)
     launches0 = B.bmlp_launch_count(h)
