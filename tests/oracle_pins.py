@@ -258,6 +258,33 @@ def check_perceptron_golden():
     assert cpr.tolist() == d["cpr"], cpr.tolist()
 
 
+def check_cp_monotone(seed=12):
+    """Alg. 3 l.2-4 with one CP tuple (mu, k) and no reinforcement: every
+    hidden weight of neuron k moves by 2 a^mu_i rho_{k,y} unless that would
+    cross the bound h_max (then it stays), no other weight moves, and the
+    pattern's stability delta_k = z_k rho_{k,y} does not decrease: each sign
+    flip of a visible weight of k raises it by exactly 2."""
+    rng = np.random.default_rng(seed)
+    for trial in range(300):
+        Kp, K, c = int(rng.integers(3, 40)), int(rng.integers(2, 12)), int(rng.integers(2, 5))
+        h_max = 7 if trial % 3 == 0 else 255
+        H = (2 * rng.integers(-(h_max + 1) // 2, (h_max + 1) // 2, (Kp, K)) + 1).astype(np.int32)
+        a = rng.choice([-1, 1], (1, Kp)).astype(np.int8)
+        P = rng.choice([-1, 1], (K, c)).astype(np.int8)
+        y = np.array([rng.integers(0, c)], np.int32)
+        k = int(rng.integers(0, K))
+        H2 = O.perceptron_update(H, a, y, P, np.array([[k]], np.int32), h_max, 0.0, seed, 1, 0)
+        rho = int(P[k, y[0]])
+        step = 2 * a[0].astype(np.int32) * rho
+        want = H.copy()
+        want[:, k] = np.where(np.abs(H[:, k] + step) <= h_max, H[:, k] + step, H[:, k])
+        assert np.array_equal(H2, want), trial
+        s_old, s_new = np.where(H[:, k] > 0, 1, -1), np.where(H2[:, k] > 0, 1, -1)
+        d_old = int((a[0] * s_old).sum()) * rho
+        d_new = int((a[0] * s_new).sum()) * rho
+        assert d_new - d_old == 2 * int((s_old != s_new).sum()) >= 0, trial
+
+
 def _ceil_frac(x: Fraction) -> int:
     return -((-x.numerator) // x.denominator)
 
@@ -671,6 +698,7 @@ ALL_CHECKS = [
     check_select_golden,
     check_select_special,
     check_perceptron_golden,
+    check_cp_monotone,
     check_threshold_exact,
     check_reinforce_rate,
     check_event_law,
