@@ -463,6 +463,63 @@ def run_ours(args):
     return 0
 
 
+ENGINE_NAMES = {1: "popc", 2: "tcgen05_e4m3", 3: "b1_mma_sync", 4: "s8_mma_sync"}
+# iterations of each peak kernel's timed launch (tens of milliseconds each)
+PEAK_ITERS = {1: 20000, 2: 20000, 3: 20000, 4: 20000}
+
+
+def engine_bakeoff(dev, reps=20):
+    """The forward contraction (Alg. 1 l.8, Table 3's XNOR/popcount term) on
+    every unit sm_103a offers: each unit's measured peak (bit-pairs/s over the
+    device), and one 8192 -> 8192 layer at the training batch (100 patterns)
+    and at the evaluation sweep's batch (65,536 patterns) on each engine that
+    has a layer kernel, timed between CUDA events (average of `reps`
+    launches after 3 untimed ones).  tcgen05.mma.kind::i8 does not exist on
+    sm_103a, so +-1 as int8 runs only on the legacy mma.sync path, which has a
+    peak kernel here but no layer kernel."""
+    import torch
+
+    from paper_2412_00119_gb300 import bmlp as B
+
+    out = {"peaks": {}, "layer_8192x8192": {}}
+    for e, name in ENGINE_NAMES.items():
+        rate, ms = B.bmlp_engine_peak(e, PEAK_ITERS[e])
+        out["peaks"][name] = {"bitpairs_per_s": rate, "tbitpairs_per_s": rate / 1e12, "ms": ms}
+    widths = (8192, 8192)
+    model = B.BMLP(widths, 10, seed=1, bs=100)
+    st = torch.cuda.current_stream(dev)
+    for M in (100, EVAL_BATCH):
+        xa = torch.from_numpy(W.random_packed(77, M, widths[0]).view(np.int64)).to(dev)
+        ya = torch.empty((M, W.words(widths[1])), dtype=torch.int64, device=dev)
+        bp = float(M) * widths[0] * widths[1]
+        row = {}
+        for e in (1, 2, 3):
+            name = ENGINE_NAMES[e]
+            for _ in range(3):
+                B.bmlp_layer_forward_engine(model.h, 1, e, xa, ya, stream=st)
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(st)
+            for _ in range(reps if M <= 128 else 3):
+                B.bmlp_layer_forward_engine(model.h, 1, e, xa, ya, stream=st)
+            e1.record(st)
+            torch.cuda.synchronize()
+            us = e0.elapsed_time(e1) * 1e3 / (reps if M <= 128 else 3)
+            pk = out["peaks"][name]["bitpairs_per_s"]
+            row[name] = {"us": us, "tbitpairs_per_s": bp / us / 1e6,
+                         "frac_of_engine_peak": bp / (us * 1e-6) / pk}
+        out["layer_8192x8192"]["M%d" % M] = row
+    model.close()
+    return out
+
+
+def run_bakeoff(args):
+    import torch
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    print(json.dumps({"engines": engine_bakeoff(dev)}), flush=True)
+    return 0
+
+
 def run_ncu_case(args):
     """Small case for profiler captures: the 8192->8192x4->10 model trained on
     N mini-batches twice (the second pass is the one to capture)."""
@@ -531,7 +588,11 @@ def main(argv=None):
                     help="run only the expansion front end on N x 1000 uint8 patterns")
     ap.add_argument("--frontend-shape", default="784,1024", metavar="D,K",
                     help="inputs and width of the expansion layer for --frontend-case")
+    ap.add_argument("--bakeoff", action="store_true",
+                    help="run only the contraction-engine comparison (peaks and layer times)")
     args = ap.parse_args(argv)
+    if args.bakeoff:
+        return run_bakeoff(args)
     if args.ncu_case:
         return run_ncu_case(args)
     if args.frontend_case:

@@ -84,6 +84,12 @@ extern "C" {
 #define BMLP_FWD_AUTO 0     /* library's choice */
 #define BMLP_FWD_POPC 1     /* CUDA-core XOR + popcount */
 #define BMLP_FWD_TCGEN05 2  /* 5th-gen tensor cores, +-1 as e4m3, fp32 accumulate (exact) */
+/* Further contraction units, measured by bmlp_engine_peak (and, for B1MMA,
+ * bmlp_layer_forward_engine) for the engine comparison; training uses POPC or
+ * TCGEN05.  tcgen05.mma.kind::i8 does not exist on sm_103a, so +-1 as int8 on
+ * tensor cores is the legacy mma.sync path (S8MMA). */
+#define BMLP_FWD_B1MMA 3    /* mma.sync m16n8k256 .b1 xor.popc (legacy tensor path) */
+#define BMLP_FWD_S8MMA 4    /* mma.sync m16n8k32 .s8, +-1 as int8 (legacy tensor path) */
 
 typedef struct bmlp bmlp_t;
 
@@ -129,7 +135,11 @@ void bmlp_destroy(bmlp_t* h);
  * flags & BMLP_EPOCH_END: afterwards set E = (last-layer 01-loss count since the
  * previous epoch end) / (patterns since then) and p_r <- p_r sqrt(E).
  * n_errors_out (host, may be NULL): last-layer 01-loss count of these n
- * patterns, measured in the training forward pass.  n == 0 is a no-op. */
+ * patterns, measured in the training forward pass.  n == 0 is a no-op.
+ * If a bounded device-side wait of a training forward pass expires (tensor-
+ * core engine), that mini-batch and every later one until the expiry is
+ * reported change neither H nor W (no marks, no update; the step counter
+ * still advances); the next call that synchronises returns BMLP_ETIMEOUT. */
 int bmlp_train(bmlp_t* h, const uint64_t* x_packed, const int32_t* labels, int64_t n,
                uint32_t flags, void* cuda_stream, int64_t* n_errors_out);
 
@@ -213,6 +223,15 @@ int bmlp_expand_sign(const uint8_t* x, int64_t n, int32_t D, const uint64_t* E, 
 int bmlp_layer_forward(bmlp_t* h, int32_t layer, const uint64_t* a_in, int64_t n,
                        uint64_t* a_out, void* cuda_stream);
 
+/* bmlp_layer_forward on an engine chosen per call (the engine comparison of
+ * the forward contraction, Alg. 1 l.8-9; Table 3 counts its XNOR/popcount
+ * work): engine BMLP_FWD_POPC, BMLP_FWD_TCGEN05 or BMLP_FWD_B1MMA, whatever
+ * the handle's own engine.  Same arguments, layouts and results as
+ * bmlp_layer_forward (every engine gives the same bits); BMLP_EINVAL for
+ * another engine (BMLP_FWD_S8MMA has no layer kernel). */
+int bmlp_layer_forward_engine(bmlp_t* h, int32_t layer, int32_t engine, const uint64_t* a_in,
+                              int64_t n, uint64_t* a_out, void* cuda_stream);
+
 /* Copy layer `layer` (1..L) to host buffers (each may be NULL; formats above),
  * plus the current p_r and step counter t (mini-batches since creation). */
 int bmlp_get_state(const bmlp_t* h, int32_t layer, int16_t* H_out, uint64_t* W_out,
@@ -265,12 +284,14 @@ int bmlp_debug_last_step(const bmlp_t* h, int32_t layer, int16_t* Z, uint64_t* A
 /* Failure-path probe of the bounded device waits (no counterpart in the
  * paper): one CTA initialises an mbarrier and waits on its first phase with
  * the same bounded wait the tensor-core kernels use, limited to `seconds`
- * (0 < seconds <= 10) of SM clock.  arrive != 0: one arrival completes the
- * phase first, so the wait succeeds.  arrive == 0: nothing arrives, the wait
+ * (0 < seconds <= 10) of SM clock.  arrive > 0: one arrival completes the
+ * phase first, so the wait succeeds.  arrive <= 0: nothing arrives, the wait
  * gives up when the limit expires, the kernel counts it as a timeout and
- * returns (no trap, no fault; the context stays usable).  Synchronises, then
- * returns BMLP_ETIMEOUT if any timeout is pending (and clears it), else
- * BMLP_OK. */
+ * returns (no trap, no fault; the context stays usable).  Synchronises; then,
+ * for arrive >= 0, returns BMLP_ETIMEOUT if any timeout is pending (and clears
+ * it), else BMLP_OK; for arrive < 0 returns BMLP_OK and leaves the expiry
+ * pending, as an expired wait inside a training step would (the next call
+ * that synchronises reports it). */
 int bmlp_debug_wait_probe(bmlp_t* h, int32_t arrive, double seconds);
 
 /* Per-kernel timing.  every = 0: off.  every = S > 0: every S-th training
@@ -301,6 +322,36 @@ int64_t bmlp_launch_count(const bmlp_t* h);
 int bmlp_update_stats(bmlp_t* h, int64_t* rows_out, int64_t* streamed_out, int64_t* bytes_out,
                       int32_t reset);
 
+/* Failure injection for the allocation paths (no counterpart in the paper;
+ * it tests the library's clean-up without a GPU fault).  After
+ * bmlp_debug_fail_alloc(n), n >= 1, the n-th memory allocation the library
+ * makes from then on -- counting every cudaMalloc of a device buffer and the
+ * pinned host block of bmlp_create, in any handle of the process -- fails as
+ * if memory were exhausted: the call that needed it returns BMLP_ENOMEM
+ * ("... (injected)"), a half-built handle is freed whole, and the injection
+ * disarms itself.  n = 0 disarms it.  BMLP_EINVAL for n < 0.
+ * bmlp_debug_alloc_stats: the number of allocations the library holds now,
+ * over every live handle of the process, and their bytes (either output may
+ * be NULL); a failed bmlp_create leaves both where they were.  Host only;
+ * neither call touches the device. */
+int bmlp_debug_fail_alloc(int64_t nth);
+int bmlp_debug_alloc_stats(int64_t* live_allocs, int64_t* live_bytes);
+
+/* Peak rate of one contraction unit on the current device (the engine
+ * comparison for the forward XNOR/popcount term of Table 3; Alg. 1 l.8):
+ * a kernel that keeps its operands on chip and issues only that unit's
+ * instruction, `iters` iterations per thread (or per MMA-issuing thread),
+ * timed between CUDA events after one untimed launch.  engine: BMLP_FWD_POPC
+ * (32-bit XOR + popcount on CUDA cores, 32 bit-pairs each), BMLP_FWD_TCGEN05
+ * (tcgen05.mma kind::f8f6f4 e4m3, M128 N256 K32), BMLP_FWD_B1MMA
+ * (mma.sync m16n8k256 b1 xor.popc), BMLP_FWD_S8MMA (mma.sync m16n8k32 s8).
+ * *bitpairs_per_s: multiply-accumulates (bit-pairs) per second over the whole
+ * device; *ms_out (may be NULL): the timed launch.  Synchronises the device;
+ * allocates a few bytes.  No handle (errors: bmlp_last_error(NULL));
+ * BMLP_EINVAL for an unknown engine or iters outside 1..2^31; BMLP_ETIMEOUT
+ * if the tcgen05 kernel's bounded completion wait expired. */
+int bmlp_engine_peak(int32_t engine, int64_t iters, double* bitpairs_per_s, double* ms_out);
+
 /* Forward-only evaluation that allocates no memory.  The paper has no
  * counterpart: this is bmlp_predict with its scratch moved into the library,
  * for callers that cannot call cudaMalloc -- code running in a host callback,
@@ -312,8 +363,9 @@ int bmlp_update_stats(bmlp_t* h, int64_t* rows_out, int64_t* streamed_out, int64
  * exits.  Results equal bmlp_predict's.
  *   n * ceil(max_l K_l / 64) must not exceed 1,048,576 (n <= 8192 for
  *   8192-wide layers); a larger n returns BMLP_EINVAL before any work.
- *   x_packed and labels_out must be device pointers (staging host buffers
- *   would allocate); host pointers return BMLP_EINVAL.
+ *   x_packed and labels_out must be device pointers on the current device
+ *   (or managed memory): staging host buffers would allocate; host pointers
+ *   and other devices' pointers return BMLP_EINVAL.
  *   The first call on a device looks up the array's device address once
  *   (cudaGetSymbolAddress); make that first call before any stream capture.
  *   Every call shares the array and it keeps the last call's contents (each

@@ -28,7 +28,7 @@ BMLP_ETIMEOUT = -4
 BMLP_ESTATE = -5
 BMLP_ENODEV = -6
 BMLP_EPOCH_END = 1
-BMLP_FWD_AUTO, BMLP_FWD_POPC, BMLP_FWD_TCGEN05 = 0, 1, 2
+BMLP_FWD_AUTO, BMLP_FWD_POPC, BMLP_FWD_TCGEN05, BMLP_FWD_B1MMA, BMLP_FWD_S8MMA = 0, 1, 2, 3, 4
 BMLP_GROUPS_CONTIGUOUS, BMLP_GROUPS_FIXED, BMLP_GROUPS_RESHUFFLED = 0, 1, 2
 PROFILE_KINDS = ("train_forward", "cls_select", "update", "eval_forward", "eval_out", "copy",
                  "r_events")
@@ -82,6 +82,10 @@ SIGNATURES = [
     ("bmlp_expand_weights", C.c_int, [C.c_uint64, C.c_int32, C.c_int32, _vp, _vp]),
     ("bmlp_expand_sign", C.c_int, [_vp, C.c_int64, C.c_int32, _vp, C.c_int32, _vp, _vp]),
     ("bmlp_debug_wait_probe", C.c_int, [_vp, C.c_int32, C.c_double]),
+    ("bmlp_engine_peak", C.c_int, [C.c_int32, C.c_int64, _f64p, _f64p]),
+    ("bmlp_debug_fail_alloc", C.c_int, [C.c_int64]),
+    ("bmlp_debug_alloc_stats", C.c_int, [_i64p, _i64p]),
+    ("bmlp_layer_forward_engine", C.c_int, [_vp, C.c_int32, C.c_int32, _vp, C.c_int64, _vp, _vp]),
 ]
 
 
@@ -219,15 +223,45 @@ def bmlp_expand_sign(x, E, K, out, stream=None):
     _check(lib().bmlp_expand_sign(_ptr(x), n, D, _ptr(E), K, _ptr(out), _stream(stream)), None)
 
 
-def bmlp_debug_wait_probe(h, arrive, seconds=0.05):
-    """Run the bounded-wait probe; raises BmlpError(BMLP_ETIMEOUT) if it expired."""
-    _check(lib().bmlp_debug_wait_probe(h, 1 if arrive else 0, float(seconds)), h)
+def bmlp_debug_wait_probe(h, arrive, seconds=0.05, leave_pending=False):
+    """Run the bounded-wait probe; raises BmlpError(BMLP_ETIMEOUT) if it expired.
+    leave_pending: nothing arrives and the expiry is left for the next
+    synchronising call to report."""
+    a = -1 if leave_pending else (1 if arrive else 0)
+    _check(lib().bmlp_debug_wait_probe(h, a, float(seconds)), h)
 
 
 def bmlp_layer_forward(h, layer, a_in, a_out, n=None, stream=None):
     """a_out = sign(a_in W_layer), packed rows on the device."""
     n = a_out.shape[0] if n is None else n
     _check(lib().bmlp_layer_forward(h, layer, _ptr(a_in), n, _ptr(a_out), _stream(stream)), h)
+
+
+def bmlp_layer_forward_engine(h, layer, engine, a_in, a_out, n=None, stream=None):
+    """bmlp_layer_forward on the given engine (BMLP_FWD_POPC / TCGEN05 / B1MMA)."""
+    n = a_out.shape[0] if n is None else n
+    _check(lib().bmlp_layer_forward_engine(h, layer, engine, _ptr(a_in), n, _ptr(a_out),
+                                           _stream(stream)), h)
+
+
+def bmlp_debug_fail_alloc(nth):
+    """Arm (nth >= 1) or disarm (0) the one-shot failure of the nth allocation."""
+    _check(lib().bmlp_debug_fail_alloc(int(nth)), None)
+
+
+def bmlp_debug_alloc_stats():
+    """(allocations the library holds, their bytes), over all live handles."""
+    n, b = C.c_int64(), C.c_int64()
+    _check(lib().bmlp_debug_alloc_stats(C.byref(n), C.byref(b)), None)
+    return n.value, b.value
+
+
+def bmlp_engine_peak(engine, iters):
+    """(bit-pairs per second over the device, ms of the timed launch) of one
+    contraction unit's peak kernel."""
+    bp, ms = C.c_double(), C.c_double()
+    _check(lib().bmlp_engine_peak(engine, iters, C.byref(bp), C.byref(ms)), None)
+    return bp.value, ms.value
 
 
 def bmlp_update_stats(h, reset=False):

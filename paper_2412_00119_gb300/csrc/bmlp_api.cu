@@ -10,6 +10,7 @@
 // an NVTX range named after it (header-only NVTX v3: a no-op unless a tracing
 // tool is attached).
 #include <algorithm>
+#include <atomic>
 #include <cmath>
 #include <cstddef>
 #include <cstdarg>
@@ -27,6 +28,20 @@ using namespace bk;
 namespace {
 
 thread_local std::string g_create_error;
+
+// Process-wide accounting of the memory the library holds (every handle's
+// device buffers and pinned host block), and the one-shot injected failure of
+// the n-th allocation from the moment bmlp_debug_fail_alloc armed it.
+std::atomic<int64_t> g_live_allocs{0}, g_live_bytes{0};
+std::atomic<int64_t> g_fail_at{0}, g_alloc_seq{0};
+
+// True when this allocation is the armed one (the injection then disarms).
+bool injected_alloc_failure() {
+  if (g_fail_at.load() <= 0) return false;
+  const int64_t seq = ++g_alloc_seq;
+  int64_t at = g_fail_at.load();
+  return seq == at && g_fail_at.compare_exchange_strong(at, 0);
+}
 
 // NVTX range for the lifetime of an entry point call.
 struct TraceRange {
@@ -55,6 +70,7 @@ struct bmlp {
   Ctrl* dCtrl = nullptr;
   RTables* dRT = nullptr;
   std::vector<void*> allocs;
+  int64_t held_bytes = 0;  // device bytes in allocs (+ the pinned host block)
   // evaluation scratch (grown on demand)
   uint64_t* evA[2] = {nullptr, nullptr};
   int64_t evCap = 0;
@@ -110,9 +126,14 @@ int cuda_fail(bmlp_t* h, cudaError_t e, const char* what) {
 template <typename T>
 int dalloc(bmlp_t* h, T** p, size_t count) {
   void* q = nullptr;
-  cudaError_t e = cudaMalloc(&q, count * sizeof(T) > 0 ? count * sizeof(T) : 16);
+  const size_t bytes = count * sizeof(T) > 0 ? count * sizeof(T) : 16;
+  if (injected_alloc_failure()) return fail(h, BMLP_ENOMEM, "cudaMalloc of %zu bytes failed (injected)", bytes);
+  cudaError_t e = cudaMalloc(&q, bytes);
   if (e != cudaSuccess) return cuda_fail(h, e, "cudaMalloc");
   h->allocs.push_back(q);
+  h->held_bytes += (int64_t)bytes;
+  g_live_allocs += 1;
+  g_live_bytes += (int64_t)bytes;
   *p = static_cast<T*>(q);
   return BMLP_OK;
 }
@@ -536,10 +557,14 @@ int bmlp_create(const int32_t* widths, int32_t n_widths, int32_t classes, int16_
     return bail(rc);
   P.ctrl = h->dCtrl;
   P.rt = h->dRT;
+  if (injected_alloc_failure())
+    return bail(fail(h, BMLP_ENOMEM, "cudaMallocHost failed (injected)"));
   if (cudaMallocHost(&h->hostPinned, 4 * sizeof(unsigned long long)) != cudaSuccess) {
     h->hostPinned = nullptr;
     return bail(fail(h, BMLP_ENOMEM, "cudaMallocHost failed"));
   }
+  g_live_allocs += 1;
+  g_live_bytes += (int64_t)(4 * sizeof(unsigned long long));
   // initial state (Alg. 1 l.2)
   for (int l = 1; l <= L; ++l) {
     DevLayer& D = P.layer[l - 1];
@@ -583,7 +608,13 @@ void bmlp_destroy(bmlp_t* h) {
   if (h->evJoin) cudaEventDestroy(h->evJoin);
   for (auto e : h->evPool) cudaEventDestroy(e);
   for (void* p : h->allocs) cudaFree(p);
-  if (h->hostPinned) cudaFreeHost(h->hostPinned);
+  g_live_allocs -= (int64_t)h->allocs.size();
+  g_live_bytes -= h->held_bytes;
+  if (h->hostPinned) {
+    cudaFreeHost(h->hostPinned);
+    g_live_allocs -= 1;
+    g_live_bytes -= (int64_t)(4 * sizeof(unsigned long long));
+  }
   delete h;
 }
 
@@ -911,6 +942,41 @@ int bmlp_layer_forward(bmlp_t* h, int32_t layer, const uint64_t* a_in, int64_t n
   return prof_collect(h, st);
 }
 
+int bmlp_layer_forward_engine(bmlp_t* h, int32_t layer, int32_t engine, const uint64_t* a_in,
+                              int64_t n, uint64_t* a_out, void* cuda_stream) {
+  TraceRange trace("bmlp_layer_forward_engine");
+  if (!h) return BMLP_EINVAL;
+  h->err.clear();
+  if (layer < 1 || layer > h->L) return fail(h, BMLP_EINVAL, "layer must be in 1..%d", h->L);
+  if (engine != BMLP_FWD_POPC && engine != BMLP_FWD_TCGEN05 && engine != BMLP_FWD_B1MMA)
+    return fail(h, BMLP_EINVAL, "engine %d has no layer kernel", engine);
+  if (n < 0) return fail(h, BMLP_EINVAL, "n < 0");
+  if (n == 0) return BMLP_OK;
+  if (!a_in || !a_out || !is_device_ptr(a_in) || !is_device_ptr(a_out))
+    return fail(h, BMLP_EINVAL, "a_in and a_out must be device pointers");
+  if (engine == BMLP_FWD_TCGEN05) CK(h, prepare_forward_eval_tc());
+  cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
+  const DevLayer& D = h->hp.layer[layer - 1];
+  for (int64_t s0 = 0; s0 < n; s0 += kEvalChunk) {
+    const int64_t m = std::min(kEvalChunk, n - s0);
+    const uint64_t* in = a_in + s0 * D.nw_in;
+    uint64_t* out = a_out + s0 * D.nw_out;
+    prof_begin(h, kProfEvalFwd, st);
+    if (engine == BMLP_FWD_TCGEN05)
+      launch_forward_eval_tc(in, m, D.nw_in, D.W, D.Kout, D.Kin, out, D.nw_out,
+                             &h->dCtrl->timeouts, st);
+    else if (engine == BMLP_FWD_B1MMA)
+      CK(h, launch_forward_b1(in, m, D.nw_in, D.W, D.Kout, D.Kin, out, D.nw_out, st));
+    else
+      k_forward_eval<<<eval_forward_grid(m, D.Kout), eval_forward_block(), 0, st>>>(
+          in, m, D.nw_in, D.W, D.Kout, D.Kin, out, D.nw_out);
+    prof_end(h, st);
+    CK(h, cudaGetLastError());
+    h->launches += 1;
+  }
+  return prof_collect(h, st);
+}
+
 int bmlp_debug_wait_probe(bmlp_t* h, int32_t arrive, double seconds) {
   if (!h) return BMLP_EINVAL;
   h->err.clear();
@@ -918,9 +984,10 @@ int bmlp_debug_wait_probe(bmlp_t* h, int32_t arrive, double seconds) {
   int khz = 0;
   CK(h, cudaDeviceGetAttribute(&khz, cudaDevAttrClockRate, h->device));
   const unsigned long long limit = (unsigned long long)(seconds * 1e3 * (double)khz);
-  launch_wait_probe(&h->dCtrl->timeouts, arrive ? 1 : 0, limit, 0);
+  launch_wait_probe(&h->dCtrl->timeouts, arrive > 0 ? 1 : 0, limit, 0);
   CK(h, cudaGetLastError());
   CK(h, cudaDeviceSynchronize());
+  if (arrive < 0) return BMLP_OK;  // the expiry stays pending for the next synchronising call
   uint32_t t = 0;
   CK(h, cudaMemcpy(&t, &h->dCtrl->timeouts, sizeof(t), cudaMemcpyDeviceToHost));
   if (t != 0) {
@@ -928,6 +995,67 @@ int bmlp_debug_wait_probe(bmlp_t* h, int32_t arrive, double seconds) {
     return fail(h, BMLP_ETIMEOUT, "a bounded device-side wait expired");
   }
   return BMLP_OK;
+}
+
+int bmlp_debug_fail_alloc(int64_t nth) {
+  if (nth < 0) return fail(nullptr, BMLP_EINVAL, "nth must be >= 0");
+  g_fail_at.store(0);
+  g_alloc_seq.store(0);
+  g_fail_at.store(nth);
+  return BMLP_OK;
+}
+
+int bmlp_debug_alloc_stats(int64_t* live_allocs, int64_t* live_bytes) {
+  if (live_allocs) *live_allocs = g_live_allocs.load();
+  if (live_bytes) *live_bytes = g_live_bytes.load();
+  return BMLP_OK;
+}
+
+int bmlp_engine_peak(int32_t engine, int64_t iters, double* bitpairs_per_s, double* ms_out) {
+  TraceRange trace("bmlp_engine_peak");
+  g_create_error.clear();
+  if (!bitpairs_per_s) return fail(nullptr, BMLP_EINVAL, "bitpairs_per_s is NULL");
+  if (engine != BMLP_FWD_POPC && engine != BMLP_FWD_TCGEN05 && engine != BMLP_FWD_B1MMA &&
+      engine != BMLP_FWD_S8MMA)
+    return fail(nullptr, BMLP_EINVAL, "unknown engine %d", engine);
+  if (iters < 1 || iters > (int64_t)1 << 31) return fail(nullptr, BMLP_EINVAL, "iters out of range");
+  int dev = 0, sms = 0;
+  CK(nullptr, cudaGetDevice(&dev));
+  CK(nullptr, cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
+  int* sink = nullptr;
+  unsigned int* tmo = nullptr;
+  cudaEvent_t e0 = nullptr, e1 = nullptr;
+  int rc = BMLP_OK;
+  double bp = 0.0;
+  float ms = 0.f;
+  auto step = [&](cudaError_t x, const char* what) {
+    if (rc == BMLP_OK && x != cudaSuccess) rc = cuda_fail(nullptr, x, what);
+  };
+  step(cudaMalloc(&sink, sizeof(int) * 8 * (size_t)sms), "cudaMalloc");
+  step(cudaMalloc(&tmo, sizeof(unsigned int)), "cudaMalloc");
+  if (rc == BMLP_OK) step(cudaMemset(tmo, 0, sizeof(unsigned int)), "cudaMemset");
+  if (rc == BMLP_OK) step(cudaEventCreate(&e0), "cudaEventCreate");
+  if (rc == BMLP_OK) step(cudaEventCreate(&e1), "cudaEventCreate");
+  // one untimed launch (clocks up, first-launch costs paid), then the timed one
+  if (rc == BMLP_OK)
+    step(launch_engine_peak(engine, std::max<int64_t>(1, iters / 4), sms, sink, tmo, 0, &bp), "peak kernel");
+  if (rc == BMLP_OK) step(cudaEventRecord(e0, 0), "cudaEventRecord");
+  if (rc == BMLP_OK) step(launch_engine_peak(engine, iters, sms, sink, tmo, 0, &bp), "peak kernel");
+  if (rc == BMLP_OK) step(cudaEventRecord(e1, 0), "cudaEventRecord");
+  if (rc == BMLP_OK) step(cudaEventSynchronize(e1), "peak kernel");
+  if (rc == BMLP_OK) step(cudaEventElapsedTime(&ms, e0, e1), "cudaEventElapsedTime");
+  unsigned int t = 0;
+  if (rc == BMLP_OK) step(cudaMemcpy(&t, tmo, sizeof(t), cudaMemcpyDeviceToHost), "cudaMemcpy");
+  if (rc == BMLP_OK && t != 0) rc = fail(nullptr, BMLP_ETIMEOUT, "a bounded device-side wait expired");
+  if (rc == BMLP_OK) {
+    *bitpairs_per_s = bp / ((double)ms * 1e-3);
+    if (ms_out) *ms_out = ms;
+  }
+  if (e0) cudaEventDestroy(e0);
+  if (e1) cudaEventDestroy(e1);
+  if (sink) cudaFree(sink);
+  if (tmo) cudaFree(tmo);
+  return rc;
 }
 
 int bmlp_debug_last_step(const bmlp_t* hc, int32_t layer, int16_t* Z, uint64_t* A, uint8_t* mark,
@@ -1001,5 +1129,9 @@ int bmlp_internal_eval_view(const bmlp_t* h, const bk::StepParams** params, int*
 }
 
 int bmlp_internal_fail(bmlp_t* h, int code, const char* msg) { return fail(h, code, "%s", msg); }
+
+void bmlp_internal_clear_error(bmlp_t* h) {
+  if (h) h->err.clear();
+}
 
 void bmlp_internal_count_launches(bmlp_t* h, int64_t n) { h->launches += n; }

@@ -242,6 +242,15 @@ void launch_forward_eval_tc(const uint64_t* A, int64_t M, int nw_in, const uint6
                             int Kin, uint64_t* Aout, int nw_out, unsigned int* timeouts,
                             cudaStream_t st);
 
+// One layer on the b1 mma.sync path (kern_forward_b1.cu): Aout (M x nw_out)
+// = packed sign(A W^T), sign(0) = +1, pad bits 0.
+cudaError_t launch_forward_b1(const uint64_t* A, int64_t M, int nw_in, const uint64_t* W, int N,
+                              int Kin, uint64_t* Aout, int nw_out, cudaStream_t st);
+// Peak-rate kernel of one contraction engine (BMLP_FWD_*): launches it on
+// `sms` SMs' worth of CTAs and returns the bit-pairs (MACs) it performs.
+cudaError_t launch_engine_peak(int engine, int64_t iters, int sms, int* sink, unsigned int* timeouts,
+                               cudaStream_t st, double* bitpairs);
+
 // Launch helpers implemented in the kernel files (grid shapes live next to the
 // kernels they describe).
 dim3 train_forward_grid(int bs, int Kout);

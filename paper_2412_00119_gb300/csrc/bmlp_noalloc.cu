@@ -46,6 +46,7 @@ int noalloc_scratch(uint64_t** out) {
 // Defined in bmlp_api.cu: the model geometry this entry point needs.
 int bmlp_internal_eval_view(const bmlp_t* h, const bk::StepParams** params, int* nwmax);
 int bmlp_internal_fail(bmlp_t* h, int code, const char* msg);
+void bmlp_internal_clear_error(bmlp_t* h);
 void bmlp_internal_count_launches(bmlp_t* h, int64_t n);
 
 extern "C" int bmlp_predict_noalloc(bmlp_t* h, const uint64_t* x_packed, int64_t n,
@@ -53,18 +54,26 @@ extern "C" int bmlp_predict_noalloc(bmlp_t* h, const uint64_t* x_packed, int64_t
   const bk::StepParams* P = nullptr;
   int nwmax = 0;
   if (bmlp_internal_eval_view(h, &P, &nwmax) != BMLP_OK) return BMLP_EINVAL;
+  bmlp_internal_clear_error(h);
   if (n < 0) return bmlp_internal_fail(h, BMLP_EINVAL, "n < 0");
   if (n == 0) return BMLP_OK;
   if (!x_packed || !labels_out) return bmlp_internal_fail(h, BMLP_EINVAL, "x or labels_out is NULL");
-  if (n * (int64_t)nwmax > kNoallocWords)
+  // nwmax >= 1; the quotient form cannot overflow for any caller-supplied n
+  if (n > kNoallocWords / nwmax)
     return bmlp_internal_fail(h, BMLP_EINVAL,
                               "n exceeds the fixed scratch: at most 1048576 / ceil(max K_l / 64) rows");
+  int cur_dev = 0;
+  if (cudaGetDevice(&cur_dev) != cudaSuccess) {
+    (void)cudaGetLastError();
+    return bmlp_internal_fail(h, BMLP_ECUDA, "cudaGetDevice failed");
+  }
   cudaPointerAttributes a;
   for (const void* p : {static_cast<const void*>(x_packed), static_cast<const void*>(labels_out)}) {
     if (cudaPointerGetAttributes(&a, p) != cudaSuccess ||
-        (a.type != cudaMemoryTypeDevice && a.type != cudaMemoryTypeManaged)) {
+        !(a.type == cudaMemoryTypeManaged || (a.type == cudaMemoryTypeDevice && a.device == cur_dev))) {
       (void)cudaGetLastError();
-      return bmlp_internal_fail(h, BMLP_EINVAL, "x and labels_out must be device pointers");
+      return bmlp_internal_fail(h, BMLP_EINVAL,
+                                "x and labels_out must be device pointers on the current device");
     }
   }
   uint64_t* scratch = nullptr;

@@ -44,6 +44,14 @@ __global__ void __launch_bounds__(kClsThreads) k_cls_select(const StepParams* __
   const int64_t start = batch_start(P);
   const int64_t bsz = batch_size(P, start);
   if (mu >= bsz) return;
+  if (ctrl->timeouts != 0u) {
+    // a bounded wait of this step's forward pass expired (or an earlier one
+    // is not yet reported): Z and A are not valid, so the pattern is marked
+    // for nothing; with every mark 0 the update leaves H and W as they are
+    // and only advances the step counters
+    if (threadIdx.x == 0) Ly.mark[mu] = 0;
+    return;
+  }
   const int c = P->c;
   __shared__ int yh[BMLP_MAX_CLASSES];
   __shared__ int s_mark, s_y;
@@ -428,6 +436,9 @@ __global__ void __launch_bounds__(kUpdThreads, 4) k_update(const StepParams* __r
   const uint32_t s = ctrl->s;
   const int64_t start = (int64_t)s * P->bs;
   const int bsz = (int)batch_size(P, start);
+  // an expired bounded wait in this step's forward pass: no CP, no R (the
+  // selection kernel marked nothing either); the counters still advance
+  const bool step_failed = ctrl->timeouts != 0u;
   __syncthreads();
 
   const int c = P->c;
@@ -456,7 +467,7 @@ __global__ void __launch_bounds__(kUpdThreads, 4) k_update(const StepParams* __r
     for (int gr = base; gr < min(base + kRowChunk, rows_total); ++gr) {
       int li = 0;
       while (li + 1 < P->L && gr >= P->layer[li + 1].row_base) ++li;
-      if (ctrl->any_mark[li] == 0u) continue;   // M_l empty: no CP, no R
+      if (step_failed || ctrl->any_mark[li] == 0u) continue;   // M_l empty: no CP, no R
       const DevLayer& Ly = P->layer[li];
       const int k = gr - Ly.row_base;
       const int gamma = Ly.gamma;

@@ -123,3 +123,25 @@ def test_null_handle_calls_fail_cleanly():
     assert lib.bmlp_get_state(None, 1, None, None, None, None, None) == B.BMLP_EINVAL
     assert lib.bmlp_launch_count(None) == -1
     lib.bmlp_destroy(None)
+    assert lib.bmlp_layer_forward_engine(None, 1, 1, None, 0, None, None) == B.BMLP_EINVAL
+    assert lib.bmlp_predict_noalloc(None, None, 0, None, None) == B.BMLP_EINVAL
+
+
+def test_engine_peak_rejects_bad_arguments():
+    lib = pkg.lib()
+    with pytest.raises(B.BmlpError) as ei:
+        B.bmlp_engine_peak(99, 10)
+    assert ei.value.code == B.BMLP_EINVAL and "engine" in str(ei.value)
+    with pytest.raises(B.BmlpError):
+        B.bmlp_engine_peak(B.BMLP_FWD_POPC, 0)
+    assert lib.bmlp_engine_peak(B.BMLP_FWD_POPC, 10, None, None) == B.BMLP_EINVAL
+
+
+def test_alloc_injection_host_side():
+    """Arming and disarming the injected allocation failure and reading the
+    live-allocation counters need no device; no handle exists here."""
+    assert B.bmlp_debug_alloc_stats() == (0, 0)
+    with pytest.raises(B.BmlpError):
+        B.bmlp_debug_fail_alloc(-1)
+    B.bmlp_debug_fail_alloc(3)
+    B.bmlp_debug_fail_alloc(0)

@@ -385,7 +385,7 @@ def test_zero_patterns_is_a_noop():
 
 # -- the workload shapes at full width ------------------------------------------
 
-def _full_width(key, steps=None, n_test=None, sweep=False, fwd=B.BMLP_FWD_AUTO):
+def _full_width(key, steps=None, n_test=None, sweep=False, fwd=B.BMLP_FWD_AUTO, epochs=1):
     cfg = W.CONFIGS[key]
     n = cfg.n_train if steps is None else steps * 100
     xp = W.make_inputs(cfg, "train", n)
@@ -393,10 +393,12 @@ def _full_width(key, steps=None, n_test=None, sweep=False, fwd=B.BMLP_FWD_AUTO):
     y = W.teacher_labels_pm1(teacher, W.unpack(xp, cfg.widths[0]))
     gpu = B.BMLP(cfg.widths, cfg.classes, seed=cfg.model_seed, bs=100, fwd_impl=fwd)
     ref = O.OracleModel(list(cfg.widths), cfg.classes, seed=cfg.model_seed, bs=100)
-    eg = gpu.train(dev_x(xp), dev_y(y), epoch_end=steps is None, count_errors=True)
-    er = ref.train(W.unpack(xp, cfg.widths[0]), y, epoch_end=steps is None)
-    assert eg == er
-    assert_same_state(gpu, ref, key)
+    xd, yd, xo = dev_x(xp), dev_y(y), W.unpack(xp, cfg.widths[0])
+    for e in range(epochs):
+        eg = gpu.train(xd, yd, epoch_end=steps is None, count_errors=True)
+        er = ref.train(xo, y, epoch_end=steps is None)
+        assert eg == er, (key, e, eg, er)
+        assert_same_state(gpu, ref, "%s epoch %d" % (key, e + 1))
     if n_test:
         xt = W.make_inputs(cfg, "test", n_test)
         o = torch.empty(n_test, dtype=torch.int32, device=DEV)
@@ -416,8 +418,11 @@ def test_c1_784_256_full_epoch():
     _full_width("C1", n_test=500)
 
 
-def test_c2_784_1024x3_first_epoch():
-    _full_width("C2", n_test=2000)
+def test_c2_784_1024x3_two_epochs():
+    """Both of the first two epochs of the 784 -> 1024 x3 -> 10 workload
+    against the live oracle, element by element: the second epoch runs at the
+    p_r that the first epoch's end rescaled (Alg. 1 l.21)."""
+    _full_width("C2", n_test=2000, epochs=2)
 
 
 def test_c3_3072_2048x3_prefix():
