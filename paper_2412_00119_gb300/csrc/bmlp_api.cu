@@ -257,7 +257,7 @@ int enqueue_step(bmlp_t* h, cudaStream_t st, bool fork, bool chained = false) {
     }
     prof_begin(h, kProfTrainFwd, st);
     if (h->fwd_impl == BMLP_FWD_TCGEN05)
-      CK(h, launch_train_forward_tc(l > 1, h->K[l], st, fork && (l > 1 || chained), h->dP, l));
+      CK(h, launch_train_forward_tc(h->K[l], st, fork && (l > 1 || chained), h->dP, l));
     else
       k_train_forward<<<train_forward_grid(h->bs, h->K[l]), train_forward_block(), 0, st>>>(h->dP, l);
     prof_end(h, st);
@@ -528,12 +528,6 @@ int bmlp_create(const int32_t* widths, int32_t n_widths, int32_t classes, int16_
     if (group_mode != BMLP_GROUPS_CONTIGUOUS &&
         ((rc = dalloc(h, &D.member, (size_t)D.Kout)) || (rc = dalloc(h, &D.group_of, (size_t)D.Kout))))
       return bail(rc);
-    D.AE = nullptr;
-    if (fwd == BMLP_FWD_TCGEN05 && l < L) {
-      if ((rc = dalloc(h, &D.AE, act_tile_bytes(D.Kout))) != BMLP_OK) return bail(rc);
-      cudaError_t ez = cudaMemset(D.AE, 0, act_tile_bytes(D.Kout));
-      if (ez != cudaSuccess) return bail(cuda_fail(h, ez, "cudaMemset"));
-    }
   }
   P.rows_total = rows_total;
   P.ev_ctas_total = ev_cta;

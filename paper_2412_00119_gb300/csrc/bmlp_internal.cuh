@@ -25,12 +25,7 @@ namespace bk {
 //   Z    int16 [bs][K_out]        pre-activations of the current mini-batch
 //   A    uint64 [bs][nw_out]      packed activations a_l of the current mini-batch
 //   mark uint8 [bs]               1 iff the pattern is in M_l
-//   sel  int16 [bs][G]            selected neuron per (pattern, group), -1 = none
-//   AE   uint8 [ceil(K_out/128)][128][128]  (tcgen05 engine, l < L) the
-//                                 activations of the mini-batch as e4m3 +-1 (0 past
-//                                 K_out), in the 128B-swizzled K-major image of
-//                                 128 patterns x 128 K-elements per tile that the
-//                                 next layer's MMA reads; rows >= bs are zero
+//   sel  int16 [G][bs]            selected neuron per (group, pattern), -1 = none
 // ---------------------------------------------------------------------------
 struct DevLayer {
   int16_t* H;
@@ -42,7 +37,6 @@ struct DevLayer {
   uint64_t* A;
   uint8_t* mark;
   int16_t* sel;       // [G][bs] selected neuron per group and pattern, or -1 (group-major)
-  uint8_t* AE;
   int16_t* member;    // [K_out] group order (neuron at position j), or null: contiguous groups
   int16_t* group_of;  // [K_out] group of neuron k (with member)
   int32_t Kin, Kout, nw_in, nw_out, ldh, gamma, G;
@@ -215,13 +209,12 @@ __global__ void k_transpose_rho(const int8_t* rho, int8_t* rhoT, int Kout, int c
 __global__ void k_repack_w(const int16_t* H, uint64_t* W, int Kin, int Kout, int ldh, int nw_in,
                            int h_max, int hb);
 // Tensor-core forward (tcgen05, +-1 as e4m3, exact fp32 sums), training layer l;
-// needs bs <= 128.  tiles: take the A operand from layer l-1's AE image.
+// needs bs <= 128.  The activations of layer l - 1 (the inputs for l = 1) are
+// read as packed bits.
 size_t train_forward_tc_smem();
 cudaError_t prepare_train_forward_tc();
 // pdl: launched with the programmatic-stream-serialization attribute.
-cudaError_t launch_train_forward_tc(bool tiles, int Kout, cudaStream_t st, bool pdl,
-                                   const StepParams* P, int l);
-size_t act_tile_bytes(int K);  // bytes of an AE image for K activations
+cudaError_t launch_train_forward_tc(int Kout, cudaStream_t st, bool pdl, const StepParams* P, int l);
 // Median binarisation of n x K fp32 patterns into n x nw packed words.
 void launch_binarize_median(const float* x, int64_t n, int K, int nw, uint64_t* out,
                             cudaStream_t st);

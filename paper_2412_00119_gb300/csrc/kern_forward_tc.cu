@@ -1,45 +1,53 @@
 // kern_forward_tc.cu -- tensor-core forward contraction of the BMLP
-// (Alg. 1 l.8-9) on sm_103a with tcgen05.
+// (Alg. 1 l.8-9) on sm_103a with tcgen05, for one training mini-batch.
 //
 //   z^mu_k = sum_i a^mu_i w_ik,  a, w in {-1, +1}
 //
 // is computed exactly as an e4m3 x e4m3 -> fp32 matrix product: +-1 are exact
-// in e4m3 (0x38 / 0xB8), pad elements are 0x00, and every partial sum is an
-// integer of magnitude <= K_in < 2^24, exact in fp32 whatever the order.
+// in e4m3 (0x38 / 0xB8), padded weight elements are 0x00, and every partial
+// sum is an integer of magnitude <= K_in < 2^24, exact in fp32 in any order.
 //
-// Tiling.  A tcgen05.mma of M = 128 rows costs about the same time for N = 64
-// as for N = 256, so the kernel uses the widest instruction: a tile is the
-// whole mini-batch (<= 128 patterns, rows >= bs unused) x TN = 256 neurons.
-// To keep every SM busy with only K_out / 256 tiles, the K range is split
-// across a cluster of kSplit = 4 CTAs: CTA r of the cluster accumulates
-// k-blocks [r nkb / 4, (r + 1) nkb / 4) in TMEM, writes its 128 x 256 fp32
-// partial to its own shared memory, and after a cluster barrier reduces the
-// four partials of its 64 columns through distributed shared memory
-// (mapa + ld.shared::cluster) and writes them out.
+// Tiling.  A tile is the whole mini-batch (MMA M = 128 rows; rows >= bs are
+// computed and never read) x TN = 256 neurons.  The K range is split across a
+// cluster of kSplit = 4 CTAs so that every SM has work with only K_out / 256
+// tiles: CTA r of the cluster accumulates k-blocks [r nkb / 4, (r+1) nkb / 4)
+// (128 K-elements each) in TMEM.
 //
-// Pipeline of a CTA (4-stage ring of 48 KB stages, 128 K-elements each):
-//   - 16 producer warps expand the bit-packed visible weights (W, neurons x
-//     words: 256 rows x 2 words = one 64-bit item per thread) into the K-major
-//     SWIZZLE_128B layout the MMA reads (16-byte chunk c of row r stored at
-//     chunk c ^ (r % 8)); for layer 1 they also expand the caller's packed
-//     inputs (A).  Bit words are loaded kPrefetch stages ahead into registers.
-//     Each producer warp arrives once on the stage's "full" mbarrier after
-//     every lane's proxy fence.
-//   - For layers l >= 2 the A operand arrives pre-expanded: the epilogue of
-//     layer l - 1 writes its activations as e4m3 in the swizzled stage image
-//     (one 16 KB tile per 128 K-elements, DevLayer::AE), and one thread pulls
-//     each tile with a bulk copy that completes on the same barrier.
-//   - 1 MMA thread waits on "full", issues tcgen05.mma.kind::f8f6f4 (M = 128,
-//     N = 256, K = 32) four times per stage into a 128 x 256 fp32 accumulator
-//     in TMEM, and commits to the stage's "empty" mbarrier.
-//   - Epilogue: tcgen05.ld -> shared partial (int16: a partial sum is an
-//     integer of magnitude <= K_in <= 32767), rows < bs only; cluster barrier; reduction of
-//     this CTA's 64 columns over the 4 partials; z (int16), packed sign bits
-//     and, for the next layer, the e4m3 tile image; cluster barrier again so
-//     that no CTA leaves while a peer still reads its partial.
+// Operands.  The tensor core can take the A operand from tensor memory, and
+// that is where the activations go; only the weights pass through shared
+// memory.  A pipeline that stages both operands in shared memory writes and
+// reads every byte of both there, and on this shape shared-memory bandwidth,
+// not the tensor core, sets the pace.  Per k-block:
+//   - 16 producer warps expand the packed visible weights of the tile's 256
+//     neuron rows into a 32 KB stage in the 128B-swizzled K-major layout the
+//     MMA reads (16-byte chunk c of row r at chunk c ^ (r % 8)), two threads
+//     per row, 64 K-elements each; and expand the packed activation bits of
+//     the 128 pattern rows into TMEM with tcgen05.st: warp w writes the lanes
+//     32 (w % 4) .. 32 (w % 4) + 31 that its lane quarter may access and
+//     K-elements 32 (w / 4) .. + 31 of the block, i.e. 8 TMEM columns (four
+//     e4m3 per 32-bit column) from one 32-bit piece of bits;
+//   - bit words are loaded kPrefetch k-blocks ahead into registers;
+//   - each producer warp waits for its TMEM stores, fences its shared-memory
+//     stores for the async proxy and arrives once on the stage's "full"
+//     mbarrier;
+//   - one MMA thread waits on "full" and issues four tcgen05.mma.kind::f8f6f4
+//     (M = 128, N = 256, K = 32; A from TMEM, B from the stage) into the
+//     128 x 256 fp32 accumulator, then commits to the stage's "empty" mbarrier.
+//   TMEM: accumulator in columns 0 .. 255, kStages activation stages of 32
+//   columns above it.  Shared memory: kStages weight stages.
+// Epilogue.  tcgen05.ld -> partials in shared memory (offset 16-bit lanes,
+// two per word, so that 32-bit adds sum two elements at once), laid out by the
+// CTA that owns each 64-column slice (CTA r of the cluster finalises neurons
+// 64 r .. 64 r + 63 of the tile); one cluster barrier; then each CTA pushes
+// its three foreign slices into their owners' slices with bulk reduce-adds
+// (cp.reduce.async.bulk .add, shared::cta -> shared::cluster), which complete
+// on the owner's mbarrier; the owner waits for the three, and writes z
+// (int16) and the packed sign bits of its 64 neurons.  A CTA leaves only after
+// its outgoing bulk reads have completed and its own slice has received all
+// three adds, so no second cluster barrier is needed.
 // Every mbarrier wait is bounded; the first expiry sets a shared flag that
 // stops every other wait, the kernel counts the failure in the control block
-// (host: BMLP_ETIMEOUT), still passes both cluster barriers, releases its TMEM
+// (host: BMLP_ETIMEOUT), still passes the cluster barrier, releases its TMEM
 // and returns.
 #include "tc_common.cuh"
 
@@ -51,32 +59,40 @@ using namespace tc;
 constexpr int TM = 128;           // MMA M: patterns (rows >= bsz unused)
 constexpr int TN = 256;           // MMA N: neurons per tile
 constexpr int kSplit = 4;         // CTAs per cluster, each a quarter of K
-constexpr int kStages = 4;
-constexpr int kPrefetch = 4;      // stages of bit-words held in registers ahead
-constexpr int kProducers = 512;   // 16 warps: the epilogue's partial and reduction
-// producer warps of the mainloop: one thread per stage row -- 256 weight rows,
-// plus 128 input rows on layer 1
-template <bool kTiles>
-constexpr int kRowWarps = kTiles ? 8 : 12;
+constexpr int kStages = 6;        // weight stages in shared memory, activation stages in TMEM
+constexpr int kPrefetch = 8;      // k-blocks of bit words held in registers ahead
+constexpr int kProducers = 512;   // 16 warps
 constexpr int THREADS = kProducers + 32;
-constexpr int A_BYTES = TM * KB;  // 16 KB
-constexpr int B_BYTES = TN * KB;  // 32 KB
-constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-constexpr int TMEM_COLS = TN;
-constexpr int PSTRIDE = TN + 8;   // int16 per partial row (+16 B: no bank conflicts)
-constexpr int kCols = TN / kSplit;  // columns reduced by one CTA
-static_assert(TM * PSTRIDE * 2 <= kStages * STAGE_BYTES, "partial must fit in the stages");
+constexpr int B_BYTES = TN * KB;  // 32 KB weight stage
+constexpr int kAccCols = TN;      // fp32 accumulator columns
+constexpr int kStageCols = KB / 4;  // TMEM columns of one activation stage (4 e4m3 per column)
+constexpr int TMEM_COLS = 512;
+static_assert(kAccCols + kStages * kStageCols <= TMEM_COLS, "TMEM budget");
+constexpr int kCols = TN / kSplit;  // neurons finalised by one CTA
 static_assert(kCols == 64, "one CTA writes one packed activation word per row");
+// A CTA's partial covers at most ceil(ceil(K_in / 128) / 4) <= 64 k-blocks of
+// 128 elements (K_in <= 32767), so it is an integer in [-8192, 8192]; stored
+// with the offset kOff = 8192 in a 16-bit lane, two lanes per 32-bit word, the
+// kSplit = 4 offset partials of an element sum to z + 4 kOff, which lies in
+// [1, 65535] because |z| <= K_in <= 32767 -- so 32-bit adds of the packed
+// words never carry from one lane into the next.
+constexpr uint32_t kOff = 8192;
+constexpr int kSliceRow = 2 * kCols + 16;  // bytes per pattern row of a partial slice (+16: banks)
+constexpr int kSliceBytes = TM * kSliceRow;
+static_assert(kSplit * kSliceBytes <= kStages * B_BYTES, "partials must fit in the stages");
+static_assert(kSliceRow % 16 == 0, "bulk copies move multiples of 16 bytes");
 
 struct __align__(8) TcShared {
   unsigned long long full[kStages];   // the producers filled stage s
   unsigned long long empty[kStages];  // the MMAs that read stage s completed
   unsigned long long done;            // all MMAs completed
+  unsigned long long red;             // the three peers' slices were added into ours
   uint32_t tmem_base;
   int failed;
+  int red_failed;                     // only the wait on `red` sets this one
 };
 
-constexpr size_t kSmemBytes = 1024 /*alignment slack*/ + kStages * STAGE_BYTES + sizeof(TcShared);
+constexpr size_t kSmemBytes = 1024 /*alignment slack*/ + kStages * B_BYTES + sizeof(TcShared);
 
 constexpr uint32_t kIdesc = tc::idesc_f8(TM, TN);
 
@@ -91,20 +107,38 @@ __device__ __forceinline__ void cluster_sync_all() {
                ::: "memory");
 }
 
-__device__ __forceinline__ uint4 ld_peer_u4(uint32_t local_addr, uint32_t rank) {
+__device__ __forceinline__ uint32_t peer_addr(uint32_t local_addr, uint32_t rank) {
   uint32_t a;
   asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(a) : "r"(local_addr), "r"(rank));
-  uint4 v;
-  asm volatile("ld.shared::cluster.v4.u32 {%0, %1, %2, %3}, [%4];"
-               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(a) : "memory");
-  return v;
+  return a;
 }
 
-// z of a packed int16 pair (low half first)
-__device__ __forceinline__ int lo16(uint32_t p) { return (int)(int16_t)(p & 0xFFFFu); }
-__device__ __forceinline__ int hi16(uint32_t p) { return (int)(int16_t)(p >> 16); }
+// MMA with the A operand in tensor memory (lane = row, four e4m3 per column).
+__device__ __forceinline__ void mma_f8_tmem_a(uint32_t tmem_d, uint32_t tmem_a, uint64_t bdesc,
+                                              uint32_t accumulate) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], [%1], %2, %3, p;\n}"
+      ::"r"(tmem_d), "r"(tmem_a), "l"(bdesc), "r"(kIdesc), "r"(accumulate));
+}
 
-template <bool kTiles>
+// 64 K-elements of one row (bits 0..63 of x) as sixteen TMEM columns of e4m3.
+__device__ __forceinline__ void tmem_store_row64(uint32_t taddr, uint64_t x) {
+  uint32_t v[16];
+  const uint32_t lo = (uint32_t)x, hi = (uint32_t)(x >> 32);
+#pragma unroll
+  for (int c = 0; c < 8; ++c) {
+    v[c] = e4m3_quad<0>(lo >> (4 * c));
+    v[8 + c] = e4m3_quad<0>(hi >> (4 * c));
+  }
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, "
+      "%12, %13, %14, %15, %16};"
+      ::"r"(taddr), "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]),
+        "r"(v[7]), "r"(v[8]), "r"(v[9]), "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]),
+        "r"(v[15]) : "memory");
+}
+
 __global__ void __cluster_dims__(kSplit, 1, 1) __launch_bounds__(THREADS, 1)
     k_train_forward_tc(const StepParams* __restrict__ P, int l);
 
@@ -113,43 +147,24 @@ __global__ void __cluster_dims__(kSplit, 1, 1) __launch_bounds__(THREADS, 1)
 size_t train_forward_tc_smem() { return kSmemBytes; }
 
 cudaError_t prepare_train_forward_tc() {
-  cudaError_t e = cudaFuncSetAttribute(k_train_forward_tc<false>,
-                                       cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
-  if (e != cudaSuccess) return e;
-  return cudaFuncSetAttribute(k_train_forward_tc<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  return cudaFuncSetAttribute(k_train_forward_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
                               (int)kSmemBytes);
 }
 
-cudaError_t launch_train_forward_tc(bool tiles, int Kout, cudaStream_t st, bool pdl,
-                                   const StepParams* P, int l) {
+cudaError_t launch_train_forward_tc(int Kout, cudaStream_t st, bool pdl, const StepParams* P, int l) {
   const dim3 grid((unsigned)(((Kout + TN - 1) / TN) * kSplit));
-  if (tiles)
-    return launch_kernel(k_train_forward_tc<true>, grid, dim3(THREADS), kSmemBytes, st, pdl, P, l);
-  return launch_kernel(k_train_forward_tc<false>, grid, dim3(THREADS), kSmemBytes, st, pdl, P, l);
+  return launch_kernel(k_train_forward_tc, grid, dim3(THREADS), kSmemBytes, st, pdl, P, l);
 }
-
-size_t act_tile_bytes(int K) { return (size_t)((K + KB - 1) / KB) * A_BYTES; }
 
 namespace {
 
-template <bool kTiles>
 __global__ void __cluster_dims__(kSplit, 1, 1) __launch_bounds__(THREADS, 1)
     k_train_forward_tc(const StepParams* __restrict__ P, int l) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* base = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-  TcShared* sh = reinterpret_cast<TcShared*>(base + kStages * STAGE_BYTES);
+  TcShared* sh = reinterpret_cast<TcShared*>(base + kStages * B_BYTES);
   const DevLayer& Ly = P->layer[l - 1];
-  // the mini-batch index is advanced by the previous step's update kernel; a
-  // layer >= 2 launch reads it after the wait below, layer 1 (which zeroes
-  // the pattern rows >= M in its prologue) before anything else
-  int64_t start = 0;
-  int M = 0;
-  if (!kTiles) {
-    pdl_wait();
-    start = (int64_t)P->ctrl->s * P->bs;
-    M = (int)min((int64_t)P->bs, P->n - start);
-  }
   const uint32_t rank = cluster_rank();
   const int n0 = (int)(blockIdx.x / kSplit) * TN;
   const int N = Ly.Kout, Kin = Ly.Kin, nw = Ly.nw_in;
@@ -160,27 +175,21 @@ __global__ void __cluster_dims__(kSplit, 1, 1) __launch_bounds__(THREADS, 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   volatile int* failed = &sh->failed;
 
-  // zero the pattern rows >= M and neuron rows >= NB of every stage once; the
-  // producers never write them (their products land in unused rows/columns)
+  // weight rows >= NB of every stage are zero (never written by the producers)
   for (int s = 0; s < kStages; ++s) {
-    if (!kTiles) {
-      uint4* a4 = reinterpret_cast<uint4*>(base + s * STAGE_BYTES);
-      for (int i = M * (KB / 16) + threadIdx.x; i < TM * (KB / 16); i += THREADS)
-        a4[i] = make_uint4(0, 0, 0, 0);
-    }
-    uint4* b4 = reinterpret_cast<uint4*>(base + s * STAGE_BYTES + A_BYTES);
+    uint4* b4 = reinterpret_cast<uint4*>(base + s * B_BYTES);
     for (int i = NB * (KB / 16) + threadIdx.x; i < TN * (KB / 16); i += THREADS)
       b4[i] = make_uint4(0, 0, 0, 0);
   }
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
-      // one arrival per row-producer warp, plus (kTiles) the tile copy's
-      // expect_tx arrival
-      mbar_init(&sh->full[s], kRowWarps<kTiles> + (kTiles ? 1 : 0));
+      mbar_init(&sh->full[s], kProducers / 64);   // one arrival per warp of the owning group
       mbar_init(&sh->empty[s], 1);
     }
     mbar_init(&sh->done, 1);
+    mbar_init(&sh->red, 1);
     sh->failed = 0;
+    sh->red_failed = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   if (warp == 0) {
@@ -193,62 +202,88 @@ __global__ void __cluster_dims__(kSplit, 1, 1) __launch_bounds__(THREADS, 1)
   __syncthreads();
   asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
   const uint32_t tmem = sh->tmem_base;
-  if (kTiles) {
-    // everything above depends on no earlier kernel; the activations, the
-    // mini-batch index and this layer's outputs (read by the previous step's
-    // update) do
-    pdl_wait();
-    start = (int64_t)P->ctrl->s * P->bs;
-    M = (int)min((int64_t)P->bs, P->n - start);
+
+  // ---------------- producer roles ----------------
+  // Two groups of eight warps take alternate k-blocks (group g: k = g, g + 2,
+  // ...; with an even kStages each stage slot belongs to one group), so one
+  // group's store fences and barrier arrival overlap the other group's
+  // expansion.  Within a group, thread t = 32 w + lane (w = warp % 8) expands
+  // weight row t of the tile (128 K-elements, eight 16-byte chunks) and 64
+  // K-elements (half w / 4) of activation row 32 (w % 4) + lane, the TMEM lane
+  // its warp may access.
+  const int grp = (warp >> 3) & 1, gw = warp & 7;
+  const int r = 32 * gw + lane;
+  const int q = gw & 3, j2 = gw >> 2;
+  const int m = 32 * q + lane;
+  const uint64_t* wsrc = (warp < 16 && r < NB) ? Ly.W + (int64_t)(n0 + r) * nw : nullptr;
+  const bool wvec = (nw % 2 == 0) && (reinterpret_cast<uintptr_t>(Ly.W) % 16 == 0);
+  const uint64_t* aprev = (l == 1) ? P->x : P->layer[l - 2].A;
+  const int bs = P->bs;
+  const int64_t ncall = P->n;
+  auto load_w = [&](int kb) -> uint4 {
+    if (wsrc == nullptr || kb >= kb0 + nk) return make_uint4(0, 0, 0, 0);
+    if (wvec) return __ldg(reinterpret_cast<const uint4*>(wsrc) + kb);
+    const uint64_t lo = 2 * kb < nw ? __ldg(wsrc + 2 * kb) : 0ull;
+    const uint64_t hi = 2 * kb + 1 < nw ? __ldg(wsrc + 2 * kb + 1) : 0ull;
+    return make_uint4((uint32_t)lo, (uint32_t)(lo >> 32), (uint32_t)hi, (uint32_t)(hi >> 32));
+  };
+  constexpr int kPf = kPrefetch / 2;   // own k-blocks held ahead (every other k-block)
+  uint4 pw[kPf];
+  // Layers >= 2: the weights (the previous step's update), the batch index
+  // and every pointer were written two or more launches back, so they are
+  // read before waiting for the previous layer, whose activations are read
+  // after.  Layer 1 waits first: its weights and batch index come from the
+  // update launched just before it.
+  int64_t start = 0;
+  int M = 0;
+  if (l > 1) {
+    start = (int64_t)P->ctrl->s * bs;
+    M = (int)min((int64_t)bs, ncall - start);
+#pragma unroll
+    for (int i = 0; i < kPf; ++i) pw[i] = load_w(kb0 + grp + 2 * i);
+  }
+  pdl_wait();
+  if (l == 1) {
+    start = (int64_t)P->ctrl->s * bs;
+    M = (int)min((int64_t)bs, ncall - start);
+#pragma unroll
+    for (int i = 0; i < kPf; ++i) pw[i] = load_w(kb0 + grp + 2 * i);
   }
   pdl_trigger();
-  const uint64_t* A = (l == 1) ? P->x + start * P->nw0 : P->layer[l - 2].A;
+  const uint64_t* A = (l == 1) ? aprev + start * P->nw0 : aprev;
 
-  if (threadIdx.x < 32 * kRowWarps<kTiles>) {
-    // ---------------- producers: one thread per stage row ----------------
-    // threads 0 .. 255: weight rows (neurons n0 ..); layer 1 also threads
-    // 256 .. 383: input rows (patterns 0 .. M - 1); per k-block the thread
-    // loads the row's two bit words (one 16-byte load when the rows are
-    // 16-byte aligned) and expands them into the row's eight 16-byte chunks
-    const int p = threadIdx.x;
-    const bool isW = p < TN;
-    const int r = isW ? p : p - TN;
-    const uint64_t* src = nullptr;
-    if (isW && r < NB) src = Ly.W + (int64_t)(n0 + r) * nw;
-    if (!isW && !kTiles && r < M) src = A + (int64_t)r * nw;
-    const bool vec = (nw % 2 == 0) && src != nullptr && (reinterpret_cast<uintptr_t>(src) % 16 == 0);
-    const uint32_t row_off = (isW ? (uint32_t)A_BYTES : 0u) + (uint32_t)(r * KB);
-    const int swz = r & 7;
-    auto load = [&](int kb) -> uint4 {
-      if (src == nullptr || kb >= kb0 + nk) return make_uint4(0, 0, 0, 0);
-      if (vec) return __ldg(reinterpret_cast<const uint4*>(src) + kb);
-      const uint64_t lo = __ldg(src + 2 * kb);
-      const uint64_t hi = 2 * kb + 1 < nw ? __ldg(src + 2 * kb + 1) : 0ull;
-      return make_uint4((uint32_t)lo, (uint32_t)(lo >> 32), (uint32_t)hi, (uint32_t)(hi >> 32));
+  if (threadIdx.x < kProducers) {
+    // ---------------- producers ----------------
+    const uint64_t* asrc = (m < M) ? A + (int64_t)m * nw : nullptr;
+    auto load_a = [&](int kb) -> uint64_t {
+      const int ai = 2 * kb + j2;
+      return (asrc != nullptr && kb < kb0 + nk && ai < nw) ? __ldg(asrc + ai) : 0ull;
     };
-    uint4 pre[kPrefetch];
+    uint64_t pa[kPf];
 #pragma unroll
-    for (int d = 0; d < kPrefetch; ++d) pre[d] = load(kb0 + d);
-
-    for (int k0 = 0; k0 < nk; k0 += kPrefetch) {
+    for (int i = 0; i < kPf; ++i) pa[i] = load_a(kb0 + grp + 2 * i);
+    const uint32_t alane = (uint32_t)(32 * q) << 16;
+    const uint32_t woff = (uint32_t)(r * KB);
+    const int swz = r & 7;
+    for (int i0 = 0; grp + 2 * i0 < nk; i0 += kPf) {
 #pragma unroll
-      for (int d = 0; d < kPrefetch; ++d) {
-        const int k = k0 + d;
+      for (int d = 0; d < kPf; ++d) {
+        const int k = grp + 2 * (i0 + d);
         if (k >= nk) break;
         const int kb = kb0 + k;
         const int s = k % kStages;
         if (k >= kStages &&
             !__all_sync(kFull, mbar_wait(&sh->empty[s], (uint32_t)((k / kStages - 1) & 1), failed)))
           break;
-        uint8_t* stage = base + s * STAGE_BYTES;
-        if (kTiles && threadIdx.x == 0) {
-          // A: the pre-expanded activation tile of this k-block
-          mbar_arrive_tx(&sh->full[s], A_BYTES);
-          bulk_g2s(stage, P->layer[l - 2].AE + (size_t)kb * A_BYTES, A_BYTES, &sh->full[s]);
-        }
-        if (src != nullptr) {
-          uint8_t* row = stage + row_off;
-          const uint32_t x[4] = {pre[d].x, pre[d].y, pre[d].z, pre[d].w};
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+        // activation row m, K-elements 64 j2 .. 64 j2 + 63 -> 16 TMEM columns
+        // (rows >= M hold whatever: their outputs are never read; K-elements
+        // past K_in meet zero weights)
+        tmem_store_row64(tmem + alane + (uint32_t)(kAccCols + kStageCols * s + 16 * j2), pa[d]);
+        // weight row r -> shared memory; elements at K >= K_in are 0
+        if (wsrc != nullptr) {
+          uint8_t* row = base + s * B_BYTES + woff;
+          const uint32_t x[4] = {pw[d].x, pw[d].y, pw[d].z, pw[d].w};
           const int valid = Kin - KB * kb;
           if (valid >= KB) {
 #pragma unroll
@@ -261,9 +296,13 @@ __global__ void __cluster_dims__(kSplit, 1, 1) __launch_bounds__(THREADS, 1)
                   chunk16_masked(x[c >> 1] >> (16 * (c & 1)), valid - 16 * c);
           }
         }
-        pre[d] = load(kb + kPrefetch);
-        // every writer orders its stores for the async proxy; one arrival per warp
+        pw[d] = load_w(kb + 2 * kPf);
+        pa[d] = load_a(kb + 2 * kPf);
+        // TMEM stores complete, shared-memory stores ordered for the async
+        // proxy, then one arrival per warp
+        asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
         __syncwarp();
         if (lane == 0) mbar_arrive(&sh->full[s]);
       }
@@ -275,29 +314,32 @@ __global__ void __cluster_dims__(kSplit, 1, 1) __launch_bounds__(THREADS, 1)
       const int s = k % kStages;
       if (!mbar_wait(&sh->full[s], (uint32_t)((k / kStages) & 1), failed)) break;
       asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-      const uint8_t* sa = base + s * STAGE_BYTES;
-      const uint64_t ad = smem_desc(smem_u32(sa));
-      const uint64_t bd = smem_desc(smem_u32(sa + A_BYTES));
+      const uint64_t bd = smem_desc(smem_u32(base + s * B_BYTES));
+      const uint32_t ta = tmem + (uint32_t)(kAccCols + kStageCols * s);
 #pragma unroll
-      for (int j = 0; j < KB / 32; ++j)   // K = 32 bytes per MMA: +2 in the address field
-        mma_f8<kIdesc>(tmem, ad + 2 * j, bd + 2 * j, (k > 0 || j > 0) ? 1u : 0u);
+      for (int j = 0; j < KB / 32; ++j)   // K = 32 per MMA: 8 TMEM columns, +2 in the B address field
+        mma_f8_tmem_a(tmem, ta + 8 * j, bd + 2 * j, (k > 0 || j > 0) ? 1u : 0u);
       mma_commit(&sh->empty[s]);
     }
     if (nk > 0 && !*failed) mma_commit(&sh->done);
   }
 
-  // ---------------- partial accumulator -> shared memory ----------------
-  // (the stages are free: every MMA that read them has completed)
-  int16_t* part = reinterpret_cast<int16_t*>(base);
+  // ---------------- partial accumulator -> shared-memory slices ----------------
+  // (the stages are free: every MMA that read them has completed).  Slice r
+  // holds columns 64 r .. 64 r + 63 of every pattern row as int32.
+  uint8_t* slices = base;
+  if (threadIdx.x == 0 && M > 0)
+    mbar_arrive_tx(&sh->red, (uint32_t)((kSplit - 1) * M * kSliceRow));
   if (threadIdx.x < kProducers) {
     bool go = nk > 0 && !*failed && mbar_wait(&sh->done, 0, failed);
     go = __all_sync(kFull, go);   // tcgen05.ld is warp-collective
     if (go) asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
     const int sub = warp & 3;     // TMEM lanes 32 sub .. 32 sub + 31
-    const int m = 32 * sub + lane;
+    const int mrow = 32 * sub + lane;
+    const int dst = warp >> 2;    // this warp's 64 columns belong to cluster CTA dst
 #pragma unroll
-    for (int half = 0; half < 2; ++half) {
-      const int col0 = 64 * (warp >> 2) + 32 * half;
+    for (int hh = 0; hh < 2; ++hh) {
+      const int col0 = 64 * dst + 32 * hh;
       uint32_t v[32];
       if (go) {
         asm volatile(
@@ -315,51 +357,70 @@ __global__ void __cluster_dims__(kSplit, 1, 1) __launch_bounds__(THREADS, 1)
 #pragma unroll
         for (int j = 0; j < 32; ++j) v[j] = 0u;  // empty K range (or a failed wait): 0
       }
-      if (m < M) {
+      if (mrow < M) {
         uint32_t pk[16];
 #pragma unroll
         for (int j = 0; j < 16; ++j)
-          pk[j] = ((uint32_t)__float2int_rn(__uint_as_float(v[2 * j])) & 0xFFFFu) |
-                  ((uint32_t)__float2int_rn(__uint_as_float(v[2 * j + 1])) << 16);
-        uint4* dst = reinterpret_cast<uint4*>(part + m * PSTRIDE + col0);
+          pk[j] = (((uint32_t)__float2int_rn(__uint_as_float(v[2 * j])) + kOff) & 0xFFFFu) |
+                  (((uint32_t)__float2int_rn(__uint_as_float(v[2 * j + 1])) + kOff) << 16);
+        uint4* out = reinterpret_cast<uint4*>(slices + dst * kSliceBytes + mrow * kSliceRow +
+                                              2 * (32 * hh));
 #pragma unroll
-        for (int q = 0; q < 4; ++q) dst[q] = make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]);
+        for (int c = 0; c < 4; ++c) out[c] = make_uint4(pk[4 * c], pk[4 * c + 1], pk[4 * c + 2], pk[4 * c + 3]);
       }
     }
   }
+  // the slices are visible to the bulk-copy proxy, and every CTA of the
+  // cluster has written its own slice before anyone adds into it
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
   asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
   cluster_sync_all();
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
 
-  // ---------------- reduction of this CTA's 64 columns ----------------
+  // ---------------- push the three foreign slices to their owners ----------------
+  // (one thread in each of three warps, so the three bulk copies are issued
+  // together)
+  if (lane == 0 && warp >= 1 && warp < kSplit && M > 0) {
+    {
+      const uint32_t peer = (rank + (uint32_t)warp) % kSplit;
+      const uint32_t src = smem_u32(slices + peer * kSliceBytes);
+      const uint32_t dstp = peer_addr(src, peer);  // the owner's own slice, same offset
+      const uint32_t bar = peer_addr(smem_u32(&sh->red), peer);
+      asm volatile(
+          "cp.reduce.async.bulk.shared::cluster.shared::cta.mbarrier::complete_tx::bytes.add.u32 "
+          "[%0], [%1], %2, [%3];"
+          ::"r"(dstp), "r"(src), "r"((uint32_t)(M * kSliceRow)), "r"(bar) : "memory");
+    }
+    asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+  }
+
+  // ---------------- this CTA's 64 neurons: z, sign bits ----------------
   if (threadIdx.x < kProducers) {
-    const int m = threadIdx.x >> 2;              // pattern row
-    const int c0 = kCols * (int)rank + 16 * (threadIdx.x & 3);  // column in the tile
-    const int nf = n0 + c0;                      // first neuron of the 16
-    if (m < M) {
-      int acc[16];
+    // waited for even after a failure elsewhere: the peers always push their
+    // three slices, and this CTA must outlive those writes into its memory
+    const bool ok = M > 0 && mbar_wait(&sh->red, 0, &sh->red_failed) && !*failed;
+    const int mrow = threadIdx.x >> 2;             // pattern row
+    const int c16 = 16 * (threadIdx.x & 3);        // 16 of the slice's 64 columns
+    const int nf = n0 + kCols * (int)rank + c16;   // first neuron of the 16
+    if (ok && mrow < M) {
+      const uint4* in = reinterpret_cast<const uint4*>(slices + rank * kSliceBytes + mrow * kSliceRow +
+                                                       2 * c16);
+      int zz[16];
 #pragma unroll
-      for (int j = 0; j < 16; ++j) acc[j] = 0;
-      const uint32_t local = smem_u32(part + m * PSTRIDE + c0);
+      for (int c = 0; c < 2; ++c) {
+        const uint4 v = in[c];
+        const uint32_t w4[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
-      for (int q = 0; q < kSplit; ++q) {
-#pragma unroll
-        for (int h = 0; h < 2; ++h) {
-          const uint4 v = ld_peer_u4(local + 16u * h, (uint32_t)q);
-          acc[8 * h + 0] += lo16(v.x);
-          acc[8 * h + 1] += hi16(v.x);
-          acc[8 * h + 2] += lo16(v.y);
-          acc[8 * h + 3] += hi16(v.y);
-          acc[8 * h + 4] += lo16(v.z);
-          acc[8 * h + 5] += hi16(v.z);
-          acc[8 * h + 6] += lo16(v.w);
-          acc[8 * h + 7] += hi16(v.w);
+        for (int e = 0; e < 4; ++e) {
+          zz[8 * c + 2 * e] = (int)(w4[e] & 0xFFFFu) - (int)(kSplit * kOff);
+          zz[8 * c + 2 * e + 1] = (int)(w4[e] >> 16) - (int)(kSplit * kOff);
         }
       }
-      int16_t* zrow = Ly.Z + (int64_t)m * N;
+      int16_t* zrow = Ly.Z + (int64_t)mrow * N;
       uint32_t bits = 0, zp[8];
 #pragma unroll
       for (int j = 0; j < 16; ++j) {
-        const int z = acc[j];
+        const int z = zz[j];
         if (nf + j < N && z >= 0) bits |= 1u << j;
         if (j & 1) zp[j >> 1] |= (uint32_t)(z & 0xFFFF) << 16;
         else zp[j >> 1] = (uint32_t)(z & 0xFFFF);
@@ -375,31 +436,15 @@ __global__ void __cluster_dims__(kSplit, 1, 1) __launch_bounds__(THREADS, 1)
           if (nf + j < N) zrow[nf + j] = (int16_t)(zp[j >> 1] >> (16 * (j & 1)));
       }
       if ((nf >> 4) < 4 * Ly.nw_out)   // pad groups of the last word get 0 bits
-        reinterpret_cast<uint16_t*>(Ly.A + (int64_t)m * Ly.nw_out)[nf >> 4] = (uint16_t)bits;
-      if (Ly.AE != nullptr && nf / KB < (N + KB - 1) / KB) {
-        // the same 16 activations as e4m3 (+1 0x38, -1 0xB8, past N 0x00) in the
-        // swizzled tile image that the next layer's stages copy verbatim
-        uint32_t q4[4];
-#pragma unroll
-        for (int b = 0; b < 4; ++b) {
-          uint32_t word = 0;
-#pragma unroll
-          for (int j = 0; j < 4; ++j) {
-            const int jj = 4 * b + j;
-            const uint32_t e = (nf + jj < N) ? (((bits >> jj) & 1u) ? 0x38u : 0xB8u) : 0u;
-            word |= e << (8 * j);
-          }
-          q4[b] = word;
-        }
-        const int c = (nf % KB) / 16;
-        uint8_t* dst = Ly.AE + (size_t)(nf / KB) * A_BYTES + (size_t)m * KB + 16 * (c ^ (m & 7));
-        *reinterpret_cast<uint4*>(dst) = make_uint4(q4[0], q4[1], q4[2], q4[3]);
-      }
+        reinterpret_cast<uint16_t*>(Ly.A + (int64_t)mrow * Ly.nw_out)[nf >> 4] = (uint16_t)bits;
     }
   }
-  cluster_sync_all();   // no CTA leaves while a peer still reads its partial
+  // outgoing bulk reads done before the shared memory goes away
+  if (lane == 0 && warp >= 1 && warp < kSplit && M > 0)
+    asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
+  __syncthreads();
   asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-  if (threadIdx.x == 0 && *failed) atomicAdd(&P->ctrl->timeouts, 1u);
+  if (threadIdx.x == 0 && (*failed || sh->red_failed)) atomicAdd(&P->ctrl->timeouts, 1u);
   if (warp == 0)
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(TMEM_COLS) : "memory");
 }

@@ -278,6 +278,9 @@ CASES = {
                                  group_mode=1),
     "groups_reshuffled_wide": dict(widths=(256, 1024), classes=10, n_train=400, gamma=[64],
                                    group_mode=2),
+    # the widest input the int16 pre-activations allow: the largest split-K
+    # partials of the tensor-core forward (|partial| = 8192)
+    "widest_input": dict(widths=(32767, 64), classes=4, n_train=200, teacher_hidden=8),
 }
 
 
