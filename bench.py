@@ -11,10 +11,14 @@ than L2, so no flush is needed between steps.
 
 Printed (rank 0, one JSON line): samples/s over all ranks, XNOR-popcount
 Gbop/s, the roofline of the dominant kernel measured live with CUDA events on
-a sample of the timed mini-batches, the oracle's CPU throughput on a bounded
+a sample of the timed mini-batches, the whole training step against its
+roofline (HBM bytes the step touches and the forward's bit-pairs at the peak
+of the engine that runs them), the oracle's CPU throughput on a bounded
 sample, the end-to-end number through the C-ABI with host (pinned) buffers,
-SM clocks sampled during the timed region, and the forward-only evaluation
-sweep (65,536 samples at batch 65,536).
+SM clocks sampled during the timed region, the forward-only evaluation sweep
+(65,536 samples at batch 65,536), the comparison of the units that can run
+the forward contraction (peaks and one 8192 x 8192 layer at 100 and 65,536
+patterns), and the same figures for the four other workloads.
 
 --impl reference times the CPU oracle (plain C, all host cores) on the same
 workload, one 100-sample mini-batch per step.
@@ -47,9 +51,12 @@ CONFIG_KEY = "C5"
 SAMPLES_PER_STEP = 100_000
 STEPS_PER_EPOCH = 10
 EVAL_BATCH = 65_536
-# sampled mini-batches for the per-kernel figures: one in 50, i.e. 20 per
-# step of 1,000 mini-batches
-PROFILE_EVERY = 50
+# sampled mini-batches for the per-kernel figures: one in 100, i.e. 10 per
+# step of 1,000 mini-batches (a sampled mini-batch runs kernel by kernel
+# between CUDA events instead of inside the captured graphs)
+PROFILE_EVERY = 100
+# the other workloads: oracle mini-batches timed for their CPU baseline
+CONFIG_ORACLE_MINIBATCHES = {"C1": 20, "C2": 10, "C3": 4, "C4": 2}
 
 # HBM traffic of one k_update launch of the timed region, from an ncu capture
 # of this bench (dram__bytes_read.sum + dram__bytes_write.sum, one pass; see
@@ -68,6 +75,35 @@ EVAL_TRAFFIC_SRC_SHA = "f8b34ceea49eb88e"
 def bitpairs_per_sample(widths, classes):
     """Forward XNOR bit-pairs per pattern: sum_l K_l (K_{l-1} + c) (Table 3)."""
     return sum(widths[l] * (widths[l - 1] + classes) for l in range(1, len(widths)))
+
+
+def forward_weight_bytes(widths):
+    """Packed visible weights the forward passes of one mini-batch read."""
+    return sum(widths[l] * ((widths[l - 1] + 63) // 64) * 8 for l in range(1, len(widths)))
+
+
+def step_roofline(ms_per_mb, upd_bytes_per_mb, widths, classes, hbm_gbs, mac_peak, popc_peak,
+                  engine):
+    """The whole training step (one mini-batch of 100) against its roofline:
+    HBM bytes = what the update touched (H of the rows with a CP tuple read and
+    written, their W rows written, the sparse reinforcement events of the
+    other rows; counted by the kernel) + the packed weights the forward reads;
+    compute = the forward's bit-pairs at the peak of the engine that runs
+    them.  t_roof = max(HBM time, compute time); frac = t_roof / measured.
+    The same step against the CUDA-core popcount peak is reported beside it."""
+    nbytes = upd_bytes_per_mb + forward_weight_bytes(widths)
+    bp = 100 * bitpairs_per_sample(widths, classes)
+    t_meas = ms_per_mb * 1e-3
+    t_hbm = nbytes / (hbm_gbs * 1e9)
+    t_cmp = bp / mac_peak
+    t_popc = bp / popc_peak
+    t_roof = max(t_hbm, t_cmp)
+    return {"bound": "hbm" if t_hbm >= t_cmp else engine, "frac": t_roof / t_meas,
+            "us_measured": t_meas * 1e6, "us_roof": t_roof * 1e6, "hbm_bytes": nbytes,
+            "us_hbm": t_hbm * 1e6, "us_compute": t_cmp * 1e6, "engine": engine,
+            "achieved_gbs": nbytes / t_meas / 1e9, "peak_gbs": hbm_gbs,
+            "vs_popcount_peak": {"us_popc": t_popc * 1e6,
+                                 "frac": max(t_hbm, t_popc) / t_meas}}
 
 
 def update_bytes_per_launch(widths):
@@ -373,7 +409,7 @@ def run_ours(args):
     # end-to-end through the C-ABI with host (pinned) buffers
     x_host = torch.from_numpy(xp.view(np.int64)).pin_memory()
     y_host = yd.cpu().pin_memory()
-    n_e2e = max(1, min(args.steps, 5))
+    n_e2e = max(1, args.steps)
     barrier()
     torch.cuda.synchronize()
     t0 = time.perf_counter()
@@ -426,6 +462,18 @@ def run_ours(args):
         "roofline": eroof,
     }
 
+    mac_peak = (FP8_PER_BF16 * bf16_tf_sus if tc else 0.0) * 1e12 / 2.0
+    sroof = step_roofline(step_ms_mb, upd_bytes, cfg.widths, cfg.classes, hbm_gbs,
+                          mac_peak if tc else popc_peak, popc_peak,
+                          "tensor (e4m3)" if tc else "alu (popcount)")
+    sroof["peak_source"] = (peak_src + " HBM copy; compute: bf16 sustained x 2 (e4m3 / bf16 nominal)"
+                            if tc else peak_src + " HBM copy; compute: SM max clock x 152 x 16 POPC x 32")
+
+    engines = engine_bakeoff(dev) if not args.no_extras else None
+    configs = ({k: config_figures(k, dev, hbm_gbs, mac_peak if tc else popc_peak, popc_peak,
+                                  None if args.no_cpu_baseline else os.cpu_count() or 1)
+                for k in ("C1", "C2", "C3", "C4")} if not args.no_extras else None)
+
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         cpu = cpu_baseline(cfg, W.unpack(xp[:100], cfg.widths[0]),
@@ -445,6 +493,7 @@ def run_ours(args):
                    "l2": "inputs larger than L2 (1 GB stream, 512 MiB hidden weights)"},
         "gbops": 2 * bp * value / 1e9,
         "roofline": roofline,
+        "step_roofline": sroof,
         "kernels": {k: {kk: vv for kk, vv in v.items()} for k, v in kernels.items()},
         "kernel_ms_per_minibatch": per_mb, "ms_per_minibatch": step_ms_mb,
         "cpu_baseline": cpu,
@@ -454,6 +503,8 @@ def run_ours(args):
         "gpu_launches": launches,
         "clocks": clk.summary(),
         "eval": eval_info,
+        "engines": engines,
+        "configs": configs,
     }
     if rank == 0:
         print(json.dumps(line), flush=True)
@@ -461,6 +512,57 @@ def run_ours(args):
     if world > 1:
         dist.destroy_process_group()
     return 0
+
+
+def config_figures(key, dev, hbm_gbs, mac_peak, popc_peak, threads):
+    """Throughput of one of the other workloads on this GPU: its whole
+    training set for one epoch (after an untimed epoch that captures the
+    graphs), timed between CUDA events; the step roofline as for the stress
+    workload; and the CPU oracle on a bounded number of its mini-batches."""
+    import torch
+
+    from paper_2412_00119_gb300 import bmlp as B
+
+    cfg = W.CONFIGS[key]
+    st = torch.cuda.current_stream(dev)
+    xp = W.make_inputs(cfg, "train")
+    xd = torch.from_numpy(xp.view(np.int64)).to(dev)
+    yd = W.teacher_labels_packed_torch(W.make_teacher(cfg), xd, cfg.widths[0])
+    n = cfg.n_train
+    model = B.BMLP(cfg.widths, cfg.classes, seed=cfg.model_seed, bs=100)
+    B.bmlp_train(model.h, xd, yd, n, B.BMLP_EPOCH_END, st)
+    B.bmlp_update_stats(model.h, reset=True)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    e0.record(st)
+    B.bmlp_train(model.h, xd, yd, n, B.BMLP_EPOCH_END, st)
+    e1.record(st)
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1)
+    _, _, ubytes = B.bmlp_update_stats(model.h, reset=True)
+    engine = ("tensor (e4m3)" if model.info["fwd_impl"] == B.BMLP_FWD_TCGEN05 else "alu (popcount)")
+    model.close()
+    n_mb = n // 100
+    out = {"workload": "%s train: %s->%d, bs 100, %d training samples; timed: the second epoch"
+                       % (key, "->".join(map(str, cfg.widths)), cfg.classes, n),
+           "samples_per_s": n / (ms / 1e3), "ms_per_epoch": ms,
+           "gbops": 2 * bitpairs_per_sample(cfg.widths, cfg.classes) * n / (ms / 1e3) / 1e9,
+           "step_roofline": step_roofline(ms / n_mb, ubytes / n_mb, cfg.widths, cfg.classes,
+                                          hbm_gbs, mac_peak, popc_peak, engine)}
+    if threads:
+        import oracle as O
+        cores = O.set_threads(threads)
+        mbs = CONFIG_ORACLE_MINIBATCHES[key]
+        xo = W.unpack(xp[:100 * mbs], cfg.widths[0])
+        yo = yd[:100 * mbs].cpu().numpy().astype(np.int32)
+        ref = O.OracleModel(list(cfg.widths), cfg.classes, seed=cfg.model_seed, bs=100)
+        t0 = time.perf_counter()
+        ref.train(xo, yo)
+        dt = time.perf_counter() - t0
+        ref.close()
+        out["cpu_baseline"] = {"value": 100 * mbs / dt, "unit": "samples/s", "cores": cores,
+                               "kind": "oracle", "sample": "first %d mini-batches of 100" % mbs}
+    return out
 
 
 ENGINE_NAMES = {1: "popc", 2: "tcgen05_e4m3", 3: "b1_mma_sync", 4: "s8_mma_sync"}
@@ -582,6 +684,8 @@ def main(argv=None):
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-extras", action="store_true",
+                    help="skip the engine comparison and the other workloads' figures")
     ap.add_argument("--ncu-case", type=int, default=0, metavar="N",
                     help="run only a small N-mini-batch case (for profiler captures)")
     ap.add_argument("--frontend-case", type=int, default=0, metavar="N",

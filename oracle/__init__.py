@@ -135,6 +135,10 @@ def _declare(L):
                                        C.c_int32, _i32p, C.c_int32, C.c_int32, C.c_int32,
                                        C.c_double, C.c_uint64, C.c_int32, C.c_uint32]
     L.or_perceptron_update.restype = None
+    L.or_perceptron_update_at.argtypes = [_i32p, C.c_int32, C.c_int32, C.c_int32, _i8p, _i32p, _i8p,
+                                          C.c_int32, _i32p, C.c_int32, C.c_int32, C.c_int32,
+                                          C.c_double, C.c_uint64, C.c_int32, C.c_uint32]
+    L.or_perceptron_update_at.restype = None
     L.or_create.argtypes = [_i32p, C.c_int32, C.c_int32, C.c_int32, C.c_uint64, C.c_int32,
                             C.c_int32, C.c_int32, C.c_double, _i32p, C.POINTER(C.c_void_p)]
     L.or_create.restype = C.c_int
@@ -297,9 +301,11 @@ def group_members(seed, l, K, mode, t=0):
     return out
 
 
-def perceptron_update(H, a_prev, y, P, sel, h_max, q, seed, l, t):
+def perceptron_update(H, a_prev, y, P, sel, h_max, q, seed, l, t, k0=0):
     """Alg. 3 on a copy of H (K_prev x K), reinforcement probability q.
-    Returns the updated H."""
+    k0: H and P hold neurons k0 .. k0 + K - 1 of the layer, sel holds neuron
+    indices of the layer (or -1), and the reinforcement stream is keyed by
+    those indices.  Returns the updated H."""
     H = np.array(H, dtype=np.int32, order="C", copy=True)
     a_prev = _c(a_prev, np.int8)
     y = _c(y, np.int32)
@@ -307,9 +313,9 @@ def perceptron_update(H, a_prev, y, P, sel, h_max, q, seed, l, t):
     sel = _c(sel, np.int32)
     Kp, K = H.shape
     b, G = sel.shape
-    lib().or_perceptron_update(_p(H, _i32p), Kp, K, _p(a_prev, _i8p), _p(y, _i32p), _p(P, _i8p),
-                               P.shape[1], _p(sel, _i32p), b, G, h_max, float(q), seed, l,
-                               t & 0xFFFFFFFF)
+    lib().or_perceptron_update_at(_p(H, _i32p), Kp, K, k0, _p(a_prev, _i8p), _p(y, _i32p),
+                                  _p(P, _i8p), P.shape[1], _p(sel, _i32p), b, G, h_max, float(q),
+                                  seed, l, t & 0xFFFFFFFF)
     return H
 
 

@@ -400,16 +400,21 @@ void or_select(const int32_t* z, int32_t b, int32_t K, const int8_t* P, int32_t 
 /* ------------------------------------------------------------------------ */
 
 /* Clipped perceptron over U_l, in (mu, g) order (O8), then reinforcement of
- * every h of the layer with probability q at step t (O9, O10).  H: K_prev x K. */
-void or_perceptron_update(int32_t* H, int32_t K_prev, int32_t K, const int8_t* a_prev,
-                          const int32_t* y, const int8_t* P, int32_t c, const int32_t* sel,
-                          int32_t b, int32_t G, int32_t h_max, double q, uint64_t seed,
-                          int32_t l, uint32_t t) {
+ * every h of the layer with probability q at step t (O9, O10), for the
+ * neurons k0 .. k0 + K - 1 of layer l (the whole layer: k0 = 0).  H: K_prev x K
+ * (column j = neuron k0 + j); P: K x c (row j = neuron k0 + j); sel holds
+ * neuron indices of the layer (k0 <= k < k0 + K) or -1.  The reinforcement
+ * stream of a neuron is keyed by its index in the layer (Alg. 3 l.5-12, O9). */
+void or_perceptron_update_at(int32_t* H, int32_t K_prev, int32_t K, int32_t k0, const int8_t* a_prev,
+                             const int32_t* y, const int8_t* P, int32_t c, const int32_t* sel,
+                             int32_t b, int32_t G, int32_t h_max, double q, uint64_t seed,
+                             int32_t l, uint32_t t) {
   /* Clipped Perceptron, Alg. 3 l.2-4 */
   for (int32_t mu = 0; mu < b; mu++)
     for (int32_t g = 0; g < G; g++) {
       int32_t k = sel[(int64_t)mu * G + g];
       if (k < 0) continue;
+      k -= k0;
       int32_t rho = P[(int64_t)k * c + y[mu]];
       for (int32_t i = 0; i < K_prev; i++) {
         int32_t* h = &H[(int64_t)i * K + k];
@@ -422,7 +427,7 @@ void or_perceptron_update(int32_t* H, int32_t K_prev, int32_t K, const int8_t* a
     uint8_t* fire = (uint8_t*)malloc((size_t)(K_prev > 0 ? K_prev : 1));
 #pragma omp for schedule(static)
     for (int32_t k = 0; k < K; k++) {
-      or_r_events(seed, l, k, t, K_prev, q, fire);
+      or_r_events(seed, l, k0 + k, t, K_prev, q, fire);
       for (int32_t i = 0; i < K_prev; i++)
         if (fire[i]) {
           int32_t* h = &H[(int64_t)i * K + k];
@@ -431,6 +436,13 @@ void or_perceptron_update(int32_t* H, int32_t K_prev, int32_t K, const int8_t* a
     }
     free(fire);
   }
+}
+
+void or_perceptron_update(int32_t* H, int32_t K_prev, int32_t K, const int8_t* a_prev,
+                          const int32_t* y, const int8_t* P, int32_t c, const int32_t* sel,
+                          int32_t b, int32_t G, int32_t h_max, double q, uint64_t seed,
+                          int32_t l, uint32_t t) {
+  or_perceptron_update_at(H, K_prev, K, 0, a_prev, y, P, c, sel, b, G, h_max, q, seed, l, t);
 }
 
 /* ------------------------------------------------------------------------ */

@@ -74,3 +74,154 @@ def test_bench_arithmetic():
     # int16 H read + write (8192 x 8192 x 2 x 2 bytes) + packed W (8192 x 128 x 8) per layer
     assert bench.update_bytes_per_launch(w) == 4 * (8192 * 8192 * 4 + 8192 * 128 * 8)
     assert bench.update_bytes_per_launch((784, 256)) == 256 * (13 * 64 * 4 + 13 * 8)
+
+
+# -- neuron sharding (paper_2412_00119_gb300.sharding) ------------------------------
+
+def _sharded_worker(rank, world, port, out, *args):
+    try:
+        _sharded_run(rank, world, port, out, *args)
+    except Exception as e:   # reported to the test instead of a silent timeout
+        out.put(("error", rank, repr(e)))
+        raise
+
+
+def _sharded_run(rank, world, port, out, widths, classes, gammas, n, bs, epochs, seed):
+    """One rank of a neuron-sharded training run, every step of the rule taken
+    from the oracle on this rank's slice of every layer; the only exchange is
+    the all-gather of the slices' activations (Sec. 3.1)."""
+    import numpy as np
+    import torch
+    import torch.distributed as dist
+
+    import oracle as O
+    import workloads as W
+    from paper_2412_00119_gb300 import sharding as S
+
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port))
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    O.set_threads(1)
+    L = len(widths) - 1
+    plan = S.neuron_slices(widths, gammas, world)
+    mine = plan[rank]
+    cfg = W.small_config(widths, classes, n, 0, teacher_hidden=16, number=61)
+    tr = W.make_split(cfg, "train")
+    x, y = tr.pm1(), tr.y
+    full = O.OracleModel(list(widths), classes, seed=seed, bs=bs, gamma=list(gammas))
+    H = [full.H(l)[:, mine[l - 1][0]:mine[l - 1][1]].copy() for l in range(1, L + 1)]
+    P = [full.P(l) for l in range(1, L + 1)]
+    full.close()
+    p_r, t, gathered = 0.5, 0, 0
+    errs = []
+    for _ in range(epochs):
+        err = 0
+        for s0 in range(0, n, bs):
+            xb, yb = x[s0:s0 + bs], y[s0:s0 + bs]
+            a_prev, ins, zs, marks = xb, [], [], []
+            for l in range(1, L + 1):
+                k0, k1 = mine[l - 1]
+                z, a = O.layer_forward(a_prev, H[l - 1])
+                # all-gather of the slices' activations (padded to the widest slice)
+                wmax = max(p[l - 1][1] - p[l - 1][0] for p in plan)
+                buf = torch.zeros((len(yb), wmax), dtype=torch.int8)
+                buf[:, :k1 - k0] = torch.from_numpy(a)
+                parts = [torch.zeros_like(buf) for _ in range(world)]
+                dist.all_gather(parts, buf)
+                gathered += 1
+                a_full = np.concatenate([parts[r][:, :plan[r][l - 1][1] - plan[r][l - 1][0]].numpy()
+                                         for r in range(world)], axis=1)
+                yhat = O.local_output(a_full, P[l - 1])
+                _, ell, _, mark = O.local_loss(yhat, yb, widths[l])
+                if l == L:
+                    err += int(ell.sum())
+                ins.append(a_prev)
+                zs.append(z)
+                marks.append(mark)
+                a_prev = a_full
+            for l in range(1, L + 1):
+                if not marks[l - 1].any():
+                    continue   # O6: no update of a layer with an empty M_l
+                k0, k1 = mine[l - 1]
+                if k1 == k0:
+                    continue
+                Ps = P[l - 1][k0:k1]
+                sel = O.select(zs[l - 1], Ps, yb, marks[l - 1], gammas[l - 1])
+                sel = np.where(sel >= 0, sel + k0, -1)
+                H[l - 1] = O.perceptron_update(H[l - 1], ins[l - 1], yb, Ps, sel, 255,
+                                               O.reinforce_prob(p_r, widths[l]), seed, l, t, k0=k0)
+            t += 1
+        errs.append(err)
+        p_r = p_r * np.sqrt(err / n)   # Alg. 1 l.21: the same error count on every rank
+    got = [None] * world
+    dist.all_gather_object(got, [h.tobytes() for h in H])
+    if rank == 0:
+        out.put((errs, p_r, t, gathered, got, plan))
+    dist.destroy_process_group()
+
+
+@pytest.mark.parametrize("world,widths,gammas", [
+    (2, (130, 256, 192), (64, 32)),      # unequal slices of layer 2 (3 units of 64)
+    (2, (70, 64, 128), (64, 64)),        # one layer with a single unit: one rank idle there
+    (3, (96, 384, 200), (64, 8)),        # three ranks; 200 = 3 units of 64 + a remainder of 8
+])
+def test_neuron_sharded_training_equals_one_rank(world, widths, gammas):
+    """Neuron-sharded training on gloo ranks -- each rank the oracle's steps on
+    its slices, one all-gather of activations per layer and mini-batch -- gives
+    the single-rank oracle's hidden weights, error counts and p_r bit for bit
+    over two epochs (the reinforcement stream is keyed by the neuron's index in
+    its layer, so the slices draw what one model draws)."""
+    import numpy as np
+
+    import oracle as O
+    import workloads as W
+
+    classes, n, bs, epochs, seed = 10, 240, 40, 2, 17
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    port = _free_port()
+    args = (world, port, q, widths, classes, gammas, n, bs, epochs, seed)
+    procs = [ctx.Process(target=_sharded_worker, args=(r,) + args) for r in range(world)]
+    for p in procs:
+        p.start()
+    res = q.get(timeout=300)
+    assert res[0] != "error", res
+    errs, p_r, t, gathered, got, plan = res
+    for p in procs:
+        p.join(timeout=60)
+        assert p.exitcode == 0
+    L = len(widths) - 1
+    assert gathered == L * epochs * (n // bs)   # one exchange per layer and mini-batch
+    cfg = W.small_config(widths, classes, n, 0, teacher_hidden=16, number=61)
+    tr = W.make_split(cfg, "train")
+    ref = O.OracleModel(list(widths), classes, seed=seed, bs=bs, gamma=list(gammas))
+    ref_errs = [ref.train(tr.pm1(), tr.y, epoch_end=True) for _ in range(epochs)]
+    assert errs == ref_errs
+    assert p_r == ref.p_r and t == ref.step
+    for l in range(1, L + 1):
+        k = widths[l - 1]
+        parts = [np.frombuffer(got[r][l - 1], np.int32).reshape(k, -1) for r in range(world)]
+        assert np.array_equal(np.concatenate(parts, axis=1), ref.H(l)), "layer %d" % l
+    ref.close()
+
+
+def test_neuron_slices_plan():
+    from paper_2412_00119_gb300 import sharding as S
+    widths, gammas = (784, 8192, 8192, 4096, 100), (64, 64, 128, 100)
+    for world in (1, 2, 3, 4, 8):
+        plan = S.neuron_slices(widths, gammas, world)
+        assert len(plan) == world
+        for l in range(1, len(widths)):
+            K, unit = widths[l], S.slice_unit(gammas[l - 1])
+            edges = [plan[r][l - 1] for r in range(world)]
+            assert edges[0][0] == 0 and edges[-1][1] == K
+            for r in range(world - 1):
+                assert edges[r][1] == edges[r + 1][0]              # contiguous cover
+            for a, b in edges:
+                assert a % unit == 0                                # whole groups and words
+                assert (b - a) % gammas[l - 1] == 0
+            sizes = [b - a for a, b in edges]
+            assert max(sizes) - min(sizes) <= unit + K % unit       # balanced to one unit
+    assert S.slice_unit(64) == 64 and S.slice_unit(100) == 1600 and S.slice_unit(96) == 192
+    assert S.gather_words_per_step((8192,) * 5, 100) == 4 * 100 * 128
+    with pytest.raises(ValueError):
+        S.neuron_slices((10, 9), (2,), 2)
