@@ -16,7 +16,8 @@ CSRC = os.path.join(HERE, "csrc")
 ROOT = os.path.dirname(HERE)
 LIB = os.path.join(HERE, "libbmlp.so")
 SOURCES = ["bmlp_api.cu", "bmlp_noalloc.cu", "kern_forward.cu", "kern_forward_tc.cu", "kern_eval_tc.cu",
-           "kern_update.cu", "kern_binarize.cu", "kern_expand.cu", "kern_peaks.cu", "kern_forward_b1.cu"]
+           "kern_update.cu", "kern_binarize.cu", "kern_expand.cu", "kern_peaks.cu", "kern_forward_b1.cu",
+           "kern_update_ws.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC,-ffp-contract=off",
          "--expt-relaxed-constexpr", "-I", os.path.join(ROOT, "include")]

@@ -88,6 +88,7 @@ struct bmlp {
   cudaEvent_t evFork = nullptr, evJoin = nullptr;
   int updCtas = 0;
   size_t updSmem = 0;
+  int update_impl = BMLP_UPD_ROWS;  // kernel of the hidden-weight update
   // profiling
   bool profiling = false;       // events around the kernels being enqueued now
   int32_t profEvery = 0;        // 0 off, 1 every mini-batch, S every S-th mini-batch
@@ -281,7 +282,10 @@ int enqueue_step(bmlp_t* h, cudaStream_t st, bool fork, bool chained = false) {
   }
   if (fork) CK(h, cudaStreamWaitEvent(st, h->evJoin, 0));
   prof_begin(h, kProfUpd, st);
-  CK(h, launch_update(update_hb_mode(h->h_max, h->hp.hb), (unsigned)h->updCtas, h->updSmem, st, fork,
+  if (h->update_impl == BMLP_UPD_STREAM)
+    CK(h, launch_update_ws(update_hb_mode(h->h_max, h->hp.hb), (unsigned)h->updCtas, st, fork, h->dP));
+  else
+    CK(h, launch_update(update_hb_mode(h->h_max, h->hp.hb), (unsigned)h->updCtas, h->updSmem, st, fork,
                       h->dP, h->hp.key0, h->hp.key1));
   prof_end(h, st);
   CK(h, cudaGetLastError());
@@ -449,6 +453,12 @@ int bmlp_create(const int32_t* widths, int32_t n_widths, int32_t classes, int16_
   if (r_den < 0 || r_num < 0) return fail(nullptr, BMLP_EINVAL, "r must be non-negative");
   const double p_r0 = hp.p_r0 < 0 ? 0.5 : hp.p_r0;
   if (!(p_r0 >= 0.0) || !std::isfinite(p_r0)) return fail(nullptr, BMLP_EINVAL, "p_r0 invalid");
+  int upd = hp.update_impl;
+  if (upd == BMLP_UPD_AUTO) upd = bs <= 128 ? BMLP_UPD_STREAM : BMLP_UPD_ROWS;
+  if (upd != BMLP_UPD_ROWS && upd != BMLP_UPD_STREAM)
+    return fail(nullptr, BMLP_EINVAL, "update_impl %d not available", hp.update_impl);
+  if (upd == BMLP_UPD_STREAM && bs > 128)
+    return fail(nullptr, BMLP_EINVAL, "update_impl STREAM needs bs <= 128");
   int fwd = hp.fwd_impl;
   if (fwd == BMLP_FWD_AUTO) fwd = bs <= 128 ? BMLP_FWD_TCGEN05 : BMLP_FWD_POPC;
   if (fwd != BMLP_FWD_POPC && fwd != BMLP_FWD_TCGEN05)
@@ -488,6 +498,7 @@ int bmlp_create(const int32_t* widths, int32_t n_widths, int32_t classes, int16_
   }
   h->L = L; h->c = classes; h->h_max = h_max; h->bs = bs; h->r_num = r_num; h->r_den = r_den;
   h->fwd_impl = fwd; h->seed = seed; h->p_r = p_r0;
+  h->update_impl = upd;
   h->group_mode = group_mode; h->max_K = max_K;
   h->K.assign(widths, widths + n_widths);
   h->gamma = gam;
@@ -513,6 +524,7 @@ int bmlp_create(const int32_t* widths, int32_t n_widths, int32_t classes, int16_
     D.ev_cta_base = ev_cta;
     ev_cta += (D.Kout + kEvRowsPerCta - 1) / kEvRowsPerCta;
     D.nblk = (D.Kin + 63) / 64;
+    D.ev_stride = (D.nblk + 1) & ~1;
     if ((rc = dalloc(h, &D.H, (size_t)D.Kout * D.ldh)) ||
         (rc = dalloc(h, &D.W, (size_t)D.Kout * D.nw_in)) ||
         (rc = dalloc(h, &D.PT, (size_t)classes * D.nw_out)) ||
@@ -522,7 +534,7 @@ int bmlp_create(const int32_t* widths, int32_t n_widths, int32_t classes, int16_
         (rc = dalloc(h, &D.A, (size_t)bs * D.nw_out)) ||
         (rc = dalloc(h, &D.mark, (size_t)bs)) ||
         (rc = dalloc(h, &D.sel, (size_t)bs * D.G)) ||
-        (rc = dalloc(h, &D.EV, (size_t)D.Kout * D.nblk)))
+        (rc = dalloc(h, &D.EV, (size_t)D.Kout * D.ev_stride)))
       return bail(rc);
     D.member = D.group_of = nullptr;
     if (group_mode != BMLP_GROUPS_CONTIGUOUS &&
@@ -544,6 +556,12 @@ int bmlp_create(const int32_t* widths, int32_t n_widths, int32_t classes, int16_
       return bail(cuda_fail(h, ea != cudaSuccess ? ea : cudaErrorInvalidConfiguration,
                             "update kernel occupancy"));
     h->updCtas = per_sm * prop.multiProcessorCount;
+    if (upd == BMLP_UPD_STREAM) {
+      // one CTA per SM (its slot ring fills most of the shared memory)
+      if ((ea = prepare_update_ws()) != cudaSuccess)
+        return bail(cuda_fail(h, ea, "streaming update kernel shared memory attribute"));
+      h->updCtas = prop.multiProcessorCount;
+    }
     P.upd_ctas_total = h->updCtas;
   }
   if ((rc = dalloc(h, &h->dP, 1)) || (rc = dalloc(h, &h->dCtrl, 1)) ||
@@ -903,6 +921,12 @@ int bmlp_get_info(const bmlp_t* h, int32_t* n_layers, int32_t* widths_out, int32
   if (gamma_out) for (int l = 1; l <= h->L; ++l) gamma_out[l - 1] = h->gamma[l];
   if (bs) *bs = h->bs;
   if (fwd_impl) *fwd_impl = h->fwd_impl;
+  return BMLP_OK;
+}
+
+int bmlp_get_update_impl(const bmlp_t* h, int32_t* update_impl) {
+  if (!h || !update_impl) return BMLP_EINVAL;
+  *update_impl = h->update_impl;
   return BMLP_OK;
 }
 

@@ -43,8 +43,9 @@ struct DevLayer {
   int32_t ev_cta_base;   // first CTA of this layer in the event-draw grid
   int32_t row_base;      // first row of this layer in the update's row numbering
   int32_t nblk;          // blocks of 64 inputs per neuron row (ceil(K_in / 64))
-  uint64_t* EV;          // [K_out][nblk] reinforcement events of the current step,
+  uint64_t* EV;          // [K_out][ev_stride] reinforcement events of the current step,
                          // bit i % 64 of word i / 64 = input i reinforced
+  int32_t ev_stride;     // words per EV row: nblk rounded up to even (16-byte rows)
 };
 
 // Device-resident step control.  The update kernel's last CTA advances t and s
@@ -239,6 +240,12 @@ void launch_forward_eval_tc(const uint64_t* A, int64_t M, int nw_in, const uint6
 // = packed sign(A W^T), sign(0) = +1, pad bits 0.
 cudaError_t launch_forward_b1(const uint64_t* A, int64_t M, int nw_in, const uint64_t* W, int N,
                               int Kin, uint64_t* Aout, int nw_out, cudaStream_t st);
+// The update with its memory traffic driven by bulk copies into a ring of
+// shared-memory slots (kern_update_ws.cu); mini-batches of at most 128; one
+// CTA per SM (grid = the SM count).
+size_t update_ws_smem();
+cudaError_t prepare_update_ws();
+cudaError_t launch_update_ws(int hb_mode, unsigned grid, cudaStream_t st, bool pdl, const StepParams* P);
 // Peak-rate kernel of one contraction engine (BMLP_FWD_*): launches it on
 // `sms` SMs' worth of CTAs and returns the bit-pairs (MACs) it performs.
 cudaError_t launch_engine_peak(int engine, int64_t iters, int sms, int* sink, unsigned int* timeouts,

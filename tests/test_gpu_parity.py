@@ -53,12 +53,14 @@ def assert_same_state(gpu, ref, where=""):
 
 def run_pair(widths, classes, n_train, n_test=64, epochs=2, seed=5, bs=100, gamma=None, h_max=255,
              r=(1, 4), p_r0=0.5, gen="bias", host=False, profiling=False, teacher_hidden=16,
-             data_number=99, fwd=B.BMLP_FWD_AUTO, group_mode=0):
+             data_number=99, fwd=B.BMLP_FWD_AUTO, group_mode=0, update_impl=B.BMLP_UPD_AUTO):
     cfg = W.small_config(widths, classes, n_train, n_test, gen=gen, teacher_hidden=teacher_hidden,
                          number=data_number)
     tr = W.make_split(cfg, "train")
     gpu = B.BMLP(widths, classes, h_max=h_max, seed=seed, bs=bs, r=r, p_r0=p_r0, gamma=gamma,
-                 fwd_impl=fwd, group_mode=group_mode)
+                 fwd_impl=fwd, group_mode=group_mode, update_impl=update_impl)
+    assert gpu.info["update_impl"] == (update_impl if update_impl else
+                                       (B.BMLP_UPD_STREAM if bs <= 128 else B.BMLP_UPD_ROWS))
     assert gpu.info["fwd_impl"] == (fwd if fwd else
                                     (B.BMLP_FWD_TCGEN05 if bs <= 128 else B.BMLP_FWD_POPC))
     ref = O.OracleModel(list(widths), classes, h_max=h_max, seed=seed, bs=bs, r=r, p_r0=p_r0,
@@ -291,6 +293,18 @@ def test_small_case(name, engine):
     if engine == "tcgen05" and kw.get("bs", 100) > 128:
         pytest.skip("the tcgen05 forward takes mini-batches of at most 128")
     gpu, _ = run_pair(fwd=ENGINES[engine], **kw)
+    gpu.close()
+
+
+ROWS_CASES = ["ragged_3layer", "tail_batch", "h_max_3_clipping", "h_max_1", "hundred_classes",
+              "groups_reshuffled", "always_reinforce", "multi_tile_k", "widest_input"]
+
+
+@pytest.mark.parametrize("name", ROWS_CASES)
+def test_small_case_rows_update(name):
+    """The same cases with the per-warp-rows update kernel (the one used for
+    mini-batches above 128) in place of the bulk-copy-fed one."""
+    gpu, _ = run_pair(update_impl=B.BMLP_UPD_ROWS, **CASES[name])
     gpu.close()
 
 
