@@ -37,8 +37,8 @@ namespace {
 
 using namespace upd;
 
-constexpr int kWsSched = 8;                  // scheduler warps
-constexpr int kWsCons = 16;                  // consumer warps
+constexpr int kWsSched = 4;                  // scheduler warps
+constexpr int kWsCons = 24;                  // consumer warps
 constexpr int kWsGroups = 4;                 // consumer groups, each on its own slots
 constexpr int kWsPerGroup = kWsCons / kWsGroups;
 static_assert(kWsSched % kWsGroups == 0, "group g takes the slots of schedulers g, g + kWsGroups, ...");
