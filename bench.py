@@ -6,8 +6,9 @@ trained on a seeded 1,000,000-sample stream of i.i.d. +-1 inputs labelled by a
 100,000 consecutive samples (1,000 mini-batches: forward, local classifiers,
 selection, CP + R + repack of every layer); every 10th step closes the epoch
 (p_r rescale), so ten steps are one pass over the stream.  The stream (1 GB
-packed) and the model state (512 MiB of int16 hidden weights) are far larger
-than L2, so no flush is needed between steps.
+packed) and the model state (256 MiB of hidden weights, bit-sliced at one
+byte per weight for h_max = 255) are far larger than L2, so no flush is needed
+between steps.
 
 Printed (rank 0, one JSON line): samples/s over all ranks, XNOR-popcount
 Gbop/s, the roofline of the dominant kernel measured live with CUDA events on
@@ -58,12 +59,13 @@ PROFILE_EVERY = 100
 # the other workloads: oracle mini-batches timed for their CPU baseline
 CONFIG_ORACLE_MINIBATCHES = {"C1": 20, "C2": 10, "C3": 4, "C4": 2}
 
-# HBM traffic of one k_update launch of the timed region, from an ncu capture
-# of this bench (dram__bytes_read.sum + dram__bytes_write.sum, one pass; see
-# profiles/k_update_c5.md), valid while the kernel source hashes to
+# HBM traffic of one k_update_ws launch of the timed region, from an ncu
+# capture of this bench (dram__bytes_read.sum + dram__bytes_write.sum, one
+# pass; see profiles/k_update_ws_c5.md), valid while the kernel sources hash to
 # UPDATE_TRAFFIC_SRC_SHA; otherwise reported as null.
-UPDATE_TRAFFIC_BYTES = 463_731_712 + 383_939_840  # dram read + write of one timed-region launch (ncu)
-UPDATE_TRAFFIC_SRC_SHA = "8d7fd0f8e4d76002"
+UPDATE_TRAFFIC_BYTES = None
+UPDATE_TRAFFIC_SRC_SHA = ""
+UPDATE_SOURCES = ("kern_update_ws.cu", "update_common.cuh")
 # The same for one 8192 -> 8192 k_forward_eval_tc launch at 65,536 patterns
 # (profiles/k_forward_eval_tc_c5eval.md), keyed to the kernel and its shared
 # tcgen05 header.  Part of the 67 MB output is still in the write-back L2 when
@@ -106,13 +108,26 @@ def step_roofline(ms_per_mb, upd_bytes_per_mb, widths, classes, hbm_gbs, mac_pea
                                  "frac": max(t_hbm, t_popc) / t_meas}}
 
 
-def update_bytes_per_launch(widths):
-    """Algorithmic HBM bytes of one update launch (all layers active): int16 H
-    read + write of every row, packed W row written."""
+def hidden_planes(h_max):
+    """Bit-planes stored per group of 32 hidden weights: the bits of h_max
+    rounded up to a power of two."""
+    nbits = max(1, int(h_max).bit_length())
+    p = 1
+    while p < nbits:
+        p *= 2
+    return p
+
+
+def update_bytes_per_launch(widths, h_max=255):
+    """Algorithmic HBM bytes of one update launch (all layers active): the
+    bit-sliced H of every row read and written (rows padded to 16 bytes),
+    the packed W row written."""
     b = 0
     for l in range(1, len(widths)):
+        ngrp = (widths[l - 1] + 31) // 32
+        ldh = (ngrp * hidden_planes(h_max) + 3) // 4 * 4
         nw = (widths[l - 1] + 63) // 64
-        b += widths[l] * (nw * 64 * 2 * 2 + nw * 8)
+        b += widths[l] * (2 * 4 * ldh + nw * 8)
     return b
 
 
@@ -376,7 +391,7 @@ def run_ours(args):
     bp_layer = 100 * cfg.widths[1] * cfg.widths[0]  # bit-pairs of one 8192x8192 forward launch
     popc_peak = popc_peak_bitpairs(sm_max_mhz)
     traffic = None
-    if UPDATE_TRAFFIC_BYTES is not None and UPDATE_TRAFFIC_SRC_SHA == src_sha("kern_update.cu"):
+    if UPDATE_TRAFFIC_BYTES is not None and UPDATE_TRAFFIC_SRC_SHA == src_sha(*UPDATE_SOURCES):
         traffic = UPDATE_TRAFFIC_BYTES
     kernels = {
         "update": {"bound": "hbm", "achieved": upd_bytes / upd_avg_s / 1e9, "peak": hbm_gbs,
@@ -403,7 +418,7 @@ def run_ours(args):
     dom_key = "update" if dominant == "update" else "train_forward"
     roofline = {k: v for k, v in kernels[dom_key].items() if k in
                 ("bound", "achieved", "peak", "unit", "frac", "traffic", "peak_source")}
-    roofline["kernel"] = {"update": "k_update",
+    roofline["kernel"] = {"update": "k_update_ws",
                           "train_forward": "k_train_forward_tc" if tc else "k_train_forward"}[dom_key]
 
     # end-to-end through the C-ABI with host (pinned) buffers
@@ -484,13 +499,15 @@ def run_ours(args):
         "metric": "training samples/sec", "value": value, "unit": "samples/s",
         "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_max / args.steps,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
-        "dtype": ("b1 (+-1 bits; forward as e4m3 x e4m3 -> fp32 on tcgen05, exact) + int16 hidden weights"
-                  if tc else "b1 (u64-packed XOR/popcount) + int16 hidden weights"), "data": "synthetic",
+        "dtype": ("b1 (+-1 bits; forward as e4m3 x e4m3 -> fp32 on tcgen05, exact) + bit-sliced "
+                  "integer hidden weights (8 planes)" if tc else
+                  "b1 (u64-packed XOR/popcount) + bit-sliced integer hidden weights (8 planes)"),
+        "data": "synthetic",
         "config": {"workload": "C5 train: 8192->8192x4->10, bs 100, 1,000,000-sample i.i.d. "
                                "stream, teacher 8192->1024->10; step = 100,000 samples",
                    "model": cfg.name, "global_batch": 100 * world, "seq_len": 0,
                    "parallelism": "replicas x%d (independent seeds)" % world,
-                   "l2": "inputs larger than L2 (1 GB stream, 512 MiB hidden weights)"},
+                   "l2": "inputs larger than L2 (1 GB stream, 256 MiB hidden weights)"},
         "gbops": 2 * bp * value / 1e9,
         "roofline": roofline,
         "step_roofline": sroof,

@@ -102,17 +102,7 @@ typedef struct bmlp_hparams {
   const int32_t* gamma;  /* L group sizes, each dividing K_l; NULL -> Sec. 4.3 rule */
   int32_t fwd_impl;      /* BMLP_FWD_*; 0 -> auto */
   int32_t group_mode;    /* BMLP_GROUPS_*: group membership of Alg. 2 (Sec. 4.3); 0 -> contiguous */
-  int32_t update_impl;   /* BMLP_UPD_*: kernel of the hidden-weight update; 0 -> auto */
 } bmlp_hparams;
-
-/* Kernels of the hidden-weight update (Alg. 3 and the repack of W); both
- * compute the same bits.  ROWS: every warp loads and updates its own neuron
- * rows.  STREAM: scheduler warps fill a ring of shared-memory slots by bulk
- * copies, consumer warps update from there (mini-batches of at most 128).
- * AUTO: STREAM when bs <= 128, else ROWS. */
-#define BMLP_UPD_AUTO 0
-#define BMLP_UPD_ROWS 1
-#define BMLP_UPD_STREAM 2
 
 /* Group membership (Sec. 4.3: by the permutation symmetry of a hidden layer
  * its groups may be any fixed random partition, or one redrawn at every
@@ -256,9 +246,6 @@ int bmlp_set_state(bmlp_t* h, int32_t layer, const int16_t* H_in, double p_r, in
 /* Model shape: any output may be NULL.  widths_out: L + 1 values; gamma_out: L. */
 int bmlp_get_info(const bmlp_t* h, int32_t* n_layers, int32_t* widths_out, int32_t* classes,
                   int32_t* gamma_out, int32_t* bs, int32_t* fwd_impl);
-
-/* The update kernel the handle uses (BMLP_UPD_ROWS or BMLP_UPD_STREAM). */
-int bmlp_get_update_impl(const bmlp_t* h, int32_t* update_impl);
 
 /* One-line description of the last error on this handle ("" if none).  With
  * h == NULL: the last error of a call that had no handle (e.g. bmlp_create). */

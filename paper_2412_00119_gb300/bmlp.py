@@ -30,7 +30,6 @@ BMLP_ENODEV = -6
 BMLP_EPOCH_END = 1
 BMLP_FWD_AUTO, BMLP_FWD_POPC, BMLP_FWD_TCGEN05, BMLP_FWD_B1MMA, BMLP_FWD_S8MMA = 0, 1, 2, 3, 4
 BMLP_GROUPS_CONTIGUOUS, BMLP_GROUPS_FIXED, BMLP_GROUPS_RESHUFFLED = 0, 1, 2
-BMLP_UPD_AUTO, BMLP_UPD_ROWS, BMLP_UPD_STREAM = 0, 1, 2
 PROFILE_KINDS = ("train_forward", "cls_select", "update", "eval_forward", "eval_out", "copy",
                  "r_events")
 
@@ -46,7 +45,7 @@ class BmlpError(RuntimeError):
 class bmlp_hparams(C.Structure):
     _fields_ = [("bs", C.c_int32), ("r_num", C.c_int32), ("r_den", C.c_int32),
                 ("p_r0", C.c_double), ("gamma", C.POINTER(C.c_int32)), ("fwd_impl", C.c_int32),
-                ("group_mode", C.c_int32), ("update_impl", C.c_int32)]
+                ("group_mode", C.c_int32)]
 
 
 _lib = None
@@ -85,7 +84,6 @@ SIGNATURES = [
     ("bmlp_debug_wait_probe", C.c_int, [_vp, C.c_int32, C.c_double]),
     ("bmlp_engine_peak", C.c_int, [C.c_int32, C.c_int64, _f64p, _f64p]),
     ("bmlp_debug_fail_alloc", C.c_int, [C.c_int64]),
-    ("bmlp_get_update_impl", C.c_int, [_vp, _i32p]),
     ("bmlp_debug_alloc_stats", C.c_int, [_i64p, _i64p]),
     ("bmlp_layer_forward_engine", C.c_int, [_vp, C.c_int32, C.c_int32, _vp, C.c_int64, _vp, _vp]),
 ]
@@ -150,7 +148,7 @@ def _stream(stream):
 # -- the C-ABI, one Python function per entry point ------------------------------
 
 def bmlp_create(widths, classes, h_max=255, seed=0, bs=100, r=(1, 4), p_r0=0.5, gamma=None,
-                fwd_impl=BMLP_FWD_AUTO, group_mode=BMLP_GROUPS_CONTIGUOUS, update_impl=BMLP_UPD_AUTO):
+                fwd_impl=BMLP_FWD_AUTO, group_mode=BMLP_GROUPS_CONTIGUOUS):
     w = (C.c_int32 * len(widths))(*[int(v) for v in widths])
     hp = bmlp_hparams()
     hp.bs = bs
@@ -162,7 +160,6 @@ def bmlp_create(widths, classes, h_max=255, seed=0, bs=100, r=(1, 4), p_r0=0.5, 
         hp.gamma = C.cast(g, _i32p)
     hp.fwd_impl = fwd_impl
     hp.group_mode = group_mode
-    hp.update_impl = update_impl
     h = _vp()
     rc = lib().bmlp_create(w, len(widths), classes, h_max, seed & (2 ** 64 - 1), C.byref(hp), C.byref(h))
     _check(rc, None)
@@ -274,12 +271,6 @@ def bmlp_update_stats(h, reset=False):
     return r.value, st.value, by.value
 
 
-def bmlp_get_update_impl(h):
-    v = C.c_int32()
-    _check(lib().bmlp_get_update_impl(h, C.byref(v)), h)
-    return v.value
-
-
 def bmlp_get_info(h):
     L = C.c_int32()
     lib().bmlp_get_info(h, C.byref(L), None, None, None, None, None)
@@ -370,12 +361,10 @@ class BMLP:
     """Owning wrapper of a bmlp_t handle."""
 
     def __init__(self, widths, classes, h_max=255, seed=0, bs=100, r=(1, 4), p_r0=0.5,
-                 gamma=None, fwd_impl=BMLP_FWD_AUTO, group_mode=BMLP_GROUPS_CONTIGUOUS,
-                 update_impl=BMLP_UPD_AUTO):
+                 gamma=None, fwd_impl=BMLP_FWD_AUTO, group_mode=BMLP_GROUPS_CONTIGUOUS):
         self.h = bmlp_create(widths, classes, h_max, seed, bs, r, p_r0, gamma, fwd_impl,
-                             group_mode, update_impl)
+                             group_mode)
         self.info = bmlp_get_info(self.h)
-        self.info["update_impl"] = bmlp_get_update_impl(self.h)
 
     def close(self):
         if getattr(self, "h", None):

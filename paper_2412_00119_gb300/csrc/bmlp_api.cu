@@ -22,6 +22,7 @@
 #include <nvtx3/nvToolsExt.h>
 
 #include "bmlp_internal.cuh"
+#include "update_common.cuh"
 
 using namespace bk;
 
@@ -88,7 +89,6 @@ struct bmlp {
   cudaEvent_t evFork = nullptr, evJoin = nullptr;
   int updCtas = 0;
   size_t updSmem = 0;
-  int update_impl = BMLP_UPD_ROWS;  // kernel of the hidden-weight update
   // profiling
   bool profiling = false;       // events around the kernels being enqueued now
   int32_t profEvery = 0;        // 0 off, 1 every mini-batch, S every S-th mini-batch
@@ -282,11 +282,7 @@ int enqueue_step(bmlp_t* h, cudaStream_t st, bool fork, bool chained = false) {
   }
   if (fork) CK(h, cudaStreamWaitEvent(st, h->evJoin, 0));
   prof_begin(h, kProfUpd, st);
-  if (h->update_impl == BMLP_UPD_STREAM)
-    CK(h, launch_update_ws(update_hb_mode(h->h_max, h->hp.hb), (unsigned)h->updCtas, st, fork, h->dP));
-  else
-    CK(h, launch_update(update_hb_mode(h->h_max, h->hp.hb), (unsigned)h->updCtas, h->updSmem, st, fork,
-                      h->dP, h->hp.key0, h->hp.key1));
+  CK(h, launch_update_ws(h->hp.nplanes, h->h_max, (unsigned)h->updCtas, st, fork, h->dP));
   prof_end(h, st);
   CK(h, cudaGetLastError());
   return BMLP_OK;
@@ -453,12 +449,6 @@ int bmlp_create(const int32_t* widths, int32_t n_widths, int32_t classes, int16_
   if (r_den < 0 || r_num < 0) return fail(nullptr, BMLP_EINVAL, "r must be non-negative");
   const double p_r0 = hp.p_r0 < 0 ? 0.5 : hp.p_r0;
   if (!(p_r0 >= 0.0) || !std::isfinite(p_r0)) return fail(nullptr, BMLP_EINVAL, "p_r0 invalid");
-  int upd = hp.update_impl;
-  if (upd == BMLP_UPD_AUTO) upd = bs <= 128 ? BMLP_UPD_STREAM : BMLP_UPD_ROWS;
-  if (upd != BMLP_UPD_ROWS && upd != BMLP_UPD_STREAM)
-    return fail(nullptr, BMLP_EINVAL, "update_impl %d not available", hp.update_impl);
-  if (upd == BMLP_UPD_STREAM && bs > 128)
-    return fail(nullptr, BMLP_EINVAL, "update_impl STREAM needs bs <= 128");
   int fwd = hp.fwd_impl;
   if (fwd == BMLP_FWD_AUTO) fwd = bs <= 128 ? BMLP_FWD_TCGEN05 : BMLP_FWD_POPC;
   if (fwd != BMLP_FWD_POPC && fwd != BMLP_FWD_TCGEN05)
@@ -491,14 +481,13 @@ int bmlp_create(const int32_t* widths, int32_t n_widths, int32_t classes, int16_
   cudaDeviceProp prop;
   cudaFuncAttributes fa;
   if (cudaGetDeviceProperties(&prop, h->device) != cudaSuccess || prop.major != 10 ||
-      update_kernel_attributes(&fa, 0) != cudaSuccess) {
+      update_kernel_image(&fa) != cudaSuccess) {
     (void)cudaGetLastError();
     delete h;
     return fail(nullptr, BMLP_ENODEV, "device has no sm_103a kernel image (needs a GB300)");
   }
   h->L = L; h->c = classes; h->h_max = h_max; h->bs = bs; h->r_num = r_num; h->r_den = r_den;
   h->fwd_impl = fwd; h->seed = seed; h->p_r = p_r0;
-  h->update_impl = upd;
   h->group_mode = group_mode; h->max_K = max_K;
   h->K.assign(widths, widths + n_widths);
   h->gamma = gam;
@@ -509,8 +498,8 @@ int bmlp_create(const int32_t* widths, int32_t n_widths, int32_t classes, int16_
   std::memset(&P, 0, sizeof(P));
   P.L = L; P.c = classes; P.bs = bs; P.h_max = h_max; P.r_num = r_num; P.r_den = r_den;
   P.nw0 = words_of(widths[0]);
-  P.hb = 1;
-  while ((1 << P.hb) < h_max + 1) ++P.hb;
+  P.nbits = upd::bits_of(h_max);
+  P.nplanes = upd::planes_of(P.nbits);
   P.key0 = (uint32_t)(seed & 0xffffffffu);
   P.key1 = (uint32_t)(seed >> 32);
   int ev_cta = 0, rows_total = 0;
@@ -518,7 +507,9 @@ int bmlp_create(const int32_t* widths, int32_t n_widths, int32_t classes, int16_
     DevLayer& D = P.layer[l - 1];
     D.Kin = h->K[l - 1]; D.Kout = h->K[l];
     D.nw_in = words_of(D.Kin); D.nw_out = words_of(D.Kout);
-    D.ldh = 64 * D.nw_in; D.gamma = gam[l]; D.G = D.Kout / D.gamma;
+    D.ngrp = (D.Kin + 31) / 32;
+    D.ldh = (D.ngrp * P.nplanes + 3) & ~3;
+    D.gamma = gam[l]; D.G = D.Kout / D.gamma;
     D.row_base = rows_total;
     rows_total += D.Kout;
     D.ev_cta_base = ev_cta;
@@ -545,23 +536,13 @@ int bmlp_create(const int32_t* widths, int32_t n_widths, int32_t classes, int16_
   P.ev_ctas_total = ev_cta;
   P.nblk_max = 0;
   for (int l = 1; l <= L; ++l) P.nblk_max = std::max(P.nblk_max, (widths[l - 1] + 63) / 64);
-  h->updSmem = update_smem_bytes(bs, P.nblk_max);
   {
-    cudaError_t ea = update_kernel_attributes(&fa, h->updSmem);
+    // the update grid is persistent, one CTA per SM (its slot ring fills most
+    // of the shared memory)
+    h->updSmem = update_ws_smem(P.nplanes);
+    const cudaError_t ea = prepare_update_ws();
     if (ea != cudaSuccess) return bail(cuda_fail(h, ea, "update kernel shared memory attribute"));
-    // the update grid is persistent: as many CTAs as fit on the device at once
-    int per_sm = 0;
-    ea = update_kernel_occupancy(update_hb_mode(h_max, P.hb), h->updSmem, &per_sm);
-    if (ea != cudaSuccess || per_sm < 1)
-      return bail(cuda_fail(h, ea != cudaSuccess ? ea : cudaErrorInvalidConfiguration,
-                            "update kernel occupancy"));
-    h->updCtas = per_sm * prop.multiProcessorCount;
-    if (upd == BMLP_UPD_STREAM) {
-      // one CTA per SM (its slot ring fills most of the shared memory)
-      if ((ea = prepare_update_ws()) != cudaSuccess)
-        return bail(cuda_fail(h, ea, "streaming update kernel shared memory attribute"));
-      h->updCtas = prop.multiProcessorCount;
-    }
+    h->updCtas = prop.multiProcessorCount;
     P.upd_ctas_total = h->updCtas;
   }
   if ((rc = dalloc(h, &h->dP, 1)) || (rc = dalloc(h, &h->dCtrl, 1)) ||
@@ -580,9 +561,11 @@ int bmlp_create(const int32_t* widths, int32_t n_widths, int32_t classes, int16_
   // initial state (Alg. 1 l.2)
   for (int l = 1; l <= L; ++l) {
     DevLayer& D = P.layer[l - 1];
-    const int64_t n1 = (int64_t)D.Kout * (D.ldh >> 3);
-    k_init_hw<<<(unsigned)((n1 + 255) / 256), 256>>>(D.H, D.W, D.Kin, D.Kout, D.ldh, D.nw_in, l,
-                                                       P.key0, P.key1, h_max, P.hb);
+    const int64_t n1 = (int64_t)D.Kout * D.ngrp;
+    cudaMemsetAsync(D.H, 0, sizeof(uint32_t) * D.Kout * D.ldh);
+    cudaMemsetAsync(D.W, 0, sizeof(uint64_t) * D.Kout * D.nw_in);
+    k_init_hw<<<(unsigned)((n1 + 255) / 256), 256>>>(D.H, D.W, D.Kin, D.Kout, D.ldh, D.ngrp, P.nplanes,
+                                                       l, P.key0, P.key1, h_max);
     const int64_t n2 = (int64_t)D.Kout * classes;
     k_init_rho<<<(unsigned)((n2 + 255) / 256), 256>>>(D.rho, D.Kout, classes, l, P.key0, P.key1);
     const int64_t n3 = (int64_t)classes * D.nw_out;
@@ -851,12 +834,20 @@ int bmlp_get_state(const bmlp_t* hc, int32_t layer, int16_t* H_out, uint64_t* W_
   CK(h, cudaDeviceSynchronize());
   const DevLayer& D = h->hp.layer[layer - 1];
   if (H_out) {
-    CK(h, cudaMemcpy2D(H_out, sizeof(int16_t) * D.Kin, D.H, sizeof(int16_t) * D.ldh,
-                       sizeof(int16_t) * D.Kin, D.Kout, cudaMemcpyDeviceToHost));
-    // lattice index -> h
-    const int base = 1 << h->hp.hb;
-    const int64_t cnt = (int64_t)D.Kout * D.Kin;
-    for (int64_t i = 0; i < cnt; ++i) H_out[i] = (int16_t)(2 * ((int)H_out[i] - base) - h->h_max);
+    // bit-sliced lattice indices -> h = 2u - h_max
+    std::vector<uint32_t> planes((size_t)D.Kout * D.ldh);
+    CK(h, cudaMemcpy(planes.data(), D.H, sizeof(uint32_t) * planes.size(), cudaMemcpyDeviceToHost));
+    const int np = h->hp.nplanes;
+    for (int64_t k = 0; k < D.Kout; ++k) {
+      const uint32_t* row = planes.data() + (size_t)k * D.ldh;
+      int16_t* out = H_out + k * D.Kin;
+      for (int i = 0; i < D.Kin; ++i) {
+        const uint32_t* grp = row + (size_t)(i >> 5) * np;
+        int u = 0;
+        for (int p = 0; p < np; ++p) u |= (int)((grp[p] >> (i & 31)) & 1u) << p;
+        out[i] = (int16_t)(2 * u - h->h_max);
+      }
+    }
   }
   if (W_out) CK(h, cudaMemcpy(W_out, D.W, sizeof(uint64_t) * D.Kout * D.nw_in, cudaMemcpyDeviceToHost));
   if (P_out) CK(h, cudaMemcpy(P_out, D.rho, (size_t)D.Kout * h->c, cudaMemcpyDeviceToHost));
@@ -885,16 +876,23 @@ int bmlp_set_state(bmlp_t* h, int32_t layer, const int16_t* H_in, double p_r, in
   if (step >= 0 && (!(p_r >= 0.0) || !std::isfinite(p_r))) return fail(h, BMLP_ESTATE, "p_r invalid");
   CK(h, cudaDeviceSynchronize());
   if (H_in) {
-    // h -> lattice index
-    const int base = 1 << h->hp.hb;
-    const int64_t cnt = (int64_t)D.Kout * D.Kin;
-    std::vector<int16_t> v((size_t)cnt);
-    for (int64_t i = 0; i < cnt; ++i) v[(size_t)i] = (int16_t)((H_in[i] + h->h_max) / 2 + base);
-    CK(h, cudaMemcpy2D(D.H, sizeof(int16_t) * D.ldh, v.data(), sizeof(int16_t) * D.Kin,
-                       sizeof(int16_t) * D.Kin, D.Kout, cudaMemcpyHostToDevice));
-    const int64_t nwt = (int64_t)D.Kout * D.nw_in;
-    k_repack_w<<<(unsigned)((nwt + 255) / 256), 256>>>(D.H, D.W, D.Kin, D.Kout, D.ldh, D.nw_in,
-                                                       h->h_max, h->hp.hb);
+    // h -> bit-sliced lattice index u = (h + h_max)/2 (padding 0)
+    const int np = h->hp.nplanes;
+    std::vector<uint32_t> planes((size_t)D.Kout * D.ldh, 0u);
+    for (int64_t k = 0; k < D.Kout; ++k) {
+      uint32_t* row = planes.data() + (size_t)k * D.ldh;
+      const int16_t* in = H_in + k * D.Kin;
+      for (int i = 0; i < D.Kin; ++i) {
+        const int u = (in[i] + h->h_max) / 2;
+        uint32_t* grp = row + (size_t)(i >> 5) * np;
+        for (int p = 0; p < np; ++p) grp[p] |= (uint32_t)((u >> p) & 1) << (i & 31);
+      }
+    }
+    CK(h, cudaMemcpy(D.H, planes.data(), sizeof(uint32_t) * planes.size(), cudaMemcpyHostToDevice));
+    const int64_t nwt = (int64_t)D.Kout * D.ngrp;
+    CK(h, cudaMemset(D.W, 0, sizeof(uint64_t) * D.Kout * D.nw_in));
+    k_repack_w<<<(unsigned)((nwt + 255) / 256), 256>>>(D.H, D.W, D.Kin, D.Kout, D.ldh, D.ngrp, np,
+                                                       h->h_max);
     CK(h, cudaGetLastError());
     h->launches += 1;
   }
@@ -921,12 +919,6 @@ int bmlp_get_info(const bmlp_t* h, int32_t* n_layers, int32_t* widths_out, int32
   if (gamma_out) for (int l = 1; l <= h->L; ++l) gamma_out[l - 1] = h->gamma[l];
   if (bs) *bs = h->bs;
   if (fwd_impl) *fwd_impl = h->fwd_impl;
-  return BMLP_OK;
-}
-
-int bmlp_get_update_impl(const bmlp_t* h, int32_t* update_impl) {
-  if (!h || !update_impl) return BMLP_EINVAL;
-  *update_impl = h->update_impl;
   return BMLP_OK;
 }
 

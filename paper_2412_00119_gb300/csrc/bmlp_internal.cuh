@@ -11,13 +11,19 @@ namespace bk {
 
 // ---------------------------------------------------------------------------
 // HBM layout of one layer l (K_in = K_{l-1}, K_out = K_l):
-//   H    int16 [K_out][ldh]      hidden weights, neuron-major; ldh = 64*nw_in;
-//                                 entries i >= K_in are padding (never read as weights).
-//                                 A weight h (odd, |h| <= h_max) is stored as its
-//                                 lattice index v = (h + h_max)/2 + 2^hb, where 2^hb
-//                                 is the least power of two >= h_max + 1 (hb >= 1), so
-//                                 v lies in [2^hb, 2^hb + h_max], h > 0 iff
-//                                 v >= 2^hb + (h_max + 1)/2, and an event moves v by 1
+//   H    uint32 [K_out][ldh]     hidden weights, neuron-major, bit-sliced: a weight h
+//                                 (odd, |h| <= h_max) is stored as its lattice index
+//                                 u = (h + h_max)/2 in [0, h_max], a CP or R event
+//                                 moves u by +-1 with clamping, and h > 0 iff
+//                                 u >= (h_max + 1)/2.  Inputs are grouped by 32:
+//                                 group g of row k (inputs 32 g .. 32 g + 31) is
+//                                 nplanes words, word p holding bit p of u of the 32
+//                                 weights (bit j <-> input 32 g + j); nbits planes are
+//                                 used (the bits of h_max), nplanes = nbits rounded
+//                                 up to a power of two (unused planes 0); ldh =
+//                                 ngrp * nplanes rounded up to a multiple of 4 words
+//                                 (16-byte rows).  Inputs i >= K_in hold u = 0 and
+//                                 are never stepped
 //   W    uint64 [K_out][nw_in]    packed sign(H), bit (i%64) of word i/64 = (h_ik > 0)
 //   PT   uint64 [c][nw_out]       packed P_l^T, bit (k%64) of word k/64 = (rho_kj > 0)
 //   rho  int8  [K_out][c]         P_l itself, for the stability rho_{k,y}
@@ -28,7 +34,7 @@ namespace bk {
 //   sel  int16 [G][bs]            selected neuron per (group, pattern), -1 = none
 // ---------------------------------------------------------------------------
 struct DevLayer {
-  int16_t* H;
+  uint32_t* H;
   uint64_t* W;
   uint64_t* PT;
   int8_t* rho;
@@ -40,6 +46,7 @@ struct DevLayer {
   int16_t* member;    // [K_out] group order (neuron at position j), or null: contiguous groups
   int16_t* group_of;  // [K_out] group of neuron k (with member)
   int32_t Kin, Kout, nw_in, nw_out, ldh, gamma, G;
+  int32_t ngrp;          // groups of 32 inputs per neuron row (ceil(K_in / 32))
   int32_t ev_cta_base;   // first CTA of this layer in the event-draw grid
   int32_t row_base;      // first row of this layer in the update's row numbering
   int32_t nblk;          // blocks of 64 inputs per neuron row (ceil(K_in / 64))
@@ -92,11 +99,11 @@ struct StepParams {
   Ctrl* ctrl;
   int32_t L, c, bs, h_max, r_num, r_den, nw0, upd_ctas_total, ev_ctas_total;
   int32_t rows_total;           // sum of K_l over the layers (update rows)
-  int32_t hb;                   // lattice-index offset exponent (see H above)
+  int32_t nbits, nplanes;       // bit-planes of H used / stored per group (see H above)
   uint32_t key0, key1;          // Philox key = (seed mod 2^32, seed div 2^32)
 };
 
-constexpr int kUpdThreads = 256;
+
 constexpr int kClsThreads = 512;
 
 // ---------------------------------------------------------------------------
@@ -162,18 +169,6 @@ __device__ __forceinline__ int clip_h(int h, int h_max) {
 __global__ void k_train_forward(const StepParams* P, int l);
 // Local classifier, 01-loss, margin, marks, and the group selection, all layers.
 __global__ void k_cls_select(const StepParams* P);
-// CP + R + repack of every layer with a non-empty M_l, then advance the step.
-// (key0, key1) = the Philox key, passed by value so that the round keys are
-// kernel-uniform.  kPow2: h_max + 1 is a power of two (both clip bounds are bit
-// boundaries of the lattice index).
-// hb_mode: 8 when h_max = 255 (compile-time lattice exponent), -1 for another
-// h_max + 1 that is a power of two, 0 otherwise (update_hb_mode).
-// pdl: launched with the programmatic-stream-serialization attribute.
-cudaError_t launch_update(int hb_mode, unsigned grid, size_t smem, cudaStream_t st, bool pdl,
-                          const StepParams* P, uint32_t key0, uint32_t key1);
-inline int update_hb_mode(int h_max, int hb) {
-  return ((h_max + 1) & h_max) != 0 ? 0 : (hb == 8 ? 8 : -1);
-}
 // Group order of every layer with a random partition (DevLayer::member /
 // group_of); redraw: keyed by the current step (else by step 0).
 cudaError_t prepare_group_order(int max_K);  // shared-memory attribute, once
@@ -184,14 +179,6 @@ void launch_r_events(unsigned grid, cudaStream_t st, const StepParams* P, uint32
                      uint32_t key1);
 constexpr int kEvRowsPerCta = 4;   // one warp per row
 constexpr int kEvThreads = 32 * kEvRowsPerCta;
-// Attributes of the update kernel; smem > 0 also raises its dynamic shared
-// memory limit to smem bytes.
-cudaError_t update_kernel_attributes(cudaFuncAttributes* fa, size_t smem);
-// Dynamic shared memory of the update kernel for mini-batches of bs and rows
-// of at most nblk_max blocks of 64 inputs.
-size_t update_smem_bytes(int bs, int nblk_max);
-// CTAs of the update kernel that fit on one SM at once.
-cudaError_t update_kernel_occupancy(int hb_mode, size_t smem, int* per_sm);
 // Generic forward for evaluation: A (M x nw_in) against W -> Aout (M x nw_out).
 __global__ void k_forward_eval(const uint64_t* __restrict__ A, int64_t M, int nw_in,
                                const uint64_t* __restrict__ W, int N, int Kin,
@@ -201,14 +188,14 @@ __global__ void k_predict_out(const uint64_t* __restrict__ A, int64_t M, int nw,
                               const uint64_t* __restrict__ PT, int c, int K,
                               int32_t* __restrict__ out);
 // Initialisation of H, W of one layer and rho, PT.
-__global__ void k_init_hw(int16_t* H, uint64_t* W, int Kin, int Kout, int ldh, int nw_in,
-                          int l, uint32_t key0, uint32_t key1, int h_max, int hb);
+__global__ void k_init_hw(uint32_t* H, uint64_t* W, int Kin, int Kout, int ldh, int ngrp, int nplanes,
+                          int l, uint32_t key0, uint32_t key1, int h_max);
 __global__ void k_init_rho(int8_t* rho, int Kout, int c, int l, uint32_t key0, uint32_t key1);
 __global__ void k_pack_pt(const int8_t* rho, uint64_t* PT, int Kout, int c, int nw_out);
 __global__ void k_transpose_rho(const int8_t* rho, int8_t* rhoT, int Kout, int c);
 // Re-derive W from H for one layer (after set_state).
-__global__ void k_repack_w(const int16_t* H, uint64_t* W, int Kin, int Kout, int ldh, int nw_in,
-                           int h_max, int hb);
+__global__ void k_repack_w(const uint32_t* H, uint64_t* W, int Kin, int Kout, int ldh, int ngrp,
+                           int nplanes, int h_max);
 // Tensor-core forward (tcgen05, +-1 as e4m3, exact fp32 sums), training layer l;
 // needs bs <= 128.  The activations of layer l - 1 (the inputs for l = 1) are
 // read as packed bits.
@@ -240,12 +227,17 @@ void launch_forward_eval_tc(const uint64_t* A, int64_t M, int nw_in, const uint6
 // = packed sign(A W^T), sign(0) = +1, pad bits 0.
 cudaError_t launch_forward_b1(const uint64_t* A, int64_t M, int nw_in, const uint64_t* W, int N,
                               int Kin, uint64_t* Aout, int nw_out, cudaStream_t st);
-// The update with its memory traffic driven by bulk copies into a ring of
-// shared-memory slots (kern_update_ws.cu); mini-batches of at most 128; one
-// CTA per SM (grid = the SM count).
-size_t update_ws_smem();
+// CP + R + repack of every layer with a non-empty M_l, then advance the step
+// (kern_update_ws.cu): bulk copies into a ring of shared-memory slots, the
+// bit-sliced steps by consumer warps; one CTA per SM (grid = the SM count).
+// pdl: launched with the programmatic-stream-serialization attribute.
+// nplanes: DevLayer's planes per group (StepParams::nplanes).
+size_t update_ws_smem(int nplanes);
 cudaError_t prepare_update_ws();
-cudaError_t launch_update_ws(int hb_mode, unsigned grid, cudaStream_t st, bool pdl, const StepParams* P);
+cudaError_t launch_update_ws(int nplanes, int h_max, unsigned grid, cudaStream_t st, bool pdl,
+                             const StepParams* P);
+// Attributes of the update kernel: fails when the library holds no sm_103a image.
+cudaError_t update_kernel_image(cudaFuncAttributes* fa);
 // Peak-rate kernel of one contraction engine (BMLP_FWD_*): launches it on
 // `sms` SMs' worth of CTAs and returns the bit-pairs (MACs) it performs.
 cudaError_t launch_engine_peak(int engine, int64_t iters, int sms, int* sink, unsigned int* timeouts,

@@ -18,18 +18,20 @@
 // memory.  A pipeline that stages both operands in shared memory writes and
 // reads every byte of both there, and on this shape shared-memory bandwidth,
 // not the tensor core, sets the pace.  Per k-block:
-//   - 16 producer warps expand the packed visible weights of the tile's 256
-//     neuron rows into a 32 KB stage in the 128B-swizzled K-major layout the
-//     MMA reads (16-byte chunk c of row r at chunk c ^ (r % 8)), two threads
-//     per row, 64 K-elements each; and expand the packed activation bits of
-//     the 128 pattern rows into TMEM with tcgen05.st: warp w writes the lanes
-//     32 (w % 4) .. 32 (w % 4) + 31 that its lane quarter may access and
-//     K-elements 32 (w / 4) .. + 31 of the block, i.e. 8 TMEM columns (four
-//     e4m3 per 32-bit column) from one 32-bit piece of bits;
-//   - bit words are loaded kPrefetch k-blocks ahead into registers;
+//   - 16 producer warps in two groups of eight take alternate k-blocks; in a
+//     group, thread t expands the packed visible weights of neuron row t of
+//     the tile (128 K-elements) into a 32 KB stage in the 128B-swizzled
+//     K-major layout the MMA reads (16-byte chunk c of row r at chunk
+//     c ^ (r % 8)), and 64 K-elements of one pattern row into TMEM with
+//     tcgen05.st: warp w writes the lanes 32 (w % 4) .. 32 (w % 4) + 31 that
+//     its lane quarter may access and K-elements 64 (w / 4) .. + 63 of the
+//     block, i.e. 16 TMEM columns (four e4m3 per 32-bit column) from one
+//     64-bit word of bits;
+//   - bit words are loaded kPrefetch k-blocks ahead into registers (each
+//     group holds its own k-blocks);
 //   - each producer warp waits for its TMEM stores, fences its shared-memory
 //     stores for the async proxy and arrives once on the stage's "full"
-//     mbarrier;
+//     mbarrier (eight arrivals complete a stage);
 //   - one MMA thread waits on "full" and issues four tcgen05.mma.kind::f8f6f4
 //     (M = 128, N = 256, K = 32; A from TMEM, B from the stage) into the
 //     128 x 256 fp32 accumulator, then commits to the stage's "empty" mbarrier.
@@ -326,7 +328,8 @@ __global__ void __cluster_dims__(kSplit, 1, 1) __launch_bounds__(THREADS, 1)
 
   // ---------------- partial accumulator -> shared-memory slices ----------------
   // (the stages are free: every MMA that read them has completed).  Slice r
-  // holds columns 64 r .. 64 r + 63 of every pattern row as int32.
+  // holds columns 64 r .. 64 r + 63 of every pattern row as 16-bit lanes
+  // offset by kOff, two per 32-bit word.
   uint8_t* slices = base;
   if (threadIdx.x == 0 && M > 0)
     mbar_arrive_tx(&sh->red, (uint32_t)((kSplit - 1) * M * kSliceRow));

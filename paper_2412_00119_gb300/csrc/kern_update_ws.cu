@@ -1,34 +1,40 @@
 // kern_update_ws.cu -- the hidden-weight update of one training step (Alg. 3:
-// clipped perceptron and reinforcement; Sec. 3.1: W = sign(H) re-packed in
-// the same pass) with its memory traffic driven by bulk copies.
+// clipped perceptron, then reinforcement; Sec. 3.1: W = sign(H) re-packed in
+// the same pass), with its memory traffic driven by bulk copies.
+//
+// The hidden weights are bit-sliced (DevLayer::H, update_common.cuh): a group
+// of 32 inputs of a neuron row is kP words, word p holding bit p of the
+// lattice index u = (h + h_max)/2 of the 32 weights.  A clipped step of +-1
+// is a ripple of word operations through the planes, on 32 weights at once.
+// The perceptron step of a tuple (mu, rho) moves weight i up where
+// a^mu_i rho_{k,y^mu} = +1 and down elsewhere, so its direction word is the
+// group's activation word, complemented when rho = -1; reinforcement moves
+// the weights of its events away from 0, so its direction word is the
+// group's h > 0 lanes, which is also the group's W word (a step away from 0
+// never flips a sign).
 //
 // The update streams every hidden weight of every neuron row that received a
-// CP tuple: read, a few integer steps, write.  In a kernel where each warp
-// loads its own row, the loads it can keep in flight bound the memory rate,
-// and the CP arithmetic delays them.  Here the two are split between warps:
-//   - kWsSched scheduler warps take rows from the step's row counter, find the
+// CP tuple: read, the steps, write.
+//   - kSched scheduler warps take rows from the step's row counter, find the
 //     row's CP tuples (Alg. 2's selections of the neuron's group; labels in
 //     shared memory), and fill one slot of a shared-memory ring per segment
-//     of kSegW hidden weights: bulk copies (cp.async.bulk, completing on the
-//     slot's "full" mbarrier) of the segment's hidden weights, of its part of
-//     the reinforcement-event bitmap, and of the first kActT tuples'
-//     activation bytes, plus the tuple list and a header;
-//   - kWsCons consumer warps, in kWsGroups groups that take different slots
-//     at once (group g the slots of schedulers g, g + kWsGroups, ...): each
-//     lane applies the tuples to its chunks of 8 weights in the slot and
-//     writes the chunk's W byte (reinforcement never flips a sign, so W is
-//     final after CP); after a group barrier the lanes apply the segment's few
-//     reinforcement events in the slot; one bulk copy writes the segment's H
-//     back to global memory, and the warps release the slot ("empty").
-// A row without tuple occupies a slot with its event bitmap only; its events
-// are applied as single-weight read-modify-writes and its W is unchanged
-// (reinforcement never flips a sign).  Slots are used in sequence order,
-// scheduler j filling sequence numbers j, j + kWsSched, ...; a scheduler that
-// finds no more rows fills one END slot, after which the consumers skip its
-// numbers.  The per-chunk arithmetic is that of k_update (update_common.cuh).
-// Every mbarrier wait is bounded; an expiry stops the CTA's loops, waits
-// (bounded) for the copies it issued, and is counted in the control block.
-// The last CTA to finish advances the step counters.
+//     of the row: bulk copies (cp.async.bulk, completing on the slot's "full"
+//     mbarrier) of the segment's planes, of its part of the reinforcement-
+//     event bitmap and of the first tuples' activation words, plus the tuple
+//     list and a header;
+//   - consumer group j (kPerGroup warps) takes the slots of scheduler j in
+//     order: each lane holds two groups of 32 weights at a time, applies the
+//     tuples in ascending mu, then the reinforcement events (Alg. 3 applies R
+//     after CP), writes the W word, and puts the planes back into the slot;
+//     one bulk copy writes the segment back to global memory, and the slot
+//     is released ("empty").
+// A row without tuple occupies a slot with its event bitmap only: its groups
+// with an event are stepped in place in global memory, and its W is
+// unchanged.  Layers with an empty M_l are skipped (no CP, no R).  Every
+// mbarrier wait is bounded; an expiry stops the CTA's loops (a consumer group
+// decides together, so no barrier is left waiting), waits (bounded) for the
+// copies it issued, and is counted in the control block.  The last CTA to
+// finish advances the step counters.
 #include "tc_common.cuh"
 #include "update_common.cuh"
 
@@ -37,78 +43,107 @@ namespace {
 
 using namespace upd;
 
-constexpr int kWsSched = 4;                  // scheduler warps
-constexpr int kWsCons = 24;                  // consumer warps
-constexpr int kWsGroups = 4;                 // consumer groups, each on its own slots
-constexpr int kWsPerGroup = kWsCons / kWsGroups;
-static_assert(kWsSched % kWsGroups == 0, "group g takes the slots of schedulers g, g + kWsGroups, ...");
-constexpr int kWsThreads = 32 * (kWsSched + kWsCons);
-constexpr int kWsSlots = 8;                  // ring slots, a multiple of kWsSched
-static_assert(kWsSlots % kWsSched == 0, "each slot belongs to one scheduler warp");
-constexpr int kSegW = 8192;                  // hidden weights per segment (one slot)
-constexpr int kActT = 4;                     // tuples whose activation bytes are staged
-constexpr int kMaxT = 128;                   // tuples per row at most (mini-batches <= 128)
+constexpr int kSched = 4;                     // scheduler warps
+constexpr int kPerGroup = 4;                  // consumer warps per group; group j serves scheduler j
+constexpr int kCons = kSched * kPerGroup;
+constexpr int kThreads = 32 * (kSched + kCons);
+constexpr int kGroupLanes = 32 * kPerGroup;
+constexpr int kMaxT = BMLP_MAX_BS;            // CP tuples of one row at most
+constexpr int kActStage = 4096;               // staged activation bytes per slot
+constexpr int kMaxSlots = 12;
+constexpr int kSmemLimit = 232448;            // dynamic shared memory of one CTA at most
 
 enum SlotType : int { kSlotRow = 0, kSlotSparse = 1, kSlotEnd = 2 };
 
 struct SlotMeta {
-  int16_t* hrow;         // the segment's first hidden weight in global memory
-  uint8_t* wrow;         // its first W byte
-  const uint8_t* aprev;  // the layer's input activations (row 0, byte 0 of the segment)
-  int type, n_t;         // slot type, CP tuples of the row
-  int nin;               // real inputs of the segment
-  int ch0;               // chunk offset of the segment in its row
-  int arow_bytes;        // bytes per activation row
-  int act_smem;          // activation bytes of the first min(n_t, kActT) tuples staged
-  int nseg;              // stored hidden weights of the segment (row padding included)
+  uint32_t* hrow;          // the segment's first plane word in global memory
+  uint32_t* wrow;          // the W word (32 bits) of the segment's first group
+  const uint32_t* aprev;   // pattern 0's activation word of the segment's first group
+  int type, n_t;           // slot type, CP tuples of the row
+  int ng;                  // groups of the segment
+  uint32_t last_mask;      // valid inputs of the segment's last group
+  int arow_words;          // 32-bit words per activation row
+  int nstage;              // tuples whose activation words are staged in the slot
+  int nwords;              // stored plane words of the segment (row padding included)
   int pad;
 };
 
-constexpr int kOffH = 0;                              // kSegW int16
-constexpr int kOffEv = kOffH + 2 * kSegW;             // kSegW / 64 uint64
-constexpr int kOffAct = kOffEv + kSegW / 8;           // kActT x kSegW / 8 bytes
-constexpr int kOffTup = kOffAct + kActT * (kSegW / 8);  // kMaxT int32
-constexpr int kOffMeta = kOffTup + 4 * kMaxT;
-constexpr int kSlotBytes = (kOffMeta + (int)sizeof(SlotMeta) + 127) & ~127;
+// Slot layout for kP planes per group: planes, event bits, staged activation
+// words, tuple list (uint16: mu | 0x8000 when rho = -1), header.
+template <int kP>
+struct Geo {
+  static constexpr int kSegG = (2048 / kP) < 1024 ? (2048 / kP) : 1024;  // groups per segment
+  static constexpr int kHBytes = 4 * kP * kSegG;
+  static constexpr int kEvBytes = 4 * kSegG;
+  static constexpr int kActT = kActStage / (4 * kSegG);   // tuples staged at most
+  static constexpr int kOffEv = kHBytes;
+  static constexpr int kOffAct = kOffEv + kEvBytes;
+  static constexpr int kOffTup = kOffAct + kActStage;
+  static constexpr int kOffMeta = kOffTup + 2 * kMaxT;
+  static constexpr int kSlotBytes = (kOffMeta + (int)sizeof(SlotMeta) + 127) & ~127;
+};
 
 struct __align__(16) WsShared {
-  unsigned long long full[kWsSlots];
-  unsigned long long empty[kWsSlots];
-  uint4 db[256];                   // packed CP steps per activation byte (rho = +1)
-  int y[kMaxT];                    // labels of the mini-batch (bad ones as 0)
-  int list[kWsSched][kMaxT];       // a scheduler's tuple scan
-  unsigned long long stats[3];     // rows visited, rows streamed, algorithmic bytes
-  int issued[kWsSlots];            // last use of each slot with copies issued (-1: none)
+  unsigned long long full[kMaxSlots];
+  unsigned long long empty[kMaxSlots];
+  int16_t y[kMaxT];                   // labels of the mini-batch (bad ones as 0)
+  uint16_t list[kSched][kMaxT];       // a scheduler's tuple scan
+  unsigned long long stats[3];        // rows visited, rows streamed, algorithmic bytes
+  int issued[kMaxSlots];              // last use of each slot with copies issued (-1: none)
   int failed;
 };
 
-constexpr size_t kWsSmemBytes = 128 /*alignment slack*/ + (size_t)kWsSlots * kSlotBytes + sizeof(WsShared);
+template <int kP>
+struct Ring {
+  static constexpr int kSlots =
+      128 + 12 * Geo<kP>::kSlotBytes + (int)sizeof(WsShared) <= kSmemLimit ? 12 : 8;
+  static_assert(kSlots % kSched == 0, "each slot belongs to one scheduler");
+  static constexpr size_t kSmem = 128 /*alignment slack*/ + (size_t)kSlots * Geo<kP>::kSlotBytes +
+                                  sizeof(WsShared);
+  static_assert(kSmem <= (size_t)kSmemLimit, "slot ring too large");
+};
 
-__device__ __forceinline__ uint8_t* slot_ptr(uint8_t* ring, int s) { return ring + (size_t)s * kSlotBytes; }
+__device__ __forceinline__ uint8_t* slot_ptr(uint8_t* ring, int s, int slot_bytes) {
+  return ring + (size_t)s * slot_bytes;
+}
 
-// barrier of the kWsPerGroup warps of consumer group g (named barriers 1..)
+// barrier of the kPerGroup warps of consumer group g (named barriers 1..)
 __device__ __forceinline__ void group_sync(int g) {
-  asm volatile("bar.sync %0, %1;" ::"r"(1 + g), "r"(32 * kWsPerGroup) : "memory");
+  asm volatile("bar.sync %0, %1;" ::"r"(1 + g), "r"(kGroupLanes) : "memory");
+}
+
+// the same barrier, returning whether v held on every thread of the group
+__device__ __forceinline__ bool group_all(int g, bool v) {
+  uint32_t r;
+  asm volatile(
+      "{\n .reg .pred p, q;\n setp.ne.u32 p, %1, 0;\n"
+      " bar.red.and.pred q, %2, %3, p;\n selp.u32 %0, 1, 0, q;\n}"
+      : "=r"(r) : "r"((uint32_t)v), "r"(1 + g), "r"(kGroupLanes) : "memory");
+  return r != 0u;
 }
 
 // ---------------------------------------------------------------------------
-// Scheduler warp: rows -> slots.
+// Scheduler warp j: rows -> slots j, j + kSched, ... (sequence numbers
+// j, j + kSched, ...).
 // ---------------------------------------------------------------------------
+template <int kP>
 __device__ __forceinline__ void ws_scheduler(const StepParams* __restrict__ P, WsShared* sh,
                                              uint8_t* ring, int j, int lane, int64_t start, int bsz,
                                              bool step_failed) {
+  using G = Geo<kP>;
+  constexpr int kSlots = Ring<kP>::kSlots;
   Ctrl* ctrl = P->ctrl;
   volatile int* failed = &sh->failed;
   const int c = P->c;
   const int rows_total = P->rows_total;
-  int* list = sh->list[j];
+  uint16_t* list = sh->list[j];
   uint32_t seq = (uint32_t)j;
   uint64_t st_rows = 0, st_streamed = 0, st_bytes = 0;
-  // acquire the slot of sequence number seq (wait until the consumers released its previous use)
+  // acquire the slot of sequence number q (its previous use released)
   auto acquire = [&](uint32_t q) -> bool {
-    const uint32_t u = q / kWsSlots;
+    const uint32_t u = q / kSlots;
     if (u == 0) return true;
-    return __all_sync(kFull, tc::mbar_wait(&sh->empty[q % kWsSlots], (u - 1) & 1u, failed));
+    return __all_sync(kFull, tc::mbar_wait(&sh->empty[q % kSlots], (u - 1) & 1u, failed));
   };
   // the ticket of the next row is taken while the current row is scanned
   int next = 0;
@@ -128,91 +163,92 @@ __device__ __forceinline__ void ws_scheduler(const StepParams* __restrict__ P, W
     const DevLayer& Ly = P->layer[li];
     const int k = gr - Ly.row_base;
     const int g = Ly.group_of ? (int)Ly.group_of[k] : k / Ly.gamma;
-    // ---- CP tuples of neuron k, ascending mu ----
-    // the group's selections of all (<= 128) patterns and, for c <= 32, the
-    // neuron's row of P_l are loaded together: one round trip
+    // ---- CP tuples of neuron k, ascending mu: the patterns whose selection
+    // in group g is k; for c <= 32 the neuron's row of P_l comes in one load
     int n_t = 0;
     const int16_t* selg = Ly.sel + (int64_t)g * P->bs;
     const int rho_lane = (c <= 32 && lane < c) ? (int)Ly.rho[(int64_t)k * c + lane] : 0;
-    int sv[kMaxT / 32];
+#pragma unroll 1
+    for (int m0 = 0; m0 < bsz; m0 += 128) {
+      int sv[4];
 #pragma unroll
-    for (int q = 0; q < kMaxT / 32; ++q) {
-      const int m = 32 * q + lane;
-      sv[q] = (m < bsz) ? (int)selg[m] : -1;
-    }
-#pragma unroll
-    for (int q = 0; q < kMaxT / 32; ++q) {
-      const int m = 32 * q + lane;
-      const bool hit = sv[q] == k;
-      const unsigned bal = __ballot_sync(kFull, hit);
-      if (bal != 0u) {
-        const int yv = hit ? sh->y[m] : 0;
-        const int rs = __shfl_sync(kFull, rho_lane, yv & 31);
-        if (hit) {
-          const int rho = (c <= 32) ? rs : (int)Ly.rho[(int64_t)k * c + yv];
-          list[n_t + __popc(bal & ((1u << lane) - 1u))] = m | ((rho > 0) ? 0 : 0x10000);
-        }
+      for (int q = 0; q < 4; ++q) {
+        const int m = m0 + 32 * q + lane;
+        sv[q] = (m < bsz) ? (int)selg[m] : -1;
       }
-      n_t += __popc(bal);
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const int m = m0 + 32 * q + lane;
+        const bool hit = sv[q] == k;
+        const unsigned bal = __ballot_sync(kFull, hit);
+        if (bal != 0u) {
+          const int yv = hit ? (int)sh->y[m] : 0;
+          const int rs = __shfl_sync(kFull, rho_lane, yv & 31);
+          if (hit) {
+            const int rho = (c <= 32) ? rs : (int)Ly.rho[(int64_t)k * c + yv];
+            list[n_t + __popc(bal & ((1u << lane) - 1u))] = (uint16_t)(m | ((rho > 0) ? 0 : 0x8000));
+          }
+        }
+        n_t += __popc(bal);
+      }
     }
     __syncwarp();
     st_rows += 1;
-    const int Kin = Ly.Kin;
-    const uint8_t* aprev = (li == 0) ? reinterpret_cast<const uint8_t*>(P->x + start * P->nw0)
-                                     : reinterpret_cast<const uint8_t*>(P->layer[li - 1].A);
-    const uint32_t arow_bytes = (uint32_t)Ly.nw_in * 8u;
-    const bool act_ok = (arow_bytes % 16u == 0) && (reinterpret_cast<uintptr_t>(aprev) % 16u == 0);
+    const int ngrp = Ly.ngrp;
+    const uint32_t* aprev = (li == 0) ? reinterpret_cast<const uint32_t*>(P->x + start * P->nw0)
+                                      : reinterpret_cast<const uint32_t*>(P->layer[li - 1].A);
+    const int arow_words = 2 * Ly.nw_in;
+    const bool act_ok = (arow_words % 4 == 0) && (reinterpret_cast<uintptr_t>(aprev) % 16u == 0);
     if (n_t > 0) {
       st_streamed += 1;
-      st_bytes += 4ull * (uint64_t)Ly.ldh + 8ull * (uint64_t)Ly.nw_in;
+      st_bytes += 8ull * (uint64_t)Ly.ldh + 8ull * (uint64_t)Ly.nw_in;   // H read + write, W write
     }
-    // ---- one slot per segment of kSegW hidden weights ----
-    for (int w0 = 0; w0 < Kin; w0 += kSegW) {
+    const uint32_t* evrow = reinterpret_cast<const uint32_t*>(Ly.EV + (int64_t)k * Ly.ev_stride);
+    // ---- one slot per segment of kSegG groups ----
+#pragma unroll 1
+    for (int g0 = 0; g0 < ngrp; g0 += G::kSegG) {
       if (!acquire(seq)) break;
-      const int s = (int)(seq % kWsSlots);
-      uint8_t* sl = slot_ptr(ring, s);
-      SlotMeta* meta = reinterpret_cast<SlotMeta*>(sl + kOffMeta);
-      const int nseg = min(kSegW, Ly.ldh - w0);                 // stored weights (multiple of 64)
-      const int nevw = min(kSegW / 64, Ly.ev_stride - w0 / 64);  // event words (even)
-      const int nact = min(kSegW / 8, (int)arow_bytes - w0 / 8); // activation bytes
-      const int nstage = (n_t > 0 && act_ok) ? min(n_t, kActT) : 0;
-      for (int q = lane; q < n_t; q += 32) reinterpret_cast<int*>(sl + kOffTup)[q] = list[q];
+      const int s = (int)(seq % kSlots);
+      uint8_t* sl = slot_ptr(ring, s, G::kSlotBytes);
+      SlotMeta* meta = reinterpret_cast<SlotMeta*>(sl + G::kOffMeta);
+      const int ng = min(G::kSegG, ngrp - g0);
+      const int nwords = min(G::kSegG * kP, Ly.ldh - g0 * kP);              // a multiple of 4
+      const uint32_t ev_bytes = (uint32_t)min(4 * G::kSegG, 8 * Ly.ev_stride - 4 * g0);
+      const uint32_t act_bytes = (uint32_t)min(4 * G::kSegG, 4 * arow_words - 4 * g0);
+      const int nstage = (n_t > 0 && act_ok) ? min(n_t, G::kActT) : 0;
+      for (int q = lane; q < n_t; q += 32) reinterpret_cast<uint16_t*>(sl + G::kOffTup)[q] = list[q];
       if (lane == 0) {
-        meta->hrow = Ly.H + (int64_t)k * Ly.ldh + w0;
-        meta->wrow = reinterpret_cast<uint8_t*>(Ly.W + (int64_t)k * Ly.nw_in) + w0 / 8;
-        meta->aprev = aprev + w0 / 8;
+        meta->hrow = Ly.H + (int64_t)k * Ly.ldh + (int64_t)g0 * kP;
+        meta->wrow = reinterpret_cast<uint32_t*>(Ly.W + (int64_t)k * Ly.nw_in) + g0;
+        meta->aprev = aprev + g0;
         meta->type = n_t > 0 ? kSlotRow : kSlotSparse;
         meta->n_t = n_t;
-        meta->nin = min(kSegW, Kin - w0);
-        meta->ch0 = w0 / 8;
-        meta->arow_bytes = (int)arow_bytes;
-        meta->act_smem = nstage > 0 ? 1 : 0;
-        meta->nseg = nseg;
+        meta->ng = ng;
+        meta->last_mask = (g0 + ng == ngrp) ? group_mask(ngrp - 1, Ly.Kin) : kFull;
+        meta->arow_words = arow_words;
+        meta->nstage = nstage;
+        meta->nwords = nwords;
       }
       __syncwarp();
       if (lane == 0) {
-        const uint32_t ev_bytes = 8u * (uint32_t)nevw;
-        const uint32_t h_bytes = n_t > 0 ? 2u * (uint32_t)nseg : 0u;
-        const uint32_t a_bytes = (uint32_t)nstage * (uint32_t)((nact + 15) & ~15);
-        tc::mbar_arrive_tx(&sh->full[s], ev_bytes + h_bytes + a_bytes);
-        sh->issued[s] = (int)(seq / kWsSlots);
-        tc::bulk_g2s(sl + kOffEv, Ly.EV + (int64_t)k * Ly.ev_stride + w0 / 64, ev_bytes, &sh->full[s]);
-        if (n_t > 0)
-          tc::bulk_g2s(sl + kOffH, Ly.H + (int64_t)k * Ly.ldh + w0, h_bytes, &sh->full[s]);
+        const uint32_t h_bytes = n_t > 0 ? 4u * (uint32_t)nwords : 0u;
+        tc::mbar_arrive_tx(&sh->full[s], ev_bytes + h_bytes + (uint32_t)nstage * act_bytes);
+        sh->issued[s] = (int)(seq / kSlots);
+        tc::bulk_g2s(sl + G::kOffEv, evrow + g0, ev_bytes, &sh->full[s]);
+        if (n_t > 0) tc::bulk_g2s(sl, meta->hrow, h_bytes, &sh->full[s]);
         for (int q = 0; q < nstage; ++q)
-          tc::bulk_g2s(sl + kOffAct + q * (kSegW / 8),
-                       aprev + (size_t)(list[q] & 0xFFFF) * arow_bytes + w0 / 8,
-                       (uint32_t)((nact + 15) & ~15), &sh->full[s]);
+          tc::bulk_g2s(sl + G::kOffAct + q * (4 * G::kSegG),
+                       aprev + (size_t)(list[q] & 0x7FFF) * arow_words + g0, act_bytes, &sh->full[s]);
       }
-      seq += kWsSched;
+      seq += kSched;
     }
     next = __shfl_sync(kFull, next, 0);
   }
-  // no more rows: an END slot for the consumers (released by nobody)
+  // no more rows: an END slot for consumer group j (released by nobody)
   if (acquire(seq)) {
-    const int s = (int)(seq % kWsSlots);
+    const int s = (int)(seq % kSlots);
     if (lane == 0) {
-      reinterpret_cast<SlotMeta*>(slot_ptr(ring, s) + kOffMeta)->type = kSlotEnd;
+      reinterpret_cast<SlotMeta*>(slot_ptr(ring, s, G::kSlotBytes) + G::kOffMeta)->type = kSlotEnd;
       tc::mbar_arrive(&sh->full[s]);
     }
   }
@@ -224,145 +260,101 @@ __device__ __forceinline__ void ws_scheduler(const StepParams* __restrict__ P, W
 }
 
 // ---------------------------------------------------------------------------
-// Consumer warp ci: slots -> hidden weights and W.  Each slot's chunks of 8
-// weights are dealt to the kWsCons x 32 consumer lanes, two per lane at a
-// time (chunks c and c + kWsCons * 32), so the tuple loop is shared.
+// Consumer warp ci of group ci / kPerGroup: the slots of its scheduler ->
+// hidden weights and W.  The segment's groups are dealt to the group's
+// kGroupLanes lanes, two per lane at a time (g and g + kGroupLanes), so the
+// tuple loop is shared.
 // ---------------------------------------------------------------------------
-template <int kHb>
+template <int kP, bool kOnes>
 __device__ __forceinline__ void ws_consumer(const StepParams* __restrict__ P, WsShared* sh,
                                             uint8_t* ring, int ci, int lane) {
+  using G = Geo<kP>;
+  constexpr int kSlots = Ring<kP>::kSlots;
   volatile int* failed = &sh->failed;
-  Enc E;
-  E.h_max = P->h_max;
-  E.hb = P->hb;
-  E.base = 1 << P->hb;
-  Lanes<kHb> LN;
-  LN.hb_rt = P->hb;
-  LN.over_pair = (uint32_t)(E.base + E.h_max + 1) * kLaneOne;
-  LN.pos_pair = (uint32_t)(E.base + (E.h_max + 1) / 2) * kLaneOne;
-  const uint32_t pos_from = (uint32_t)(E.base + (E.h_max + 1) / 2);  // lattice index of h = +1
-  const uint32_t v_top = (uint32_t)(E.base + E.h_max);
-  constexpr int kStride = kWsPerGroup * 32;   // chunk distance between a lane's two chunks
-  const int grp = ci / kWsPerGroup, wi = ci % kWsPerGroup;
-  // the schedulers whose slots this group takes: grp, grp + kWsGroups, ...
-  unsigned mine = 0;
-  for (int j = grp; j < kWsSched; j += kWsGroups) mine |= 1u << j;
+  const Sliced<kP, kOnes> S(P->h_max);
+  const int grp = ci / kPerGroup, wi = ci % kPerGroup;
+  const int ti = wi * 32 + lane;
   uint64_t sparse_bytes = 0;
-  unsigned finished = 0;
 #pragma unroll 1
-  for (uint32_t seq = (uint32_t)grp; finished != mine; seq += kWsGroups) {
-    const int j = (int)(seq % kWsSched);
-    if ((finished >> j) & 1u) continue;
-    const int s = (int)(seq % kWsSlots);
-    if (!__all_sync(kFull, tc::mbar_wait(&sh->full[s], (seq / kWsSlots) & 1u, failed))) break;
-    uint8_t* sl = slot_ptr(ring, s);
-    const SlotMeta meta = *reinterpret_cast<const SlotMeta*>(sl + kOffMeta);
-    if (meta.type == kSlotEnd) {
-      finished |= 1u << j;
-      continue;
-    }
-    int16_t* hrow = meta.hrow;
-    const uint64_t* ev = reinterpret_cast<const uint64_t*>(sl + kOffEv);
+  for (uint32_t seq = (uint32_t)grp;; seq += kSched) {
+    const int s = (int)(seq % kSlots);
+    const bool ok = tc::mbar_wait(&sh->full[s], (seq / kSlots) & 1u, failed);
+    if (!group_all(grp, ok)) break;
+    uint8_t* sl = slot_ptr(ring, s, G::kSlotBytes);
+    const SlotMeta meta = *reinterpret_cast<const SlotMeta*>(sl + G::kOffMeta);
+    if (meta.type == kSlotEnd) break;
+    const uint32_t* ev = reinterpret_cast<const uint32_t*>(sl + G::kOffEv);
+    const int ng = meta.ng;
     if (meta.type == kSlotSparse) {
-      // a row without tuple: its reinforcement events as single-weight RMWs
-      const int nblk = (meta.nin + 63) / 64;
-      for (int b = wi * 32 + lane; b < nblk; b += kStride) {
-        uint64_t mask = ev[b];
-        sparse_bytes += 4ull * (uint64_t)__popcll(mask);
+      // a row without tuple: the groups with an event, stepped in global memory
 #pragma unroll 1
-        while (mask != 0ull) {
-          const int bit = __ffsll((long long)mask) - 1;
-          mask &= mask - 1ull;
-          int16_t* hp = hrow + 64 * b + bit;
-          const uint32_t v = (uint16_t)*hp;
-          *hp = (int16_t)((v >= pos_from) ? min(v + 1u, v_top) : max(v - 1u, (uint32_t)E.base));
-        }
+      for (int gi = ti; gi < ng; gi += kGroupLanes) {
+        const uint32_t e = ev[gi] & (gi == ng - 1 ? meta.last_mask : kFull);
+        if (e == 0u) continue;
+        uint32_t* hp = meta.hrow + (size_t)gi * kP;
+        uint32_t u[kP];
+        load_planes<kP>(u, hp);
+        S.step(u, S.positive(u), e);
+        store_planes<kP>(hp, u);
+        sparse_bytes += 8ull * kP;
       }
     } else {
       const int n_t = meta.n_t;
-      const int32_t* tl = reinterpret_cast<const int32_t*>(sl + kOffTup);
-      const uint8_t* act = sl + kOffAct;
-      const int nin = meta.nin;                    // real inputs of the segment
-      const int nch = (nin + 7) >> 3;              // chunks holding at least one input
-      const int full = nin >> 3;                   // chunks of 8 real inputs
-      const int ch0 = meta.ch0;                    // chunk offset of the segment in the row
-      const uint32_t arow_bytes = (uint32_t)meta.arow_bytes;
-      const uint8_t* aseg = meta.aprev;            // activation row 0 at the segment's first byte
-      const uint8_t* aprev = aseg - ch0;           // ... at the row's first byte
-      const int nstage = meta.act_smem ? min(n_t, kActT) : 0;
-      uint8_t* wrow = meta.wrow;
-      const uint4* hs = reinterpret_cast<const uint4*>(sl + kOffH);
+      const uint16_t* tl = reinterpret_cast<const uint16_t*>(sl + G::kOffTup);
+      const uint32_t* act = reinterpret_cast<const uint32_t*>(sl + G::kOffAct);
+      const uint32_t* aseg = meta.aprev;
+      const int arow_words = meta.arow_words;
+      const int nstage = meta.nstage;
+      uint32_t* hs = reinterpret_cast<uint32_t*>(sl);
 #pragma unroll 1
-      for (int cb = wi * 32; cb < nch; cb += 2 * kStride) {
-        int chv[2];
-        bool live[2];
-        uint4 w[2];
+      for (int ga = ti; ga < ng; ga += 2 * kGroupLanes) {
+        const int gb = ga + kGroupLanes;
+        const bool live1 = gb < ng;
+        const uint32_t en0 = (ga == ng - 1) ? meta.last_mask : kFull;
+        const uint32_t en1 = live1 ? ((gb == ng - 1) ? meta.last_mask : kFull) : 0u;
+        uint32_t u0[kP], u1[kP];
+        load_planes<kP>(u0, hs + (size_t)ga * kP);
+        if (live1) load_planes<kP>(u1, hs + (size_t)gb * kP);
+        else {
 #pragma unroll
-        for (int u = 0; u < 2; ++u) {
-          chv[u] = cb + u * kStride + lane;
-          live[u] = chv[u] < nch;
-          w[u] = live[u] ? hs[chv[u]] : make_uint4(0, 0, 0, 0);
+          for (int p = 0; p < kP; ++p) u1[p] = 0u;
         }
-        const uint4 w_in[2] = {w[0], w[1]};
         // ---- CP tuples, ascending mu ----
 #pragma unroll 1
         for (int q = 0; q < n_t; ++q) {
-          const int e = tl[q];
-          const uint32_t xm = (e & 0x10000) ? 0xFFu : 0u;   // rho = -1: ~byte
-          const uint8_t* arow = aseg + (size_t)(e & 0xFFFF) * arow_bytes;
-#pragma unroll
-          for (int u = 0; u < 2; ++u) {
-            uint32_t byte = 0u;
-            if (live[u]) byte = q < nstage ? act[q * (kSegW / 8) + chv[u]] : arow[chv[u]];
-            const uint4 d = sh->db[(byte ^ xm) & 0xFFu];
-            w[u].x = LN.clip(w[u].x + d.x);
-            w[u].y = LN.clip(w[u].y + d.y);
-            w[u].z = LN.clip(w[u].z + d.z);
-            w[u].w = LN.clip(w[u].w + d.w);
+          const uint32_t e = tl[q];
+          const uint32_t xm = (e & 0x8000u) ? kFull : 0u;   // rho = -1: complement
+          uint32_t a0, a1 = 0u;
+          if (q < nstage) {
+            a0 = act[q * G::kSegG + ga];
+            if (live1) a1 = act[q * G::kSegG + gb];
+          } else {
+            const uint32_t* arow = aseg + (size_t)(e & 0x7FFFu) * arow_words;
+            a0 = arow[ga];
+            if (live1) a1 = arow[gb];
           }
+          S.step(u0, a0 ^ xm, en0);
+          S.step(u1, a1 ^ xm, en1);
         }
-        // ---- W bytes (reinforcement never flips a sign, so W is final
-        // after CP), H back into the slot ----
-#pragma unroll
-        for (int u = 0; u < 2; ++u) {
-          if (!live[u]) continue;
-          uint32_t wbyte = LN.w_byte(w[u]);
-          if (chv[u] >= full) {
-            // the partly padded last chunk of the row: CP per weight, from the row as loaded
-            const ChunkOut o = chunk_scalar(w_in[u], ch0 + chv[u], nin - 8 * chv[u], tl, n_t, aprev,
-                                            arow_bytes, E, 0u);
-            w[u] = o.w;
-            wbyte = o.wbyte;
-          }
-          reinterpret_cast<uint4*>(sl + kOffH)[chv[u]] = w[u];
-          wrow[chv[u]] = (uint8_t)wbyte;
+        // ---- R: the events step away from 0; W = the lanes with h > 0 ----
+        const uint32_t pos0 = S.positive(u0) & en0;
+        const uint32_t pos1 = S.positive(u1) & en1;
+        S.step(u0, pos0, ev[ga] & en0);
+        if (live1) S.step(u1, pos1, ev[gb] & en1);
+        meta.wrow[ga] = pos0;
+        store_planes<kP>(hs + (size_t)ga * kP, u0);
+        if (live1) {
+          meta.wrow[gb] = pos1;
+          store_planes<kP>(hs + (size_t)gb * kP, u1);
         }
       }
-      // ---- R, after every CP of the segment: the row's few events, applied in
-      // the slot (lanes take event words) ----
-      group_sync(grp);
-      {
-        int16_t* hseg = reinterpret_cast<int16_t*>(sl + kOffH);
-        const int nblk = (nin + 63) / 64;
-        for (int b = wi * 32 + lane; b < nblk; b += kStride) {
-          uint64_t mask = ev[b];
-#pragma unroll 1
-          while (mask != 0ull) {
-            const int bit = __ffsll((long long)mask) - 1;
-            mask &= mask - 1ull;
-            int16_t* hp = hseg + 64 * b + bit;
-            const uint32_t v = (uint16_t)*hp;
-            *hp = (int16_t)((v >= pos_from) ? min(v + 1u, v_top) : max(v - 1u, (uint32_t)E.base));
-          }
-        }
-      }
-      // the slot's H to global memory in one bulk copy (the generic-proxy
+      // the slot's planes to global memory in one bulk copy (the generic-proxy
       // writes above are fenced for the copy engine by every writer)
       asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
       group_sync(grp);
       if (wi == 0 && lane == 0) {
         asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;"
-                     ::"l"(hrow), "r"(tc::smem_u32(sl + kOffH)), "r"((uint32_t)(2 * meta.nseg)) : "memory");
+                     ::"l"(meta.hrow), "r"(tc::smem_u32(sl)), "r"((uint32_t)(4 * meta.nwords)) : "memory");
         asm volatile("cp.async.bulk.commit_group;" ::: "memory");
         asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");   // the slot may be refilled
       }
@@ -370,38 +362,27 @@ __device__ __forceinline__ void ws_consumer(const StepParams* __restrict__ P, Ws
     __syncwarp();
     if (lane == 0) tc::mbar_arrive(&sh->empty[s]);
   }
-  // the group's bulk stores of H complete before the kernel ends
+  // the group's bulk stores complete before the kernel ends
   if (wi == 0 && lane == 0) asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
   if (sparse_bytes) atomicAdd(&sh->stats[2], sparse_bytes);
 }
 
-template <int kHb>
-__global__ void __launch_bounds__(kWsThreads, 1) k_update_ws(const StepParams* __restrict__ P) {
+template <int kP, bool kOnes>
+__global__ void __launch_bounds__(kThreads, 1) k_update_ws(const StepParams* __restrict__ P) {
+  using G = Geo<kP>;
+  constexpr int kSlots = Ring<kP>::kSlots;
   extern __shared__ uint8_t ws_raw[];
   uint8_t* ring = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(ws_raw) + 127) &
                                              ~static_cast<uintptr_t>(127));
-  WsShared* sh = reinterpret_cast<WsShared*>(ring + (size_t)kWsSlots * kSlotBytes);
+  WsShared* sh = reinterpret_cast<WsShared*>(ring + (size_t)kSlots * G::kSlotBytes);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   Ctrl* ctrl = P->ctrl;
-  // tables and barriers: independent of every earlier kernel
-  if (threadIdx.x < 256) {
-    // db[b]: the +-1 lattice steps of the 8 weights of a chunk whose activation
-    // byte is b, for rho = +1 (rho = -1 indexes with ~b), two lanes per word
-    // (d_lo + 2^16 d_hi: one 32-bit add steps both lanes)
-    const int b = threadIdx.x;
-    uint32_t wv[4];
-#pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      const int d0 = ((b >> (2 * q)) & 1) ? 1 : -1, d1 = ((b >> (2 * q + 1)) & 1) ? 1 : -1;
-      wv[q] = (uint32_t)(d0 + 65536 * d1);
-    }
-    sh->db[b] = make_uint4(wv[0], wv[1], wv[2], wv[3]);
-  }
-  if (threadIdx.x < kWsSlots) sh->issued[threadIdx.x] = -1;
+  // barriers: independent of every earlier kernel
+  if (threadIdx.x < kSlots) sh->issued[threadIdx.x] = -1;
   if (threadIdx.x == 0) {
-    for (int q = 0; q < kWsSlots; ++q) {
+    for (int q = 0; q < kSlots; ++q) {
       tc::mbar_init(&sh->full[q], 1);
-      tc::mbar_init(&sh->empty[q], kWsPerGroup);
+      tc::mbar_init(&sh->empty[q], kPerGroup);
     }
     sh->stats[0] = sh->stats[1] = sh->stats[2] = 0ull;
     sh->failed = 0;
@@ -417,17 +398,17 @@ __global__ void __launch_bounds__(kWsThreads, 1) k_update_ws(const StepParams* _
   // an expired bounded wait in this step's forward pass: no CP, no R (the
   // selection kernel marked nothing either); the counters still advance
   const bool step_failed = ctrl->timeouts != 0u;
-  for (int i = threadIdx.x; i < bsz; i += kWsThreads) {
+  for (int i = threadIdx.x; i < bsz; i += kThreads) {
     const int yv = P->y[start + i];
-    sh->y[i] = (yv < 0 || yv >= P->c) ? 0 : yv;   // memory-safe stand-in; the host reports bad labels
+    sh->y[i] = (int16_t)((yv < 0 || yv >= P->c) ? 0 : yv);   // memory-safe stand-in; the host reports bad labels
   }
   __syncthreads();
-  if (warp < kWsSched)
-    ws_scheduler(P, sh, ring, warp, lane, start, bsz, step_failed);
+  if (warp < kSched)
+    ws_scheduler<kP>(P, sh, ring, warp, lane, start, bsz, step_failed);
   else
-    ws_consumer<kHb>(P, sh, ring, warp - kWsSched, lane);
+    ws_consumer<kP, kOnes>(P, sh, ring, warp - kSched, lane);
   __syncthreads();
-  if (sh->failed && threadIdx.x < kWsSlots && sh->issued[threadIdx.x] >= 0) {
+  if (sh->failed && threadIdx.x < kSlots && sh->issued[threadIdx.x] >= 0) {
     // after an expired wait: the copies issued into this slot land before the
     // CTA's shared memory goes away (a wait of its own, bounded)
     int own = 0;
@@ -453,27 +434,54 @@ __global__ void __launch_bounds__(kWsThreads, 1) k_update_ws(const StepParams* _
   }
 }
 
-}  // namespace
-
-size_t update_ws_smem() { return kWsSmemBytes; }
-
-cudaError_t prepare_update_ws() {
-  cudaError_t e = cudaFuncSetAttribute(k_update_ws<8>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       (int)kWsSmemBytes);
-  if (e != cudaSuccess) return e;
-  e = cudaFuncSetAttribute(k_update_ws<-1>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                           (int)kWsSmemBytes);
-  if (e != cudaSuccess) return e;
-  return cudaFuncSetAttribute(k_update_ws<0>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              (int)kWsSmemBytes);
+template <int kP, bool kOnes>
+cudaError_t set_smem() {
+  return cudaFuncSetAttribute(k_update_ws<kP, kOnes>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              (int)Ring<kP>::kSmem);
 }
 
-cudaError_t launch_update_ws(int hb_mode, unsigned grid, cudaStream_t st, bool pdl, const StepParams* P) {
-  if (hb_mode == 8)
-    return launch_kernel(k_update_ws<8>, dim3(grid), dim3(kWsThreads), kWsSmemBytes, st, pdl, P);
-  if (hb_mode != 0)
-    return launch_kernel(k_update_ws<-1>, dim3(grid), dim3(kWsThreads), kWsSmemBytes, st, pdl, P);
-  return launch_kernel(k_update_ws<0>, dim3(grid), dim3(kWsThreads), kWsSmemBytes, st, pdl, P);
+template <int kP, bool kOnes>
+cudaError_t launch_one(unsigned grid, cudaStream_t st, bool pdl, const StepParams* P) {
+  return launch_kernel(k_update_ws<kP, kOnes>, dim3(grid), dim3(kThreads), Ring<kP>::kSmem, st, pdl, P);
+}
+
+}  // namespace
+
+size_t update_ws_smem(int nplanes) {
+  switch (nplanes) {
+    case 1: return Ring<1>::kSmem;
+    case 2: return Ring<2>::kSmem;
+    case 4: return Ring<4>::kSmem;
+    case 8: return Ring<8>::kSmem;
+    default: return Ring<16>::kSmem;
+  }
+}
+
+cudaError_t prepare_update_ws() {
+  cudaError_t e;
+  if ((e = set_smem<1, true>()) != cudaSuccess || (e = set_smem<2, true>()) != cudaSuccess ||
+      (e = set_smem<4, true>()) != cudaSuccess || (e = set_smem<4, false>()) != cudaSuccess ||
+      (e = set_smem<8, true>()) != cudaSuccess || (e = set_smem<8, false>()) != cudaSuccess ||
+      (e = set_smem<16, false>()) != cudaSuccess)
+    return e;
+  return cudaSuccess;
+}
+
+cudaError_t update_kernel_image(cudaFuncAttributes* fa) {
+  return cudaFuncGetAttributes(fa, k_update_ws<8, true>);
+}
+
+cudaError_t launch_update_ws(int nplanes, int h_max, unsigned grid, cudaStream_t st, bool pdl,
+                             const StepParams* P) {
+  const bool ones = h_max == (1 << nplanes) - 1;
+  switch (nplanes) {
+    case 1: return launch_one<1, true>(grid, st, pdl, P);
+    case 2: return launch_one<2, true>(grid, st, pdl, P);
+    case 4: return ones ? launch_one<4, true>(grid, st, pdl, P) : launch_one<4, false>(grid, st, pdl, P);
+    case 8: return ones ? launch_one<8, true>(grid, st, pdl, P) : launch_one<8, false>(grid, st, pdl, P);
+    case 16: return launch_one<16, false>(grid, st, pdl, P);
+    default: return cudaErrorInvalidValue;
+  }
 }
 
 }  // namespace bk

@@ -1,8 +1,16 @@
-// update_common.cuh -- per-chunk arithmetic of the hidden-weight update
-// (Alg. 3: clipped perceptron, reinforcement, and the repack of W = sign(H),
-// Sec. 3.1) shared by the update kernels.  A chunk is 8 consecutive hidden
-// weights of one neuron row (16 bytes of int16 lattice indices v = (h +
-// h_max)/2 + 2^hb, two 16-bit lanes per 32-bit word; see DevLayer::H).
+// update_common.cuh -- bit-sliced arithmetic on the hidden weights, shared by
+// the update, initialisation and repack kernels (Alg. 3: the clipped
+// perceptron and reinforcement steps; Sec. 3.1: W = sign(H)).
+//
+// A group is 32 weights of one neuron row held as kP 32-bit planes u[0..kP):
+// bit j of u[p] is bit p of the lattice index u_j = (h_j + h_max)/2 of weight
+// j (DevLayer::H).  h_j moves by 2 per event, so u_j moves by 1, clipped to
+// [0, h_max]; h_j > 0 iff u_j >= (h_max + 1)/2.  One step of +-1 on all 32
+// weights is a ripple through the planes: the lanes that move flip plane 0,
+// and a lane's carry (moving up) or borrow (moving down) reaches plane p + 1
+// while its bit p was 1 (up) or 0 (down).  The clip removes from the moving
+// lanes those already at h_max (moving up) or at 0 (moving down): no lane
+// leaves [0, h_max], so no carry passes the top plane.
 #pragma once
 
 #include "bmlp_internal.cuh"
@@ -10,128 +18,118 @@
 namespace bk {
 namespace upd {
 
-constexpr uint32_t kLaneTop = 0x80008000u;
-constexpr uint32_t kLaneOne = 0x00010001u;
 constexpr unsigned kFull = 0xffffffffu;
 
-__device__ __forceinline__ uint32_t lane_v(const uint4& w, int j) {
-  const uint32_t word = (j < 2) ? w.x : (j < 4) ? w.y : (j < 6) ? w.z : w.w;
-  return (word >> (16 * (j & 1))) & 0xFFFFu;
+// Planes used by the lattice index of h_max (the bits of h_max) and stored per
+// group (that count rounded up to a power of two: 1, 2, 4, 8 or 16).
+__host__ __device__ inline int bits_of(int h_max) {
+  int b = 1;
+  while ((1 << b) <= h_max) ++b;
+  return b;
+}
+__host__ __device__ inline int planes_of(int nbits) {
+  int p = 1;
+  while (p < nbits) p <<= 1;
+  return p;
 }
 
-__device__ __forceinline__ void set_lane_v(uint4& w, int j, uint32_t v) {
-  const int sh = 16 * (j & 1);
-  const uint32_t m = ~(0xFFFFu << sh), x = (v & 0xFFFFu) << sh;
-  if (j < 2) w.x = (w.x & m) | x;
-  else if (j < 4) w.y = (w.y & m) | x;
-  else if (j < 6) w.z = (w.z & m) | x;
-  else w.w = (w.w & m) | x;
-}
-
-struct ChunkOut {
-  uint4 w;
-  uint32_t wbyte;
+// A constant broadcast to 32 lanes, plane by plane: m[p] = all ones where
+// bit p of v is set.
+template <int kP>
+struct PlaneConst {
+  uint32_t m[kP];
+  __device__ __forceinline__ explicit PlaneConst(int v) {
+#pragma unroll
+    for (int p = 0; p < kP; ++p) m[p] = ((v >> p) & 1) ? kFull : 0u;
+  }
 };
 
-struct Enc {
-  int h_max, hb, base;  // v = (h + h_max)/2 + base, base = 2^hb
-  __device__ __forceinline__ int dec(uint32_t v) const { return 2 * ((int)v - base) - h_max; }
-  __device__ __forceinline__ uint32_t enc(int h) const { return (uint32_t)((h + h_max) / 2 + base); }
+// kOnes: h_max = 2^kP - 1, every stored plane is used, the upper bound is
+// all ones and h > 0 is the top plane.
+template <int kP, bool kOnes>
+struct Sliced {
+  PlaneConst<kP> hm;  // h_max
+  PlaneConst<kP> pm;  // (h_max + 1)/2, the lattice index of h = +1
+  __device__ __forceinline__ explicit Sliced(int h_max) : hm(h_max), pm((h_max + 1) / 2) {}
+
+  // lanes with u == h_max
+  __device__ __forceinline__ uint32_t at_top(const uint32_t (&u)[kP]) const {
+    uint32_t r = kFull;
+#pragma unroll
+    for (int p = 0; p < kP; ++p) r &= kOnes ? u[p] : ~(u[p] ^ hm.m[p]);
+    return r;
+  }
+  // lanes with u > 0
+  __device__ __forceinline__ uint32_t nonzero(const uint32_t (&u)[kP]) const {
+    uint32_t r = 0u;
+#pragma unroll
+    for (int p = 0; p < kP; ++p) r |= u[p];
+    return r;
+  }
+  // The lanes of en step: up where d is set, down elsewhere; a lane at the
+  // bound in its direction stays.
+  __device__ __forceinline__ void step(uint32_t (&u)[kP], uint32_t d, uint32_t en) const {
+    const uint32_t top = at_top(u), nz = nonzero(u);
+    uint32_t k = en & ((d & ~top) | (~d & nz));
+    const uint32_t nd = ~d;
+#pragma unroll
+    for (int p = 0; p < kP; ++p) {
+      const uint32_t nk = k & (u[p] ^ nd);  // carry on 1 (up) / borrow on 0 (down)
+      u[p] ^= k;
+      k = nk;
+    }
+  }
+  // lanes with h > 0, i.e. u >= (h_max + 1)/2
+  __device__ __forceinline__ uint32_t positive(const uint32_t (&u)[kP]) const {
+    if (kOnes) return u[kP - 1];
+    uint32_t gt = 0u, eq = kFull;
+#pragma unroll
+    for (int p = kP - 1; p >= 0; --p) {
+      gt |= eq & u[p] & ~pm.m[p];
+      eq &= ~(u[p] ^ pm.m[p]);
+    }
+    return gt | eq;
+  }
 };
 
-// Per-weight path (rule as printed, on decoded h): CP, then R for the inputs
-// whose bit of `fire` is set, and W, for the first `nvalid` weights of the
-// chunk.  Taken only by the ragged last chunk of a row; its loops stay rolled.
-__device__ __forceinline__ ChunkOut chunk_scalar(uint4 w, int ch, int nvalid, const int32_t* list,
-                                                 int n_t, const uint8_t* aprev, uint32_t arow_bytes,
-                                                 Enc E, uint32_t fire) {
-#pragma unroll 1
-  for (int q = 0; q < n_t; ++q) {
-    const int e = list[q];
-    const int m = e & 0xFFFF;
-    const int rho = (e & 0x10000) ? -1 : 1;
-    const uint32_t byte = aprev[(size_t)m * arow_bytes + ch];
-#pragma unroll 1
-    for (int j = 0; j < nvalid; ++j) {
-      const int step = ((byte >> j) & 1u) ? rho : -rho;
-      set_lane_v(w, j, E.enc(clip_h(E.dec(lane_v(w, j)) + 2 * step, E.h_max)));
+// The kP planes of one group (16-byte aligned for kP >= 4).
+template <int kP>
+__device__ __forceinline__ void load_planes(uint32_t (&u)[kP], const uint32_t* src) {
+  if constexpr (kP >= 4) {
+#pragma unroll
+    for (int q = 0; q < kP / 4; ++q) {
+      const uint4 v = reinterpret_cast<const uint4*>(src)[q];
+      u[4 * q] = v.x; u[4 * q + 1] = v.y; u[4 * q + 2] = v.z; u[4 * q + 3] = v.w;
     }
+  } else if constexpr (kP == 2) {
+    const uint2 v = *reinterpret_cast<const uint2*>(src);
+    u[0] = v.x; u[1] = v.y;
+  } else {
+    u[0] = *src;
   }
-  ChunkOut out;
-  out.wbyte = 0;
-#pragma unroll 1
-  for (int j = 0; j < nvalid; ++j) {
-    int h = E.dec(lane_v(w, j));
-    if ((fire >> j) & 1u) {
-      h = clip_h(h + (h > 0 ? 2 : -2), E.h_max);
-      set_lane_v(w, j, E.enc(h));
-    }
-    out.wbyte |= (h > 0 ? 1u : 0u) << j;
-  }
-  out.w = w;
-  return out;
 }
 
-// bit 15 of every lane of w equal to the lane value of cpair (exact, carry-free)
-__device__ __forceinline__ uint32_t eq_flags(uint32_t w, uint32_t cpair) {
-  const uint32_t x = w ^ cpair;
-  return ~(((x & 0x7FFF7FFFu) + 0x7FFF7FFFu) | x) & kLaneTop;
+template <int kP>
+__device__ __forceinline__ void store_planes(uint32_t* dst, const uint32_t (&u)[kP]) {
+  if constexpr (kP >= 4) {
+#pragma unroll
+    for (int q = 0; q < kP / 4; ++q)
+      reinterpret_cast<uint4*>(dst)[q] = make_uint4(u[4 * q], u[4 * q + 1], u[4 * q + 2], u[4 * q + 3]);
+  } else if constexpr (kP == 2) {
+    *reinterpret_cast<uint2*>(dst) = make_uint2(u[0], u[1]);
+  } else {
+    *dst = u[0];
+  }
 }
-
-// Gather bit 15 of the 8 lanes into a byte (lane j -> bit j).
-__device__ __forceinline__ uint32_t gather_top(uint32_t a, uint32_t b, uint32_t c, uint32_t d) {
-  const uint32_t p0 = __byte_perm(a, b, 0x7531) & 0x80808080u;
-  const uint32_t p1 = __byte_perm(c, d, 0x7531) & 0x80808080u;
-  return ((p0 * 0x00204081u) >> 28) | (((p1 * 0x00204081u) >> 28) << 4);
-}
-
-// kHb > 0: h_max + 1 = 2^kHb, a compile-time exponent; kHb = -1: h_max + 1 a
-// power of two given at run time; kHb = 0: any odd h_max.
-template <int kHb>
-struct Lanes {
-  static constexpr bool kPow2 = kHb != 0;
-  int hb_rt;
-  __device__ __forceinline__ int hb() const { return kHb > 0 ? kHb : hb_rt; }
-  uint32_t over_pair;  // pair(2^hb + h_max + 1), used when !kPow2
-  uint32_t pos_pair;   // pair(2^hb + (h_max + 1)/2), used when !kPow2
-  // lanes that left [2^hb, 2^hb + h_max] by one step go back
-  __device__ __forceinline__ uint32_t clip(uint32_t v) const {
-    if (kPow2) {
-      const uint32_t t = (v >> hb()) & 0x00030003u;  // 0 under, 1 inside, 2 over
-      return v + kLaneOne - t;
-    } else {
-      const uint32_t under = (~v >> hb()) & kLaneOne;
-      return v + under - (eq_flags(v, over_pair) >> 15);
-    }
-  }
-  // bit 15 of each lane = (h > 0)
-  __device__ __forceinline__ uint32_t pos_top(uint32_t v) const {
-    if (kPow2) return (v << (16 - hb())) & kLaneTop;
-    return ((v | kLaneTop) - pos_pair) & kLaneTop;
-  }
-  // lanes with f = 1 (f: 0 or 1 per lane) step away from 0, then clip
-  __device__ __forceinline__ uint32_t reinforce(uint32_t v, uint32_t f) const {
-    const uint32_t p = pos_top(v) >> 15;
-    return clip(v + (f & p) - (f & ~p));
-  }
-  // W byte of a chunk (lane j -> bit j = h_j > 0)
-  __device__ __forceinline__ uint32_t w_byte(const uint4& w) const {
-    if (kPow2) {
-      // move each lane's sign bit (bit hb - 1) to bit 7 of the lane's low byte;
-      // the low bytes of the 8 lanes then hold the 8 sign bits at bit 7
-      const int sh = 8 - hb();
-      const uint32_t x = sh >= 0 ? w.x << sh : w.x >> -sh, y = sh >= 0 ? w.y << sh : w.y >> -sh;
-      const uint32_t z = sh >= 0 ? w.z << sh : w.z >> -sh, u = sh >= 0 ? w.w << sh : w.w >> -sh;
-      const uint32_t p0 = __byte_perm(x, y, 0x6420) & 0x80808080u;
-      const uint32_t p1 = __byte_perm(z, u, 0x6420) & 0x80808080u;
-      return ((p0 * 0x00204081u) >> 28) | (((p1 * 0x00204081u) >> 28) << 4);
-    }
-    return gather_top(pos_top(w.x), pos_top(w.y), pos_top(w.z), pos_top(w.w));
-  }
-};
 
 __device__ __forceinline__ uint32_t word_of(const uint4& v, int i) {
   return i == 0 ? v.x : (i == 1 ? v.y : (i == 2 ? v.z : v.w));
+}
+
+// Valid-input mask of group g of a row of Kin inputs.
+__host__ __device__ __forceinline__ uint32_t group_mask(int g, int Kin) {
+  const int n = Kin - 32 * g;
+  return n >= 32 ? 0xffffffffu : (n <= 0 ? 0u : ((1u << n) - 1u));
 }
 
 }  // namespace upd

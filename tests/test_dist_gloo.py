@@ -71,9 +71,16 @@ def test_bench_arithmetic():
     import bench
     w = (8192, 8192, 8192, 8192, 8192)
     assert bench.bitpairs_per_sample(w, 10) == 4 * 8192 * (8192 + 10)
-    # int16 H read + write (8192 x 8192 x 2 x 2 bytes) + packed W (8192 x 128 x 8) per layer
-    assert bench.update_bytes_per_launch(w) == 4 * (8192 * 8192 * 4 + 8192 * 128 * 8)
-    assert bench.update_bytes_per_launch((784, 256)) == 256 * (13 * 64 * 4 + 13 * 8)
+    # bit-sliced H (8 planes of 32 weights: one byte per weight) read + write
+    # (8192 x 8192 x 1 x 2 bytes) + packed W (8192 x 128 x 8) per layer
+    assert bench.update_bytes_per_launch(w) == 4 * (8192 * 8192 * 2 + 8192 * 128 * 8)
+    # 25 groups x 8 planes = 200 words per row; one plane (h_max = 1): 25 words
+    # padded to 28; 16 planes (h_max = 257): 400 words
+    assert bench.update_bytes_per_launch((784, 256)) == 256 * (2 * 4 * 200 + 13 * 8)
+    assert bench.update_bytes_per_launch((784, 256), h_max=1) == 256 * (2 * 4 * 28 + 13 * 8)
+    assert bench.update_bytes_per_launch((784, 256), h_max=257) == 256 * (2 * 4 * 400 + 13 * 8)
+    assert [bench.hidden_planes(h) for h in (1, 3, 5, 7, 15, 17, 255, 257, 16383)] == \
+        [1, 2, 4, 4, 4, 8, 8, 16, 16]
 
 
 # -- neuron sharding (paper_2412_00119_gb300.sharding) ------------------------------

@@ -53,14 +53,12 @@ def assert_same_state(gpu, ref, where=""):
 
 def run_pair(widths, classes, n_train, n_test=64, epochs=2, seed=5, bs=100, gamma=None, h_max=255,
              r=(1, 4), p_r0=0.5, gen="bias", host=False, profiling=False, teacher_hidden=16,
-             data_number=99, fwd=B.BMLP_FWD_AUTO, group_mode=0, update_impl=B.BMLP_UPD_AUTO):
+             data_number=99, fwd=B.BMLP_FWD_AUTO, group_mode=0):
     cfg = W.small_config(widths, classes, n_train, n_test, gen=gen, teacher_hidden=teacher_hidden,
                          number=data_number)
     tr = W.make_split(cfg, "train")
     gpu = B.BMLP(widths, classes, h_max=h_max, seed=seed, bs=bs, r=r, p_r0=p_r0, gamma=gamma,
-                 fwd_impl=fwd, group_mode=group_mode, update_impl=update_impl)
-    assert gpu.info["update_impl"] == (update_impl if update_impl else
-                                       (B.BMLP_UPD_STREAM if bs <= 128 else B.BMLP_UPD_ROWS))
+                 fwd_impl=fwd, group_mode=group_mode)
     assert gpu.info["fwd_impl"] == (fwd if fwd else
                                     (B.BMLP_FWD_TCGEN05 if bs <= 128 else B.BMLP_FWD_POPC))
     ref = O.OracleModel(list(widths), classes, h_max=h_max, seed=seed, bs=bs, r=r, p_r0=p_r0,
@@ -283,6 +281,19 @@ CASES = {
     # the widest input the int16 pre-activations allow: the largest split-K
     # partials of the tensor-core forward (|partial| = 8192)
     "widest_input": dict(widths=(32767, 64), classes=4, n_train=200, teacher_hidden=8),
+    # every plane count of the bit-sliced hidden weights (1, 2, 4, 8, 16 planes;
+    # h_max = 2^planes - 1 or not), rows of several update segments (4096
+    # inputs per segment at 16 planes, 8192 at 8), and rows of up to 1024 CP
+    # tuples (gamma = 1, bs = 1024)
+    "h_max_7_clipping": dict(widths=(96, 64), classes=4, n_train=400, h_max=7, p_r0=1.0),
+    "h_max_15_clipping": dict(widths=(300, 128), classes=5, n_train=400, h_max=15, p_r0=1.0),
+    "h_max_127": dict(widths=(200, 96), classes=4, n_train=300, h_max=127, p_r0=1.0),
+    "h_max_257_two_segments": dict(widths=(5000, 64), classes=4, n_train=200, h_max=257,
+                                   teacher_hidden=8),
+    "h_max_16383": dict(widths=(130, 64), classes=4, n_train=300, h_max=16383, p_r0=2.0),
+    "two_segments_255": dict(widths=(9000, 64), classes=4, n_train=200, teacher_hidden=8),
+    "bs_max_gamma_1": dict(widths=(64, 16), classes=4, n_train=2048, bs=1024, gamma=[1]),
+    "bs_300": dict(widths=(256, 128), classes=4, n_train=900, bs=300, gamma=[64]),
 }
 
 
@@ -293,18 +304,6 @@ def test_small_case(name, engine):
     if engine == "tcgen05" and kw.get("bs", 100) > 128:
         pytest.skip("the tcgen05 forward takes mini-batches of at most 128")
     gpu, _ = run_pair(fwd=ENGINES[engine], **kw)
-    gpu.close()
-
-
-ROWS_CASES = ["ragged_3layer", "tail_batch", "h_max_3_clipping", "h_max_1", "hundred_classes",
-              "groups_reshuffled", "always_reinforce", "multi_tile_k", "widest_input"]
-
-
-@pytest.mark.parametrize("name", ROWS_CASES)
-def test_small_case_rows_update(name):
-    """The same cases with the per-warp-rows update kernel (the one used for
-    mini-batches above 128) in place of the bulk-copy-fed one."""
-    gpu, _ = run_pair(update_impl=B.BMLP_UPD_ROWS, **CASES[name])
     gpu.close()
 
 
@@ -482,15 +481,23 @@ def test_update_stats_count_rows_and_bytes():
     B.bmlp_update_stats(gpu.h, reset=True)
     gpu.train(dev_x(tr.xp), dev_y(tr.y))
     rows, streamed, nbytes = B.bmlp_update_stats(gpu.h, reset=True)
-    want_rows = want_streamed = 0
+    want_rows = 0
+    per_layer = []
     for l in (1, 2):
         _, _, mark, sel = B.bmlp_debug_last_step(gpu.h, l)
+        per_layer.append(np.unique(sel[sel >= 0]).size if mark.any() else 0)
         if mark.any():
             want_rows += widths[l]
-            want_streamed += np.unique(sel[sel >= 0]).size
+    want_streamed = sum(per_layer)
     assert rows == want_rows and streamed == want_streamed, (rows, want_rows, streamed, want_streamed)
-    row_bytes = [4 * 64 * ((widths[l - 1] + 63) // 64) + 8 * ((widths[l - 1] + 63) // 64) for l in (1, 2)]
-    assert nbytes >= streamed * min(row_bytes) and (nbytes - streamed * min(row_bytes)) % 4 == 0
+    # a streamed row: its bit-sliced H (8 planes per 32 inputs at h_max = 255,
+    # rows padded to 16 bytes) read and written, its packed W row written; a
+    # row without tuple: 2 x 32 bytes per group of 32 weights with an event
+    ldh = [((widths[l - 1] + 31) // 32 * 8 + 3) // 4 * 4 for l in (1, 2)]
+    row_bytes = [2 * 4 * ldh[l - 1] + 8 * ((widths[l - 1] + 63) // 64) for l in (1, 2)]
+    assert row_bytes == [2 * 4 * 56 + 8 * 4, 2 * 4 * 40 + 8 * 3]
+    streamed_bytes = per_layer[0] * row_bytes[0] + per_layer[1] * row_bytes[1]
+    assert nbytes >= streamed_bytes and (nbytes - streamed_bytes) % 64 == 0, (nbytes, streamed_bytes)
     assert B.bmlp_update_stats(gpu.h) == (0, 0, 0)
     gpu.close()
 
