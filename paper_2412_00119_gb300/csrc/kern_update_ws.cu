@@ -23,18 +23,17 @@
 //     event bitmap and of the first tuples' activation words, plus the tuple
 //     list and a header;
 //   - consumer group j (kPerGroup warps) takes the slots of scheduler j in
-//     order: each lane holds two groups of 32 weights at a time, applies the
-//     tuples in ascending mu, then the reinforcement events (Alg. 3 applies R
-//     after CP), writes the W word, and puts the planes back into the slot;
-//     one bulk copy writes the segment back to global memory, and the slot
-//     is released ("empty").
+//     order: each lane holds two groups of 32 weights at a time in
+//     registers, applies the tuples in ascending mu, then the reinforcement
+//     events (Alg. 3 applies R after CP), and writes the planes and the W
+//     word to global memory; each warp releases the slot ("empty") when it
+//     has read its part, without waiting for the other warps.
 // A row without tuple occupies a slot with its event bitmap only: its groups
 // with an event are stepped in place in global memory, and its W is
 // unchanged.  Layers with an empty M_l are skipped (no CP, no R).  Every
-// mbarrier wait is bounded; an expiry stops the CTA's loops (a consumer group
-// decides together, so no barrier is left waiting), waits (bounded) for the
-// copies it issued, and is counted in the control block.  The last CTA to
-// finish advances the step counters.
+// mbarrier wait is bounded; an expiry stops the CTA's loops, waits (bounded)
+// for the copies it issued, and is counted in the control block.  The last
+// CTA to finish advances the step counters.
 #include "tc_common.cuh"
 #include "update_common.cuh"
 
@@ -107,25 +106,20 @@ __device__ __forceinline__ uint8_t* slot_ptr(uint8_t* ring, int s, int slot_byte
   return ring + (size_t)s * slot_bytes;
 }
 
-// barrier of the kPerGroup warps of consumer group g (named barriers 1..)
-__device__ __forceinline__ void group_sync(int g) {
-  asm volatile("bar.sync %0, %1;" ::"r"(1 + g), "r"(kGroupLanes) : "memory");
-}
-
-// the same barrier, returning whether v held on every thread of the group
-__device__ __forceinline__ bool group_all(int g, bool v) {
-  uint32_t r;
-  asm volatile(
-      "{\n .reg .pred p, q;\n setp.ne.u32 p, %1, 0;\n"
-      " bar.red.and.pred q, %2, %3, p;\n selp.u32 %0, 1, 0, q;\n}"
-      : "=r"(r) : "r"((uint32_t)v), "r"(1 + g), "r"(kGroupLanes) : "memory");
-  return r != 0u;
-}
-
 // ---------------------------------------------------------------------------
 // Scheduler warp j: rows -> slots j, j + kSched, ... (sequence numbers
-// j, j + kSched, ...).
+// j, j + kSched, ...).  Rows are pipelined one deep: while row r is turned
+// into slots, the selections of row r + 1 (its ticket taken one row earlier)
+// are in flight, and the ticket of row r + 2 is taken.
 // ---------------------------------------------------------------------------
+struct RowFetch {
+  int gr;          // global row number (>= rows_total: none)
+  int li, k;       // layer index, neuron
+  int sv[4];       // this lane's selections of patterns 32 q + lane (the first 128)
+  int rho_lane;    // rho_{k, lane} for c <= 32
+  bool skip;       // M_l empty, or the step's forward pass failed: no CP, no R
+};
+
 template <int kP>
 __device__ __forceinline__ void ws_scheduler(const StepParams* __restrict__ P, WsShared* sh,
                                              uint8_t* ring, int j, int lane, int64_t start, int bsz,
@@ -135,65 +129,98 @@ __device__ __forceinline__ void ws_scheduler(const StepParams* __restrict__ P, W
   Ctrl* ctrl = P->ctrl;
   volatile int* failed = &sh->failed;
   const int c = P->c;
+  const int L = P->L;
   const int rows_total = P->rows_total;
   uint16_t* list = sh->list[j];
   uint32_t seq = (uint32_t)j;
   uint64_t st_rows = 0, st_streamed = 0, st_bytes = 0;
+  // lane i < L holds layer i's first row and its "M_l non-empty" flag
+  const int rb_lane = lane < L ? P->layer[lane].row_base : 0;
+  const unsigned am_lane = lane < L ? ctrl->any_mark[lane] : 0u;
   // acquire the slot of sequence number q (its previous use released)
   auto acquire = [&](uint32_t q) -> bool {
     const uint32_t u = q / kSlots;
     if (u == 0) return true;
     return __all_sync(kFull, tc::mbar_wait(&sh->empty[q % kSlots], (u - 1) & 1u, failed));
   };
-  // the ticket of the next row is taken while the current row is scanned
-  int next = 0;
-  if (lane == 0) next = (int)atomicAdd(&ctrl->upd_next, 1u);
-  next = __shfl_sync(kFull, next, 0);
+  // issue the loads of row gr (consumed one row later)
+  auto fetch = [&](int gr) -> RowFetch {
+    RowFetch f;
+    f.gr = gr;
+    f.li = __popc(__ballot_sync(kFull, lane >= 1 && lane < L && gr >= rb_lane));
+    f.skip = gr >= rows_total || step_failed || __shfl_sync(kFull, am_lane, f.li) == 0u;
+    f.k = 0;
+    f.rho_lane = 0;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) f.sv[q] = -1;
+    if (!f.skip) {
+      const DevLayer& Ly = P->layer[f.li];
+      f.k = gr - Ly.row_base;
+      const int g = Ly.group_of ? (int)Ly.group_of[f.k] : f.k / Ly.gamma;
+      const int16_t* selg = Ly.sel + (int64_t)g * P->bs;
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const int m = 32 * q + lane;
+        if (m < bsz) f.sv[q] = (int)selg[m];
+      }
+      if (c <= 32 && lane < c) f.rho_lane = (int)Ly.rho[(int64_t)f.k * c + lane];
+    }
+    return f;
+  };
+  // tuples from selections sv of patterns m0 + 32 q + lane, appended to list
+  auto scan4 = [&](const RowFetch& f, const int (&sv)[4], int m0, int n_t) -> int {
+    const DevLayer& Ly = P->layer[f.li];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const int m = m0 + 32 * q + lane;
+      const bool hit = sv[q] == f.k;
+      const unsigned bal = __ballot_sync(kFull, hit);
+      if (bal != 0u) {
+        const int yv = hit ? (int)sh->y[m] : 0;
+        const int rs = __shfl_sync(kFull, f.rho_lane, yv & 31);
+        if (hit) {
+          const int rho = (c <= 32) ? rs : (int)Ly.rho[(int64_t)f.k * c + yv];
+          list[n_t + __popc(bal & ((1u << lane) - 1u))] = (uint16_t)(m | ((rho > 0) ? 0 : 0x8000));
+        }
+      }
+      n_t += __popc(bal);
+    }
+    return n_t;
+  };
+  int ticket = 0;
+  if (lane == 0) ticket = (int)atomicAdd(&ctrl->upd_next, 1u);
+  RowFetch cur = fetch(__shfl_sync(kFull, ticket, 0));
+  if (lane == 0) ticket = (int)atomicAdd(&ctrl->upd_next, 1u);
 #pragma unroll 1
-  while (true) {
-    const int gr = next;
-    if (gr >= rows_total || *failed) break;
-    if (lane == 0) next = (int)atomicAdd(&ctrl->upd_next, 1u);
-    int li = 0;
-    while (li + 1 < P->L && gr >= P->layer[li + 1].row_base) ++li;
-    if (step_failed || ctrl->any_mark[li] == 0u) {   // M_l empty: no CP, no R
-      next = __shfl_sync(kFull, next, 0);
+  while (cur.gr < rows_total && !*failed) {
+    const RowFetch nxt = fetch(__shfl_sync(kFull, ticket, 0));
+    if (lane == 0) ticket = (int)atomicAdd(&ctrl->upd_next, 1u);
+    if (cur.skip) {
+      cur = nxt;
       continue;
     }
-    const DevLayer& Ly = P->layer[li];
-    const int k = gr - Ly.row_base;
-    const int g = Ly.group_of ? (int)Ly.group_of[k] : k / Ly.gamma;
+    const DevLayer& Ly = P->layer[cur.li];
+    const int k = cur.k;
     // ---- CP tuples of neuron k, ascending mu: the patterns whose selection
-    // in group g is k; for c <= 32 the neuron's row of P_l comes in one load
-    int n_t = 0;
-    const int16_t* selg = Ly.sel + (int64_t)g * P->bs;
-    const int rho_lane = (c <= 32 && lane < c) ? (int)Ly.rho[(int64_t)k * c + lane] : 0;
+    // in its group is k ----
+    int n_t = scan4(cur, cur.sv, 0, 0);
+    if (bsz > 128) {
+      const int g = Ly.group_of ? (int)Ly.group_of[k] : k / Ly.gamma;
+      const int16_t* selg = Ly.sel + (int64_t)g * P->bs;
 #pragma unroll 1
-    for (int m0 = 0; m0 < bsz; m0 += 128) {
-      int sv[4];
+      for (int m0 = 128; m0 < bsz; m0 += 128) {
+        int sv[4];
 #pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        const int m = m0 + 32 * q + lane;
-        sv[q] = (m < bsz) ? (int)selg[m] : -1;
-      }
-#pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        const int m = m0 + 32 * q + lane;
-        const bool hit = sv[q] == k;
-        const unsigned bal = __ballot_sync(kFull, hit);
-        if (bal != 0u) {
-          const int yv = hit ? (int)sh->y[m] : 0;
-          const int rs = __shfl_sync(kFull, rho_lane, yv & 31);
-          if (hit) {
-            const int rho = (c <= 32) ? rs : (int)Ly.rho[(int64_t)k * c + yv];
-            list[n_t + __popc(bal & ((1u << lane) - 1u))] = (uint16_t)(m | ((rho > 0) ? 0 : 0x8000));
-          }
+        for (int q = 0; q < 4; ++q) {
+          const int m = m0 + 32 * q + lane;
+          sv[q] = (m < bsz) ? (int)selg[m] : -1;
         }
-        n_t += __popc(bal);
+        n_t = scan4(cur, sv, m0, n_t);
       }
     }
     __syncwarp();
     st_rows += 1;
+    const int li = cur.li;
     const int ngrp = Ly.ngrp;
     const uint32_t* aprev = (li == 0) ? reinterpret_cast<const uint32_t*>(P->x + start * P->nw0)
                                       : reinterpret_cast<const uint32_t*>(P->layer[li - 1].A);
@@ -242,7 +269,7 @@ __device__ __forceinline__ void ws_scheduler(const StepParams* __restrict__ P, W
       }
       seq += kSched;
     }
-    next = __shfl_sync(kFull, next, 0);
+    cur = nxt;
   }
   // no more rows: an END slot for consumer group j (released by nobody)
   if (acquire(seq)) {
@@ -263,13 +290,17 @@ __device__ __forceinline__ void ws_scheduler(const StepParams* __restrict__ P, W
 // Consumer warp ci of group ci / kPerGroup: the slots of its scheduler ->
 // hidden weights and W.  The segment's groups are dealt to the group's
 // kGroupLanes lanes, two per lane at a time (g and g + kGroupLanes), so the
-// tuple loop is shared.
+// tuple loop is shared.  The warps of a group do not wait for one another:
+// each reads its part of the slot, releases it (the slot's "empty" barrier
+// counts the group's warps), and writes planes and W words to global memory
+// from registers.
 // ---------------------------------------------------------------------------
 template <int kP, bool kOnes>
 __device__ __forceinline__ void ws_consumer(const StepParams* __restrict__ P, WsShared* sh,
                                             uint8_t* ring, int ci, int lane) {
   using G = Geo<kP>;
   constexpr int kSlots = Ring<kP>::kSlots;
+  constexpr int kPerLane = G::kSegG / kGroupLanes;   // groups of a segment per lane at most
   volatile int* failed = &sh->failed;
   const Sliced<kP, kOnes> S(P->h_max);
   const int grp = ci / kPerGroup, wi = ci % kPerGroup;
@@ -278,92 +309,88 @@ __device__ __forceinline__ void ws_consumer(const StepParams* __restrict__ P, Ws
 #pragma unroll 1
   for (uint32_t seq = (uint32_t)grp;; seq += kSched) {
     const int s = (int)(seq % kSlots);
-    const bool ok = tc::mbar_wait(&sh->full[s], (seq / kSlots) & 1u, failed);
-    if (!group_all(grp, ok)) break;
+    if (!__all_sync(kFull, tc::mbar_wait(&sh->full[s], (seq / kSlots) & 1u, failed))) break;
     uint8_t* sl = slot_ptr(ring, s, G::kSlotBytes);
     const SlotMeta meta = *reinterpret_cast<const SlotMeta*>(sl + G::kOffMeta);
     if (meta.type == kSlotEnd) break;
     const uint32_t* ev = reinterpret_cast<const uint32_t*>(sl + G::kOffEv);
     const int ng = meta.ng;
     if (meta.type == kSlotSparse) {
-      // a row without tuple: the groups with an event, stepped in global memory
-#pragma unroll 1
-      for (int gi = ti; gi < ng; gi += kGroupLanes) {
-        const uint32_t e = ev[gi] & (gi == ng - 1 ? meta.last_mask : kFull);
-        if (e == 0u) continue;
-        uint32_t* hp = meta.hrow + (size_t)gi * kP;
+      // a row without tuple: the event words are read and the slot released,
+      // then the groups with an event are stepped in global memory
+      uint32_t evs[kPerLane];
+#pragma unroll
+      for (int q = 0; q < kPerLane; ++q) {
+        const int gi = ti + q * kGroupLanes;
+        evs[q] = gi < ng ? ev[gi] & (gi == ng - 1 ? meta.last_mask : kFull) : 0u;
+      }
+      __syncwarp();
+      if (lane == 0) tc::mbar_arrive(&sh->empty[s]);
+#pragma unroll
+      for (int q = 0; q < kPerLane; ++q) {
+        if (evs[q] == 0u) continue;
+        uint32_t* hp = meta.hrow + (size_t)(ti + q * kGroupLanes) * kP;
         uint32_t u[kP];
         load_planes<kP>(u, hp);
-        S.step(u, S.positive(u), e);
+        S.step(u, S.positive(u), evs[q]);
         store_planes<kP>(hp, u);
         sparse_bytes += 8ull * kP;
       }
-    } else {
-      const int n_t = meta.n_t;
-      const uint16_t* tl = reinterpret_cast<const uint16_t*>(sl + G::kOffTup);
-      const uint32_t* act = reinterpret_cast<const uint32_t*>(sl + G::kOffAct);
-      const uint32_t* aseg = meta.aprev;
-      const int arow_words = meta.arow_words;
-      const int nstage = meta.nstage;
-      uint32_t* hs = reinterpret_cast<uint32_t*>(sl);
+      continue;
+    }
+    const int n_t = meta.n_t;
+    const uint16_t* tl = reinterpret_cast<const uint16_t*>(sl + G::kOffTup);
+    const uint32_t* act = reinterpret_cast<const uint32_t*>(sl + G::kOffAct);
+    const uint32_t* aseg = meta.aprev;
+    const int arow_words = meta.arow_words;
+    const int nstage = meta.nstage;
+    const uint32_t* hs = reinterpret_cast<const uint32_t*>(sl);
 #pragma unroll 1
-      for (int ga = ti; ga < ng; ga += 2 * kGroupLanes) {
-        const int gb = ga + kGroupLanes;
-        const bool live1 = gb < ng;
-        const uint32_t en0 = (ga == ng - 1) ? meta.last_mask : kFull;
-        const uint32_t en1 = live1 ? ((gb == ng - 1) ? meta.last_mask : kFull) : 0u;
-        uint32_t u0[kP], u1[kP];
-        load_planes<kP>(u0, hs + (size_t)ga * kP);
-        if (live1) load_planes<kP>(u1, hs + (size_t)gb * kP);
-        else {
+    for (int ga = ti; ga < ng; ga += 2 * kGroupLanes) {
+      const int gb = ga + kGroupLanes;
+      const bool live1 = gb < ng;
+      const uint32_t en0 = (ga == ng - 1) ? meta.last_mask : kFull;
+      const uint32_t en1 = live1 ? ((gb == ng - 1) ? meta.last_mask : kFull) : 0u;
+      uint32_t u0[kP], u1[kP];
+      load_planes<kP>(u0, hs + (size_t)ga * kP);
+      if (live1) load_planes<kP>(u1, hs + (size_t)gb * kP);
+      else {
 #pragma unroll
-          for (int p = 0; p < kP; ++p) u1[p] = 0u;
-        }
-        // ---- CP tuples, ascending mu ----
-#pragma unroll 1
-        for (int q = 0; q < n_t; ++q) {
-          const uint32_t e = tl[q];
-          const uint32_t xm = (e & 0x8000u) ? kFull : 0u;   // rho = -1: complement
-          uint32_t a0, a1 = 0u;
-          if (q < nstage) {
-            a0 = act[q * G::kSegG + ga];
-            if (live1) a1 = act[q * G::kSegG + gb];
-          } else {
-            const uint32_t* arow = aseg + (size_t)(e & 0x7FFFu) * arow_words;
-            a0 = arow[ga];
-            if (live1) a1 = arow[gb];
-          }
-          S.step(u0, a0 ^ xm, en0);
-          S.step(u1, a1 ^ xm, en1);
-        }
-        // ---- R: the events step away from 0; W = the lanes with h > 0 ----
-        const uint32_t pos0 = S.positive(u0) & en0;
-        const uint32_t pos1 = S.positive(u1) & en1;
-        S.step(u0, pos0, ev[ga] & en0);
-        if (live1) S.step(u1, pos1, ev[gb] & en1);
-        meta.wrow[ga] = pos0;
-        store_planes<kP>(hs + (size_t)ga * kP, u0);
-        if (live1) {
-          meta.wrow[gb] = pos1;
-          store_planes<kP>(hs + (size_t)gb * kP, u1);
-        }
+        for (int p = 0; p < kP; ++p) u1[p] = 0u;
       }
-      // the slot's planes to global memory in one bulk copy (the generic-proxy
-      // writes above are fenced for the copy engine by every writer)
-      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-      group_sync(grp);
-      if (wi == 0 && lane == 0) {
-        asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;"
-                     ::"l"(meta.hrow), "r"(tc::smem_u32(sl)), "r"((uint32_t)(4 * meta.nwords)) : "memory");
-        asm volatile("cp.async.bulk.commit_group;" ::: "memory");
-        asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");   // the slot may be refilled
+      const uint32_t r0 = ev[ga] & en0, r1 = live1 ? ev[gb] & en1 : 0u;
+      // ---- CP tuples, ascending mu ----
+#pragma unroll 1
+      for (int q = 0; q < n_t; ++q) {
+        const uint32_t e = tl[q];
+        const uint32_t xm = (e & 0x8000u) ? kFull : 0u;   // rho = -1: complement
+        uint32_t a0, a1 = 0u;
+        if (q < nstage) {
+          a0 = act[q * G::kSegG + ga];
+          if (live1) a1 = act[q * G::kSegG + gb];
+        } else {
+          const uint32_t* arow = aseg + (size_t)(e & 0x7FFFu) * arow_words;
+          a0 = arow[ga];
+          if (live1) a1 = arow[gb];
+        }
+        S.step(u0, a0 ^ xm, en0);
+        S.step(u1, a1 ^ xm, en1);
+      }
+      // ---- R: the events step away from 0; W = the lanes with h > 0 ----
+      const uint32_t pos0 = S.positive(u0) & en0;
+      const uint32_t pos1 = S.positive(u1) & en1;
+      S.step(u0, pos0, r0);
+      S.step(u1, pos1, r1);
+      meta.wrow[ga] = pos0;
+      store_planes<kP>(meta.hrow + (size_t)ga * kP, u0);
+      if (live1) {
+        meta.wrow[gb] = pos1;
+        store_planes<kP>(meta.hrow + (size_t)gb * kP, u1);
       }
     }
     __syncwarp();
     if (lane == 0) tc::mbar_arrive(&sh->empty[s]);
   }
-  // the group's bulk stores complete before the kernel ends
-  if (wi == 0 && lane == 0) asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
   if (sparse_bytes) atomicAdd(&sh->stats[2], sparse_bytes);
 }
 
