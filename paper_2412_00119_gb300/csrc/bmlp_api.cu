@@ -282,7 +282,7 @@ int enqueue_step(bmlp_t* h, cudaStream_t st, bool fork, bool chained = false) {
   }
   if (fork) CK(h, cudaStreamWaitEvent(st, h->evJoin, 0));
   prof_begin(h, kProfUpd, st);
-  CK(h, launch_update_ws(h->hp.nplanes, h->h_max, (unsigned)h->updCtas, st, fork, h->dP));
+  CK(h, launch_update_ws(h->hp.nplanes, h->h_max, h->bs, (unsigned)h->updCtas, st, fork, h->dP));
   prof_end(h, st);
   CK(h, cudaGetLastError());
   return BMLP_OK;
@@ -539,7 +539,7 @@ int bmlp_create(const int32_t* widths, int32_t n_widths, int32_t classes, int16_
   {
     // the update grid is persistent, one CTA per SM (its slot ring fills most
     // of the shared memory)
-    h->updSmem = update_ws_smem(P.nplanes);
+    h->updSmem = update_ws_smem(P.nplanes, bs);
     const cudaError_t ea = prepare_update_ws();
     if (ea != cudaSuccess) return bail(cuda_fail(h, ea, "update kernel shared memory attribute"));
     h->updCtas = prop.multiProcessorCount;

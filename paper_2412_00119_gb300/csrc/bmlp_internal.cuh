@@ -231,10 +231,11 @@ cudaError_t launch_forward_b1(const uint64_t* A, int64_t M, int nw_in, const uin
 // (kern_update_ws.cu): bulk copies into a ring of shared-memory slots, the
 // bit-sliced steps by consumer warps; one CTA per SM (grid = the SM count).
 // pdl: launched with the programmatic-stream-serialization attribute.
-// nplanes: DevLayer's planes per group (StepParams::nplanes).
-size_t update_ws_smem(int nplanes);
+// nplanes: DevLayer's planes per group (StepParams::nplanes); bs: the
+// mini-batch size (the tuple lists of the slot ring).
+size_t update_ws_smem(int nplanes, int bs);
 cudaError_t prepare_update_ws();
-cudaError_t launch_update_ws(int nplanes, int h_max, unsigned grid, cudaStream_t st, bool pdl,
+cudaError_t launch_update_ws(int nplanes, int h_max, int bs, unsigned grid, cudaStream_t st, bool pdl,
                              const StepParams* P);
 // Attributes of the update kernel: fails when the library holds no sm_103a image.
 cudaError_t update_kernel_image(cudaFuncAttributes* fa);

@@ -42,14 +42,13 @@ namespace {
 
 using namespace upd;
 
-constexpr int kSched = 4;                     // scheduler warps
-constexpr int kPerGroup = 4;                  // consumer warps per group; group j serves scheduler j
+constexpr int kSched = 8;                     // scheduler warps
+constexpr int kPerGroup = 2;                  // consumer warps per group; group j serves scheduler j
 constexpr int kCons = kSched * kPerGroup;
 constexpr int kThreads = 32 * (kSched + kCons);
 constexpr int kGroupLanes = 32 * kPerGroup;
 constexpr int kMaxT = BMLP_MAX_BS;            // CP tuples of one row at most
-constexpr int kActStage = 4096;               // staged activation bytes per slot
-constexpr int kMaxSlots = 12;
+constexpr int kMaxSlots = 24;
 constexpr int kSmemLimit = 232448;            // dynamic shared memory of one CTA at most
 
 enum SlotType : int { kSlotRow = 0, kSlotSparse = 1, kSlotEnd = 2 };
@@ -68,21 +67,35 @@ struct SlotMeta {
 };
 
 // Slot layout for kP planes per group: planes, event bits, staged activation
-// words, tuple list (uint16: mu | 0x8000 when rho = -1), header.
+// words, tuple list (uint16: mu | 0x8000 when rho = -1; 2 bs bytes), header.
 template <int kP>
 struct Geo {
   static constexpr int kSegG = (2048 / kP) < 1024 ? (2048 / kP) : 1024;  // groups per segment
   static constexpr int kHBytes = 4 * kP * kSegG;
   static constexpr int kEvBytes = 4 * kSegG;
-  static constexpr int kActT = kActStage / (4 * kSegG);   // tuples staged at most
+  static constexpr int kActBytes = 4 * kSegG;                   // one pattern's words of a segment
+  static constexpr int kActT = 2048 / kActBytes > 1 ? 2048 / kActBytes : 1;  // tuples staged at most
   static constexpr int kOffEv = kHBytes;
   static constexpr int kOffAct = kOffEv + kEvBytes;
-  static constexpr int kOffTup = kOffAct + kActStage;
-  static constexpr int kOffMeta = kOffTup + 2 * kMaxT;
-  static constexpr int kSlotBytes = (kOffMeta + (int)sizeof(SlotMeta) + 127) & ~127;
+  static constexpr int kOffTup = kOffAct + kActT * kActBytes;
+};
+
+// What the schedulers read of a layer, copied to shared memory at the start
+// (the parameter block's cache lines do not survive in the small L1 that the
+// slot ring leaves, and every row reads several of them in sequence).
+struct LayerSh {
+  uint32_t* H;
+  uint64_t* W;
+  const uint64_t* EV;
+  const int16_t* sel;
+  const int8_t* rho;
+  const int16_t* group_of;
+  const uint32_t* aprev;   // the layer's input activations of this mini-batch, row 0
+  int row_base, gamma, ngrp, ldh, nw_in, ev_stride, Kin, pad;
 };
 
 struct __align__(16) WsShared {
+  LayerSh lay[BMLP_MAX_LAYERS];
   unsigned long long full[kMaxSlots];
   unsigned long long empty[kMaxSlots];
   int16_t y[kMaxT];                   // labels of the mini-batch (bad ones as 0)
@@ -92,15 +105,25 @@ struct __align__(16) WsShared {
   int failed;
 };
 
-template <int kP>
+// The ring for a mini-batch size: as many slots as fit in the shared memory
+// (a multiple of kSched, at most kMaxSlots); the host sizes the launch with
+// the same function.
 struct Ring {
-  static constexpr int kSlots =
-      128 + 12 * Geo<kP>::kSlotBytes + (int)sizeof(WsShared) <= kSmemLimit ? 12 : 8;
-  static_assert(kSlots % kSched == 0, "each slot belongs to one scheduler");
-  static constexpr size_t kSmem = 128 /*alignment slack*/ + (size_t)kSlots * Geo<kP>::kSlotBytes +
-                                  sizeof(WsShared);
-  static_assert(kSmem <= (size_t)kSmemLimit, "slot ring too large");
+  int slot_bytes, nslots, off_meta;
+  size_t smem;   // dynamic shared memory of the launch (128 bytes of alignment slack)
 };
+
+template <int kP>
+__host__ __device__ __forceinline__ Ring ring_of(int bs) {
+  Ring r;
+  r.off_meta = Geo<kP>::kOffTup + ((2 * bs + 15) & ~15);
+  r.slot_bytes = (r.off_meta + (int)sizeof(SlotMeta) + 127) & ~127;
+  int n = (kSmemLimit - 128 - (int)sizeof(WsShared)) / r.slot_bytes;
+  n = n < kMaxSlots ? n : kMaxSlots;
+  r.nslots = n / kSched * kSched;
+  r.smem = 128 + (size_t)r.nslots * r.slot_bytes + sizeof(WsShared);
+  return r;
+}
 
 __device__ __forceinline__ uint8_t* slot_ptr(uint8_t* ring, int s, int slot_bytes) {
   return ring + (size_t)s * slot_bytes;
@@ -122,26 +145,27 @@ struct RowFetch {
 
 template <int kP>
 __device__ __forceinline__ void ws_scheduler(const StepParams* __restrict__ P, WsShared* sh,
-                                             uint8_t* ring, int j, int lane, int64_t start, int bsz,
+                                             uint8_t* ring, const Ring R, int j, int lane, int bsz,
                                              bool step_failed) {
   using G = Geo<kP>;
-  constexpr int kSlots = Ring<kP>::kSlots;
+  const uint32_t nslots = (uint32_t)R.nslots;
   Ctrl* ctrl = P->ctrl;
   volatile int* failed = &sh->failed;
   const int c = P->c;
   const int L = P->L;
+  const int bs = P->bs;
   const int rows_total = P->rows_total;
   uint16_t* list = sh->list[j];
   uint32_t seq = (uint32_t)j;
   uint64_t st_rows = 0, st_streamed = 0, st_bytes = 0;
   // lane i < L holds layer i's first row and its "M_l non-empty" flag
-  const int rb_lane = lane < L ? P->layer[lane].row_base : 0;
+  const int rb_lane = lane < L ? sh->lay[lane].row_base : 0;
   const unsigned am_lane = lane < L ? ctrl->any_mark[lane] : 0u;
   // acquire the slot of sequence number q (its previous use released)
   auto acquire = [&](uint32_t q) -> bool {
-    const uint32_t u = q / kSlots;
+    const uint32_t u = q / nslots;
     if (u == 0) return true;
-    return __all_sync(kFull, tc::mbar_wait(&sh->empty[q % kSlots], (u - 1) & 1u, failed));
+    return __all_sync(kFull, tc::mbar_wait(&sh->empty[q % nslots], (u - 1) & 1u, failed));
   };
   // issue the loads of row gr (consumed one row later)
   auto fetch = [&](int gr) -> RowFetch {
@@ -154,10 +178,10 @@ __device__ __forceinline__ void ws_scheduler(const StepParams* __restrict__ P, W
 #pragma unroll
     for (int q = 0; q < 4; ++q) f.sv[q] = -1;
     if (!f.skip) {
-      const DevLayer& Ly = P->layer[f.li];
+      const LayerSh& Ly = sh->lay[f.li];
       f.k = gr - Ly.row_base;
       const int g = Ly.group_of ? (int)Ly.group_of[f.k] : f.k / Ly.gamma;
-      const int16_t* selg = Ly.sel + (int64_t)g * P->bs;
+      const int16_t* selg = Ly.sel + (int64_t)g * bs;
 #pragma unroll
       for (int q = 0; q < 4; ++q) {
         const int m = 32 * q + lane;
@@ -169,7 +193,7 @@ __device__ __forceinline__ void ws_scheduler(const StepParams* __restrict__ P, W
   };
   // tuples from selections sv of patterns m0 + 32 q + lane, appended to list
   auto scan4 = [&](const RowFetch& f, const int (&sv)[4], int m0, int n_t) -> int {
-    const DevLayer& Ly = P->layer[f.li];
+    const LayerSh& Ly = sh->lay[f.li];
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
       const int m = m0 + 32 * q + lane;
@@ -199,14 +223,14 @@ __device__ __forceinline__ void ws_scheduler(const StepParams* __restrict__ P, W
       cur = nxt;
       continue;
     }
-    const DevLayer& Ly = P->layer[cur.li];
+    const LayerSh& Ly = sh->lay[cur.li];
     const int k = cur.k;
     // ---- CP tuples of neuron k, ascending mu: the patterns whose selection
     // in its group is k ----
     int n_t = scan4(cur, cur.sv, 0, 0);
     if (bsz > 128) {
       const int g = Ly.group_of ? (int)Ly.group_of[k] : k / Ly.gamma;
-      const int16_t* selg = Ly.sel + (int64_t)g * P->bs;
+      const int16_t* selg = Ly.sel + (int64_t)g * bs;
 #pragma unroll 1
       for (int m0 = 128; m0 < bsz; m0 += 128) {
         int sv[4];
@@ -220,10 +244,8 @@ __device__ __forceinline__ void ws_scheduler(const StepParams* __restrict__ P, W
     }
     __syncwarp();
     st_rows += 1;
-    const int li = cur.li;
     const int ngrp = Ly.ngrp;
-    const uint32_t* aprev = (li == 0) ? reinterpret_cast<const uint32_t*>(P->x + start * P->nw0)
-                                      : reinterpret_cast<const uint32_t*>(P->layer[li - 1].A);
+    const uint32_t* aprev = Ly.aprev;
     const int arow_words = 2 * Ly.nw_in;
     const bool act_ok = (arow_words % 4 == 0) && (reinterpret_cast<uintptr_t>(aprev) % 16u == 0);
     if (n_t > 0) {
@@ -235,13 +257,13 @@ __device__ __forceinline__ void ws_scheduler(const StepParams* __restrict__ P, W
 #pragma unroll 1
     for (int g0 = 0; g0 < ngrp; g0 += G::kSegG) {
       if (!acquire(seq)) break;
-      const int s = (int)(seq % kSlots);
-      uint8_t* sl = slot_ptr(ring, s, G::kSlotBytes);
-      SlotMeta* meta = reinterpret_cast<SlotMeta*>(sl + G::kOffMeta);
+      const int s = (int)(seq % nslots);
+      uint8_t* sl = slot_ptr(ring, s, R.slot_bytes);
+      SlotMeta* meta = reinterpret_cast<SlotMeta*>(sl + R.off_meta);
       const int ng = min(G::kSegG, ngrp - g0);
       const int nwords = min(G::kSegG * kP, Ly.ldh - g0 * kP);              // a multiple of 4
       const uint32_t ev_bytes = (uint32_t)min(4 * G::kSegG, 8 * Ly.ev_stride - 4 * g0);
-      const uint32_t act_bytes = (uint32_t)min(4 * G::kSegG, 4 * arow_words - 4 * g0);
+      const uint32_t act_bytes = (uint32_t)min(G::kActBytes, 4 * arow_words - 4 * g0);
       const int nstage = (n_t > 0 && act_ok) ? min(n_t, G::kActT) : 0;
       for (int q = lane; q < n_t; q += 32) reinterpret_cast<uint16_t*>(sl + G::kOffTup)[q] = list[q];
       if (lane == 0) {
@@ -260,11 +282,11 @@ __device__ __forceinline__ void ws_scheduler(const StepParams* __restrict__ P, W
       if (lane == 0) {
         const uint32_t h_bytes = n_t > 0 ? 4u * (uint32_t)nwords : 0u;
         tc::mbar_arrive_tx(&sh->full[s], ev_bytes + h_bytes + (uint32_t)nstage * act_bytes);
-        sh->issued[s] = (int)(seq / kSlots);
+        sh->issued[s] = (int)(seq / nslots);
         tc::bulk_g2s(sl + G::kOffEv, evrow + g0, ev_bytes, &sh->full[s]);
         if (n_t > 0) tc::bulk_g2s(sl, meta->hrow, h_bytes, &sh->full[s]);
         for (int q = 0; q < nstage; ++q)
-          tc::bulk_g2s(sl + G::kOffAct + q * (4 * G::kSegG),
+          tc::bulk_g2s(sl + G::kOffAct + q * G::kActBytes,
                        aprev + (size_t)(list[q] & 0x7FFF) * arow_words + g0, act_bytes, &sh->full[s]);
       }
       seq += kSched;
@@ -273,9 +295,9 @@ __device__ __forceinline__ void ws_scheduler(const StepParams* __restrict__ P, W
   }
   // no more rows: an END slot for consumer group j (released by nobody)
   if (acquire(seq)) {
-    const int s = (int)(seq % kSlots);
+    const int s = (int)(seq % nslots);
     if (lane == 0) {
-      reinterpret_cast<SlotMeta*>(slot_ptr(ring, s, G::kSlotBytes) + G::kOffMeta)->type = kSlotEnd;
+      reinterpret_cast<SlotMeta*>(slot_ptr(ring, s, R.slot_bytes) + R.off_meta)->type = kSlotEnd;
       tc::mbar_arrive(&sh->full[s]);
     }
   }
@@ -297,10 +319,10 @@ __device__ __forceinline__ void ws_scheduler(const StepParams* __restrict__ P, W
 // ---------------------------------------------------------------------------
 template <int kP, bool kOnes>
 __device__ __forceinline__ void ws_consumer(const StepParams* __restrict__ P, WsShared* sh,
-                                            uint8_t* ring, int ci, int lane) {
+                                            uint8_t* ring, const Ring R, int ci, int lane) {
   using G = Geo<kP>;
-  constexpr int kSlots = Ring<kP>::kSlots;
-  constexpr int kPerLane = G::kSegG / kGroupLanes;   // groups of a segment per lane at most
+  const uint32_t nslots = (uint32_t)R.nslots;
+  constexpr int kPerLane = (G::kSegG + kGroupLanes - 1) / kGroupLanes;   // groups of a segment per lane at most
   volatile int* failed = &sh->failed;
   const Sliced<kP, kOnes> S(P->h_max);
   const int grp = ci / kPerGroup, wi = ci % kPerGroup;
@@ -308,10 +330,10 @@ __device__ __forceinline__ void ws_consumer(const StepParams* __restrict__ P, Ws
   uint64_t sparse_bytes = 0;
 #pragma unroll 1
   for (uint32_t seq = (uint32_t)grp;; seq += kSched) {
-    const int s = (int)(seq % kSlots);
-    if (!__all_sync(kFull, tc::mbar_wait(&sh->full[s], (seq / kSlots) & 1u, failed))) break;
-    uint8_t* sl = slot_ptr(ring, s, G::kSlotBytes);
-    const SlotMeta meta = *reinterpret_cast<const SlotMeta*>(sl + G::kOffMeta);
+    const int s = (int)(seq % nslots);
+    if (!__all_sync(kFull, tc::mbar_wait(&sh->full[s], (seq / nslots) & 1u, failed))) break;
+    uint8_t* sl = slot_ptr(ring, s, R.slot_bytes);
+    const SlotMeta meta = *reinterpret_cast<const SlotMeta*>(sl + R.off_meta);
     if (meta.type == kSlotEnd) break;
     const uint32_t* ev = reinterpret_cast<const uint32_t*>(sl + G::kOffEv);
     const int ng = meta.ng;
@@ -326,15 +348,21 @@ __device__ __forceinline__ void ws_consumer(const StepParams* __restrict__ P, Ws
       }
       __syncwarp();
       if (lane == 0) tc::mbar_arrive(&sh->empty[s]);
+      // two groups at a time, both loads first, so that their latencies overlap
 #pragma unroll
-      for (int q = 0; q < kPerLane; ++q) {
-        if (evs[q] == 0u) continue;
-        uint32_t* hp = meta.hrow + (size_t)(ti + q * kGroupLanes) * kP;
-        uint32_t u[kP];
-        load_planes<kP>(u, hp);
-        S.step(u, S.positive(u), evs[q]);
-        store_planes<kP>(hp, u);
-        sparse_bytes += 8ull * kP;
+      for (int q0 = 0; q0 < kPerLane; q0 += 2) {
+        uint32_t u[2][kP];
+#pragma unroll
+        for (int d = 0; d < 2 && q0 + d < kPerLane; ++d)
+          if (evs[q0 + d] != 0u)
+            load_planes<kP>(u[d], meta.hrow + (size_t)(ti + (q0 + d) * kGroupLanes) * kP);
+#pragma unroll
+        for (int d = 0; d < 2 && q0 + d < kPerLane; ++d) {
+          if (evs[q0 + d] == 0u) continue;
+          S.step(u[d], S.positive(u[d]), evs[q0 + d]);
+          store_planes<kP>(meta.hrow + (size_t)(ti + (q0 + d) * kGroupLanes) * kP, u[d]);
+          sparse_bytes += 8ull * kP;
+        }
       }
       continue;
     }
@@ -366,8 +394,8 @@ __device__ __forceinline__ void ws_consumer(const StepParams* __restrict__ P, Ws
         const uint32_t xm = (e & 0x8000u) ? kFull : 0u;   // rho = -1: complement
         uint32_t a0, a1 = 0u;
         if (q < nstage) {
-          a0 = act[q * G::kSegG + ga];
-          if (live1) a1 = act[q * G::kSegG + gb];
+          a0 = act[q * (G::kActBytes / 4) + ga];
+          if (live1) a1 = act[q * (G::kActBytes / 4) + gb];
         } else {
           const uint32_t* arow = aseg + (size_t)(e & 0x7FFFu) * arow_words;
           a0 = arow[ga];
@@ -396,18 +424,18 @@ __device__ __forceinline__ void ws_consumer(const StepParams* __restrict__ P, Ws
 
 template <int kP, bool kOnes>
 __global__ void __launch_bounds__(kThreads, 1) k_update_ws(const StepParams* __restrict__ P) {
-  using G = Geo<kP>;
-  constexpr int kSlots = Ring<kP>::kSlots;
+  const Ring R = ring_of<kP>(P->bs);
+  const int nslots = R.nslots;
   extern __shared__ uint8_t ws_raw[];
   uint8_t* ring = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(ws_raw) + 127) &
                                              ~static_cast<uintptr_t>(127));
-  WsShared* sh = reinterpret_cast<WsShared*>(ring + (size_t)kSlots * G::kSlotBytes);
+  WsShared* sh = reinterpret_cast<WsShared*>(ring + (size_t)nslots * R.slot_bytes);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   Ctrl* ctrl = P->ctrl;
   // barriers: independent of every earlier kernel
-  if (threadIdx.x < kSlots) sh->issued[threadIdx.x] = -1;
+  if (threadIdx.x < nslots) sh->issued[threadIdx.x] = -1;
   if (threadIdx.x == 0) {
-    for (int q = 0; q < kSlots; ++q) {
+    for (int q = 0; q < nslots; ++q) {
       tc::mbar_init(&sh->full[q], 1);
       tc::mbar_init(&sh->empty[q], kPerGroup);
     }
@@ -425,17 +453,27 @@ __global__ void __launch_bounds__(kThreads, 1) k_update_ws(const StepParams* __r
   // an expired bounded wait in this step's forward pass: no CP, no R (the
   // selection kernel marked nothing either); the counters still advance
   const bool step_failed = ctrl->timeouts != 0u;
+  if (threadIdx.x < P->L) {
+    const int li = threadIdx.x;
+    const DevLayer& D = P->layer[li];
+    LayerSh& o = sh->lay[li];
+    o.H = D.H; o.W = D.W; o.EV = D.EV; o.sel = D.sel; o.rho = D.rho; o.group_of = D.group_of;
+    o.aprev = li == 0 ? reinterpret_cast<const uint32_t*>(P->x + start * P->nw0)
+                      : reinterpret_cast<const uint32_t*>(P->layer[li - 1].A);
+    o.row_base = D.row_base; o.gamma = D.gamma; o.ngrp = D.ngrp; o.ldh = D.ldh; o.nw_in = D.nw_in;
+    o.ev_stride = D.ev_stride; o.Kin = D.Kin; o.pad = 0;
+  }
   for (int i = threadIdx.x; i < bsz; i += kThreads) {
     const int yv = P->y[start + i];
     sh->y[i] = (int16_t)((yv < 0 || yv >= P->c) ? 0 : yv);   // memory-safe stand-in; the host reports bad labels
   }
   __syncthreads();
   if (warp < kSched)
-    ws_scheduler<kP>(P, sh, ring, warp, lane, start, bsz, step_failed);
+    ws_scheduler<kP>(P, sh, ring, R, warp, lane, bsz, step_failed);
   else
-    ws_consumer<kP, kOnes>(P, sh, ring, warp - kSched, lane);
+    ws_consumer<kP, kOnes>(P, sh, ring, R, warp - kSched, lane);
   __syncthreads();
-  if (sh->failed && threadIdx.x < kSlots && sh->issued[threadIdx.x] >= 0) {
+  if (sh->failed && threadIdx.x < nslots && sh->issued[threadIdx.x] >= 0) {
     // after an expired wait: the copies issued into this slot land before the
     // CTA's shared memory goes away (a wait of its own, bounded)
     int own = 0;
@@ -464,23 +502,23 @@ __global__ void __launch_bounds__(kThreads, 1) k_update_ws(const StepParams* __r
 template <int kP, bool kOnes>
 cudaError_t set_smem() {
   return cudaFuncSetAttribute(k_update_ws<kP, kOnes>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              (int)Ring<kP>::kSmem);
+                              kSmemLimit);
 }
 
 template <int kP, bool kOnes>
-cudaError_t launch_one(unsigned grid, cudaStream_t st, bool pdl, const StepParams* P) {
-  return launch_kernel(k_update_ws<kP, kOnes>, dim3(grid), dim3(kThreads), Ring<kP>::kSmem, st, pdl, P);
+cudaError_t launch_one(unsigned grid, size_t smem, cudaStream_t st, bool pdl, const StepParams* P) {
+  return launch_kernel(k_update_ws<kP, kOnes>, dim3(grid), dim3(kThreads), smem, st, pdl, P);
 }
 
 }  // namespace
 
-size_t update_ws_smem(int nplanes) {
+size_t update_ws_smem(int nplanes, int bs) {
   switch (nplanes) {
-    case 1: return Ring<1>::kSmem;
-    case 2: return Ring<2>::kSmem;
-    case 4: return Ring<4>::kSmem;
-    case 8: return Ring<8>::kSmem;
-    default: return Ring<16>::kSmem;
+    case 1: return ring_of<1>(bs).smem;
+    case 2: return ring_of<2>(bs).smem;
+    case 4: return ring_of<4>(bs).smem;
+    case 8: return ring_of<8>(bs).smem;
+    default: return ring_of<16>(bs).smem;
   }
 }
 
@@ -498,15 +536,18 @@ cudaError_t update_kernel_image(cudaFuncAttributes* fa) {
   return cudaFuncGetAttributes(fa, k_update_ws<8, true>);
 }
 
-cudaError_t launch_update_ws(int nplanes, int h_max, unsigned grid, cudaStream_t st, bool pdl,
+cudaError_t launch_update_ws(int nplanes, int h_max, int bs, unsigned grid, cudaStream_t st, bool pdl,
                              const StepParams* P) {
   const bool ones = h_max == (1 << nplanes) - 1;
+  const size_t smem = update_ws_smem(nplanes, bs);
   switch (nplanes) {
-    case 1: return launch_one<1, true>(grid, st, pdl, P);
-    case 2: return launch_one<2, true>(grid, st, pdl, P);
-    case 4: return ones ? launch_one<4, true>(grid, st, pdl, P) : launch_one<4, false>(grid, st, pdl, P);
-    case 8: return ones ? launch_one<8, true>(grid, st, pdl, P) : launch_one<8, false>(grid, st, pdl, P);
-    case 16: return launch_one<16, false>(grid, st, pdl, P);
+    case 1: return launch_one<1, true>(grid, smem, st, pdl, P);
+    case 2: return launch_one<2, true>(grid, smem, st, pdl, P);
+    case 4: return ones ? launch_one<4, true>(grid, smem, st, pdl, P)
+                        : launch_one<4, false>(grid, smem, st, pdl, P);
+    case 8: return ones ? launch_one<8, true>(grid, smem, st, pdl, P)
+                        : launch_one<8, false>(grid, smem, st, pdl, P);
+    case 16: return launch_one<16, false>(grid, smem, st, pdl, P);
     default: return cudaErrorInvalidValue;
   }
 }
