@@ -47,6 +47,7 @@ constexpr int kPerGroup = 2;                  // consumer warps per group; group
 constexpr int kCons = kSched * kPerGroup;
 constexpr int kThreads = 32 * (kSched + kCons);
 constexpr int kGroupLanes = 32 * kPerGroup;
+constexpr int kGroupsInFlight = 2;            // groups of 32 weights per consumer lane at once (kP <= 8)
 constexpr int kMaxT = BMLP_MAX_BS;            // CP tuples of one row at most
 constexpr int kMaxSlots = 24;
 constexpr int kSmemLimit = 232448;            // dynamic shared memory of one CTA at most
@@ -74,7 +75,7 @@ struct Geo {
   static constexpr int kHBytes = 4 * kP * kSegG;
   static constexpr int kEvBytes = 4 * kSegG;
   static constexpr int kActBytes = 4 * kSegG;                   // one pattern's words of a segment
-  static constexpr int kActT = 2048 / kActBytes > 1 ? 2048 / kActBytes : 1;  // tuples staged at most
+  static constexpr int kActT = 4096 / kActBytes > 1 ? 4096 / kActBytes : 1;  // tuples staged at most
   static constexpr int kOffEv = kHBytes;
   static constexpr int kOffAct = kOffEv + kEvBytes;
   static constexpr int kOffTup = kOffAct + kActT * kActBytes;
@@ -99,29 +100,33 @@ struct __align__(16) WsShared {
   unsigned long long full[kMaxSlots];
   unsigned long long empty[kMaxSlots];
   int16_t y[kMaxT];                   // labels of the mini-batch (bad ones as 0)
-  uint16_t list[kSched][kMaxT];       // a scheduler's tuple scan
   unsigned long long stats[3];        // rows visited, rows streamed, algorithmic bytes
   int issued[kMaxSlots];              // last use of each slot with copies issued (-1: none)
   int failed;
 };
 
 // The ring for a mini-batch size: as many slots as fit in the shared memory
-// (a multiple of kSched, at most kMaxSlots); the host sizes the launch with
-// the same function.
+// (a multiple of kSched, at most kMaxSlots), followed by the schedulers' tuple
+// scans (kSched lists of bs entries) and WsShared; the host sizes the launch
+// with the same function.
 struct Ring {
   int slot_bytes, nslots, off_meta;
-  size_t smem;   // dynamic shared memory of the launch (128 bytes of alignment slack)
+  int list_bytes;   // one scheduler's tuple scan
+  size_t smem;      // dynamic shared memory of the launch (128 bytes of alignment slack)
 };
 
 template <int kP>
 __host__ __device__ __forceinline__ Ring ring_of(int bs) {
   Ring r;
-  r.off_meta = Geo<kP>::kOffTup + ((2 * bs + 15) & ~15);
+  const int tup = (2 * bs + 15) & ~15;
+  r.off_meta = Geo<kP>::kOffTup + tup;
   r.slot_bytes = (r.off_meta + (int)sizeof(SlotMeta) + 127) & ~127;
-  int n = (kSmemLimit - 128 - (int)sizeof(WsShared)) / r.slot_bytes;
+  r.list_bytes = tup;
+  const int fixed = 128 + kSched * r.list_bytes + (int)sizeof(WsShared);
+  int n = (kSmemLimit - fixed) / r.slot_bytes;
   n = n < kMaxSlots ? n : kMaxSlots;
   r.nslots = n / kSched * kSched;
-  r.smem = 128 + (size_t)r.nslots * r.slot_bytes + sizeof(WsShared);
+  r.smem = (size_t)fixed + (size_t)r.nslots * r.slot_bytes;
   return r;
 }
 
@@ -155,7 +160,7 @@ __device__ __forceinline__ void ws_scheduler(const StepParams* __restrict__ P, W
   const int L = P->L;
   const int bs = P->bs;
   const int rows_total = P->rows_total;
-  uint16_t* list = sh->list[j];
+  uint16_t* list = reinterpret_cast<uint16_t*>(ring + (size_t)R.nslots * R.slot_bytes + (size_t)j * R.list_bytes);
   uint32_t seq = (uint32_t)j;
   uint64_t st_rows = 0, st_streamed = 0, st_bytes = 0;
   // lane i < L holds layer i's first row and its "M_l non-empty" flag
@@ -323,6 +328,9 @@ __device__ __forceinline__ void ws_consumer(const StepParams* __restrict__ P, Ws
   using G = Geo<kP>;
   const uint32_t nslots = (uint32_t)R.nslots;
   constexpr int kPerLane = (G::kSegG + kGroupLanes - 1) / kGroupLanes;   // groups of a segment per lane at most
+  // groups a lane holds in registers at once (more give the dependent step
+  // chains of different groups to interleave)
+  constexpr int kInFlight = kP <= 8 ? kGroupsInFlight : 2;
   volatile int* failed = &sh->failed;
   const Sliced<kP, kOnes> S(P->h_max);
   const int grp = ci / kPerGroup, wi = ci % kPerGroup;
@@ -374,46 +382,45 @@ __device__ __forceinline__ void ws_consumer(const StepParams* __restrict__ P, Ws
     const int nstage = meta.nstage;
     const uint32_t* hs = reinterpret_cast<const uint32_t*>(sl);
 #pragma unroll 1
-    for (int ga = ti; ga < ng; ga += 2 * kGroupLanes) {
-      const int gb = ga + kGroupLanes;
-      const bool live1 = gb < ng;
-      const uint32_t en0 = (ga == ng - 1) ? meta.last_mask : kFull;
-      const uint32_t en1 = live1 ? ((gb == ng - 1) ? meta.last_mask : kFull) : 0u;
-      uint32_t u0[kP], u1[kP];
-      load_planes<kP>(u0, hs + (size_t)ga * kP);
-      if (live1) load_planes<kP>(u1, hs + (size_t)gb * kP);
-      else {
+    for (int g0 = ti; g0 < ng; g0 += kInFlight * kGroupLanes) {
+      // kInFlight groups of this lane: g0 + i kGroupLanes
+      uint32_t u[kInFlight][kP], en[kInFlight], r[kInFlight];
 #pragma unroll
-        for (int p = 0; p < kP; ++p) u1[p] = 0u;
+      for (int i = 0; i < kInFlight; ++i) {
+        const int g = g0 + i * kGroupLanes;
+        const bool live = g < ng;
+        en[i] = live ? (g == ng - 1 ? meta.last_mask : kFull) : 0u;
+        if (live) load_planes<kP>(u[i], hs + (size_t)g * kP);
+        else {
+#pragma unroll
+          for (int p = 0; p < kP; ++p) u[i][p] = 0u;
+        }
+        r[i] = live ? ev[g] & en[i] : 0u;
       }
-      const uint32_t r0 = ev[ga] & en0, r1 = live1 ? ev[gb] & en1 : 0u;
       // ---- CP tuples, ascending mu ----
 #pragma unroll 1
       for (int q = 0; q < n_t; ++q) {
         const uint32_t e = tl[q];
         const uint32_t xm = (e & 0x8000u) ? kFull : 0u;   // rho = -1: complement
-        uint32_t a0, a1 = 0u;
-        if (q < nstage) {
-          a0 = act[q * (G::kActBytes / 4) + ga];
-          if (live1) a1 = act[q * (G::kActBytes / 4) + gb];
-        } else {
-          const uint32_t* arow = aseg + (size_t)(e & 0x7FFFu) * arow_words;
-          a0 = arow[ga];
-          if (live1) a1 = arow[gb];
+        const uint32_t* arow = q < nstage ? act + q * (G::kActBytes / 4)
+                                          : aseg + (size_t)(e & 0x7FFFu) * arow_words;
+#pragma unroll
+        for (int i = 0; i < kInFlight; ++i) {
+          const int g = g0 + i * kGroupLanes;
+          const uint32_t a = en[i] ? arow[g] : 0u;
+          S.step(u[i], a ^ xm, en[i]);
         }
-        S.step(u0, a0 ^ xm, en0);
-        S.step(u1, a1 ^ xm, en1);
       }
       // ---- R: the events step away from 0; W = the lanes with h > 0 ----
-      const uint32_t pos0 = S.positive(u0) & en0;
-      const uint32_t pos1 = S.positive(u1) & en1;
-      S.step(u0, pos0, r0);
-      S.step(u1, pos1, r1);
-      meta.wrow[ga] = pos0;
-      store_planes<kP>(meta.hrow + (size_t)ga * kP, u0);
-      if (live1) {
-        meta.wrow[gb] = pos1;
-        store_planes<kP>(meta.hrow + (size_t)gb * kP, u1);
+#pragma unroll
+      for (int i = 0; i < kInFlight; ++i) {
+        const int g = g0 + i * kGroupLanes;
+        const uint32_t pos = S.positive(u[i]) & en[i];
+        S.step(u[i], pos, r[i]);
+        if (en[i]) {
+          meta.wrow[g] = pos;
+          store_planes<kP>(meta.hrow + (size_t)g * kP, u[i]);
+        }
       }
     }
     __syncwarp();
@@ -429,7 +436,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_update_ws(const StepParams* __r
   extern __shared__ uint8_t ws_raw[];
   uint8_t* ring = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(ws_raw) + 127) &
                                              ~static_cast<uintptr_t>(127));
-  WsShared* sh = reinterpret_cast<WsShared*>(ring + (size_t)nslots * R.slot_bytes);
+  WsShared* sh = reinterpret_cast<WsShared*>(ring + (size_t)nslots * R.slot_bytes + (size_t)kSched * R.list_bytes);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   Ctrl* ctrl = P->ctrl;
   // barriers: independent of every earlier kernel
