@@ -71,7 +71,8 @@ struct Ctrl {
   unsigned long long upd_rows;       // neuron rows visited (layers with M_l non-empty)
   unsigned long long upd_streamed;   // rows streamed (at least one CP tuple)
   unsigned long long upd_bytes;      // algorithmic bytes: H read + write and W write of the
-                                     // streamed rows, int16 read + write per sparse event
+                                     // streamed rows, the planes of a group read + written
+                                     // per group with an event of a row without tuple
   unsigned long long layer_err[BMLP_MAX_LAYERS];  // local 01-loss count of each layer
 };
 

@@ -33,28 +33,47 @@ __device__ __forceinline__ int64_t batch_size(const StepParams* P, int64_t start
 //   mark = loss or tau * r_den < r_num * K_l                         (l.14-15)
 //   for marked mu, group g: sel = argmax_{k in g} {delta_k < 0},
 //   delta_k = z_k rho_{k,y}, ties to the lowest k; -1 if none        (Alg. 2 l.4-8)
+// Launched as a programmatic dependent of the last layer's forward pass: the
+// CTAs of layers l < L read only what kernels two or more launches back wrote
+// (their layer's Z and A, the batch index), so they do all their work before
+// waiting, overlapping that forward pass; the CTAs of layer L wait first.
+// Every CTA waits before it lets the next kernel start, so a kernel two
+// launches back has always completed.
 // ---------------------------------------------------------------------------
+__device__ __forceinline__ void cls_select_body(const StepParams* __restrict__ P, int li, int mu);
+
 __global__ void __launch_bounds__(kClsThreads) k_cls_select(const StepParams* __restrict__ P) {
   const int li = blockIdx.y;
   const int mu = blockIdx.x;
+  const bool early = li < P->L - 1;
+  if (!early) pdl_wait();
+  cls_select_body(P, li, mu);
+  if (early) pdl_wait();
+  pdl_trigger();
+}
+
+__device__ __forceinline__ void cls_select_body(const StepParams* __restrict__ P, int li, int mu) {
   const DevLayer& Ly = P->layer[li];
   Ctrl* ctrl = P->ctrl;
-  pdl_wait();
-  pdl_trigger();
   const int64_t start = batch_start(P);
   const int64_t bsz = batch_size(P, start);
   if (mu >= bsz) return;
-  if (ctrl->timeouts != 0u) {
+  __shared__ int yh[BMLP_MAX_CLASSES];
+  __shared__ int s_mark, s_y, s_timeout;
+  // one read of the counter for the whole CTA (the last forward pass may be
+  // running beside an early CTA and could raise it meanwhile)
+  if (threadIdx.x == 0) s_timeout = ctrl->timeouts != 0u;
+  __syncthreads();
+  if (s_timeout) {
     // a bounded wait of this step's forward pass expired (or an earlier one
     // is not yet reported): Z and A are not valid, so the pattern is marked
     // for nothing; with every mark 0 the update leaves H and W as they are
-    // and only advances the step counters
+    // and only advances the step counters (the update kernel also skips the
+    // step on its own reading of the counter)
     if (threadIdx.x == 0) Ly.mark[mu] = 0;
     return;
   }
   const int c = P->c;
-  __shared__ int yh[BMLP_MAX_CLASSES];
-  __shared__ int s_mark, s_y;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nwarps = blockDim.x >> 5;
 
   const uint64_t* a = Ly.A + (int64_t)mu * Ly.nw_out;
