@@ -63,8 +63,8 @@ CONFIG_ORACLE_MINIBATCHES = {"C1": 20, "C2": 10, "C3": 4, "C4": 2}
 # capture of this bench (dram__bytes_read.sum + dram__bytes_write.sum, one
 # pass; see profiles/k_update_ws_c5.md), valid while the kernel sources hash to
 # UPDATE_TRAFFIC_SRC_SHA; otherwise reported as null.
-UPDATE_TRAFFIC_BYTES = None
-UPDATE_TRAFFIC_SRC_SHA = ""
+UPDATE_TRAFFIC_BYTES = 262_359_808 + 179_019_776  # dram read + write of one timed-region launch (ncu)
+UPDATE_TRAFFIC_SRC_SHA = "5de9071d4dacc413"
 UPDATE_SOURCES = ("kern_update_ws.cu", "update_common.cuh")
 # The same for one 8192 -> 8192 k_forward_eval_tc launch at 65,536 patterns
 # (profiles/k_forward_eval_tc_c5eval.md), keyed to the kernel and its shared
