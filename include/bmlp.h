@@ -315,10 +315,12 @@ int64_t bmlp_launch_count(const bmlp_t* h);
  * (synchronises): neuron rows visited (layers with a non-empty M_l), rows
  * streamed (rows with at least one CP tuple; a row without tuple changes only
  * at its reinforcement events and keeps its W), and the algorithmic bytes the
- * rule touched: per streamed row its H read and written (int16) and its W row
- * written, per reinforcement event of a row without tuple 2 bytes read and 2
- * written.  Any output may be NULL; reset != 0 zeroes the counters after
- * reading them. */
+ * rule touched: per streamed row its hidden weights read and written as the
+ * library stores them (bit-sliced: the bits of h_max rounded up to a power of
+ * two per weight, rows padded to 16 bytes) and its W row written, per group of
+ * 32 weights with a reinforcement event in a row without tuple the group's
+ * planes read and written.  Any output may be NULL; reset != 0 zeroes the
+ * counters after reading them. */
 int bmlp_update_stats(bmlp_t* h, int64_t* rows_out, int64_t* streamed_out, int64_t* bytes_out,
                       int32_t reset);
 
