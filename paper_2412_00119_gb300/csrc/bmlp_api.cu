@@ -247,10 +247,13 @@ int enqueue_step(bmlp_t* h, cudaStream_t st, bool fork, bool chained = false) {
     launch_r_events((unsigned)h->hp.ev_ctas_total, st, h->dP, h->hp.key0, h->hp.key1);
     prof_end(h, st);
   }
+  // one hidden layer whose forward pass leaves most SMs free (at most 64
+  // CTAs): the event draws start with the step
+  const bool early = h->L == 1 && ((h->K[1] + 255) / 256) * 4 <= 64;
   for (int l = 1; l <= h->L; ++l) {
-    if (fork && l == 2) {
-      // fork after the first forward pass: its CTAs hold the SMs, and the
-      // event draws and the second pass become ready together
+    if (fork && l == (early ? 1 : 2)) {
+      // otherwise fork after the first forward pass: its CTAs hold the SMs,
+      // and the event draws and the second pass become ready together
       CK(h, cudaEventRecord(h->evFork, st));
       CK(h, cudaStreamWaitEvent(h->sideStream, h->evFork, 0));
       launch_r_events((unsigned)h->hp.ev_ctas_total, h->sideStream, h->dP, h->hp.key0, h->hp.key1);
@@ -274,7 +277,7 @@ int enqueue_step(bmlp_t* h, cudaStream_t st, bool fork, bool chained = false) {
   CK(h, launch_kernel(k_cls_select, dim3((unsigned)h->bs, (unsigned)h->L), dim3(kClsThreads), 0, st,
                       fork && h->fwd_impl == BMLP_FWD_TCGEN05, h->dP));
   prof_end(h, st);
-  if (fork && h->L == 1) {
+  if (fork && h->L == 1 && !early) {
     CK(h, cudaEventRecord(h->evFork, st));
     CK(h, cudaStreamWaitEvent(h->sideStream, h->evFork, 0));
     launch_r_events((unsigned)h->hp.ev_ctas_total, h->sideStream, h->dP, h->hp.key0, h->hp.key1);
