@@ -72,6 +72,12 @@ UPDATE_SOURCES = ("kern_update_ws.cu", "update_common.cuh")
 # the launch ends, so the write figure is below the output's size.
 EVAL_TRAFFIC_BYTES = 75_599_360 + 32_936_448
 EVAL_TRAFFIC_SRC_SHA = "f8b34ceea49eb88e"
+# The same for one 8192 -> 8192 k_train_forward_tc launch at bs 100 (a layer
+# >= 2; profiles/k_train_forward_tc_c5.md): the layer's 8 MiB of visible
+# weights and the activation words read, z and the sign bits still in the
+# write-back L2 when the launch ends.
+FWD_TRAFFIC_BYTES = 8_560_384 + 0
+FWD_TRAFFIC_SRC_SHA = "63ee748cad5467c0"
 
 
 def bitpairs_per_sample(widths, classes):
@@ -403,9 +409,13 @@ def run_ours(args):
     }
     if tc:
         fp8_sus = FP8_PER_BF16 * bf16_tf_sus
+        ftraffic = None
+        if (FWD_TRAFFIC_BYTES is not None and cfg.widths[0] == cfg.widths[1] == 8192
+                and FWD_TRAFFIC_SRC_SHA == src_sha("kern_forward_tc.cu", "tc_common.cuh")):
+            ftraffic = FWD_TRAFFIC_BYTES
         kernels["train_forward"] = {
             "bound": "tensor", "achieved": 2 * bp_layer / fwd_avg_s / 1e12, "peak": fp8_sus,
-            "unit": "TFLOP/s", "frac": 2 * bp_layer / fwd_avg_s / 1e12 / fp8_sus, "traffic": None,
+            "unit": "TFLOP/s", "frac": 2 * bp_layer / fwd_avg_s / 1e12 / fp8_sus, "traffic": ftraffic,
             "avg_us": fwd_avg_s * 1e6, "algorithmic_flops": 2 * bp_layer,
             "peak_source": peak_src + " bf16 sustained x 2 (e4m3 / bf16 nominal)"}
     else:
