@@ -83,6 +83,27 @@ def test_bench_arithmetic():
         [1, 2, 4, 4, 4, 8, 8, 16, 16]
 
 
+def test_step_roofline_arithmetic():
+    """The whole-step roofline of the bench line: t_roof = max(HBM bytes at the
+    copy peak, the forward's bit-pairs at the engine's peak), frac = t_roof /
+    measured; the popcount-peak figure is reported beside it."""
+    import bench
+    w = (8192, 8192, 8192, 8192, 8192)
+    bp = 100 * bench.bitpairs_per_sample(w, 10)
+    fwd_bytes = bench.forward_weight_bytes(w)
+    assert fwd_bytes == 4 * 8192 * 128 * 8
+    upd = 433_000_000
+    r = bench.step_roofline(0.184, upd, w, 10, 6784.8, 3397.6e12, 161e12, "tensor (e4m3)")
+    t_hbm = (upd + fwd_bytes) / 6784.8e9
+    assert r["bound"] == "hbm" and abs(r["us_roof"] - t_hbm * 1e6) < 1e-9
+    assert abs(r["frac"] - t_hbm / 184e-6) < 1e-12
+    assert abs(r["vs_popcount_peak"]["us_popc"] - bp / 161e12 * 1e6) < 1e-9
+    assert abs(r["vs_popcount_peak"]["frac"] - max(t_hbm, bp / 161e12) / 184e-6) < 1e-12
+    # a compute-bound case names the engine
+    r2 = bench.step_roofline(0.184, 0, w, 10, 6784.8, 1e12, 161e12, "alu (popcount)")
+    assert r2["bound"] == "alu (popcount)" and abs(r2["us_compute"] - bp / 1e12 * 1e6) < 1e-6
+
+
 # -- neuron sharding (paper_2412_00119_gb300.sharding) ------------------------------
 
 def _sharded_worker(rank, world, port, out, *args):
