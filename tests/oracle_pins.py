@@ -12,8 +12,10 @@ Sources of the expected values:
   * exhaustive brute force of the +-1 dot product, N - 2 popcount(a XOR w);
   * exact rational arithmetic for the reinforcement probability and the
     sampler's thresholds, the law of independent Bernoulli(q) events (marginal
-    rate, pair independence, per-block binomial counts), a binomial bound on
-    the reinforcement rate, and the closed form of Alg. 1 l.21;
+    rate, pair independence, per-block binomial counts; and, for small blocks,
+    the exact probability of every event set against the product law), a
+    binomial bound on the reinforcement rate, and the closed form of Alg. 1
+    l.21;
   * invariants of Alg. 3 (odd h, |h| <= h_max, one lattice unit per event,
     reinforcement moves away from 0) and the learnability of a separable task;
   * the rank form of the lower median (brute force), the truncated network
@@ -401,6 +403,115 @@ def check_event_law():
         assert np.all(_events(q, 130, 20) == 1)
 
 
+def _least_with(V, tab, hi):
+    """The least j <= hi with V < tab[j], or hi + 1 when there is none (a
+    linear scan: the definition, not the oracle's search)."""
+    for j in range(hi + 1):
+        if V < int(tab[j]):
+            return j
+    return hi + 1
+
+
+def _block_law(any_, first, gap, n):
+    """Exact probability of every event set of an n-input block under the
+    block sampler of reading O9 with these thresholds, as Fractions: the
+    block draw U fires the block with measure any / 2^32; the first event is
+    at j with measure (first[j] - first[j-1]) / 2^32; after an event at p the
+    next comes g + 1 inputs later with measure (gap[g] - gap[g-1]) / 2^32 for
+    g <= n - 2 - p, and none with the rest.  Keys: tuples of positions."""
+    two32 = 1 << 32
+    law = {(): Fraction(two32 - any_, two32)}
+
+    def walk(events, prob):
+        p = events[-1]
+        if p == n - 1:
+            law[tuple(events)] = law.get(tuple(events), 0) + prob
+            return
+        gmax = n - 2 - p
+        stop = Fraction(two32 - int(gap[gmax]), two32)
+        law[tuple(events)] = law.get(tuple(events), 0) + prob * stop
+        prev = 0
+        for g in range(gmax + 1):
+            m = Fraction(int(gap[g]) - prev, two32)
+            prev = int(gap[g])
+            if m:
+                walk(events + [p + 1 + g], prob * m)
+
+    prev = 0
+    for j in range(n):
+        m = Fraction(int(first[j]) - prev, two32)
+        prev = int(first[j])
+        if m:
+            walk([j], Fraction(any_, two32) * m)
+    return law
+
+
+class _EventDraws:
+    """V_0, V_1, ... of one block: the words of Philox((b, k, (4 + r) 2^16 + l,
+    t)) for r = 0, 1, ..., in order."""
+
+    def __init__(self, b, k, l, t, key):
+        self.b, self.k, self.l, self.t, self.key = b, k, l, t, key
+        self.i = 0
+        self.words = []
+
+    def __call__(self):
+        if self.i % 4 == 0:
+            ctr = (self.b, self.k, ((4 + self.i // 4) << 16) + self.l, self.t)
+            self.words = [int(w) for w in O.philox4x32_10(ctr, self.key)]
+        v = self.words[self.i % 4]
+        self.i += 1
+        return v
+
+
+def check_sampler_exact_law():
+    """Reading O9 realises independent Bernoulli(q) events exactly up to the
+    2^-32 rounding of its thresholds: for small blocks, the exact probability
+    of every event set under the sampler (from the oracle's tables) sums to 1
+    and lies within (n + 2) 2^-31 of q^|S| (1-q)^(n-|S|).  And the oracle's
+    events are those the sampler's definition gives on its documented stream:
+    block draw U = word b % 4 of Philox((b/4, k, 3 * 2^16 + l, t)), event
+    draws V = the words of Philox((b, k, (4 + r) 2^16 + l, t)), r = 0, 1, ...,
+    key = (seed mod 2^32, seed div 2^32); the first event at the least j with
+    V < first[j]; after an event at p, the next at p + 1 + g for the least
+    g <= n - 2 - p with V < gap[g], else none."""
+    for q in (0.0044077, 0.05, 0.3, 0.77):
+        for n in (1, 2, 3, 5, 8):
+            any_, first, gap = O.r_block_tables(q, n)
+            law = _block_law(any_, first, gap, n)
+            assert sum(law.values()) == 1, (q, n)
+            tol = Fraction(n + 2, 1 << 31)
+            qf = Fraction(q)
+            for mask in range(1 << n):
+                S = tuple(i for i in range(n) if mask >> i & 1)
+                want = qf ** len(S) * (1 - qf) ** (n - len(S))
+                assert abs(law.get(S, Fraction(0)) - want) <= tol, (q, n, S)
+    seed, l, t = 0x1234_5678_9ABC_DEF1, 2, 77
+    key = (seed & 0xFFFFFFFF, seed >> 32)
+    for q, K_prev in ((0.05, 200), (0.3, 130), (0.0044077, 64)):
+        tabs = {n: O.r_block_tables(q, n) for n in {64, K_prev % 64 or 64}}
+        for k in range(40 if q > 0.01 else 160):
+            want = np.zeros(K_prev, np.uint8)
+            for b in range((K_prev + 63) // 64):
+                n = min(64, K_prev - 64 * b)
+                any_, first, gap = tabs[n]
+                U = int(O.philox4x32_10((b // 4, k, (3 << 16) + l, t), key)[b % 4])
+                if not U < any_:
+                    continue
+                V = _EventDraws(b, k, l, t, key)
+                p = _least_with(V(), first, n - 1)
+                want[64 * b + p] = 1
+                while p < n - 1:
+                    gmax = n - 2 - p
+                    g = _least_with(V(), gap, gmax)
+                    if g > gmax:
+                        break
+                    p += 1 + g
+                    want[64 * b + p] = 1
+            got = O.r_events(seed, l, k, t, K_prev, q)
+            assert np.array_equal(got, want), (q, K_prev, k)
+
+
 def check_update_invariants(seed=4):
     """One CP tuple changes each h of its neuron by exactly one lattice unit (2)
     unless clipped; reinforcement never flips a sign; h stays odd and bounded."""
@@ -702,6 +813,7 @@ ALL_CHECKS = [
     check_threshold_exact,
     check_reinforce_rate,
     check_event_law,
+    check_sampler_exact_law,
     check_update_invariants,
     check_training_invariants,
     check_no_mark_no_update,

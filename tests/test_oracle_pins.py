@@ -42,6 +42,11 @@ MUTANTS = [
     ("r_block_gate_ignored", "if (!((uint64_t)w[b % 4] < any[x])) continue;", "(void)any;"),
     ("r_one_event_per_block", "      if (g > n - 2 - p) break;", "      break;"),
     ("r_tail_uses_full_tables", "const int32_t x = (n == 64) ? 0 : 1;", "const int32_t x = 0;"),
+    ("r_event_stream_tag", "((4u + (uint32_t)(e->used / 4)) << 16)", "((5u + (uint32_t)(e->used / 4)) << 16)"),
+    ("r_first_scan_short", "while (p < n - 1 && !((uint64_t)V < first[x][p])) p++;",
+     "while (p < n - 2 && !((uint64_t)V < first[x][p])) p++;"),
+    ("r_gap_end_exclusive", "while (g <= n - 2 - p && !((uint64_t)V < gap[x][g])) g++;",
+     "while (g < n - 2 - p && !((uint64_t)V < gap[x][g])) g++;"),
     ("philox_7_rounds", "for (int round = 0; round < 10; round++)", "for (int round = 0; round < 7; round++)"),
     ("update_without_marks", "if (!any) continue; /* O6 */", "(void)any;"),
     ("gamma_ties_small", "(dist == best_dist && g > best)", "(dist == best_dist && g < best)"),
